@@ -1,0 +1,166 @@
+"""MixFP4 CPU oracle -- TEST INFRASTRUCTURE ONLY.
+
+A plain C restatement of the MixFP4 method (arXiv 2605.31035), wrapped with
+ctypes over numpy arrays.  Only ``tests/``, ``__graft_entry__.smoke()`` and the
+``cpu_baseline`` / ``--impl reference`` legs of ``bench.py`` may import this
+package.  The CUDA product path (``paper_2605_31035_gb300``) never imports it,
+and the two share no code.
+
+Function map (paper passages are cited in ``mixfp4_oracle.c``):
+  e4m3_value / e4m3_rne     E4M3 block scale grid and its RNE cast (Alg. 1)
+  fp4_value / fp4_rne       Table 1 / App. B.2 codebooks with the x2 E1M2 remap
+  quantize                  Algorithm 1 with type-in-scale packing (App. B.3)
+  dequantize                App. B.2/B.3 decode times the tensor scale
+  gemm_f64                  C = A_deq B_deq^T in float64
+  gemm_exact                App. B.1 Eq. (factor), exact integer accumulation
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "mixfp4_oracle.c")
+_LIB = os.path.join(_HERE, "liboracle.so")
+
+MODE_MIX, MODE_E2M1_ONLY, MODE_E1M2_ONLY = 0, 1, 2
+
+
+def build(force: bool = False) -> str:
+    """Compile the oracle with IEEE-strict flags (no FMA contraction)."""
+    if force or not os.path.exists(_LIB) or os.path.getmtime(_LIB) < os.path.getmtime(_SRC):
+        tmp = _LIB + f".tmp{os.getpid()}"
+        subprocess.check_call(
+            ["gcc", "-O2", "-ffp-contract=off", "-fno-fast-math", "-std=c11", "-fPIC", "-shared",
+             _SRC, "-o", tmp, "-lm"])
+        os.replace(tmp, _LIB)
+    return _LIB
+
+
+_lib = None
+
+
+def _L():
+    global _lib
+    if _lib is None:
+        lib = ctypes.CDLL(build())
+        P = ctypes.c_void_p
+        I64 = ctypes.c_int64
+        lib.oracle_e4m3_value.restype = ctypes.c_double
+        lib.oracle_e4m3_value.argtypes = [ctypes.c_int]
+        lib.oracle_e4m3_rne.restype = ctypes.c_int
+        lib.oracle_e4m3_rne.argtypes = [ctypes.c_float]
+        lib.oracle_fp4_value.restype = ctypes.c_double
+        lib.oracle_fp4_value.argtypes = [ctypes.c_int, ctypes.c_int]
+        lib.oracle_e1m2_stored_value.restype = ctypes.c_double
+        lib.oracle_e1m2_stored_value.argtypes = [ctypes.c_int]
+        lib.oracle_fp4_rne.restype = ctypes.c_int
+        lib.oracle_fp4_rne.argtypes = [ctypes.c_int, ctypes.c_float]
+        lib.oracle_quantize.restype = ctypes.c_int
+        lib.oracle_quantize.argtypes = [P, I64, I64, I64, ctypes.c_int, ctypes.c_int, P, P, P, P, P]
+        lib.oracle_dequantize.restype = None
+        lib.oracle_dequantize.argtypes = [P, P, ctypes.c_float, I64, I64, P]
+        lib.oracle_gemm_f64.restype = None
+        lib.oracle_gemm_f64.argtypes = [P, P, ctypes.c_float, P, P, ctypes.c_float, I64, I64, I64, P]
+        lib.oracle_gemm_exact.restype = None
+        lib.oracle_gemm_exact.argtypes = [P, P, ctypes.c_float, P, P, ctypes.c_float, I64, I64, I64, P]
+        lib.oracle_dequant_row_f64.restype = None
+        lib.oracle_dequant_row_f64.argtypes = [P, P, ctypes.c_float, I64, I64, P]
+        _lib = lib
+    return _lib
+
+
+def _p(a: np.ndarray):
+    assert a.flags["C_CONTIGUOUS"]
+    return a.ctypes.data_as(ctypes.c_void_p)
+
+
+def e4m3_value(code: int) -> float:
+    return _L().oracle_e4m3_value(int(code))
+
+
+def e4m3_rne(v: float) -> int:
+    return _L().oracle_e4m3_rne(float(v))
+
+
+def fp4_value(fmt: int, payload: int) -> float:
+    """fmt 0 = E2M1, 1 = E1M2 (x2 remapped)."""
+    return _L().oracle_fp4_value(int(fmt), int(payload))
+
+
+def e1m2_stored_value(payload: int) -> float:
+    return _L().oracle_e1m2_stored_value(int(payload))
+
+
+def fp4_rne(fmt: int, y: float) -> int:
+    return _L().oracle_fp4_rne(int(fmt), float(y))
+
+
+def quantize(x_bf16_bits: np.ndarray, mode: int = MODE_MIX, s32: float | None = None,
+             want_errors: bool = False):
+    """Algorithm 1 on a [rows, K] tensor given as uint16 bf16 bit patterns.
+
+    Returns (codes uint8 [rows, K/2], scales uint8 [rows, K/16], s32 float)
+    and, with want_errors, the per-block S of each candidate.
+    """
+    x = np.ascontiguousarray(x_bf16_bits, dtype=np.uint16)
+    rows, K = x.shape
+    codes = np.zeros((rows, K // 2), np.uint8)
+    scales = np.zeros((rows, K // 16), np.uint8)
+    s = np.array([0.0 if s32 is None else s32], np.float32)
+    e2 = np.zeros((rows, K // 16), np.float32)
+    e1 = np.zeros((rows, K // 16), np.float32)
+    rc = _L().oracle_quantize(_p(x), rows, K, K, int(mode), 0 if s32 is None else 1, _p(s),
+                              _p(codes), _p(scales), _p(e2), _p(e1))
+    if rc != 0:
+        raise ValueError("oracle_quantize rejected the input (non-finite value or K % 16 != 0)")
+    if want_errors:
+        return codes, scales, float(s[0]), e2, e1
+    return codes, scales, float(s[0])
+
+
+def dequantize(codes: np.ndarray, scales: np.ndarray, s32: float) -> np.ndarray:
+    codes = np.ascontiguousarray(codes, np.uint8)
+    scales = np.ascontiguousarray(scales, np.uint8)
+    rows, K = codes.shape[0], codes.shape[1] * 2
+    out = np.zeros((rows, K), np.float32)
+    _L().oracle_dequantize(_p(codes), _p(scales), float(s32), rows, K, _p(out))
+    return out
+
+
+def dequant_rows_f64(codes: np.ndarray, scales: np.ndarray, s32: float, rows) -> np.ndarray:
+    codes = np.ascontiguousarray(codes, np.uint8)
+    scales = np.ascontiguousarray(scales, np.uint8)
+    K = codes.shape[1] * 2
+    rows = list(rows)
+    out = np.zeros((len(rows), K), np.float64)
+    buf = np.zeros(K, np.float64)
+    for i, r in enumerate(rows):
+        _L().oracle_dequant_row_f64(_p(codes), _p(scales), float(s32), K, int(r), _p(buf))
+        out[i] = buf
+    return out
+
+
+def gemm_f64(a, b) -> np.ndarray:
+    """a, b: (codes, scales, s32) triples; returns C = A_deq B_deq^T (float64)."""
+    ac, as_, as32 = a
+    bc, bs, bs32 = b
+    ac, as_, bc, bs = (np.ascontiguousarray(t, np.uint8) for t in (ac, as_, bc, bs))
+    M, N, K = ac.shape[0], bc.shape[0], ac.shape[1] * 2
+    C = np.zeros((M, N), np.float64)
+    _L().oracle_gemm_f64(_p(ac), _p(as_), float(as32), _p(bc), _p(bs), float(bs32), M, N, K, _p(C))
+    return C
+
+
+def gemm_exact(a, b) -> np.ndarray:
+    """Exact App. B.1 factored GEMM, returned as float64 (rounded once)."""
+    ac, as_, as32 = a
+    bc, bs, bs32 = b
+    ac, as_, bc, bs = (np.ascontiguousarray(t, np.uint8) for t in (ac, as_, bc, bs))
+    M, N, K = ac.shape[0], bc.shape[0], ac.shape[1] * 2
+    C = np.zeros((M, N), np.longdouble)
+    _L().oracle_gemm_exact(_p(ac), _p(as_), float(as32), _p(bc), _p(bs), float(bs32), M, N, K, _p(C))
+    return C.astype(np.float64)

@@ -1,0 +1,296 @@
+/*
+ * MixFP4 CPU oracle -- TEST INFRASTRUCTURE ONLY.
+ *
+ * A plain, slow, deliberately unoptimised restatement of the MixFP4 method
+ * (arXiv 2605.31035).  Only tests/, __graft_entry__.smoke() and the
+ * cpu_baseline / reference legs of bench.py may load this library.  The CUDA
+ * product path never links, imports or calls it, and the two share no code.
+ *
+ * Build: gcc -O2 -ffp-contract=off -fPIC -shared (no fast-math, no FMA
+ * contraction) so every float operation below is one IEEE-754 binary32
+ * operation rounded to nearest-even, with subnormals.
+ *
+ * What each function follows:
+ *   fp_code_value      Eq. 1-2 (Sec. 2.1), the IEEE-like value of an S.E.M code
+ *   e4m3_*             E4M3 block scale (Sec. 2.1; Alg. 1 scale steps)
+ *   fp4_*              Table 1 (Sec. 3.1) and App. B.2 codebooks; the x2 E1M2
+ *                      remap of Sec. 3.1 / App. B.2
+ *   oracle_quantize    Algorithm 1 (MixFP4 quantization), with the type bit of
+ *                      App. B.3 (type-in-scale packing)
+ *   oracle_dequantize  App. B.2/B.3 decode (scale_ue4m3 = scale with bit 7
+ *                      cleared) times the per-tensor scale
+ *   oracle_gemm_f64    C = A_deq . B_deq^T in float64 (plain definition)
+ *   oracle_gemm_exact  App. B.1 Eq. (factor): per-block integer dot times the
+ *                      scale product, accumulated exactly in __int128
+ *
+ * Readings where the paper is silent (the same list is kept in the design doc):
+ *   R1 X_FP8 = fl32(X / s32) is an fp32 value (no FP8 cast).
+ *   R2 s8 = E4M3_RNE(fl32(blockmax / c)), c = 6 (E2M1) or 7 (E1M2): two
+ *      roundings, E4M3 with subnormals, saturating at 448.
+ *   R3 E1M2 quantizes in x2 units: magnitudes {0..7}, payload = integer.
+ *   R4 FP4 rounding is round-to-nearest of the fp32 quotient y = fl32(|a|/s8)
+ *      onto the codebook, ties to the even payload, saturating at the maximum.
+ *      The nibble sign bit is signbit(x).
+ *   R5 block error: d_i = fl32(q_i*s8 - |a_i|) (the product is exact);
+ *      S_even = fma chain over i = 0,2,..,14 from +0, S_odd over 1,3,..,15,
+ *      S = fl32(S_even + S_odd); the division by 16 of the mean is omitted.
+ *   R6 E2M1 is chosen iff S_E2M1 < S_E1M2 (strict), otherwise E1M2 with T=1.
+ *   R7 s8 == 0 gives all-zero magnitudes and d_i = -|a_i|; s32 == 0 gives a_i = 0.
+ *   R9 element 2j in the low nibble of byte j; codes [rows][K/2], scales
+ *      [rows][K/16], both K-major.
+ */
+#include <math.h>
+#include <stdint.h>
+#include <string.h>
+
+/* ---------------------------------------------------------------------------
+ * Eq. 1-2: value of a non-negative code with exponent field e, mantissa field
+ * m, W_M mantissa bits and bias B:  2^(e-B) (1 + m/2^W_M) for e >= 1,
+ * 2^(1-B) (m/2^W_M) for e == 0.
+ * ------------------------------------------------------------------------- */
+static double fp_code_value(int e, int m, int wm, int bias) {
+  double frac = (double)m / (double)(1 << wm);
+  if (e == 0) return ldexp(frac, 1 - bias);
+  return ldexp(1.0 + frac, e - bias);
+}
+
+/* E4M3 ("fn" variant, as in NVFP4): W_E=4, W_M=3, B=7; code 0x7F is NaN and
+ * is not a value.  Codes 0x00..0x7E are the 127 finite non-negative values. */
+double oracle_e4m3_value(int code7) {
+  int e = (code7 >> 3) & 0xF, m = code7 & 7;
+  return fp_code_value(e, m, 3, 7);
+}
+
+/* Round-to-nearest-even onto the E4M3 grid by exhaustive search (R2):
+ * the nearest finite value, ties to the code with an even mantissa LSB;
+ * anything above 448 saturates to 448 (the nearest finite value). */
+int oracle_e4m3_rne(float v) {
+  if (v >= 448.0f) return 0x7E;                     /* saturate (R2) */
+  int best = 0;
+  double bestd = INFINITY;
+  for (int c = 0; c <= 0x7E; ++c) {
+    double d = fabs((double)v - oracle_e4m3_value(c));
+    if (d < bestd || (d == bestd && (c & 1) == 0 && (best & 1) == 1)) {
+      best = c;
+      bestd = d;
+    }
+  }
+  return best;
+}
+
+/* Table 1 / App. B.2 codebooks.  type 0 = E2M1 (W_E=2, W_M=1, bias 1),
+ * type 1 = E1M2 (W_E=1, W_M=2, bias 0) followed by the fixed x2 remap of
+ * Sec. 3.1.  The payload is [p2 p1 p0]: E2M1 e=[p2p1], m=[p0];
+ * E1M2 e=[p2], m=[p1p0]. */
+double oracle_fp4_value(int type, int payload) {
+  if (type == 0) return fp_code_value((payload >> 1) & 3, payload & 1, 1, 1);
+  return 2.0 * fp_code_value((payload >> 2) & 1, payload & 3, 2, 0);
+}
+
+/* Stored (pre-remap) E1M2 magnitude, for the Table 1 pin. */
+double oracle_e1m2_stored_value(int payload) {
+  return fp_code_value((payload >> 2) & 1, payload & 3, 2, 0);
+}
+
+/* R4: nearest codebook magnitude to y >= 0, ties to the even payload;
+ * y above the maximum lands on the maximum (the nearest value). */
+int oracle_fp4_rne(int type, float y) {
+  if ((double)y >= oracle_fp4_value(type, 7)) return 7;  /* saturate (R4) */
+  int best = 0;
+  double bestd = INFINITY;
+  for (int p = 0; p < 8; ++p) {
+    double d = fabs((double)y - oracle_fp4_value(type, p));
+    if (d < bestd || (d == bestd && (p & 1) == 0 && (best & 1) == 1)) {
+      best = p;
+      bestd = d;
+    }
+  }
+  return best;
+}
+
+static float bf16_to_float(uint16_t h) {
+  uint32_t u = (uint32_t)h << 16;
+  float f;
+  memcpy(&f, &u, 4);
+  return f;
+}
+
+/* One candidate of Algorithm 1 for one 16-element block: scale, quantize,
+ * dequantize, error.  a[] holds X_FP8 for the block, B its block max. */
+static void candidate(int type, const float a[16], float B, int* s8code,
+                      int payload[16], float* S) {
+  float cmax = (type == 0) ? 6.0f : 7.0f;          /* largest magnitude */
+  float ratio = B / cmax;                           /* fl32(B / c) */
+  int code = oracle_e4m3_rne(ratio);                /* E4M3 RNE, R2 */
+  float s8 = (float)oracle_e4m3_value(code);        /* exact in fp32 */
+  float d[16];
+  for (int i = 0; i < 16; ++i) {
+    float mag = fabsf(a[i]);
+    float y = (s8 > 0.0f) ? mag / s8 : 0.0f;        /* fl32(|a|/s8), R7 */
+    int p = oracle_fp4_rne(type, y);                /* R4 */
+    float q = (float)oracle_fp4_value(type, p);
+    d[i] = q * s8 - mag;                            /* R5, product exact */
+    payload[i] = p;
+  }
+  float se = 0.0f, so = 0.0f;                       /* R5 order */
+  for (int i = 0; i < 16; i += 2) se = fmaf(d[i], d[i], se);
+  for (int i = 1; i < 16; i += 2) so = fmaf(d[i], d[i], so);
+  *S = se + so;
+  *s8code = code;
+}
+
+/* Algorithm 1 over a [rows][K] bf16 tensor (row stride ldx elements).
+ *   mode 0 = MixFP4, 1 = E2M1 only (NVFP4), 2 = E1M2 only (NVINT4)
+ *   scale_given 0: s32 = fl32(max|X| / 2688) is computed and written to *s32;
+ *   scale_given 1: *s32 is read.
+ * Optional err_e2m1 / err_e1m2 ([rows][K/16]) receive each block's S.
+ * Returns 0, or -1 on a non-finite input or K % 16 != 0. */
+int oracle_quantize(const uint16_t* x, int64_t rows, int64_t K, int64_t ldx,
+                    int mode, int scale_given, float* s32, uint8_t* codes,
+                    uint8_t* scales, float* err_e2m1, float* err_e1m2) {
+  if (K % 16 != 0) return -1;
+  float amax = 0.0f;
+  for (int64_t r = 0; r < rows; ++r)
+    for (int64_t k = 0; k < K; ++k) {
+      float v = bf16_to_float(x[r * ldx + k]);
+      if (!isfinite(v)) return -1;
+      if (fabsf(v) > amax) amax = fabsf(v);
+    }
+  float s = scale_given ? *s32 : amax / 2688.0f;   /* 2688 = 6*448 = 7*384 */
+  if (!scale_given) *s32 = s;
+
+  int64_t nb = K / 16;
+  for (int64_t r = 0; r < rows; ++r) {
+    for (int64_t b = 0; b < nb; ++b) {
+      float a[16], B = 0.0f;
+      int sign[16];
+      for (int i = 0; i < 16; ++i) {
+        float v = bf16_to_float(x[r * ldx + b * 16 + i]);
+        sign[i] = signbit(v) ? 1 : 0;
+        a[i] = (s > 0.0f) ? v / s : 0.0f;           /* X_FP8 = X / s32, R1, R7 */
+        if (fabsf(a[i]) > B) B = fabsf(a[i]);       /* block-max(|X_FP8|) */
+      }
+      int c2 = 0, c1 = 0, p2[16], p1[16];
+      float S2 = 0.0f, S1 = 0.0f;
+      if (mode != 2) candidate(0, a, B, &c2, p2, &S2);
+      if (mode != 1) candidate(1, a, B, &c1, p1, &S1);
+      int T;
+      if (mode == 1) T = 0;
+      else if (mode == 2) T = 1;
+      else T = (S2 < S1) ? 0 : 1;                   /* R6: strict < */
+      const int* p = T ? p1 : p2;
+      int code = T ? c1 : c2;
+      uint8_t* crow = codes + r * (K / 2) + b * 8;
+      for (int j = 0; j < 8; ++j) {
+        int lo = (sign[2 * j] << 3) | p[2 * j];
+        int hi = (sign[2 * j + 1] << 3) | p[2 * j + 1];
+        crow[j] = (uint8_t)(lo | (hi << 4));        /* R9 */
+      }
+      scales[r * nb + b] = (uint8_t)((T << 7) | code);  /* App. B.3 */
+      if (err_e2m1) err_e2m1[r * nb + b] = S2;
+      if (err_e1m2) err_e1m2[r * nb + b] = S1;
+    }
+  }
+  return 0;
+}
+
+/* Decode one element to its value in units of the block scale:
+ * sign * v(T, payload) (App. B.2, Sec. 3.1 remap). */
+static double decode_unit(uint8_t codebyte, int hi, int T) {
+  int nib = hi ? (codebyte >> 4) : (codebyte & 0xF);
+  double v = oracle_fp4_value(T, nib & 7);
+  return (nib & 8) ? -v : v;
+}
+
+/* App. B.3: the block scale is the scale byte with bit 7 forced to 0, and the
+ * type bit T = bit 7 selects the payload interpretation. */
+static double block_scale(uint8_t s) { return oracle_e4m3_value(s & 0x7F); }
+
+/* out = fl32(sign * v * s8 * s32); the product is exact in double. */
+void oracle_dequantize(const uint8_t* codes, const uint8_t* scales, float s32,
+                       int64_t rows, int64_t K, float* out) {
+  int64_t nb = K / 16;
+  for (int64_t r = 0; r < rows; ++r)
+    for (int64_t k = 0; k < K; ++k) {
+      uint8_t s = scales[r * nb + k / 16];
+      double v = decode_unit(codes[r * (K / 2) + k / 2], (int)(k & 1), s >> 7);
+      out[r * K + k] = (float)(v * block_scale(s) * (double)s32);
+    }
+}
+
+/* Plain definition: C[m][n] = sum_k A_deq[m][k] * B_deq[n][k] in float64,
+ * with A_deq = v * s8 * s32 exact in double. */
+void oracle_gemm_f64(const uint8_t* ac, const uint8_t* as, float as32,
+                     const uint8_t* bc, const uint8_t* bs, float bs32,
+                     int64_t M, int64_t N, int64_t K, double* C) {
+  int64_t nb = K / 16;
+  for (int64_t m = 0; m < M; ++m)
+    for (int64_t n = 0; n < N; ++n) {
+      double acc = 0.0;
+      for (int64_t k = 0; k < K; ++k) {
+        uint8_t sa = as[m * nb + k / 16], sb = bs[n * nb + k / 16];
+        double va = decode_unit(ac[m * (K / 2) + k / 2], (int)(k & 1), sa >> 7) *
+                    block_scale(sa) * (double)as32;
+        double vb = decode_unit(bc[n * (K / 2) + k / 2], (int)(k & 1), sb >> 7) *
+                    block_scale(sb) * (double)bs32;
+        acc += va * vb;
+      }
+      C[m * N + n] = acc;
+    }
+}
+
+/* Row m of A_deq (float64), for sampled checks at large sizes. */
+void oracle_dequant_row_f64(const uint8_t* codes, const uint8_t* scales,
+                            float s32, int64_t K, int64_t r, double* out) {
+  int64_t nb = K / 16;
+  for (int64_t k = 0; k < K; ++k) {
+    uint8_t s = scales[r * nb + k / 16];
+    out[k] = decode_unit(codes[r * (K / 2) + k / 2], (int)(k & 1), s >> 7) *
+             block_scale(s) * (double)s32;
+  }
+}
+
+/* Integer form of a block scale: s8 = mant * 2^(ex - 10), mant in [0, 15],
+ * ex in [1, 15] (Eq. 1 with the subnormal exponent 1 - B). */
+static void scale_int(uint8_t s, int* mant, int* ex) {
+  int e = (s >> 3) & 0xF, m = s & 7;
+  if (e == 0) { *mant = m; *ex = 1; }
+  else { *mant = 8 + m; *ex = e; }
+}
+
+/* Twice the decoded magnitude as an integer: E2M1 {0,1,2,3,4,6,8,12},
+ * E1M2 {0,2,...,14}. */
+static int unit2(uint8_t codebyte, int hi, int T) {
+  double v = decode_unit(codebyte, hi, T);
+  return (int)lrint(2.0 * v);
+}
+
+/* App. B.1 Eq. (factor): sum_b (sA_b sB_b) sum_i a_i b_i, with every term an
+ * integer times a power of two, accumulated exactly.  The element values are
+ * u/2 and the scales mant * 2^(ex-10), so each block contributes
+ * mantA*mantB*2^(exA+exB) * sum(uA*uB) in units of 2^-22.  The final value is
+ * total * 2^-22 * s32A * s32B, formed in long double. */
+void oracle_gemm_exact(const uint8_t* ac, const uint8_t* as, float as32,
+                       const uint8_t* bc, const uint8_t* bs, float bs32,
+                       int64_t M, int64_t N, int64_t K, long double* C) {
+  int64_t nb = K / 16;
+  for (int64_t m = 0; m < M; ++m)
+    for (int64_t n = 0; n < N; ++n) {
+      __int128 total = 0;
+      for (int64_t b = 0; b < nb; ++b) {
+        uint8_t sa = as[m * nb + b], sb = bs[n * nb + b];
+        int ma, ea, mb, eb;
+        scale_int(sa, &ma, &ea);
+        scale_int(sb, &mb, &eb);
+        int64_t dot = 0;
+        for (int i = 0; i < 16; ++i) {
+          int64_t k = b * 16 + i;
+          dot += (int64_t)unit2(ac[m * (K / 2) + k / 2], (int)(k & 1), sa >> 7) *
+                 unit2(bc[n * (K / 2) + k / 2], (int)(k & 1), sb >> 7);
+        }
+        total += (__int128)dot * ma * mb * ((__int128)1 << (ea + eb));
+      }
+      long double t = (long double)total;
+      C[m * N + n] = ldexpl(t, -22) * (long double)as32 * (long double)bs32;
+    }
+}

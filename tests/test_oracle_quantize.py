@@ -1,0 +1,268 @@
+"""Pins for the oracle's Algorithm 1 (CPU only).
+
+Checked against: hand-worked blocks (tests/golden/worked_blocks.txt), exact
+round trips of representable tensors, brute-force error minimisation in exact
+rational arithmetic, the type-in-scale encoding of App. B.3, invariances that
+hold by construction of the method, and the App. A crossover.
+"""
+import math
+import os
+from fractions import Fraction
+
+import numpy as np
+import pytest
+import torch
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+MODES = {"mix": 0, "e2m1": 1, "e1m2": 2}
+
+
+def bf16_bits_of(values):
+    t = torch.tensor(np.asarray(values, np.float32)).to(torch.bfloat16)
+    back = t.float().numpy()
+    assert np.array_equal(back, np.asarray(values, np.float32)), "fixture value not exact in bf16"
+    return t.view(torch.int16).numpy().view(np.uint16)
+
+
+def bits_to_f32(bits):
+    return (bits.astype(np.uint32) << 16).view(np.float32)
+
+
+def _cases():
+    cases, cur = [], None
+    with open(os.path.join(GOLDEN, "worked_blocks.txt")) as f:
+        for line in f:
+            line = line.strip()
+            if not line or line.startswith("#"):
+                continue
+            parts = line.split()
+            if parts[0] == "case":
+                cur = {"name": parts[1], "mode": MODES[parts[2]]}
+                cases.append(cur)
+            elif parts[0] == "x":
+                cur["x"] = [float(v) for v in parts[1:]]
+            elif parts[0] == "s32":
+                cur["s32"] = float(parts[1])
+            else:
+                cur[parts[0]] = [int(v, 16) for v in parts[1:]]
+    return cases
+
+
+@pytest.mark.parametrize("case", _cases(), ids=lambda c: c["name"])
+def test_worked_blocks(oracle, case):
+    x = bf16_bits_of(case["x"])[None, :]
+    codes, scales, s32 = oracle.quantize(x, mode=case["mode"])
+    assert s32 == case["s32"]
+    assert codes[0].tolist() == case["codes"]
+    assert scales[0].tolist() == case["scales"]
+
+
+def test_worked_block_errors(oracle):
+    """The error sums of the hand-worked block R (12288 and 1600)."""
+    case = _cases()[0]
+    x = bf16_bits_of(case["x"])[None, :]
+    _, _, _, e2, e1 = oracle.quantize(x, mode=0, want_errors=True)
+    assert e2[0].tolist()[0] == 0.0 and e1[0].tolist()[1] == 0.0
+    assert e2[0, 2] == 12288.0 and e1[0, 2] == 1600.0
+
+
+def _representable_tensor(rng, rows, nb, e_s32):
+    """X = q * s8 * s32 with s32 = 2^e_s32; each block is E2M1- or E1M2-exact
+    with block max 6*s8 or 7*s8, and one block carries the tensor max 2688*s32."""
+    x = np.zeros((rows, nb * 16), np.float64)
+    e2m1 = np.array([0, 0.5, 1, 1.5, 2, 3, 4, 6])
+    for r in range(rows):
+        for b in range(nb):
+            if r == 0 and b == 0:
+                s8, typ = 448.0, 0
+            else:
+                typ = rng.integers(0, 2)
+                # a normal E4M3 scale well inside the range
+                s8 = float((8 + rng.integers(0, 8)) * 2.0 ** rng.integers(-6, 3))
+            if typ == 0:
+                q = rng.choice(e2m1, 16)
+                q[rng.integers(0, 16)] = 6
+            else:
+                q = rng.integers(0, 8, 16).astype(np.float64)
+                q[rng.integers(0, 16)] = 7
+            sign = rng.choice([-1.0, 1.0], 16)
+            x[r, b * 16:(b + 1) * 16] = sign * q * s8 * 2.0 ** e_s32
+    return x.astype(np.float32)
+
+
+@pytest.mark.parametrize("e_s32", [-12, -3, 0, 5])
+def test_exact_round_trip(oracle, e_s32):
+    rng = np.random.default_rng(100 + e_s32)
+    x = _representable_tensor(rng, 4, 6, e_s32)
+    bits = bf16_bits_of(x)
+    codes, scales, s32, e2, e1 = oracle.quantize(bits, want_errors=True)
+    assert s32 == 2.0 ** e_s32
+    back = oracle.dequantize(codes, scales, s32)
+    assert np.array_equal(back, x)
+    chosen = np.where(scales >> 7, e1, e2)
+    assert np.all(chosen == 0.0)
+
+
+def _exact_block_errors(a_block, s8, fmt, book):
+    """Exact sum of squared errors of the codes the oracle would pick, in Fractions."""
+    out = Fraction(0)
+    for a in a_block:
+        y = Fraction(abs(a))
+        best = min(range(8), key=lambda p: (abs(Fraction(book[p]) * Fraction(s8) - y), p % 2))
+        out += (Fraction(book[best]) * Fraction(s8) - y) ** 2
+    return out
+
+
+def test_brute_force_tiny_blocks(oracle):
+    """Every code minimises |v*s8 - |a|| over all 8 payloads of its format
+    (ties to the even payload), the scale byte is the E4M3 value nearest to
+    blockmax/c (torch cast), and the selected format has the smaller exact
+    error whenever the two exact errors differ by more than fp32 noise."""
+    rng = np.random.default_rng(5)
+    grid = np.array([0, 0.25, 0.5, 0.75, 1, 1.25, 1.5, 2, 2.5, 3, 3.5, 4, 5, 6, 7, 8, 10, 12], np.float32)
+    rows, nb = 24, 8
+    x = rng.choice(grid, (rows, nb * 16)) * rng.choice([-1, 1], (rows, nb * 16))
+    x = (x * (2.0 ** rng.integers(-4, 4, (rows, 1)))).astype(np.float32)
+    x[0, 0] = 2688.0  # s32 = 1 so X_FP8 = X exactly
+    bits = bf16_bits_of(x)
+    codes, scales, s32 = oracle.quantize(bits)
+    assert s32 == 1.0
+    books = [[oracle.fp4_value(f, p) for p in range(8)] for f in (0, 1)]
+    for r in range(rows):
+        for b in range(nb):
+            a = x[r, b * 16:(b + 1) * 16].astype(np.float64)
+            T = scales[r, b] >> 7
+            s8 = oracle.e4m3_value(scales[r, b] & 0x7F)
+            B = np.float32(np.abs(a).max())
+            c = np.float32(7.0 if T else 6.0)
+            ref_code = torch.tensor([float(B / c)], dtype=torch.float32).to(torch.float8_e4m3fn)
+            assert int(ref_code.view(torch.uint8)) == scales[r, b] & 0x7F
+            book = books[T]
+            for i in range(16):
+                nib = (codes[r, b * 8 + i // 2] >> (4 * (i & 1))) & 0xF
+                assert (nib >> 3) == (1 if math.copysign(1, a[i]) < 0 else 0)
+                y = Fraction(abs(float(a[i]))) / Fraction(s8) if s8 > 0 else Fraction(0)
+                dists = [abs(Fraction(book[p]) - y) for p in range(8)]
+                best = min(range(8), key=lambda p: (dists[p], p % 2))
+                assert (nib & 7) == best, (r, b, i)
+            # exact comparison of the two candidates
+            errs = []
+            for fmt in (0, 1):
+                s8f = oracle.e4m3_value(oracle.e4m3_rne(float(np.float32(B / np.float32(6.0 if fmt == 0 else 7.0)))))
+                errs.append(_exact_block_errors(a, s8f, fmt, books[fmt]))
+            if errs[0] != errs[1] and abs(errs[0] - errs[1]) > Fraction(1, 10 ** 5) * max(errs):
+                assert T == (0 if errs[0] < errs[1] else 1), (r, b, errs)
+            if errs[0] == errs[1]:
+                assert T == 1  # strict "<" of Alg. 1: ties go to E1M2
+
+
+def test_type_bit_consistency(oracle):
+    """App. B.3: a MixFP4 block with T=0 is byte-identical to the E2M1-only
+    (NVFP4) quantization of the same block, and with T=1 to the E1M2-only one."""
+    from paper_2605_31035_gb300 import synth
+    x = synth.bf16_bits(synth.activations(32, 256, 11, 12))
+    cm, sm, s32 = oracle.quantize(x, mode=0)
+    c2, s2, s32b = oracle.quantize(x, mode=1)
+    c1, s1, s32c = oracle.quantize(x, mode=2)
+    assert s32 == s32b == s32c
+    T = (sm >> 7).astype(bool)
+    assert T.any() and (~T).any()
+    assert np.all((s2 >> 7) == 0) and np.all((s1 >> 7) == 1)
+    assert np.array_equal(sm[~T], s2[~T]) and np.array_equal(sm[T], s1[T])
+    cm_b = cm.reshape(32, -1, 8)
+    assert np.array_equal(cm_b[~T], c2.reshape(32, -1, 8)[~T])
+    assert np.array_equal(cm_b[T], c1.reshape(32, -1, 8)[T])
+
+
+def test_scaling_negation_permutation_invariance(oracle):
+    from paper_2605_31035_gb300 import synth
+    xt = synth.activations(16, 512, 21, 22)
+    base = oracle.quantize(synth.bf16_bits(xt))
+    for k in (-5, 3):
+        sc = oracle.quantize(synth.bf16_bits(xt * 2.0 ** k))
+        assert np.array_equal(sc[0], base[0]) and np.array_equal(sc[1], base[1])
+        assert sc[2] == base[2] * 2.0 ** k
+    neg = oracle.quantize(synth.bf16_bits(-xt))
+    assert np.array_equal(neg[1], base[1])
+    assert np.array_equal(neg[0], base[0] ^ 0x88)
+    perm = torch.randperm(16, generator=torch.Generator().manual_seed(3))
+    pq = oracle.quantize(synth.bf16_bits(xt[perm]))
+    assert np.array_equal(pq[0], base[0][perm.numpy()]) and np.array_equal(pq[1], base[1][perm.numpy()])
+
+
+def test_zero_and_tiny_blocks(oracle):
+    """Alg. 1 degenerate cases: an all-zero tensor (s32 = 0, every error 0,
+    ties go to E1M2) and blocks whose scale rounds to E4M3 zero."""
+    z = np.zeros((2, 32), np.uint16)
+    codes, scales, s32 = oracle.quantize(z)
+    assert s32 == 0.0 and not codes.any() and np.all(scales == 0x80)
+    codes, scales, _ = oracle.quantize(z, mode=1)
+    assert np.all(scales == 0x00)
+    negz = np.full((1, 16), 0x8000, np.uint16)  # -0.0 keeps its sign nibble
+    codes, scales, _ = oracle.quantize(negz)
+    assert np.all(codes == 0x88) and scales[0, 0] == 0x80
+    # block max far below s32 * 2^-10: both scales round to E4M3 zero
+    x = np.zeros((1, 32), np.float32)
+    x[0, 0] = 2688.0
+    x[0, 16:] = 2.0 ** -14
+    codes, scales, s32 = oracle.quantize(bf16_bits_of(x))
+    assert s32 == 1.0 and scales[0, 1] == 0x80 and not (codes[0, 8:] & 0x77).any()
+
+
+def test_rejects_bad_input(oracle):
+    with pytest.raises(ValueError):
+        oracle.quantize(np.full((1, 16), 0x7FC0, np.uint16))  # NaN
+    with pytest.raises(ValueError):
+        oracle.quantize(np.zeros((1, 24), np.uint16))
+
+
+def _crossover_equation(kappa):
+    """App. A: R_NVFP4(kappa) - R_NVINT4(kappa) with g=16, alpha=1/96, beta=1/1728."""
+    t = kappa / 6.0
+    phi = math.exp(-t * t / 2) / math.sqrt(2 * math.pi)
+    Phi = 0.5 * (1 + math.erf(t / math.sqrt(2)))
+    w = 2 * (t * phi + 1 - Phi)
+    r_fp = (w - kappa ** 2 / 16) / 96 + kappa ** 2 * (2 * Phi - 1) / 1728
+    r_int = kappa ** 2 / (12 * 49) * 15 / 16
+    return r_fp - r_int, r_int
+
+
+def test_appendix_a_crossover_constants():
+    vals = {}
+    with open(os.path.join(GOLDEN, "appendix_a_crossover.txt")) as f:
+        for line in f:
+            if line.strip() and not line.startswith("#"):
+                k, v = line.split()
+                vals[k] = float(v)
+    lo, hi = 1.5, 3.0
+    for _ in range(200):
+        mid = (lo + hi) / 2
+        if _crossover_equation(mid)[0] > 0:
+            lo = mid
+        else:
+            hi = mid
+    k = (lo + hi) / 2
+    assert abs(k - vals["kappa_star"]) < 1e-12
+    r = _crossover_equation(k)[1]
+    assert abs(r - vals["R_star"]) < 1e-14
+    assert abs(-10 * math.log10(r) - vals["QSNR_star_dB"]) < 1e-9
+
+
+def test_crest_factor_selection_trend(oracle):
+    """Statistical sanity (App. A, Sec. 2.2): MixFP4 picks E1M2 mostly for
+    flat blocks (low crest factor) and E2M1 mostly for peaked ones."""
+    g = torch.Generator().manual_seed(9)
+    z = torch.randn(512, 16 * 64, generator=g)
+    z[:, 0] = 40.0  # fixes s32 well above every block so the scale is not the limiter
+    bits = synth_bits(z)
+    _, scales, _ = oracle.quantize(bits)
+    blocks = z.reshape(512, 64, 16)[:, 1:]
+    kappa = (blocks.abs().amax(-1) / blocks.pow(2).mean(-1).sqrt()).numpy()
+    t = (scales[:, 1:] >> 7).astype(bool)
+    low, high = kappa < 2.0, kappa > 3.0
+    assert t[low].mean() > 0.6
+    assert t[high].mean() < 0.4
+
+
+def synth_bits(t):
+    return t.to(torch.bfloat16).view(torch.int16).numpy().view(np.uint16)
