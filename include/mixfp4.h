@@ -1,0 +1,133 @@
+/*
+ * mixfp4.h -- C ABI of libmixfp4.so, the GB300 (sm_103a) MixFP4 W4A4 linear
+ * layer: an online MixFP4 quantizer, its decoder, and a MixFP4 x MixFP4 GEMM.
+ *
+ * MixFP4 (arXiv 2605.31035) extends NVFP4: every 16-element block along the
+ * reduction dimension K stores sixteen 4-bit codes and one 8-bit block scale.
+ * Each code is [s | p2 p1 p0] (App. B.2): a sign bit and a 3-bit payload read
+ * as FP4 E2M1 {0,.5,1,1.5,2,3,4,6} or as FP4 E1M2 remapped x2 to {0,..,7}
+ * (Table 1, Sec. 3.1).  The scale byte carries the block's format in bit 7
+ * (T = 0 E2M1, T = 1 E1M2) and the unsigned E4M3 block scale s8 in bits 6:0
+ * (App. B.3).  A tensor adds one fp32 per-tensor scale s32 (Alg. 1).
+ * An element's value is  (-1)^s * v(T, p) * s8 * s32.
+ *
+ * Storage layout (the paper fixes none; this library's choice):
+ *   codes  uint8 [rows][K/2]   element 2j of a row in the low nibble of byte j
+ *   scales uint8 [rows][K/16]  one byte per block, blocks in K order
+ *   both row-major with no padding (row pitch K/2 and K/16 bytes).
+ *
+ * Conventions for every entry point:
+ *   - All tensor pointers are DEVICE pointers owned by the caller; the library
+ *     allocates no device memory and keeps no per-call state.
+ *   - Work is enqueued asynchronously on `stream` (a cudaStream_t; NULL = the
+ *     legacy default stream).  The return value reports argument validation
+ *     and launch errors only; results are ready once the stream is synchronised.
+ *   - Invalid arguments return a negative mixfp4_status and enqueue nothing.
+ *     No entry point traps or aborts.
+ *   - Inputs must be finite; NaN or Inf input gives unspecified codes.
+ */
+#ifndef MIXFP4_H
+#define MIXFP4_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  MIXFP4_OK = 0,
+  MIXFP4_ERR_NULL = -1,    /* a required pointer is NULL */
+  MIXFP4_ERR_SHAPE = -2,   /* a size is negative, or violates a multiple-of rule */
+  MIXFP4_ERR_ALIGN = -3,   /* a pointer or leading dimension is misaligned */
+  MIXFP4_ERR_DTYPE = -4,   /* unsupported input dtype */
+  MIXFP4_ERR_CUDA = -5,    /* a CUDA runtime call or launch failed */
+  MIXFP4_ERR_TIMEOUT = -6, /* a bounded device-side wait gave up (see status_word) */
+  MIXFP4_ERR_ARG = -7      /* an enum argument is out of range */
+} mixfp4_status;
+
+enum { MIXFP4_MODE_MIX = 0,        /* Alg. 1: per-block E2M1/E1M2 by lower MSE */
+       MIXFP4_MODE_E2M1_ONLY = 1,  /* every block E2M1, T = 0 (plain NVFP4 bits) */
+       MIXFP4_MODE_E1M2_ONLY = 2   /* every block E1M2, T = 1 (NVINT4 lattice) */ };
+
+enum { MIXFP4_SCALE_COMPUTE = 0,   /* compute s32 = fl32(max|x| / 2688), write *tensor_scale */
+       MIXFP4_SCALE_GIVEN = 1      /* read s32 from *tensor_scale */ };
+
+enum { MIXFP4_DTYPE_BF16 = 0 };
+
+/*
+ * mixfp4_quantize -- Algorithm 1 (Sec. 3.2) with type-in-scale packing (App. B.3).
+ *
+ *   s32  = fl32(max|X| / 2688)              (2688 = 6*448 = 7*384)
+ *   a_i  = fl32(x_i / s32)                   per element (0 when s32 == 0)
+ *   per 16-element block with B = max|a_i|, for c in {E2M1 (max 6), E1M2 (max 7)}:
+ *     s8_c = E4M3_RNE(fl32(B / max_c))       (subnormals, saturating at 448)
+ *     q_i  = RNE_c(fl32(|a_i| / s8_c))       nearest codebook value, ties to the
+ *                                            even payload, saturating (q = 0 if s8_c = 0)
+ *     S_c  = S_even + S_odd, fma chains of d_i^2 over even / odd i, d_i = q_i*s8_c - |a_i|
+ *   E2M1 iff S_E2M1 < S_E1M2 (strict), else E1M2 with T = 1.
+ *
+ * x            device, bf16 [rows][ldx]; 32-byte aligned; ldx % 16 == 0, ldx >= K.
+ * dtype        MIXFP4_DTYPE_BF16.
+ * rows, K      rows >= 0, K >= 0, K % 16 == 0.  rows*K == 0 is a valid no-op
+ *              (with SCALE_COMPUTE, *tensor_scale is still set to 0).
+ * codes        device, uint8 [rows][K/2], 8-byte aligned.            (output)
+ * scales       device, uint8 [rows][K/16].                           (output)
+ * tensor_scale device, one float: written (COMPUTE) or read (GIVEN).  A given
+ *              s32 must be finite and >= 0, and max|x| / s32 must be finite.
+ * workspace    device, one uint32 scratch word; required with SCALE_COMPUTE
+ *              (it receives max|x|), ignored with SCALE_GIVEN.  Calls that share
+ *              a workspace word must be ordered on the GPU.
+ * mode         MIXFP4_MODE_*.   scale_flag  MIXFP4_SCALE_*.
+ */
+int mixfp4_quantize(const void* x, int dtype, int64_t rows, int64_t K, int64_t ldx,
+                    uint8_t* codes, uint8_t* scales, float* tensor_scale,
+                    uint32_t* workspace, int mode, int scale_flag, void* stream);
+
+/*
+ * mixfp4_dequantize -- App. B.2/B.3 decode:
+ *   out[r][k] = fl32((-1)^s * v(T, p) * ue4m3(scale & 0x7F) * s32),
+ * one rounding of the exact product.
+ *
+ * codes        device, uint8 [rows][K/2], 8-byte aligned.
+ * scales       device, uint8 [rows][K/16].
+ * tensor_scale device, one float s32.
+ * rows, K      rows >= 0, K % 16 == 0.
+ * out          device, float [rows][K], 32-byte aligned.                (output)
+ */
+int mixfp4_dequantize(const uint8_t* codes, const uint8_t* scales, const float* tensor_scale,
+                      int64_t rows, int64_t K, float* out, void* stream);
+
+/*
+ * mixfp4_gemm -- MixFP4 x MixFP4 GEMM, C = A_deq . B_deq^T:
+ *   C[m][n] = s32A * s32B * sum_blocks (sA * sB) * sum_i vA_i * vB_i
+ * (App. B.1 Eq. (factor)), where each block's codes are decoded to the unified
+ * E2M2 value (Sec. 3.3, App. B.5) times its E4M3 scale -- exact in bf16 -- and
+ * contracted on the tensor cores with fp32 accumulation.
+ *
+ * a_codes/a_scales/a_ts   A = activations, M x K, quantized by mixfp4_quantize.
+ * b_codes/b_scales/b_ts   B = weights (nn.Linear layout), N x K.
+ * M, N, K      M >= 0, N >= 0, K % 256 == 0; M and N need no padding.
+ * C            device, float [M][ldc], ldc >= N, 4-byte aligned (16-byte alignment
+ *              and ldc % 4 == 0 enable vector stores).                      (output)
+ * status_word  device uint32 or NULL.  When given it is zeroed by the call and
+ *              becomes nonzero if a bounded device-side pipeline wait gave up
+ *              (C is then unspecified); the caller reads it after synchronising.
+ * Code and scale pointers must be 16-byte aligned.
+ */
+int mixfp4_gemm(const uint8_t* a_codes, const uint8_t* a_scales, const float* a_ts,
+                const uint8_t* b_codes, const uint8_t* b_scales, const float* b_ts,
+                int64_t M, int64_t N, int64_t K, float* C, int64_t ldc,
+                uint32_t* status_word, void* stream);
+
+/* Human-readable name of a mixfp4_status value (static string). */
+const char* mixfp4_status_string(int status);
+
+/* ABI version of this library (major * 100 + minor). */
+int mixfp4_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* MIXFP4_H */

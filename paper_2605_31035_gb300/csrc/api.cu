@@ -1,0 +1,104 @@
+// C ABI of libmixfp4.so (declared in include/mixfp4.h): argument validation,
+// status codes, and kernel launches.  No entry point allocates device memory.
+#include <cuda_runtime.h>
+#include <cstdint>
+
+#include "kernels.cuh"
+
+namespace {
+
+inline bool aligned(const void* p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+inline int launch_status() {
+  return cudaGetLastError() == cudaSuccess ? MIXFP4_OK : MIXFP4_ERR_CUDA;
+}
+
+}  // namespace
+
+extern "C" {
+
+int mixfp4_version(void) { return 100; }
+
+const char* mixfp4_status_string(int status) {
+  switch (status) {
+    case MIXFP4_OK: return "ok";
+    case MIXFP4_ERR_NULL: return "null pointer";
+    case MIXFP4_ERR_SHAPE: return "invalid shape";
+    case MIXFP4_ERR_ALIGN: return "misaligned pointer or leading dimension";
+    case MIXFP4_ERR_DTYPE: return "unsupported dtype";
+    case MIXFP4_ERR_CUDA: return "CUDA error";
+    case MIXFP4_ERR_TIMEOUT: return "device-side wait timed out";
+    case MIXFP4_ERR_ARG: return "argument out of range";
+    default: return "unknown status";
+  }
+}
+
+int mixfp4_quantize(const void* x, int dtype, int64_t rows, int64_t K, int64_t ldx,
+                    uint8_t* codes, uint8_t* scales, float* tensor_scale, uint32_t* workspace,
+                    int mode, int scale_flag, void* stream) {
+  if (dtype != MIXFP4_DTYPE_BF16) return MIXFP4_ERR_DTYPE;
+  if (mode < MIXFP4_MODE_MIX || mode > MIXFP4_MODE_E1M2_ONLY) return MIXFP4_ERR_ARG;
+  if (scale_flag != MIXFP4_SCALE_COMPUTE && scale_flag != MIXFP4_SCALE_GIVEN) return MIXFP4_ERR_ARG;
+  if (rows < 0 || K < 0 || K % 16 != 0 || ldx < K) return MIXFP4_ERR_SHAPE;
+  if (!tensor_scale) return MIXFP4_ERR_NULL;
+  if (scale_flag == MIXFP4_SCALE_COMPUTE && !workspace) return MIXFP4_ERR_NULL;
+  const bool empty = (rows == 0 || K == 0);
+  if (!empty && (!x || !codes || !scales)) return MIXFP4_ERR_NULL;
+  if (!empty && (!aligned(x, 32) || ldx % 16 != 0 || !aligned(codes, 8))) return MIXFP4_ERR_ALIGN;
+  if (!aligned(tensor_scale, 4) || (workspace && !aligned(workspace, 4))) return MIXFP4_ERR_ALIGN;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const int given = scale_flag == MIXFP4_SCALE_GIVEN;
+  if (empty) {
+    if (!given && cudaMemsetAsync(tensor_scale, 0, sizeof(float), s) != cudaSuccess)
+      return MIXFP4_ERR_CUDA;
+    return MIXFP4_OK;
+  }
+  const uint16_t* xb = static_cast<const uint16_t*>(x);
+  if (!given) {
+    if (cudaMemsetAsync(workspace, 0, sizeof(uint32_t), s) != cudaSuccess) return MIXFP4_ERR_CUDA;
+    mixfp4::launch_amax(xb, rows, K, ldx, workspace, s);
+    if (int st = launch_status()) return st;
+  }
+  mixfp4::launch_quantize(xb, rows, K, ldx, codes, scales, tensor_scale, workspace, mode, given, s);
+  return launch_status();
+}
+
+int mixfp4_dequantize(const uint8_t* codes, const uint8_t* scales, const float* tensor_scale,
+                      int64_t rows, int64_t K, float* out, void* stream) {
+  if (rows < 0 || K < 0 || K % 16 != 0) return MIXFP4_ERR_SHAPE;
+  if (rows == 0 || K == 0) return MIXFP4_OK;
+  if (!codes || !scales || !tensor_scale || !out) return MIXFP4_ERR_NULL;
+  if (!aligned(codes, 8) || !aligned(out, 32) || !aligned(tensor_scale, 4)) return MIXFP4_ERR_ALIGN;
+  mixfp4::launch_dequantize(codes, scales, tensor_scale, rows, K, out, static_cast<cudaStream_t>(stream));
+  return launch_status();
+}
+
+int mixfp4_gemm(const uint8_t* a_codes, const uint8_t* a_scales, const float* a_ts,
+                const uint8_t* b_codes, const uint8_t* b_scales, const float* b_ts,
+                int64_t M, int64_t N, int64_t K, float* C, int64_t ldc,
+                uint32_t* status_word, void* stream) {
+  if (M < 0 || N < 0 || K < 0 || K % 256 != 0 || ldc < N) return MIXFP4_ERR_SHAPE;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (status_word) {
+    if (!aligned(status_word, 4)) return MIXFP4_ERR_ALIGN;
+    if (cudaMemsetAsync(status_word, 0, sizeof(uint32_t), s) != cudaSuccess) return MIXFP4_ERR_CUDA;
+  }
+  if (M == 0 || N == 0) return MIXFP4_OK;
+  if (!C) return MIXFP4_ERR_NULL;
+  if (!aligned(C, 4)) return MIXFP4_ERR_ALIGN;
+  if (K == 0) {  // empty reduction: C = 0
+    if (cudaMemset2DAsync(C, (size_t)ldc * sizeof(float), 0, (size_t)N * sizeof(float), (size_t)M, s) != cudaSuccess)
+      return MIXFP4_ERR_CUDA;
+    return MIXFP4_OK;
+  }
+  if (!a_codes || !a_scales || !a_ts || !b_codes || !b_scales || !b_ts) return MIXFP4_ERR_NULL;
+  if (!aligned(a_codes, 16) || !aligned(a_scales, 16) || !aligned(b_codes, 16) ||
+      !aligned(b_scales, 16) || !aligned(a_ts, 4) || !aligned(b_ts, 4))
+    return MIXFP4_ERR_ALIGN;
+  int st = mixfp4::launch_gemm(a_codes, a_scales, a_ts, b_codes, b_scales, b_ts, M, N, K, C, ldc,
+                               status_word, s);
+  if (st) return st;
+  return launch_status();
+}
+
+}  // extern "C"

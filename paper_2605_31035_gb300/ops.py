@@ -1,0 +1,139 @@
+"""Thin ctypes binding over libmixfp4.so (C ABI in include/mixfp4.h).
+
+Each function marshals torch CUDA tensors to device pointers and the current
+stream, calls the entry point of the same name, and raises on a nonzero status.
+All arithmetic runs in the library's CUDA kernels; there is no fallback.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from dataclasses import dataclass
+
+import torch
+
+MODE_MIX, MODE_E2M1_ONLY, MODE_E1M2_ONLY = 0, 1, 2
+SCALE_COMPUTE, SCALE_GIVEN = 0, 1
+DTYPE_BF16 = 0
+
+STATUS = {0: "ok", -1: "null pointer", -2: "invalid shape", -3: "misaligned", -4: "unsupported dtype",
+          -5: "CUDA error", -6: "device-side wait timed out", -7: "argument out of range"}
+
+_LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "libmixfp4.so")
+_lib = None
+
+
+class MixFP4Error(RuntimeError):
+    def __init__(self, fn: str, status: int):
+        super().__init__(f"{fn} failed: {STATUS.get(status, status)} ({status})")
+        self.status = status
+
+
+def lib() -> ctypes.CDLL:
+    """Load libmixfp4.so; raise if it has not been built (no fallback exists)."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(_LIB_PATH):
+            raise RuntimeError(
+                f"{_LIB_PATH} is missing: build it with `python -c 'import __graft_entry__ as g; g.build()'`")
+        L = ctypes.CDLL(_LIB_PATH)
+        P, I64, I = ctypes.c_void_p, ctypes.c_int64, ctypes.c_int
+        L.mixfp4_quantize.restype = I
+        L.mixfp4_quantize.argtypes = [P, I, I64, I64, I64, P, P, P, P, I, I, P]
+        L.mixfp4_dequantize.restype = I
+        L.mixfp4_dequantize.argtypes = [P, P, P, I64, I64, P, P]
+        L.mixfp4_gemm.restype = I
+        L.mixfp4_gemm.argtypes = [P, P, P, P, P, P, I64, I64, I64, P, I64, P, P]
+        L.mixfp4_status_string.restype = ctypes.c_char_p
+        L.mixfp4_status_string.argtypes = [I]
+        L.mixfp4_version.restype = I
+        L.mixfp4_version.argtypes = []
+        _lib = L
+    return _lib
+
+
+def _ptr(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream=None):
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+def _check(fn: str, status: int):
+    if status != 0:
+        raise MixFP4Error(fn, status)
+
+
+@dataclass
+class QTensor:
+    """A MixFP4 tensor: codes [rows, K/2], scales [rows, K/16], s32 (1 float), all on one device."""
+    codes: torch.Tensor
+    scales: torch.Tensor
+    tensor_scale: torch.Tensor
+
+    @property
+    def rows(self) -> int:
+        return self.codes.shape[0]
+
+    @property
+    def K(self) -> int:
+        return self.codes.shape[1] * 2
+
+
+def empty_qtensor(rows: int, K: int, device) -> QTensor:
+    return QTensor(torch.empty(rows, K // 2, dtype=torch.uint8, device=device),
+                   torch.empty(rows, K // 16, dtype=torch.uint8, device=device),
+                   torch.empty(1, dtype=torch.float32, device=device))
+
+
+def mixfp4_quantize(x: torch.Tensor, mode: int = MODE_MIX, tensor_scale: torch.Tensor | None = None,
+                    out: QTensor | None = None, workspace: torch.Tensor | None = None,
+                    stream=None) -> QTensor:
+    """Quantize a bf16 [rows, K] CUDA tensor (row stride may exceed K).
+
+    With tensor_scale=None the per-tensor scale is computed (max|x| / 2688);
+    otherwise the given 1-element fp32 tensor is used as s32.
+    """
+    assert x.dtype == torch.bfloat16 and x.dim() == 2 and x.stride(1) == 1
+    rows, K = x.shape
+    q = out if out is not None else empty_qtensor(rows, K, x.device)
+    given = tensor_scale is not None
+    if given:
+        q.tensor_scale.copy_(tensor_scale.reshape(1))
+    ws = None
+    if not given:
+        ws = workspace if workspace is not None else torch.empty(1, dtype=torch.int32, device=x.device)
+    st = lib().mixfp4_quantize(_ptr(x), DTYPE_BF16, rows, K, x.stride(0), _ptr(q.codes), _ptr(q.scales),
+                               _ptr(q.tensor_scale), _ptr(ws), int(mode),
+                               SCALE_GIVEN if given else SCALE_COMPUTE, _stream(stream))
+    _check("mixfp4_quantize", st)
+    return q
+
+
+def mixfp4_dequantize(q: QTensor, out: torch.Tensor | None = None, stream=None) -> torch.Tensor:
+    o = out if out is not None else torch.empty(q.rows, q.K, dtype=torch.float32, device=q.codes.device)
+    st = lib().mixfp4_dequantize(_ptr(q.codes), _ptr(q.scales), _ptr(q.tensor_scale), q.rows, q.K,
+                                 _ptr(o), _stream(stream))
+    _check("mixfp4_dequantize", st)
+    return o
+
+
+def mixfp4_gemm(a: QTensor, b: QTensor, out: torch.Tensor | None = None,
+                status_word: torch.Tensor | None = None, stream=None) -> torch.Tensor:
+    """C = A_deq . B_deq^T in fp32; a is M x K, b is N x K."""
+    assert a.K == b.K
+    M, N, K = a.rows, b.rows, a.K
+    C = out if out is not None else torch.empty(M, N, dtype=torch.float32, device=a.codes.device)
+    st = lib().mixfp4_gemm(_ptr(a.codes), _ptr(a.scales), _ptr(a.tensor_scale),
+                           _ptr(b.codes), _ptr(b.scales), _ptr(b.tensor_scale),
+                           M, N, K, _ptr(C), C.stride(0), _ptr(status_word), _stream(stream))
+    _check("mixfp4_gemm", st)
+    return C
+
+
+def linear(x: torch.Tensor, w_q: QTensor, mode: int = MODE_MIX, stream=None) -> torch.Tensor:
+    """W4A4 linear: quantize the activations online, then the MixFP4 GEMM with
+    pre-quantized weights.  Returns x_deq . w_deq^T in fp32."""
+    return mixfp4_gemm(mixfp4_quantize(x, mode, stream=stream), w_q, stream=stream)

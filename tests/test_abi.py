@@ -1,0 +1,86 @@
+"""C ABI of libmixfp4.so (CPU only): the library builds and loads, exports
+every entry point include/mixfp4.h declares, and rejects invalid arguments
+with the documented status codes before touching the GPU."""
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2605_31035_gb300 import build, ops
+    build.build()
+    return ops.lib()
+
+
+def declared_functions():
+    text = open(os.path.join(ROOT, "include", "mixfp4.h")).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(mixfp4_\w+)\s*\(", text)))
+
+
+def test_exports_every_declared_symbol(lib):
+    names = declared_functions()
+    assert {"mixfp4_quantize", "mixfp4_dequantize", "mixfp4_gemm"} <= set(names)
+    for n in names:
+        assert hasattr(lib, n), n
+
+
+def test_version_and_status_strings(lib):
+    assert lib.mixfp4_version() >= 100
+    for code in range(0, -8, -1):
+        assert lib.mixfp4_status_string(code)
+    assert lib.mixfp4_status_string(0) == b"ok"
+
+
+def test_quantize_validation(lib):
+    fake = ctypes.c_void_p(1 << 20)  # never dereferenced: validation fails first
+    ws = ctypes.c_void_p(1 << 21)
+    q = lib.mixfp4_quantize
+    assert q(fake, 7, 4, 32, 32, fake, fake, fake, ws, 0, 0, None) == -4        # dtype
+    assert q(fake, 0, 4, 24, 24, fake, fake, fake, ws, 0, 0, None) == -2        # K % 16
+    assert q(fake, 0, 4, 32, 16, fake, fake, fake, ws, 0, 0, None) == -2        # ldx < K
+    assert q(fake, 0, -1, 32, 32, fake, fake, fake, ws, 0, 0, None) == -2       # rows < 0
+    assert q(fake, 0, 4, 32, 32, fake, fake, fake, ws, 3, 0, None) == -7        # mode
+    assert q(fake, 0, 4, 32, 32, fake, fake, fake, ws, 0, 2, None) == -7        # scale flag
+    assert q(None, 0, 4, 32, 32, fake, fake, fake, ws, 0, 0, None) == -1        # x null
+    assert q(fake, 0, 4, 32, 32, fake, fake, fake, None, 0, 0, None) == -1      # workspace
+    assert q(ctypes.c_void_p((1 << 20) + 2), 0, 4, 32, 32, fake, fake, fake, ws, 0, 0, None) == -3
+    assert q(fake, 0, 4, 32, 40, fake, fake, fake, ws, 0, 1, None) == -3        # ldx % 16
+
+
+def test_dequantize_and_gemm_validation(lib):
+    fake = ctypes.c_void_p(1 << 20)
+    assert lib.mixfp4_dequantize(fake, fake, fake, 4, 24, fake, None) == -2
+    assert lib.mixfp4_dequantize(None, fake, fake, 4, 32, fake, None) == -1
+    assert lib.mixfp4_dequantize(fake, fake, fake, 4, 32, ctypes.c_void_p((1 << 20) + 16), None) == -3
+    g = lib.mixfp4_gemm
+    assert g(fake, fake, fake, fake, fake, fake, 4, 4, 128, fake, 4, None, None) == -2   # K % 256
+    assert g(fake, fake, fake, fake, fake, fake, 4, 8, 256, fake, 4, None, None) == -2   # ldc < N
+    assert g(fake, fake, fake, fake, fake, fake, -1, 4, 256, fake, 4, None, None) == -2
+    assert g(fake, fake, fake, fake, fake, fake, 4, 4, 256, None, 4, None, None) == -1
+    assert g(fake, fake, fake, fake, fake, fake, 4, 4, 256, ctypes.c_void_p((1 << 20) + 2), 4, None, None) == -3
+    assert g(None, fake, fake, fake, fake, fake, 4, 4, 256, fake, 4, None, None) == -1
+
+
+def test_header_documents_each_entry_point():
+    text = open(os.path.join(ROOT, "include", "mixfp4.h")).read()
+    for name in ("mixfp4_quantize", "mixfp4_dequantize", "mixfp4_gemm"):
+        block = text[:text.index(f"int {name}(")]
+        doc = block[block.rindex("/*"):]
+        assert any(s in doc for s in ("Algorithm 1", "App. B")), name
+        assert "device" in doc.lower()
+
+
+def test_product_path_has_no_oracle_or_cpu_fallback():
+    pkg = os.path.join(ROOT, "paper_2605_31035_gb300")
+    for dirpath, _, files in os.walk(pkg):
+        for f in files:
+            if f.endswith((".py", ".cu", ".cuh", ".h")):
+                src = open(os.path.join(dirpath, f)).read()
+                assert "import oracle" not in src and "from oracle" not in src, f
+                assert "liboracle" not in src, f
