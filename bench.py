@@ -1,0 +1,421 @@
+"""Benchmark of the MixFP4 W4A4 linear layer on GB300.
+
+One step = one pass of the hot path over one batch of the Llama-3-8B
+attention-projection workload (X 2048x4096 bf16 Student-t activations with
+outlier channels, W 4096x4096 bf16 weights): amax + MixFP4 quantization of X
+(Algorithm 1), then the MixFP4 x MixFP4 GEMM against W quantized once
+beforehand.  The metric is the layer's throughput in TFLOP/s (2*M*N*K per
+step); the quantizer's GB/s on a 2^28-element activation (larger than L2) is
+reported beside it.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+With N > 1 (launched by torch.distributed.run) every rank runs an independent
+replica on its own GPU -- the layer has no cross-GPU exchange -- and rank 0
+prints ONE JSON line with the whole-job throughput (max time over ranks).
+``--impl reference`` times the plain CPU oracle on bounded samples of the same
+workload on the host cores.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "MixFP4 GEMM TFLOP/s + quantizer GB/s, each as % of GB300 roofline"
+WORKLOAD = "attn"
+QUANT_BYTES_PER_ELEM = 2.0 + 0.5 + 1.0 / 16.0   # bf16 in, nibble codes + scale bytes out
+
+
+def peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        d = json.load(open(p))
+        return {"hbm_gbs": d["hbm_gbs"], "bf16_tflops": d["bf16_tflops"],
+                "bf16_tflops_sustained": d.get("bf16_tflops_sustained"), "source": "measured"}
+    return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0, "source": "fallback"}
+
+
+def kernel_hash(name: str) -> str:
+    src = os.path.join(ROOT, "paper_2605_31035_gb300", "csrc", name)
+    return hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+
+
+def ncu_traffic(key: str, src: str):
+    """DRAM bytes per launch from a committed ncu summary, if it was taken on
+    the current kernel source; otherwise None."""
+    p = os.path.join(ROOT, "profiles", "ncu_traffic.json")
+    if not os.path.exists(p):
+        return None
+    d = json.load(open(p)).get(key)
+    if not d or d.get("source_sha") != kernel_hash(src):
+        return None
+    return d.get("dram_bytes_per_launch")
+
+
+class ClockSampler:
+    """nvidia-smi samples of SM clock and throttle reasons during the timed region."""
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+
+    def __enter__(self):
+        fd, self.path = tempfile.mkstemp(suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "100"], stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except OSError:
+            self.proc = None
+        time.sleep(0.3)
+        return self
+
+    def __exit__(self, *a):
+        if self.proc is not None:
+            time.sleep(0.2)
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self, t0: float | None = None):
+        rows = []
+        if self.path and os.path.exists(self.path):
+            for line in open(self.path):
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) < 9:
+                    continue
+                try:
+                    rows.append((float(parts[1]), float(parts[2]), parts[5:9]))
+                except ValueError:
+                    continue
+            os.unlink(self.path)
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"], "samples": 0}
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for _, _, flags in rows for i, f in enumerate(flags) if f.lower() == "active"})
+        return {"sm_mhz": statistics.median(r[0] for r in rows), "sm_max_mhz": max(r[1] for r in rows),
+                "reasons": reasons, "samples": len(rows)}
+
+
+def dist_setup(n_gpus: int):
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    if ws > 1:
+        import torch.distributed as dist
+        backend = "nccl" if os.environ.get("MIXFP4_BENCH_BACKEND", "nccl") == "nccl" else "gloo"
+        dist.init_process_group(backend)
+        return dist.get_rank(), ws, int(os.environ.get("LOCAL_RANK", "0"))
+    return 0, 1, 0
+
+
+def reduce_max(value: float, device) -> float:
+    """Max of a per-rank scalar over the job (identity without a process group)."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()):
+        return value
+    t = torch.tensor([value], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def barrier():
+    import torch.distributed as dist
+    if dist.is_available() and dist.is_initialized():
+        dist.barrier()
+
+
+# ----------------------------------------------------------------------------- ours
+def run_ours(args):
+    import torch
+    from paper_2605_31035_gb300 import build, ops, synth
+
+    rank, world, local = dist_setup(args.gpus)
+    build.build()
+    dev = torch.device(f"cuda:{local}")
+    torch.cuda.set_device(dev)
+    stream = torch.cuda.current_stream(dev)
+    lin = synth.workloads()[WORKLOAD].linears[0]
+    M, N, K = lin.M, lin.N, lin.K
+    flops = 2.0 * M * N * K
+    pk = peaks()
+
+    x_cpu = lin.make_x()
+    x = x_cpu.to(dev)
+    w_q = ops.mixfp4_quantize(lin.make_w().to(dev))          # weights quantized once
+    q_x = ops.empty_qtensor(M, K, dev)
+    ws = torch.empty(1, dtype=torch.int32, device=dev)
+    C = torch.empty(M, N, dtype=torch.float32, device=dev)
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)   # > 129 MB L2
+
+    def step():
+        ops.mixfp4_quantize(x, out=q_x, workspace=ws)
+        ops.mixfp4_gemm(q_x, w_q, out=C)
+
+    for _ in range(args.warmup):
+        flush.zero_()
+        step()
+    torch.cuda.synchronize(dev)
+
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
+    barrier()
+    torch.cuda.synchronize(dev)
+    with ClockSampler(local) as clk:
+        for i in range(args.steps):
+            flush.zero_()
+            ev[i][0].record(stream)
+            ops.mixfp4_quantize(x, out=q_x, workspace=ws)
+            ev[i][1].record(stream)
+            ops.mixfp4_gemm(q_x, w_q, out=C)
+            ev[i][2].record(stream)
+        torch.cuda.synchronize(dev)
+    barrier()
+    step_ms = [e[0].elapsed_time(e[2]) for e in ev]
+    quant_ms = [e[0].elapsed_time(e[1]) for e in ev]
+    gemm_ms = [e[1].elapsed_time(e[2]) for e in ev]
+    total_ms = reduce_max(sum(step_ms), dev)
+    ms_per_step = total_ms / args.steps
+    value = world * args.steps * flops / (total_ms * 1e-3) / 1e12
+    gemm_avg = statistics.mean(gemm_ms)
+    gemm_tflops = flops / (gemm_avg * 1e-3) / 1e12
+    quant_avg = statistics.mean(quant_ms)
+    clocks = clk.summary()
+
+    # Quantizer alone on a 2^28-element activation (512 MiB bf16 > L2), SCALE_COMPUTE.
+    xs = synth.sweep_activation(28).to(dev)
+    qs = ops.empty_qtensor(xs.shape[0], xs.shape[1], dev)
+    for _ in range(3):
+        ops.mixfp4_quantize(xs, out=qs, workspace=ws)
+    qev = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(10)]
+    for e in qev:
+        e[0].record(stream)
+        ops.mixfp4_quantize(xs, out=qs, workspace=ws)
+        e[1].record(stream)
+    torch.cuda.synchronize(dev)
+    sweep_ms = statistics.median(a.elapsed_time(b) for a, b in qev)
+    sweep_alg_gbs = xs.numel() * QUANT_BYTES_PER_ELEM / (sweep_ms * 1e-3) / 1e9
+    sweep_read_gbs = xs.numel() * (QUANT_BYTES_PER_ELEM + 2.0) / (sweep_ms * 1e-3) / 1e9
+    del xs, qs
+
+    # End to end through the public API with host buffers: pinned X in, C out.
+    x_host = x_cpu.pin_memory()
+    c_host = torch.empty(M, N, dtype=torch.float32).pin_memory()
+    x_dev = torch.empty_like(x)
+    for _ in range(3):
+        x_dev.copy_(x_host, non_blocking=True)
+        ops.linear(x_dev, w_q)
+        c_host.copy_(C, non_blocking=True)
+    torch.cuda.synchronize(dev)
+    e2e_steps = max(10, min(args.steps, 200))
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    barrier()
+    e0.record(stream)
+    for _ in range(e2e_steps):
+        x_dev.copy_(x_host, non_blocking=True)
+        ops.mixfp4_quantize(x_dev, out=q_x, workspace=ws)
+        ops.mixfp4_gemm(q_x, w_q, out=C)
+        c_host.copy_(C, non_blocking=True)
+    e1.record(stream)
+    torch.cuda.synchronize(dev)
+    e2e_ms = reduce_max(e0.elapsed_time(e1), dev)
+    e2e_value = world * e2e_steps * flops / (e2e_ms * 1e-3) / 1e12
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cpu = cpu_baseline(lin, x_cpu, budget_s=args.cpu_budget)
+
+    peak_t = pk["bf16_tflops"]
+    traffic = ncu_traffic(f"gemm_{WORKLOAD}", "gemm.cu")
+    out = {
+        "metric": METRIC, "value": round(value, 2), "unit": "TFLOP/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_per_step, 5),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic",
+        "config": {"workload": f"Llama-3-8B attention projection: X {M}x{K} . W {N}x{K} (MixFP4 W4A4)",
+                   "M": M, "N": N, "K": K, "mode": "MixFP4", "weights": "pre-quantized once",
+                   "l2": "flushed between steps (256 MiB write, outside the step events)",
+                   "parallelism": f"replicas x{world}"},
+        "roofline": {"bound": "tensor", "kernel": "mixfp4_gemm_kernel",
+                     "achieved": round(gemm_tflops, 2), "peak": peak_t, "unit": "TFLOP/s",
+                     "frac": round(gemm_tflops / peak_t, 4),
+                     "peak_kind": f"bf16 dense burst, {pk['source']} (MEASURED_PEAKS.json)",
+                     "traffic": traffic},
+        "kernels": {
+            "gemm_ms": round(gemm_avg, 5), "gemm_tflops": round(gemm_tflops, 2),
+            "quantize_with_amax_ms": round(quant_avg, 5),
+            "quantize_with_amax_gbs_alg": round(M * K * QUANT_BYTES_PER_ELEM / (quant_avg * 1e-3) / 1e9, 1),
+            "quantizer_2^28": {"ms": round(sweep_ms, 4), "alg_gbs": round(sweep_alg_gbs, 1),
+                               "alg_frac_of_hbm": round(sweep_alg_gbs / pk["hbm_gbs"], 4),
+                               "bytes_incl_amax_read_gbs": round(sweep_read_gbs, 1),
+                               "hbm_peak_gbs": pk["hbm_gbs"]}},
+        "clocks": clocks,
+        "e2e": {"value": round(e2e_value, 2), "unit": "TFLOP/s",
+                "h2d_bytes_per_step": x_host.numel() * 2, "d2h_bytes_per_step": c_host.numel() * 4,
+                "steps": e2e_steps},
+        "gpu_launches": 3 * args.steps,
+        "cpu_baseline": cpu,
+    }
+    if rank == 0:
+        print(json.dumps(out), flush=True)
+
+
+# ------------------------------------------------------------------ CPU oracle legs
+class OracleLayer:
+    """The hot path on the CPU oracle: Algorithm 1 on sampled rows of X (with
+    the full tensor's s32) and the float64 GEMM against sampled rows of W,
+    which are quantized once up front like the GPU path's weights."""
+
+    def __init__(self, lin, x_cpu, w_cpu, max_w_rows: int):
+        import numpy as np
+        import oracle
+        from paper_2605_31035_gb300 import synth
+        self.lin = lin
+        self.x_bits = synth.bf16_bits(x_cpu)
+        self.s32 = float(np.float32(np.float32(float(x_cpu.abs().max().float())) / np.float32(2688.0)))
+        ws32 = float(np.float32(np.float32(float(w_cpu.abs().max().float())) / np.float32(2688.0)))
+        self.wq = oracle.quantize(synth.bf16_bits(w_cpu[:max_w_rows]), s32=ws32)
+
+    def run(self, n_rows_x: int, n_rows_w: int, row0: int = 0):
+        """Returns (seconds, flops) of one sampled pass."""
+        import oracle
+        wq = (self.wq[0][:n_rows_w], self.wq[1][:n_rows_w], self.wq[2])
+        xs = self.x_bits[row0:row0 + n_rows_x]
+        t0 = time.perf_counter()
+        xq = oracle.quantize(xs, s32=self.s32)
+        oracle.gemm_f64(xq, wq)
+        return time.perf_counter() - t0, 2.0 * n_rows_x * n_rows_w * self.lin.K
+
+
+def _calibrated_rows(layer: OracleLayer, n_rows_x: int, budget_s: float, cap: int) -> int:
+    secs, _ = layer.run(1, 16)
+    return max(8, min(cap, int(16 * budget_s / (max(secs, 1e-4) * n_rows_x))))
+
+
+def cpu_baseline(lin, x_cpu, budget_s: float = 15.0):
+    cap = 2048
+    layer = OracleLayer(lin, x_cpu, lin.make_w()[:cap], cap)
+    n_w = _calibrated_rows(layer, 4, budget_s, cap)
+    secs, flops = layer.run(4, n_w)
+    return {"value": flops / secs / 1e12, "unit": "TFLOP/s", "cores": 1, "kind": "oracle",
+            "sample": f"Algorithm 1 on 4 rows of X + float64 GEMM vs {n_w} pre-quantized rows of W "
+                      f"(K={lin.K}), {secs:.1f} s single-threaded"}
+
+
+def run_reference(args):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    from paper_2605_31035_gb300 import synth
+    lin = synth.workloads()[WORKLOAD].linears[0]
+    x_cpu = lin.make_x()
+    cap = 1024
+    layer = OracleLayer(lin, x_cpu, lin.make_w()[:cap], cap)
+    per_step_budget = max(0.01, min(1.0, 150.0 / max(1, args.steps + args.warmup)))
+    n_w = _calibrated_rows(layer, 1, per_step_budget, cap)
+    for i in range(args.warmup):
+        layer.run(1, n_w, row0=i % lin.M)
+    tot, fl = 0.0, 0.0
+    for i in range(args.steps):
+        s, f = layer.run(1, n_w, row0=i % lin.M)
+        tot += s
+        fl += f
+    value = fl / tot / 1e12
+    out = {"metric": METRIC, "value": value, "unit": "TFLOP/s", "n_gpus": int(os.environ.get("WORLD_SIZE", "1")),
+           "steps": args.steps, "warmup": args.warmup, "ms_per_step": tot / args.steps * 1e3,
+           "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+           "data": "synthetic", "impl": "reference",
+           "config": {"workload": f"Llama-3-8B attention projection: X {lin.M}x{lin.K} . W {lin.N}x{lin.K} (MixFP4 W4A4)",
+                      "M": lin.M, "N": lin.N, "K": lin.K, "mode": "MixFP4"},
+           "cpu_baseline": {"value": value, "unit": "TFLOP/s", "cores": 1, "kind": "oracle",
+                            "sample": f"per step: Algorithm 1 on 1 row of X + float64 GEMM vs {n_w} "
+                                      f"pre-quantized rows of W (K={lin.K}), single-threaded"},
+           "gpu_launches": 0,
+           "e2e": {"value": value, "unit": "TFLOP/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(out), flush=True)
+
+
+def run_kernel_only(args):
+    """One kernel on one workload, for profilers: `--warmup` untimed launches,
+    then `--steps` launches, then exit.  Prints the CUDA-event time per launch."""
+    import torch
+    from paper_2605_31035_gb300 import build, ops, synth
+    build.build()
+    dev = torch.device("cuda:0")
+    if args.workload.startswith("sweep"):
+        x = synth.sweep_activation(int(args.workload[5:])).to(dev)
+        w = None
+    else:
+        lin = synth.workloads()[args.workload].linears[0]
+        x = lin.make_x().to(dev)
+        w = lin.make_w().to(dev)
+    ws = torch.empty(1, dtype=torch.int32, device=dev)
+    qx = ops.mixfp4_quantize(x, workspace=ws)
+    if args.kernel == "gemm":
+        qw = ops.mixfp4_quantize(w, workspace=ws)
+        C = torch.empty(x.shape[0], w.shape[0], dtype=torch.float32, device=dev)
+        fn = lambda: ops.mixfp4_gemm(qx, qw, out=C)
+        work = 2.0 * x.shape[0] * w.shape[0] * x.shape[1]
+    elif args.kernel == "quantize":
+        fn = lambda: ops.mixfp4_quantize(x, out=qx, workspace=ws)
+        work = x.numel() * QUANT_BYTES_PER_ELEM
+    else:
+        out = torch.empty(x.shape, dtype=torch.float32, device=dev)
+        fn = lambda: ops.mixfp4_dequantize(qx, out=out)
+        work = x.numel() * (0.5 + 1.0 / 16 + 4.0)
+    for _ in range(args.warmup):
+        fn()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(args.steps):
+        fn()
+    e1.record()
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / args.steps
+    unit = "TFLOP/s" if args.kernel == "gemm" else "GB/s"
+    rate = work / (ms * 1e-3) / (1e12 if args.kernel == "gemm" else 1e9)
+    print(json.dumps({"kernel": args.kernel, "workload": args.workload, "ms": round(ms, 5),
+                      "rate": round(rate, 1), "unit": unit}))
+
+
+def main(argv=None):
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=1000)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--cpu-budget", type=float, default=15.0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--kernel", choices=["gemm", "quantize", "dequantize"], default=None,
+                    help="profiling mode: launch only this kernel")
+    ap.add_argument("--workload", default=WORKLOAD,
+                    help="tiny|attn|mlp|decode|hadamard|sweepNN (kernel-only mode)")
+    args = ap.parse_args(argv)
+    if args.kernel:
+        return run_kernel_only(args)
+    if args.warmup < 3:
+        ap.error("--warmup must be >= 3")
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()
