@@ -120,6 +120,33 @@ int mixfp4_gemm(const uint8_t* a_codes, const uint8_t* a_scales, const float* a_
                 int64_t M, int64_t N, int64_t K, float* C, int64_t ldc,
                 uint32_t* status_word, void* stream);
 
+/*
+ * mixfp4_quantize_noalloc -- mixfp4_quantize with MIXFP4_SCALE_COMPUTE for
+ * callers that cannot allocate device memory.  The paper has no counterpart;
+ * this is a deployment convenience.
+ *
+ * mixfp4_quantize needs a caller-provided scratch word (`workspace`) to
+ * compute the per-tensor scale.  Callers such as an inference runtime that
+ * plans all device memory ahead of time and gives an operator only its input
+ * and output buffers, or a plugin whose execute callback must not call
+ * cudaMalloc, have no such word.  This entry point keeps it in a 256-byte
+ * file-scope device array of the library instead and allocates nothing.
+ *
+ * Arguments and results are those of mixfp4_quantize with SCALE_COMPUTE:
+ * x, dtype, rows, K, ldx, codes, scales, mode and stream as documented there;
+ * tensor_scale (device, one float) receives s32.
+ *
+ * The first call on a device looks up the array's device address for that
+ * device (make it before any stream capture).  Every call shares the array,
+ * and the array keeps the last call's contents (it is cleared before each
+ * use); calls that overlap on the GPU race on it and must be ordered.  Any
+ * shape needs one 32-bit word of the 64 the array holds; a larger need would
+ * be rejected with MIXFP4_ERR_SHAPE.
+ */
+int mixfp4_quantize_noalloc(const void* x, int dtype, int64_t rows, int64_t K, int64_t ldx,
+                            uint8_t* codes, uint8_t* scales, float* tensor_scale, int mode,
+                            void* stream);
+
 /* Human-readable name of a mixfp4_status value (static string). */
 const char* mixfp4_status_string(int status);
 
