@@ -1,21 +1,28 @@
 // MixFP4 x MixFP4 GEMM for sm_103a: C = A_deq . B_deq^T (App. B.1 Eq. (factor)).
 //
 // Per 16-element block the MixFP4 codes are decoded to the unified E2M2 value
-// (Sec. 3.3, App. B.5) times the block's E4M3 scale.  Written as 2*v*s8 that
-// product has at most 7 significant bits and lies in [2^-9, 2*7*448], so it is
-// exact in bf16; the tensor cores then contract bf16 x bf16 with fp32
-// accumulation (tcgen05.mma kind::f16, K = 16 = one block per instruction) and
-// the epilogue applies s32A * s32B / 4.
+// (Sec. 3.3, App. B.5) times the block's E4M3 scale.  Written as u * s8 with
+// u = 2v (E2M1: {0,1,2,3,4,6,8,12}, E1M2: {0,2,...,14}) the product has at most
+// 7 significant bits and lies in [2^-9, 14 * 448], so it is exact in f16; the
+// tensor cores contract f16 x f16 with fp32 accumulation (tcgen05.mma
+// kind::f16, K = 16 per instruction) and the epilogue applies s32A * s32B / 4.
 //
-// One CTA computes a 128 x 256 tile of C:
-//   warp 0      TMA producer: packed codes [rows][128 B] (128-byte swizzle) and
-//               scales [rows][16 B] for a 256-wide K slice, into a 2-deep ring;
-//   warp 1      TMEM allocator and single-thread MMA issuer (accumulator
-//               128 lanes x 256 fp32 columns in tensor memory);
-//   warps 2-13  decoders, one thread per tile row (128 A rows + 256 B rows):
-//               each turns 64 K of its row per sub-stage into bf16 in the
-//               canonical K-major no-swizzle UMMA layout, in a 2-deep ring;
-//   warps 2-9   after the K loop: epilogue, tcgen05.ld -> scale -> global fp32.
+// Work decomposition: persistent CTA pairs (clusters of 2, cta_group::2).  A
+// pair owns 256 x 256 output tiles; each CTA holds 128 rows of A and 128 rows
+// (half) of B, so each CTA decodes 256 rows per K step while its tensor core
+// produces a 128 x 256 slab.  Per CTA:
+//   warp 0      TMA producer: codes [rows][128 B] (128-byte swizzle) and
+//               scales [rows][16 B] of a 256-wide K slice into a 3-deep ring;
+//   warp 1      TMEM allocator (both CTAs); in the leader CTA also the single
+//               MMA-issuing thread.  Accumulators: 2 x (128 lanes x 256 fp32)
+//               per CTA, double-buffered across tiles;
+//   warps 2-17  decoders, two threads per operand row (128 A + 128 B), each
+//               turning 32 K of the row per sub-stage into f16 in the
+//               canonical K-major no-swizzle UMMA layout, 3-deep ring.  The
+//               leader's MMA waits for both CTAs' decoders (remote mbarrier
+//               arrivals);
+//   warps 18-21 epilogue: tcgen05.ld -> x s32A s32B / 4 -> fp32 C, overlapped
+//               with the next tile's main loop.
 // All pipeline waits are bounded; a wait that gives up records a nonzero
 // status word and the CTA drains and exits without touching C.
 #include <cuda.h>
@@ -32,24 +39,29 @@ namespace {
 
 using namespace sm100;
 
-constexpr int BM = 128;            // tile rows of A (MMA M)
-constexpr int BN = 256;            // tile rows of B (MMA N)
+constexpr int BM = 128;            // A rows per CTA (pair tile: 256)
+constexpr int BNH = 128;           // B rows per CTA (pair tile: 256)
+constexpr int TILE_M = 2 * BM, TILE_N = 2 * BNH;
 constexpr int BKC = 256;           // K per TMA code stage
 constexpr int BKD = 64;            // K per decoded sub-stage
-constexpr int kSub = BKC / BKD;    // sub-stages per code stage
-constexpr int kCodeStages = 2;
-constexpr int kDecStages = 2;
-constexpr int kDecodeWarps = (BM + BN) / 32;   // 12
-constexpr int kThreads = 32 * (2 + kDecodeWarps);
-constexpr uint32_t kTmemCols = 256;
+constexpr int kSub = BKC / BKD;
+constexpr int kCodeStages = 3;
+constexpr int kDecStages = 3;
+constexpr int kDecodeWarps = 2 * (BM + BNH) / 32;   // 16: two threads per operand row
+constexpr int kEpiWarps = 4;
+constexpr int kFirstDecodeWarp = 2;
+constexpr int kFirstEpiWarp = kFirstDecodeWarp + kDecodeWarps;  // 18
+constexpr int kThreads = 32 * (kFirstEpiWarp + kEpiWarps);      // 704
+constexpr uint32_t kAccCols = TILE_N;           // fp32 columns per accumulator
+constexpr uint32_t kTmemCols = 2 * kAccCols;    // double-buffered
 
 constexpr int A_CODE_BYTES = BM * BKC / 2;
-constexpr int B_CODE_BYTES = BN * BKC / 2;
+constexpr int B_CODE_BYTES = BNH * BKC / 2;
 constexpr int A_SCALE_BYTES = BM * BKC / 16;
-constexpr int B_SCALE_BYTES = BN * BKC / 16;
+constexpr int B_SCALE_BYTES = BNH * BKC / 16;
 constexpr int CODE_STAGE_BYTES = A_CODE_BYTES + B_CODE_BYTES + A_SCALE_BYTES + B_SCALE_BYTES;
 constexpr int A_DEC_BYTES = BM * BKD * 2;
-constexpr int B_DEC_BYTES = BN * BKD * 2;
+constexpr int B_DEC_BYTES = BNH * BKD * 2;
 constexpr int DEC_STAGE_BYTES = A_DEC_BYTES + B_DEC_BYTES;
 constexpr int OFF_DEC = kCodeStages * CODE_STAGE_BYTES;
 constexpr int OFF_BAR = OFF_DEC + kDecStages * DEC_STAGE_BYTES;
@@ -63,16 +75,17 @@ static_assert(SMEM_ALLOC <= 232448, "shared memory budget");
 //   (row / 8) * SBO + kchunk * LBO + (row % 8) * 16
 constexpr uint32_t kLBO = 128;                  // next 8 K-elements
 constexpr uint32_t kSBO = (BKD / 8) * 128;      // next 8 rows (1024 B)
-constexpr uint32_t kIdesc = idesc_bf16_f32(BM, BN);
+constexpr uint32_t kIdesc = idesc_f16_f32(TILE_M, TILE_N);
 
 constexpr uint64_t kWaitLimitNs = 1000000000ull;  // 1 s per pipeline wait
 
 struct Bars {
   uint64_t code_full[kCodeStages];
   uint64_t code_empty[kCodeStages];
-  uint64_t dec_full[kDecStages];
-  uint64_t dec_empty[kDecStages];
-  uint64_t acc_full;
+  uint64_t dec_full[kDecStages];    // leader: 2 x kDecodeWarps arrivals
+  uint64_t dec_empty[kDecStages];   // MMA commit (multicast to both CTAs)
+  uint64_t acc_full[2];             // MMA commit (multicast)
+  uint64_t acc_empty[2];            // leader: 2 x kEpiWarps arrivals
   uint64_t drain;
   uint32_t tmem_base;
   int abort;
@@ -87,41 +100,40 @@ __device__ __forceinline__ uint4 lds128(uint32_t addr) {
   asm volatile("ld.shared.v4.b32 {%0,%1,%2,%3}, [%4];" : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(addr) : "memory");
   return v;
 }
-__device__ __forceinline__ uint32_t fma_bf16x2(uint32_t a, uint32_t b, uint32_t c) {
+__device__ __forceinline__ uint32_t hmul2(uint32_t a, uint32_t b) {
   uint32_t d;
-  asm("fma.rn.bf16x2 %0, %1, %2, %3;" : "=r"(d) : "r"(a), "r"(b), "r"(c));
+  asm("mul.rn.f16x2 %0, %1, %2;" : "=r"(d) : "r"(a), "r"(b));
   return d;
-}
-__device__ __forceinline__ uint32_t bf16x2_splat(float v) {
-  uint32_t d;
-  asm("cvt.rn.bf16x2.f32 %0, %1, %1;" : "=r"(d) : "f"(v));
-  return d;
-}
-__device__ __forceinline__ uint32_t lop_xor_and(uint32_t a, uint32_t b, uint32_t mask) {
-  return a ^ (b & mask);
 }
 
-// Decode 8 consecutive codes (one 32-bit word, element 2j in the low nibble of
-// byte j) of a block to 8 bf16 values 2*v*s8 = u*s8, u = 2v:
-//   E2M1 u in {0,1,2,3,4,6,8,12}, E1M2 u in {0,2,...,14} (selected by the LUT).
-// u is looked up with prmt, turned into the bf16 128+u, and
-//   fma(128+u, s8, -128*s8) = u*s8 exactly; the nibble sign is then XORed in.
+// f16 high bytes of u = 2v by payload (the low byte of every such f16 is 0):
+//   E2M1 u = {0,1,2,3,4,6,8,12} -> 00 3C 40 42 | 44 46 48 4A
+//   E1M2 u = {0,2,4,...,14}     -> 00 40 44 46 | 48 49 4A 4B
+constexpr uint32_t kLutE2M1Lo = 0x42403C00u, kLutE2M1Hi = 0x4A484644u;
+constexpr uint32_t kLutE1M2Lo = 0x46444000u, kLutE1M2Hi = 0x4B4A4948u;
+
+// Decode one 32-bit code word (8 elements, element 2j in the low nibble of
+// byte j) of a block with f16x2 scale s2 into four f16x2 words, in the order
+// (e0,e1) (e2,e3) (e4,e5) (e6,e7): byte LUT of the payloads (prmt), the
+// nibble sign moved into bit 7 of each byte (prmt + lop3), bytes placed as f16
+// high bytes (prmt), times s8 (exact).
 __device__ __forceinline__ void decode8(uint32_t w, uint32_t lut_lo, uint32_t lut_hi, uint32_t s2,
-                                        uint32_t c2, uint32_t out[4]) {
+                                        uint32_t out[4]) {
   const uint32_t wp = w & 0x77777777u;
+  const uint32_t ws = w * 16u;
   const uint32_t u0 = prmt(lut_lo, lut_hi, wp);
-  const uint32_t u1 = prmt(lut_lo, lut_hi, wp >> 16);
-  const uint32_t ws = w << 4;
-  const uint32_t k43 = 0x43434343u;
-  const uint32_t m0 = prmt(u0, k43, 0x4140u), m1 = prmt(u0, k43, 0x4342u);
-  const uint32_t m2 = prmt(u1, k43, 0x4140u), m3 = prmt(u1, k43, 0x4342u);
-  out[0] = lop_xor_and(fma_bf16x2(m0, s2, c2), prmt(w, ws, 0x0040u), 0x80008000u);
-  out[1] = lop_xor_and(fma_bf16x2(m1, s2, c2), prmt(w, ws, 0x1050u), 0x80008000u);
-  out[2] = lop_xor_and(fma_bf16x2(m2, s2, c2), prmt(w, ws, 0x2060u), 0x80008000u);
-  out[3] = lop_xor_and(fma_bf16x2(m3, s2, c2), prmt(w, ws, 0x3070u), 0x80008000u);
+  const uint32_t u1 = prmt(lut_lo, lut_hi, __umulhi(wp, 0x10000u));
+  const uint32_t g0 = prmt(w, ws, 0x1504u);  // byte i bit 7 = sign of element i   (i = 0..3)
+  const uint32_t g1 = prmt(w, ws, 0x3726u);  // byte i bit 7 = sign of element 4+i
+  const uint32_t v0 = u0 | (g0 & 0x80808080u);
+  const uint32_t v1 = u1 | (g1 & 0x80808080u);
+  out[0] = hmul2(prmt(v0, 0u, 0x1404u), s2);
+  out[1] = hmul2(prmt(v0, 0u, 0x3424u), s2);
+  out[2] = hmul2(prmt(v1, 0u, 0x1404u), s2);
+  out[3] = hmul2(prmt(v1, 0u, 0x3424u), s2);
 }
 
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
 mixfp4_gemm_kernel(const __grid_constant__ CUtensorMap tm_ac, const __grid_constant__ CUtensorMap tm_bc,
                    const __grid_constant__ CUtensorMap tm_as, const __grid_constant__ CUtensorMap tm_bs,
                    const float* __restrict__ a_ts, const float* __restrict__ b_ts,
@@ -133,8 +145,12 @@ mixfp4_gemm_kernel(const __grid_constant__ CUtensorMap tm_ac, const __grid_const
   volatile int* abort_flag = &bars->abort;
   const uint32_t sbase = smem_u32(smem);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int m0 = blockIdx.y * BM, n0 = blockIdx.x * BN;
+  const uint32_t rank = cluster_ctarank();
+  const bool leader = rank == 0;
   const int num_kc = K / BKC;
+  const int mtiles = (M + TILE_M - 1) / TILE_M, ntiles_n = (N + TILE_N - 1) / TILE_N;
+  const int ntiles = mtiles * ntiles_n;
+  const int cluster_id = blockIdx.x >> 1, nclusters = gridDim.x >> 1;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kCodeStages; ++s) {
@@ -142,22 +158,25 @@ mixfp4_gemm_kernel(const __grid_constant__ CUtensorMap tm_ac, const __grid_const
       mbar_init(smem_u32(&bars->code_empty[s]), kDecodeWarps);
     }
     for (int s = 0; s < kDecStages; ++s) {
-      mbar_init(smem_u32(&bars->dec_full[s]), kDecodeWarps);
+      mbar_init(smem_u32(&bars->dec_full[s]), 2 * kDecodeWarps);
       mbar_init(smem_u32(&bars->dec_empty[s]), 1);
     }
-    mbar_init(smem_u32(&bars->acc_full), 1);
+    for (int s = 0; s < 2; ++s) {
+      mbar_init(smem_u32(&bars->acc_full[s]), 1);
+      mbar_init(smem_u32(&bars->acc_empty[s]), 2 * kEpiWarps);
+    }
     mbar_init(smem_u32(&bars->drain), 1);
     bars->abort = 0;
     fence_mbar_init();
   }
   if (warp == 1) {
-    tmem_alloc(smem_u32(&bars->tmem_base), kTmemCols);
-    tmem_relinquish();
+    tmem_alloc_pair(smem_u32(&bars->tmem_base), kTmemCols);
+    tmem_relinquish_pair();
   }
   tc_fence_before();
-  __syncthreads();
+  cluster_sync();  // barriers of both CTAs initialised, TMEM allocated in both
   tc_fence_after();
-  const uint32_t tmem_acc = bars->tmem_base;
+  const uint32_t tmem_base = bars->tmem_base;
 
   auto fail = [&](uint32_t code) {
     *abort_flag = 1;
@@ -173,22 +192,29 @@ mixfp4_gemm_kernel(const __grid_constant__ CUtensorMap tm_ac, const __grid_const
       tma_prefetch(&tm_bs);
       int last_phase[kCodeStages];
       for (int s = 0; s < kCodeStages; ++s) last_phase[s] = -1;
-      for (int kc = 0; kc < num_kc; ++kc) {
-        const int s = kc % kCodeStages;
-        const uint32_t ph = (kc / kCodeStages) & 1;
-        if (!mbar_wait(smem_u32(&bars->code_empty[s]), ph ^ 1, abort_flag, kWaitLimitNs)) {
-          fail(1u);
-          break;
+      int it = 0;
+      bool ok = true;
+      for (int t = cluster_id; t < ntiles && ok; t += nclusters) {
+        const int mt = t % mtiles, nt = t / mtiles;
+        const int ma = mt * TILE_M + (int)rank * BM, nb = nt * TILE_N + (int)rank * BNH;
+        for (int kc = 0; kc < num_kc; ++kc, ++it) {
+          const int s = it % kCodeStages;
+          const uint32_t ph = (it / kCodeStages) & 1;
+          if (!mbar_wait(smem_u32(&bars->code_empty[s]), ph ^ 1, abort_flag, kWaitLimitNs)) {
+            fail(1u);
+            ok = false;
+            break;
+          }
+          const uint32_t st = sbase + s * CODE_STAGE_BYTES;
+          const uint32_t fb = smem_u32(&bars->code_full[s]);
+          mbar_arrive_expect_tx(fb, CODE_STAGE_BYTES);
+          const int xk = kc * (BKC / 2), xs = kc * (BKC / 16);
+          tma_load_2d(st, &tm_ac, xk, ma, fb);
+          tma_load_2d(st + A_CODE_BYTES, &tm_bc, xk, nb, fb);
+          tma_load_2d(st + A_CODE_BYTES + B_CODE_BYTES, &tm_as, xs, ma, fb);
+          tma_load_2d(st + A_CODE_BYTES + B_CODE_BYTES + A_SCALE_BYTES, &tm_bs, xs, nb, fb);
+          last_phase[s] = (int)ph;
         }
-        const uint32_t st = sbase + s * CODE_STAGE_BYTES;
-        const uint32_t fb = smem_u32(&bars->code_full[s]);
-        mbar_arrive_expect_tx(fb, CODE_STAGE_BYTES);
-        const int xk = kc * (BKC / 2), xs = kc * (BKC / 16);
-        tma_load_2d(st, &tm_ac, xk, m0, fb);
-        tma_load_2d(st + A_CODE_BYTES, &tm_bc, xk, n0, fb);
-        tma_load_2d(st + A_CODE_BYTES + B_CODE_BYTES, &tm_as, xs, m0, fb);
-        tma_load_2d(st + A_CODE_BYTES + B_CODE_BYTES + A_SCALE_BYTES, &tm_bs, xs, n0, fb);
-        last_phase[s] = (int)ph;
       }
       if (*abort_flag) {
         // Let the copies this thread started land before the CTA may exit.
@@ -198,143 +224,170 @@ mixfp4_gemm_kernel(const __grid_constant__ CUtensorMap tm_ac, const __grid_const
       }
     }
   } else if (warp == 1) {
-    // ---------------- MMA issuer ----------------
-    if (lane == 0) {
+    // ---------------- MMA issuer (leader CTA) ----------------
+    if (leader && lane == 0) {
       int d = 0;
       uint32_t dph = 0;
       bool ok = true;
-      for (int kc = 0; kc < num_kc && ok; ++kc) {
-        for (int sub = 0; sub < kSub; ++sub) {
-          if (!mbar_wait(smem_u32(&bars->dec_full[d]), dph, abort_flag, kWaitLimitNs)) {
-            fail(2u);
-            ok = false;
-            break;
-          }
-          tc_fence_after();
-          const uint32_t abase = sbase + OFF_DEC + d * DEC_STAGE_BYTES;
-          const uint32_t bbase = abase + A_DEC_BYTES;
-#pragma unroll
-          for (int j = 0; j < BKD / 16; ++j) {
-            const uint64_t ad = smem_desc_noswizzle(abase + j * 256, kLBO, kSBO);
-            const uint64_t bd = smem_desc_noswizzle(bbase + j * 256, kLBO, kSBO);
-            mma_bf16(tmem_acc, ad, bd, kIdesc, (kc | sub | j) != 0 ? 1u : 0u);
-          }
-          mma_commit(smem_u32(&bars->dec_empty[d]));
-          if (++d == kDecStages) { d = 0; dph ^= 1; }
+      int i = 0;
+      for (int t = cluster_id; t < ntiles && ok; t += nclusters, ++i) {
+        const int ab = i & 1;
+        const uint32_t aph = (i >> 1) & 1;
+        if (!mbar_wait_cluster(smem_u32(&bars->acc_empty[ab]), aph ^ 1, abort_flag, kWaitLimitNs)) {
+          fail(2u);
+          break;
         }
+        tc_fence_after();
+        const uint32_t dtm = tmem_base + (uint32_t)ab * kAccCols;
+        for (int kc = 0; kc < num_kc && ok; ++kc) {
+          for (int sub = 0; sub < kSub; ++sub) {
+            if (!mbar_wait_cluster(smem_u32(&bars->dec_full[d]), dph, abort_flag, kWaitLimitNs)) {
+              fail(4u);
+              ok = false;
+              break;
+            }
+            tc_fence_after();
+            const uint32_t abase = sbase + OFF_DEC + d * DEC_STAGE_BYTES;
+            const uint32_t bbase = abase + A_DEC_BYTES;
+#pragma unroll
+            for (int j = 0; j < BKD / 16; ++j) {
+              const uint64_t ad = smem_desc_noswizzle(abase + j * 256, kLBO, kSBO);
+              const uint64_t bd = smem_desc_noswizzle(bbase + j * 256, kLBO, kSBO);
+              mma_f16_pair(dtm, ad, bd, kIdesc, (kc | sub | j) != 0 ? 1u : 0u);
+            }
+            mma_commit_pair(smem_u32(&bars->dec_empty[d]), 3);
+            if (++d == kDecStages) { d = 0; dph ^= 1; }
+          }
+        }
+        if (ok) mma_commit_pair(smem_u32(&bars->acc_full[ab]), 3);
       }
-      // acc_full fires when every MMA issued above has completed.  The issuer
-      // also waits for it (ignoring the abort flag), so tensor memory is never
-      // freed under a running MMA.
-      mma_commit(smem_u32(&bars->acc_full));
-      if (!mbar_wait(smem_u32(&bars->acc_full), 0, nullptr, kWaitLimitNs)) fail(32u);
+      // Every MMA issued above completes before the drain barrier fires; wait
+      // for it (ignoring the abort flag) so TMEM is never freed under an MMA.
+      mma_commit_pair(smem_u32(&bars->drain), 1);
+      if (!mbar_wait_cluster(smem_u32(&bars->drain), 0, nullptr, kWaitLimitNs)) fail(8u);
     }
-  } else {
-    // ---------------- decoders (one thread per tile row) ----------------
-    const int row = threadIdx.x - 64;  // 0..383
+  } else if (warp < kFirstEpiWarp) {
+    // ---------------- decoders (two threads per operand row) ----------------
+    const int dt = threadIdx.x - 32 * kFirstDecodeWarp;  // 0..511
+    const int row = dt & 255, half = dt >> 8;            // half: which 32 K of a sub-stage
     const bool is_a = row < BM;
     const int rl = is_a ? row : row - BM;
     const uint32_t code_off = (is_a ? 0 : A_CODE_BYTES) + rl * (BKC / 2);
     const uint32_t scale_off = A_CODE_BYTES + B_CODE_BYTES + (is_a ? 0 : A_SCALE_BYTES) + rl * (BKC / 16);
-    const uint32_t dec_off = OFF_DEC + (is_a ? 0 : A_DEC_BYTES) + (rl >> 3) * kSBO + (rl & 7) * 16;
+    const uint32_t dec_off = OFF_DEC + (is_a ? 0 : A_DEC_BYTES) + (rl >> 3) * kSBO + (rl & 7) * 16 +
+                             half * 4 * kLBO;
     const uint32_t swz = rl & 7;
+    const uint32_t dec_full_leader0 = mapa_shared(smem_u32(&bars->dec_full[0]), 0);
     int d = 0;
     uint32_t dph = 0;
+    int it = 0;
     bool ok = true;
-    for (int kc = 0; kc < num_kc && ok; ++kc) {
-      const int s = kc % kCodeStages;
-      const uint32_t ph = (kc / kCodeStages) & 1;
-      if (!mbar_wait(smem_u32(&bars->code_full[s]), ph, abort_flag, kWaitLimitNs)) {
-        fail(4u);
-        break;
-      }
-      const uint32_t st = sbase + s * CODE_STAGE_BYTES;
-      const uint4 sc = lds128(st + scale_off);
-      const uint32_t scw[4] = {sc.x, sc.y, sc.z, sc.w};
-#pragma unroll
-      for (int sub = 0; sub < kSub; ++sub) {
-        // this row's 64 codes of the sub-stage: logical 16-byte chunks 2*sub, 2*sub+1
-        const uint4 c0 = lds128(st + code_off + (((2 * sub) ^ swz) << 4));
-        const uint4 c1 = lds128(st + code_off + (((2 * sub + 1) ^ swz) << 4));
-        if (sub == kSub - 1) {
-          __syncwarp();
-          if (lane == 0) mbar_arrive(smem_u32(&bars->code_empty[s]));
-        }
-        if (!mbar_wait(smem_u32(&bars->dec_empty[d]), dph ^ 1, abort_flag, kWaitLimitNs)) {
-          fail(8u);
+    for (int t = cluster_id; t < ntiles && ok; t += nclusters) {
+      for (int kc = 0; kc < num_kc && ok; ++kc, ++it) {
+        const int s = it % kCodeStages;
+        const uint32_t ph = (it / kCodeStages) & 1;
+        if (!mbar_wait(smem_u32(&bars->code_full[s]), ph, abort_flag, kWaitLimitNs)) {
+          fail(16u);
           ok = false;
           break;
         }
-        const uint32_t w[8] = {c0.x, c0.y, c0.z, c0.w, c1.x, c1.y, c1.z, c1.w};
-        const uint32_t s4 = scw[sub];
-        const uint32_t mag = s4 & 0x7F7F7F7Fu;
-        float sv[4];
-        f16x2_to_f32(cvt_f16x2_from_e4m3x2((uint16_t)(mag & 0xFFFFu)), sv[0], sv[1]);
-        f16x2_to_f32(cvt_f16x2_from_e4m3x2((uint16_t)(mag >> 16)), sv[2], sv[3]);
-        const uint32_t dst = sbase + dec_off + d * DEC_STAGE_BYTES;
+        const uint32_t st = sbase + s * CODE_STAGE_BYTES;
+        const uint4 sc = lds128(st + scale_off);
+        const uint32_t scw[4] = {sc.x, sc.y, sc.z, sc.w};
 #pragma unroll
-        for (int b = 0; b < 4; ++b) {
-          const bool e1m2 = (s4 >> (8 * b + 7)) & 1u;
-          const uint32_t lut_lo = e1m2 ? 0x06040200u : 0x03020100u;
-          const uint32_t lut_hi = e1m2 ? 0x0E0C0A08u : 0x0C080604u;
-          const uint32_t s2 = bf16x2_splat(sv[b]);
-          const uint32_t c2 = bf16x2_splat(-128.0f * sv[b]);
+        for (int sub = 0; sub < kSub; ++sub) {
+          // this thread's 32 codes of the sub-stage: logical 16-byte chunk 2*sub + half
+          const uint4 c = lds128(st + code_off + (((2 * sub + half) ^ swz) << 4));
+          if (!mbar_wait_cluster(smem_u32(&bars->dec_empty[d]), dph ^ 1, abort_flag, kWaitLimitNs)) {
+            fail(32u);
+            ok = false;
+            break;
+          }
+          const uint32_t w[4] = {c.x, c.y, c.z, c.w};
+          // scale bytes of this thread's two blocks (blocks 4*sub + 2*half, +1)
+          const uint32_t s2b = (scw[sub] >> (16 * half)) & 0xFFFFu;
+          const uint32_t h01 = cvt_f16x2_from_e4m3x2((uint16_t)(s2b & 0x7F7Fu));
+          const uint32_t sv[2] = {prmt(h01, 0u, 0x1010u), prmt(h01, 0u, 0x3232u)};
+          const uint32_t dst = sbase + dec_off + d * DEC_STAGE_BYTES;
 #pragma unroll
-          for (int i = 0; i < 2; ++i) {
-            uint32_t o[4];
-            decode8(w[2 * b + i], lut_lo, lut_hi, s2, c2, o);
-            sts128(dst + (2 * b + i) * kLBO, o[0], o[1], o[2], o[3]);
+          for (int b = 0; b < 2; ++b) {
+            const bool e1m2 = (s2b >> (8 * b + 7)) & 1u;
+            const uint32_t lut_lo = e1m2 ? kLutE1M2Lo : kLutE2M1Lo;
+            const uint32_t lut_hi = e1m2 ? kLutE1M2Hi : kLutE2M1Hi;
+#pragma unroll
+            for (int i = 0; i < 2; ++i) {
+              uint32_t o[4];
+              decode8(w[2 * b + i], lut_lo, lut_hi, sv[b], o);
+              sts128(dst + (2 * b + i) * kLBO, o[0], o[1], o[2], o[3]);
+            }
+          }
+          fence_proxy_async_smem();
+          __syncwarp();
+          if (lane == 0) mbar_arrive_cluster(dec_full_leader0 + d * 8);
+          if (++d == kDecStages) { d = 0; dph ^= 1; }
+          if (sub == kSub - 1) {
+            // Release the code stage only now: every value loaded from it has
+            // been consumed (the decoded stores depend on it), so the TMA
+            // refill cannot overtake a pending shared-memory load.
+            __syncwarp();
+            if (lane == 0) mbar_arrive(smem_u32(&bars->code_empty[s]));
           }
         }
-        fence_proxy_async_smem();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(smem_u32(&bars->dec_full[d]));
-        if (++d == kDecStages) { d = 0; dph ^= 1; }
       }
     }
-
-    // ---------------- epilogue (warps 2-9) ----------------
-    if (warp < 10) {
-      const bool acc_ok = mbar_wait(smem_u32(&bars->acc_full), 0, abort_flag, kWaitLimitNs);
+  } else {
+    // ---------------- epilogue ----------------
+    const int q = warp & 3;  // TMEM lane quarter of this warp
+    const float sa = 0.25f * __ldg(a_ts), sb = __ldg(b_ts);
+    const bool vec_ok = ((ldc & 3) == 0) && ((reinterpret_cast<uintptr_t>(C) & 15) == 0);
+    const uint32_t acc_empty_leader0 = mapa_shared(smem_u32(&bars->acc_empty[0]), 0);
+    int i = 0;
+    for (int t = cluster_id; t < ntiles; t += nclusters, ++i) {
+      const int ab = i & 1;
+      const uint32_t aph = (i >> 1) & 1;
+      const bool acc_ok = mbar_wait_cluster(smem_u32(&bars->acc_full[ab]), aph, abort_flag, kWaitLimitNs);
       tc_fence_after();
       // tcgen05.ld is warp-collective: decide for the whole warp.
       const bool go = __all_sync(0xffffffffu, acc_ok && !*abort_flag);
-      if (!acc_ok && !*abort_flag) fail(16u);
-      if (go) {
-        const int q = warp & 3;                 // TMEM lane quarter of this warp
-        const int half = (warp - 2) >> 2;       // column half
-        const int r = m0 + q * 32 + lane;
-        const float sa = 0.25f * __ldg(a_ts), sb = __ldg(b_ts);
-        const bool vec_ok = ((ldc & 3) == 0) && ((reinterpret_cast<uintptr_t>(C) & 15) == 0);
-        for (int cc = 0; cc < BN / 2; cc += 16) {
-          const int col = half * (BN / 2) + cc;
-          uint32_t v[16];
-          tmem_ld_32x32b_x16(tmem_acc + ((uint32_t)(q * 32) << 16) + (uint32_t)col, v);
-          tmem_ld_wait();
-          if (r < M) {
-            float* crow = C + (long long)r * ldc + n0 + col;
-            float o[16];
+      if (!go) {
+        if (!acc_ok && !*abort_flag) fail(64u);
+        break;
+      }
+      const int mt = t % mtiles, nt = t / mtiles;
+      const int r = mt * TILE_M + (int)rank * BM + q * 32 + lane;
+      const int n0 = nt * TILE_N;
+      const uint32_t tbase = tmem_base + (uint32_t)ab * kAccCols + ((uint32_t)(q * 32) << 16);
+#pragma unroll 1
+      for (int col = 0; col < TILE_N; col += 32) {
+        uint32_t v[32];
+        tmem_ld_32x32b_x32(tbase + (uint32_t)col, v);
+        tmem_ld_wait();
+        if (r < M) {
+          float* crow = C + (long long)r * ldc + n0 + col;
+          float o[32];
 #pragma unroll
-            for (int i = 0; i < 16; ++i) o[i] = __fmul_rn(__fmul_rn(__uint_as_float(v[i]), sa), sb);
-            if (vec_ok && n0 + col + 16 <= N) {
+          for (int k = 0; k < 32; ++k) o[k] = __fmul_rn(__fmul_rn(__uint_as_float(v[k]), sa), sb);
+          if (vec_ok && n0 + col + 32 <= N) {
 #pragma unroll
-              for (int i = 0; i < 16; i += 4)
-                *reinterpret_cast<float4*>(crow + i) = make_float4(o[i], o[i + 1], o[i + 2], o[i + 3]);
-            } else {
-              for (int i = 0; i < 16; ++i)
-                if (n0 + col + i < N) crow[i] = o[i];
-            }
+            for (int k = 0; k < 32; k += 4)
+              *reinterpret_cast<float4*>(crow + k) = make_float4(o[k], o[k + 1], o[k + 2], o[k + 3]);
+          } else {
+            for (int k = 0; k < 32; ++k)
+              if (n0 + col + k < N) crow[k] = o[k];
           }
         }
       }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive_cluster(acc_empty_leader0 + ab * 8);
     }
   }
 
   tc_fence_before();
-  __syncthreads();
+  cluster_sync();  // both CTAs done with TMEM (and with each other's barriers)
   if (warp == 1) {
     tc_fence_after();
-    tmem_dealloc(tmem_acc, kTmemCols);
+    tmem_dealloc_pair(tmem_base, kTmemCols);
   }
 }
 
@@ -365,18 +418,29 @@ bool make_map(CUtensorMap* m, const void* base, uint64_t row_bytes, uint64_t row
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+int num_sms() {
+  static int n = 0;
+  if (!n) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0)
+      n = 148;
+  }
+  return n;
+}
+
 }  // namespace
 
 int launch_gemm(const uint8_t* a_codes, const uint8_t* a_scales, const float* a_ts,
                 const uint8_t* b_codes, const uint8_t* b_scales, const float* b_ts, int64_t M,
                 int64_t N, int64_t K, float* C, int64_t ldc, uint32_t* status_word,
                 cudaStream_t stream) {
-  if (M > (int64_t)65535 * BM || N > (1 << 30) || K > (1 << 30)) return MIXFP4_ERR_SHAPE;
+  if (M > (1 << 30) || N > (1 << 30) || K > (1 << 30)) return MIXFP4_ERR_SHAPE;
   CUtensorMap tac, tbc, tas, tbs;
   if (!make_map(&tac, a_codes, (uint64_t)K / 2, (uint64_t)M, BKC / 2, BM, CU_TENSOR_MAP_SWIZZLE_128B) ||
-      !make_map(&tbc, b_codes, (uint64_t)K / 2, (uint64_t)N, BKC / 2, BN, CU_TENSOR_MAP_SWIZZLE_128B) ||
+      !make_map(&tbc, b_codes, (uint64_t)K / 2, (uint64_t)N, BKC / 2, BNH, CU_TENSOR_MAP_SWIZZLE_128B) ||
       !make_map(&tas, a_scales, (uint64_t)K / 16, (uint64_t)M, BKC / 16, BM, CU_TENSOR_MAP_SWIZZLE_NONE) ||
-      !make_map(&tbs, b_scales, (uint64_t)K / 16, (uint64_t)N, BKC / 16, BN, CU_TENSOR_MAP_SWIZZLE_NONE))
+      !make_map(&tbs, b_scales, (uint64_t)K / 16, (uint64_t)N, BKC / 16, BNH, CU_TENSOR_MAP_SWIZZLE_NONE))
     return MIXFP4_ERR_CUDA;
   static bool attr_set = false;
   if (!attr_set) {
@@ -385,9 +449,11 @@ int launch_gemm(const uint8_t* a_codes, const uint8_t* a_scales, const float* a_
       return MIXFP4_ERR_CUDA;
     attr_set = true;
   }
-  dim3 grid((unsigned)((N + BN - 1) / BN), (unsigned)((M + BM - 1) / BM));
-  mixfp4_gemm_kernel<<<grid, kThreads, SMEM_ALLOC, stream>>>(tac, tbc, tas, tbs, a_ts, b_ts, (int)M, (int)N,
-                                                               (int)K, C, (long long)ldc, status_word);
+  const int64_t tiles = ((M + TILE_M - 1) / TILE_M) * ((N + TILE_N - 1) / TILE_N);
+  int64_t clusters = num_sms() / 2;
+  if (clusters > tiles) clusters = tiles;
+  mixfp4_gemm_kernel<<<(unsigned)(2 * clusters), kThreads, SMEM_ALLOC, stream>>>(
+      tac, tbc, tas, tbs, a_ts, b_ts, (int)M, (int)N, (int)K, C, (long long)ldc, status_word);
   return MIXFP4_OK;
 }
 

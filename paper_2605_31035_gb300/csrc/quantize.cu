@@ -19,6 +19,7 @@
 //   * E2M1 rounding uses cvt.rn.satfinite.e2m1x2 (RNE, saturating) and E4M3
 //     scale rounding cvt.rn.satfinite.e4m3x2; E1M2 rounding adds 1.5*2^23
 //     (RNE to an integer) and clamps the integer to 7.
+#include <cuda_fp16.h>
 #include <cuda_runtime.h>
 #include <cstdint>
 
@@ -42,40 +43,60 @@ __device__ __forceinline__ uint32_t lo32(u64 v) { return (uint32_t)v; }
 __device__ __forceinline__ uint32_t hi32(u64 v) { return (uint32_t)(v >> 32); }
 
 struct TensorConsts {
-  float s32;   // per-tensor scale, possibly rescaled to [1, 2)
-  float r32;   // RN(1/s32), or 0 when s32 == 0
+  float s32;     // per-tensor scale, possibly rescaled to [1, 2)
+  float r32;     // RN(1/s32), or 0 when s32 == 0
   float r6, r7;  // RN(1/6), RN(1/7)
-  int k;       // |x| is multiplied by 2^k when `scaled`
+  int k;         // |x| is multiplied by 2^k when `scaled`
   int scaled;
 };
 
-// Derive the per-tensor constants once per CTA (thread 0), broadcast via smem.
-__device__ __forceinline__ TensorConsts tensor_consts(float* tensor_scale,
-                                                      const uint32_t* amax_word, int scale_given,
-                                                      TensorConsts* sh) {
-  if (threadIdx.x == 0) {
-    float s32;
-    if (scale_given) {
-      s32 = *tensor_scale;
-    } else {
-      s32 = __fdiv_rn(__uint_as_float(*amax_word), 2688.0f);  // 6*448 = 7*384
-      if (blockIdx.x == 0) *tensor_scale = s32;
-    }
-    TensorConsts c;
-    c.scaled = !(s32 == 0.0f || (s32 >= 0x1p-20f && s32 <= 0x1p100f));
-    c.k = 0;
-    if (c.scaled) {
-      c.k = -ilogbf(s32);
-      s32 = scalbnf(s32, c.k);  // exact, now in [1, 2)
-    }
-    c.s32 = s32;
-    c.r32 = (s32 > 0.0f) ? __frcp_rn(s32) : 0.0f;
-    c.r6 = __frcp_rn(6.0f);
-    c.r7 = __frcp_rn(7.0f);
-    *sh = c;
+// Per-tensor constants, derived by every thread (a persistent thread handles
+// many blocks, so this costs a few instructions per block at most).
+__device__ __forceinline__ TensorConsts tensor_consts(float* tensor_scale, const uint32_t* amax_word,
+                                                      int scale_given) {
+  float s32;
+  if (scale_given) {
+    s32 = *tensor_scale;
+  } else {
+    s32 = __fdiv_rn(__uint_as_float(*amax_word), 2688.0f);  // 6*448 = 7*384
+    if (blockIdx.x == 0 && threadIdx.x == 0) *tensor_scale = s32;
   }
-  __syncthreads();
-  return *sh;
+  TensorConsts c;
+  c.scaled = !(s32 == 0.0f || (s32 >= 0x1p-20f && s32 <= 0x1p100f));
+  c.k = 0;
+  if (c.scaled) {
+    c.k = -ilogbf(s32);
+    s32 = scalbnf(s32, c.k);  // exact, now in [1, 2)
+  }
+  c.s32 = s32;
+  c.r32 = (s32 > 0.0f) ? __frcp_rn(s32) : 0.0f;
+  c.r6 = __frcp_rn(6.0f);
+  c.r7 = __frcp_rn(7.0f);
+  return c;
+}
+
+// E2M1 quantization of a pair (RNE, saturating): returns the byte of the two
+// nibbles (first element low) and the dequantized pair as f16x2.
+__device__ __forceinline__ uint32_t e2m1_pair(float lo, float hi, uint32_t& h2) {
+  uint32_t byte;
+  asm("{ .reg .b8 t; cvt.rn.satfinite.e2m1x2.f32 t, %2, %3; cvt.rn.f16x2.e2m1x2 %1, t; cvt.u32.u8 %0, t; }"
+      : "=r"(byte), "=r"(h2) : "f"(hi), "f"(lo));
+  return byte;
+}
+
+// Four byte values (each in the low byte of a word) packed into one word.
+__device__ __forceinline__ uint32_t pack_low_bytes(uint32_t b0, uint32_t b1, uint32_t b2, uint32_t b3) {
+  return prmt(prmt(b0, b1, 0x0040u), prmt(b2, b3, 0x0040u), 0x5410u);
+}
+
+// Sign nibble bits of 8 elements held in 4 bf16 pairs: element 2j -> bit 3 of
+// byte j, element 2j+1 -> bit 7 (the sign bits of the code word).
+__device__ __forceinline__ uint32_t sign_bits(uint32_t w0, uint32_t w1, uint32_t w2, uint32_t w3) {
+  const uint32_t x = prmt(w0, w1, 0x7351u);   // [w0.b1, w1.b1, w0.b3, w1.b3]
+  const uint32_t y = prmt(w2, w3, 0x7351u);
+  const uint32_t even = prmt(x, y, 0x5410u);  // byte j bit 7 = sign of element 2j
+  const uint32_t odd = prmt(x, y, 0x7632u);   // byte j bit 7 = sign of element 2j+1
+  return (odd & 0x80808080u) | ((even >> 4) & 0x08080808u);
 }
 
 // Algorithm 1 for one 16-element block held as 8 bf16 pairs.
@@ -87,16 +108,21 @@ __device__ __forceinline__ TensorConsts tensor_consts(float* tensor_scale,
 // whether its quotient is correctly rounded does not affect any output.  The
 // same holds for |a| < 2^-102 in the |a|/s8 step and for B < 2^-102, where
 // both block scales round to E4M3 zero anyway.
+//
+// E1M2 clamp: when s8 = E4M3(b7) is normal (>= 2^-6) and b7 = fl32(B/7) did
+// not saturate, s8 >= b7 / (1 + 2^-4), so |a|/s8 <= 7 * 1.0625 * (1 + 2^-23)
+// < 7.5 and RNE never exceeds 7; only other blocks need the clamp.
 template <int kMode, bool kScaled>
 __device__ __forceinline__ void quantize_block(const uint32_t w[8], const TensorConsts& tc,
-                                               uint32_t& code_lo, uint32_t& code_hi,
-                                               uint32_t& scale_byte) {
+                                               const float2* __restrict__ tab, uint32_t& code_lo,
+                                               uint32_t& code_hi, uint32_t& scale_byte) {
   // |x| as packed fp32 pairs (element 2j in the low lane).
   u64 a[8];
   const u64 ns32 = pack2(-tc.s32, -tc.s32), r32 = pack2(tc.r32, tc.r32);
 #pragma unroll
   for (int j = 0; j < 8; ++j) {
-    uint32_t lo = (w[j] << 16) & 0x7FFF0000u, hi = w[j] & 0x7FFF0000u;
+    const uint32_t u = w[j] & 0x7FFF7FFFu;
+    uint32_t lo = u << 16, hi = u & 0xFFFF0000u;
     if (kScaled) {
       lo = __float_as_uint(scalbnf(__uint_as_float(lo), tc.k));
       hi = __float_as_uint(scalbnf(__uint_as_float(hi), tc.k));
@@ -110,106 +136,135 @@ __device__ __forceinline__ void quantize_block(const uint32_t w[8], const Tensor
   float B = max3f(max3f(v[0], v[1], v[2]), max3f(v[3], v[4], v[5]), max3f(v[6], v[7], v[8]));
   B = max3f(B, max3f(v[9], v[10], v[11]), max3f(v[12], v[13], max3f(v[14], v[15], 0.0f)));
 
-  // Candidate block scales s8 = E4M3(fl32(B/6)), E4M3(fl32(B/7)).
-  u64 bq = div_rn2(pack2(B, B), pack2(-6.0f, -7.0f), pack2(tc.r6, tc.r7));
+  // Candidate block scales s8 = E4M3(fl32(B/6)), E4M3(fl32(B/7)) and RN(1/s8).
+  const u64 bq = div_rn2(pack2(B, B), pack2(-6.0f, -7.0f), pack2(tc.r6, tc.r7));
   float b6, b7;
   unpack2(bq, b6, b7);
   const uint32_t sc = cvt_e4m3x2(b7, b6);  // low byte: E2M1 scale code, high: E1M2
-  float s8_2, s8_1;
-  f16x2_to_f32(cvt_f16x2_from_e4m3x2((uint16_t)sc), s8_2, s8_1);
-
-  // Sign nibble bits: element 2j -> bit 3 of code byte j, 2j+1 -> bit 7.
-  uint32_t sgn[8];
-#pragma unroll
-  for (int j = 0; j < 8; ++j) sgn[j] = ((w[j] >> 12) & 0x08u) | ((w[j] >> 24) & 0x80u);
+  const uint32_t c2 = sc & 0x7Fu, c1 = (sc >> 8) & 0x7Fu;
 
   float S2 = 0.0f, S1 = 0.0f;
-  uint32_t pay2[8], pay1[8];
+  uint32_t p2lo = 0, p2hi = 0, p1lo = 0, p1hi = 0;
   if (kMode != MIXFP4_MODE_E1M2_ONLY) {
     // E2M1 candidate.
-    const float rr = (s8_2 > 0.0f) ? __frcp_rn(s8_2) : 0.0f;
-    const u64 ns8 = pack2(-s8_2, -s8_2), r8 = pack2(rr, rr);
+    const float2 t = tab[c2];
+    const u64 ns8 = pack2(-t.x, -t.x), r8 = pack2(t.y, t.y);
+    const uint16_t ns8h = __half_as_ushort(__float2half_rn(-t.x));  // exact: E4M3 values are f16 values
     u64 acc = 0;  // (+0, +0): even / odd chains
+    uint32_t e[8];
 #pragma unroll
     for (int j = 0; j < 8; ++j) {
-      u64 y = div_rn2(a[j], ns8, r8);
+      const u64 y = div_rn2(a[j], ns8, r8);
       float ylo, yhi;
       unpack2(y, ylo, yhi);
-      const uint32_t c = cvt_e2m1x2(yhi, ylo);
-      pay2[j] = c;
-      float qlo, qhi;
-      f16x2_to_f32(cvt_f16x2_from_e2m1x2(c), qlo, qhi);
-      u64 d = fma2(pack2(qlo, qhi), ns8, a[j]);  // |a| - q s8 (exact)
-      acc = fma2(d, d, acc);
+      uint32_t h2;
+      e[j] = e2m1_pair(ylo, yhi, h2);
+      if (kMode == MIXFP4_MODE_MIX) {
+        float alo, ahi, dlo, dhi;
+        unpack2(a[j], alo, ahi);
+        // d = |a| - q s8 (exact), with q taken straight from its f16 decode
+        asm("{ .reg .f16 ql, qh; mov.b32 {ql, qh}, %2;\n"
+            " fma.rn.f32.f16 %0, ql, %3, %4;\n fma.rn.f32.f16 %1, qh, %3, %5; }"
+            : "=f"(dlo), "=f"(dhi) : "r"(h2), "h"(ns8h), "f"(alo), "f"(ahi));
+        const u64 d = pack2(dlo, dhi);
+        acc = fma2(d, d, acc);
+      }
     }
-    float se, so;
-    unpack2(acc, se, so);
-    S2 = se + so;
+    p2lo = pack_low_bytes(e[0], e[1], e[2], e[3]);
+    p2hi = pack_low_bytes(e[4], e[5], e[6], e[7]);
+    if (kMode == MIXFP4_MODE_MIX) {
+      float se, so;
+      unpack2(acc, se, so);
+      S2 = se + so;
+    }
   }
   if (kMode != MIXFP4_MODE_E2M1_ONLY) {
     // E1M2 candidate (x2 units: integers 0..7).
-    const float rr = (s8_1 > 0.0f) ? __frcp_rn(s8_1) : 0.0f;
-    const u64 ns8 = pack2(-s8_1, -s8_1), r8 = pack2(rr, rr);
+    const float2 t = tab[c1];
+    const u64 ns8 = pack2(-t.x, -t.x), r8 = pack2(t.y, t.y);
     const u64 magic = pack2(12582912.0f, 12582912.0f);    // 1.5 * 2^23
     const u64 nmagic = pack2(-12582912.0f, -12582912.0f);
+    const bool clamp = !(t.x >= 0x1p-6f && b7 <= 448.0f);
     u64 acc = 0;
+    uint32_t pb[8];
 #pragma unroll
     for (int j = 0; j < 8; ++j) {
-      u64 y = div_rn2(a[j], ns8, r8);
-      u64 t = add2(y, magic);  // RNE to an integer in the low mantissa bits
-      const uint32_t tlo = min(lo32(t), 0x4B400007u), thi = min(hi32(t), 0x4B400007u);
-      pay1[j] = (tlo & 7u) | ((thi & 7u) << 4);
-      u64 q = add2(bits2(tlo, thi), nmagic);
-      u64 d = fma2(q, ns8, a[j]);
-      acc = fma2(d, d, acc);
+      const u64 y = div_rn2(a[j], ns8, r8);
+      const u64 tq = add2(y, magic);  // RNE to an integer in the low mantissa bits
+      uint32_t tlo = lo32(tq), thi = hi32(tq);
+      if (clamp) {
+        tlo = min(tlo, 0x4B400007u);
+        thi = min(thi, 0x4B400007u);
+      }
+      pb[j] = tlo + (thi << 4);  // low byte: payload pair (first element low)
+      if (kMode == MIXFP4_MODE_MIX) {
+        const u64 q = add2(bits2(tlo, thi), nmagic);
+        const u64 d = fma2(q, ns8, a[j]);
+        acc = fma2(d, d, acc);
+      }
     }
-    float se, so;
-    unpack2(acc, se, so);
-    S1 = se + so;
+    p1lo = pack_low_bytes(pb[0], pb[1], pb[2], pb[3]);
+    p1hi = pack_low_bytes(pb[4], pb[5], pb[6], pb[7]);
+    if (kMode == MIXFP4_MODE_MIX) {
+      float se, so;
+      unpack2(acc, se, so);
+      S1 = se + so;
+    }
   }
   int T;
   if (kMode == MIXFP4_MODE_E2M1_ONLY) T = 0;
   else if (kMode == MIXFP4_MODE_E1M2_ONLY) T = 1;
   else T = (S2 < S1) ? 0 : 1;  // strict "<" of Algorithm 1
 
-  code_lo = 0;
-  code_hi = 0;
-#pragma unroll
-  for (int j = 0; j < 8; ++j) {
-    uint32_t p;
-    if (kMode == MIXFP4_MODE_E2M1_ONLY) p = pay2[j];
-    else if (kMode == MIXFP4_MODE_E1M2_ONLY) p = pay1[j];
-    else p = T ? pay1[j] : pay2[j];
-    const uint32_t byte = (p | sgn[j]) & 0xFFu;
-    if (j < 4) code_lo |= byte << (8 * j);
-    else code_hi |= byte << (8 * (j - 4));
-  }
-  scale_byte = T ? (0x80u | ((sc >> 8) & 0x7Fu)) : (sc & 0x7Fu);
+  code_lo = (T ? p1lo : p2lo) | sign_bits(w[0], w[1], w[2], w[3]);
+  code_hi = (T ? p1hi : p2hi) | sign_bits(w[4], w[5], w[6], w[7]);
+  scale_byte = T ? (0x80u | c1) : c2;
 }
 
+template <bool kContig>
+__device__ __forceinline__ const uint16_t* block_src(const uint16_t* x, int64_t b, int64_t kblocks, int64_t ldx) {
+  if (kContig) return x + b * 16;
+  const int64_t row = b / kblocks;
+  return x + row * ldx + (b - row * kblocks) * 16;
+}
+
+// Persistent grid: each thread walks blocks b, b + nthr, b + 2 nthr, ... and
+// keeps the next block's 32-byte load in flight while it quantizes the
+// current one.  The first loads are issued before any set-up work.
 template <int kMode, bool kContig>
-__global__ void __launch_bounds__(kQuantThreads)
+__global__ void __launch_bounds__(kQuantThreads, 4)
 quantize_kernel(const uint16_t* __restrict__ x, int64_t nblocks, int64_t kblocks, int64_t ldx,
                 uint8_t* __restrict__ codes, uint8_t* __restrict__ scales, float* tensor_scale,
                 const uint32_t* amax_word, int scale_given) {
-  __shared__ TensorConsts sh;
-  const TensorConsts tc = tensor_consts(tensor_scale, amax_word, scale_given, &sh);
-  const int64_t b = (int64_t)blockIdx.x * kQuantThreads + threadIdx.x;
-  if (b >= nblocks) return;
-  const uint16_t* src;
-  if (kContig) {
-    src = x + b * 16;
-  } else {
-    const int64_t row = b / kblocks;
-    src = x + row * ldx + (b - row * kblocks) * 16;
+  __shared__ float2 tab[128];  // E4M3 code -> {s8, RN(1/s8)}
+  const int64_t nthr = (int64_t)gridDim.x * kQuantThreads;
+  int64_t b = (int64_t)blockIdx.x * kQuantThreads + threadIdx.x;
+  uint32_t wa[8], wb[8];
+  if (b < nblocks) ldg256_stream(block_src<kContig>(x, b, kblocks, ldx), wa);
+  if (b + nthr < nblocks) ldg256_stream(block_src<kContig>(x, b + nthr, kblocks, ldx), wb);
+  if (threadIdx.x < 128) {
+    float s8 = 0.0f, unused;
+    if (threadIdx.x < 0x7F) f16x2_to_f32(cvt_f16x2_from_e4m3x2((uint16_t)threadIdx.x), s8, unused);
+    tab[threadIdx.x] = make_float2(s8, s8 > 0.0f ? __frcp_rn(s8) : 0.0f);
   }
-  uint32_t w[8];
-  ldg256_stream(src, w);
-  uint32_t lo, hi, sb;
-  if (tc.scaled) quantize_block<kMode, true>(w, tc, lo, hi, sb);
-  else quantize_block<kMode, false>(w, tc, lo, hi, sb);
-  stg64(codes + b * 8, lo, hi);
-  scales[b] = (uint8_t)sb;
+  const TensorConsts tc = tensor_consts(tensor_scale, amax_word, scale_given);
+  __syncthreads();
+  for (; b < nblocks; b += 2 * nthr) {
+    uint32_t lo, hi, sb;
+    if (tc.scaled) quantize_block<kMode, true>(wa, tc, tab, lo, hi, sb);
+    else quantize_block<kMode, false>(wa, tc, tab, lo, hi, sb);
+    stg64(codes + b * 8, lo, hi);
+    scales[b] = (uint8_t)sb;
+    if (b + 2 * nthr < nblocks) ldg256_stream(block_src<kContig>(x, b + 2 * nthr, kblocks, ldx), wa);
+    const int64_t b1 = b + nthr;
+    if (b1 < nblocks) {
+      if (tc.scaled) quantize_block<kMode, true>(wb, tc, tab, lo, hi, sb);
+      else quantize_block<kMode, false>(wb, tc, tab, lo, hi, sb);
+      stg64(codes + b1 * 8, lo, hi);
+      scales[b1] = (uint8_t)sb;
+      if (b1 + 2 * nthr < nblocks) ldg256_stream(block_src<kContig>(x, b1 + 2 * nthr, kblocks, ldx), wb);
+    }
+  }
 }
 
 // max |x| over the tensor as the bit pattern of a non-negative fp32 (bf16
@@ -295,7 +350,10 @@ int launch_quantize(const uint16_t* x, int64_t rows, int64_t K, int64_t ldx, uin
                     uint8_t* scales, float* tensor_scale, const uint32_t* amax_word, int mode,
                     int scale_given, cudaStream_t stream) {
   const int64_t kblocks = K / 16, nblocks = rows * kblocks;
-  const int64_t grid = (nblocks + kQuantThreads - 1) / kQuantThreads;
+  // Persistent grid: 4 CTAs per SM of a 152-SM GB300, fewer for small tensors
+  // (each thread takes at least two blocks).
+  int64_t grid = (nblocks + 2 * kQuantThreads - 1) / (2 * kQuantThreads);
+  if (grid > 152 * 4) grid = 152 * 4;
   if (grid == 0) return 0;
 #define MIXFP4_LAUNCH_Q(MODE)                                                              \
   do {                                                                                     \
