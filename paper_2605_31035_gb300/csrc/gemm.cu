@@ -12,17 +12,16 @@
 // (half) of B, so each CTA decodes 256 rows per K step while its tensor core
 // produces a 128 x 256 slab.  Per CTA:
 //   warp 0      TMA producer: codes [rows][128 B] (128-byte swizzle) and
-//               scales [rows][16 B] of a 256-wide K slice into a 3-deep ring;
+//               scales [rows][16 B] of a 256-wide K slice into a 2-deep ring;
 //   warp 1      TMEM allocator (both CTAs); in the leader CTA also the single
 //               MMA-issuing thread.  Accumulators: 2 x (128 lanes x 256 fp32)
 //               per CTA, double-buffered across tiles;
-//   warps 2-17  decoders, two threads per operand row (128 A + 128 B), each
-//               turning 32 K of the row per sub-stage into f16 in the
-//               canonical K-major no-swizzle UMMA layout, 3-deep ring.  The
-//               leader's MMA waits for both CTAs' decoders (remote mbarrier
-//               arrivals);
-//   warps 18-21 epilogue: tcgen05.ld -> x s32A s32B / 4 -> fp32 C, overlapped
-//               with the next tile's main loop.
+//   decoders    kTPR threads per operand row (128 A + 128 B), each turning
+//               its share of a sub-stage's K into f16 in the canonical K-major
+//               no-swizzle UMMA layout, kDecStages-deep ring.  The leader's MMA
+//               waits for both CTAs' decoders (remote mbarrier arrivals);
+//   last 4 warps  epilogue: tcgen05.ld -> x s32A s32B / 4 -> fp32 C,
+//               overlapped with the next tile's main loop.
 // All pipeline waits are bounded; a wait that gives up records a nonzero
 // status word and the CTA drains and exits without touching C.
 #include <cuda.h>
@@ -42,16 +41,29 @@ using namespace sm100;
 constexpr int BM = 128;            // A rows per CTA (pair tile: 256)
 constexpr int BNH = 128;           // B rows per CTA (pair tile: 256)
 constexpr int TILE_M = 2 * BM, TILE_N = 2 * BNH;
-constexpr int BKC = 256;           // K per TMA code stage
-constexpr int BKD = 64;            // K per decoded sub-stage
+#ifndef MIXFP4_GEMM_BKD
+#define MIXFP4_GEMM_BKD 128
+#endif
+#ifndef MIXFP4_GEMM_DEC_STAGES
+#define MIXFP4_GEMM_DEC_STAGES 2
+#endif
+#ifndef MIXFP4_GEMM_TPR
+#define MIXFP4_GEMM_TPR 2
+#endif
+constexpr int BKC = 256;                      // K per TMA code stage
+constexpr int BKD = MIXFP4_GEMM_BKD;          // K per decoded sub-stage
 constexpr int kSub = BKC / BKD;
-constexpr int kCodeStages = 3;
-constexpr int kDecStages = 3;
-constexpr int kDecodeWarps = 2 * (BM + BNH) / 32;   // 16: two threads per operand row
+constexpr int kCodeStages = 2;
+constexpr int kDecStages = MIXFP4_GEMM_DEC_STAGES;
+constexpr int kTPR = MIXFP4_GEMM_TPR;         // decode threads per operand row
+constexpr int kChunksPerSub = BKD / 32;       // 16-byte code chunks (32 codes) per row per sub-stage
+constexpr int kChunksPerThread = kChunksPerSub / kTPR;
+static_assert(kChunksPerThread >= 1 && kChunksPerSub % kTPR == 0, "decode split");
+constexpr int kDecodeWarps = kTPR * (BM + BNH) / 32;
 constexpr int kEpiWarps = 4;
 constexpr int kFirstDecodeWarp = 2;
-constexpr int kFirstEpiWarp = kFirstDecodeWarp + kDecodeWarps;  // 18
-constexpr int kThreads = 32 * (kFirstEpiWarp + kEpiWarps);      // 704
+constexpr int kFirstEpiWarp = kFirstDecodeWarp + kDecodeWarps;
+constexpr int kThreads = 32 * (kFirstEpiWarp + kEpiWarps);
 constexpr uint32_t kAccCols = TILE_N;           // fp32 columns per accumulator
 constexpr uint32_t kTmemCols = 2 * kAccCols;    // double-buffered
 
@@ -190,8 +202,7 @@ mixfp4_gemm_kernel(const __grid_constant__ CUtensorMap tm_ac, const __grid_const
       tma_prefetch(&tm_bc);
       tma_prefetch(&tm_as);
       tma_prefetch(&tm_bs);
-      int last_phase[kCodeStages];
-      for (int s = 0; s < kCodeStages; ++s) last_phase[s] = -1;
+      int last_it = -1;  // last code-stage use issued (its copies may be in flight)
       int it = 0;
       bool ok = true;
       for (int t = cluster_id; t < ntiles && ok; t += nclusters) {
@@ -213,14 +224,15 @@ mixfp4_gemm_kernel(const __grid_constant__ CUtensorMap tm_ac, const __grid_const
           tma_load_2d(st + A_CODE_BYTES, &tm_bc, xk, nb, fb);
           tma_load_2d(st + A_CODE_BYTES + B_CODE_BYTES, &tm_as, xs, ma, fb);
           tma_load_2d(st + A_CODE_BYTES + B_CODE_BYTES + A_SCALE_BYTES, &tm_bs, xs, nb, fb);
-          last_phase[s] = (int)ph;
+          last_it = it;
         }
       }
       if (*abort_flag) {
         // Let the copies this thread started land before the CTA may exit.
-        for (int s = 0; s < kCodeStages; ++s)
-          if (last_phase[s] >= 0)
-            mbar_wait(smem_u32(&bars->code_full[s]), (uint32_t)last_phase[s], nullptr, kWaitLimitNs);
+        for (int u = last_it - kCodeStages + 1; u <= last_it; ++u)
+          if (u >= 0)
+            mbar_wait(smem_u32(&bars->code_full[u % kCodeStages]), (uint32_t)((u / kCodeStages) & 1), nullptr,
+                      kWaitLimitNs);
       }
     }
   } else if (warp == 1) {
@@ -267,15 +279,14 @@ mixfp4_gemm_kernel(const __grid_constant__ CUtensorMap tm_ac, const __grid_const
       if (!mbar_wait_cluster(smem_u32(&bars->drain), 0, nullptr, kWaitLimitNs)) fail(8u);
     }
   } else if (warp < kFirstEpiWarp) {
-    // ---------------- decoders (two threads per operand row) ----------------
-    const int dt = threadIdx.x - 32 * kFirstDecodeWarp;  // 0..511
-    const int row = dt & 255, half = dt >> 8;            // half: which 32 K of a sub-stage
+    // ---------------- decoders (kTPR threads per operand row) ----------------
+    const int dt = threadIdx.x - 32 * kFirstDecodeWarp;
+    const int row = dt & 255, part = dt >> 8;  // part: which share of a sub-stage's chunks
     const bool is_a = row < BM;
     const int rl = is_a ? row : row - BM;
     const uint32_t code_off = (is_a ? 0 : A_CODE_BYTES) + rl * (BKC / 2);
     const uint32_t scale_off = A_CODE_BYTES + B_CODE_BYTES + (is_a ? 0 : A_SCALE_BYTES) + rl * (BKC / 16);
-    const uint32_t dec_off = OFF_DEC + (is_a ? 0 : A_DEC_BYTES) + (rl >> 3) * kSBO + (rl & 7) * 16 +
-                             half * 4 * kLBO;
+    const uint32_t dec_off = OFF_DEC + (is_a ? 0 : A_DEC_BYTES) + (rl >> 3) * kSBO + (rl & 7) * 16;
     const uint32_t swz = rl & 7;
     const uint32_t dec_full_leader0 = mapa_shared(smem_u32(&bars->dec_full[0]), 0);
     int d = 0;
@@ -292,38 +303,50 @@ mixfp4_gemm_kernel(const __grid_constant__ CUtensorMap tm_ac, const __grid_const
           break;
         }
         const uint32_t st = sbase + s * CODE_STAGE_BYTES;
-        const uint4 sc = lds128(st + scale_off);
-        const uint32_t scw[4] = {sc.x, sc.y, sc.z, sc.w};
+        const uint4 sc = lds128(st + scale_off);  // the row's 16 block scales of this code stage
 #pragma unroll
         for (int sub = 0; sub < kSub; ++sub) {
-          // this thread's 32 codes of the sub-stage: logical 16-byte chunk 2*sub + half
-          const uint4 c = lds128(st + code_off + (((2 * sub + half) ^ swz) << 4));
+          uint4 c[kChunksPerThread];
+#pragma unroll
+          for (int j = 0; j < kChunksPerThread; ++j) {
+            const int chunk = sub * kChunksPerSub + part * kChunksPerThread + j;
+            c[j] = lds128(st + code_off + (((uint32_t)chunk ^ swz) << 4));
+          }
           if (!mbar_wait_cluster(smem_u32(&bars->dec_empty[d]), dph ^ 1, abort_flag, kWaitLimitNs)) {
             fail(32u);
             ok = false;
             break;
           }
-          const uint32_t w[4] = {c.x, c.y, c.z, c.w};
-          // scale bytes of this thread's two blocks (blocks 4*sub + 2*half, +1)
-          const uint32_t s2b = (scw[sub] >> (16 * half)) & 0xFFFFu;
-          const uint32_t h01 = cvt_f16x2_from_e4m3x2((uint16_t)(s2b & 0x7F7Fu));
-          const uint32_t sv[2] = {prmt(h01, 0u, 0x1010u), prmt(h01, 0u, 0x3232u)};
           const uint32_t dst = sbase + dec_off + d * DEC_STAGE_BYTES;
 #pragma unroll
-          for (int b = 0; b < 2; ++b) {
-            const bool e1m2 = (s2b >> (8 * b + 7)) & 1u;
-            const uint32_t lut_lo = e1m2 ? kLutE1M2Lo : kLutE2M1Lo;
-            const uint32_t lut_hi = e1m2 ? kLutE1M2Hi : kLutE2M1Hi;
+          for (int j = 0; j < kChunksPerThread; ++j) {
+            const int chunk = sub * kChunksPerSub + part * kChunksPerThread + j;  // 32 codes, 2 blocks
+            const int sw = chunk >> 1;  // scale word holding blocks 2*chunk, 2*chunk+1
+            const uint32_t s4 = sw == 0 ? sc.x : sw == 1 ? sc.y : sw == 2 ? sc.z : sc.w;
+            const uint32_t s2b = (s4 >> (16 * (chunk & 1))) & 0xFFFFu;
+            const uint32_t h01 = cvt_f16x2_from_e4m3x2((uint16_t)(s2b & 0x7F7Fu));
+            const uint32_t sv[2] = {prmt(h01, 0u, 0x1010u), prmt(h01, 0u, 0x3232u)};
+            const uint32_t w[4] = {c[j].x, c[j].y, c[j].z, c[j].w};
+            const int kchunk0 = (chunk - sub * kChunksPerSub) * 4;  // first 8-element K chunk
 #pragma unroll
-            for (int i = 0; i < 2; ++i) {
-              uint32_t o[4];
-              decode8(w[2 * b + i], lut_lo, lut_hi, sv[b], o);
-              sts128(dst + (2 * b + i) * kLBO, o[0], o[1], o[2], o[3]);
+            for (int b = 0; b < 2; ++b) {
+              const bool e1m2 = (s2b >> (8 * b + 7)) & 1u;
+              const uint32_t lut_lo = e1m2 ? kLutE1M2Lo : kLutE2M1Lo;
+              const uint32_t lut_hi = e1m2 ? kLutE1M2Hi : kLutE2M1Hi;
+#pragma unroll
+              for (int i = 0; i < 2; ++i) {
+                uint32_t o[4];
+                decode8(w[2 * b + i], lut_lo, lut_hi, sv[b], o);
+                sts128(dst + (kchunk0 + 2 * b + i) * kLBO, o[0], o[1], o[2], o[3]);
+              }
             }
           }
           fence_proxy_async_smem();
           __syncwarp();
-          if (lane == 0) mbar_arrive_cluster(dec_full_leader0 + d * 8);
+          if (lane == 0) {
+            if (leader) mbar_arrive(smem_u32(&bars->dec_full[d]));
+            else mbar_arrive_cluster(dec_full_leader0 + d * 8);
+          }
           if (++d == kDecStages) { d = 0; dph ^= 1; }
           if (sub == kSub - 1) {
             // Release the code stage only now: every value loaded from it has
