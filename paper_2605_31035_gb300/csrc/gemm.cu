@@ -9,19 +9,21 @@
 //
 // Work decomposition: persistent CTA pairs (clusters of 2, cta_group::2).  A
 // pair owns 256 x 256 output tiles; each CTA holds 128 rows of A and 128 rows
-// (half) of B, so each CTA decodes 256 rows per K step while its tensor core
-// produces a 128 x 256 slab.  Per CTA:
-//   warp 0      TMA producer: codes [rows][128 B] (128-byte swizzle) and
-//               scales [rows][16 B] of a 256-wide K slice into a 2-deep ring;
-//   warp 1      TMEM allocator (both CTAs); in the leader CTA also the single
-//               MMA-issuing thread.  Accumulators: 2 x (128 lanes x 256 fp32)
-//               per CTA, double-buffered across tiles;
-//   decoders    kTPR threads per operand row (128 A + 128 B), each turning
-//               its share of a sub-stage's K into f16 in the canonical K-major
-//               no-swizzle UMMA layout, kDecStages-deep ring.  The leader's MMA
-//               waits for both CTAs' decoders (remote mbarrier arrivals);
-//   last 4 warps  epilogue: tcgen05.ld -> x s32A s32B / 4 -> fp32 C,
-//               overlapped with the next tile's main loop.
+// (half) of B.  Decoded A never touches shared memory: it is written to tensor
+// memory (tcgen05.st) and the MMA reads it from there; decoded B goes through
+// shared memory.  Per CTA:
+//   warp 0        TMA producer: codes [rows][128 B] (128-byte swizzle) and
+//                 scales [rows][16 B] of a 256-wide K slice into a 2-deep ring;
+//   warp 1        TMEM allocator (both CTAs); in the leader CTA also the single
+//                 MMA-issuing thread;
+//   warps 2-9     A decoders, two threads per A row (lane quarter = warp % 4),
+//                 64 K of the row per stage -> f16 pairs in TMEM columns;
+//   warps 10-17   B decoders, two threads per B row, 64 K of the row per stage
+//                 -> f16 in the canonical K-major no-swizzle UMMA layout;
+//   warps 18-25   epilogue: tcgen05.ld -> x s32A s32B / 4 -> fp32 C.
+// TMEM per CTA (512 columns): fp32 accumulator 128 lanes x 256 columns, then
+// kDecStages A stages of 64 columns (128 K of f16 pairs).  The leader's MMA
+// waits for both CTAs' decoders (remote mbarrier arrivals).
 // All pipeline waits are bounded; a wait that gives up records a nonzero
 // status word and the CTA drains and exits without touching C.
 #include <cuda.h>
@@ -38,55 +40,50 @@ namespace {
 
 using namespace sm100;
 
-constexpr int BM = 128;            // A rows per CTA (pair tile: 256)
-constexpr int BNH = 128;           // B rows per CTA (pair tile: 256)
+constexpr int BM = 128;                       // A rows per CTA (pair tile: 256)
+constexpr int BNH = 128;                      // B rows per CTA (pair tile: 256)
 constexpr int TILE_M = 2 * BM, TILE_N = 2 * BNH;
-#ifndef MIXFP4_GEMM_BKD
-#define MIXFP4_GEMM_BKD 128
-#endif
-#ifndef MIXFP4_GEMM_DEC_STAGES
-#define MIXFP4_GEMM_DEC_STAGES 2
-#endif
-#ifndef MIXFP4_GEMM_TPR
-#define MIXFP4_GEMM_TPR 2
-#endif
 constexpr int BKC = 256;                      // K per TMA code stage
-constexpr int BKD = MIXFP4_GEMM_BKD;          // K per decoded sub-stage
+constexpr int BKD = 128;                      // K per decoded stage
 constexpr int kSub = BKC / BKD;
 constexpr int kCodeStages = 2;
-constexpr int kDecStages = MIXFP4_GEMM_DEC_STAGES;
-constexpr int kTPR = MIXFP4_GEMM_TPR;         // decode threads per operand row
-constexpr int kChunksPerSub = BKD / 32;       // 16-byte code chunks (32 codes) per row per sub-stage
+constexpr int kDecStages = 4;
+constexpr int kTPR = 2;                       // decode threads per operand row
+constexpr int kChunksPerSub = BKD / 32;       // 16-byte code chunks (32 codes) per row per stage
 constexpr int kChunksPerThread = kChunksPerSub / kTPR;
-static_assert(kChunksPerThread >= 1 && kChunksPerSub % kTPR == 0, "decode split");
-constexpr int kDecodeWarps = kTPR * (BM + BNH) / 32;
-constexpr int kEpiWarps = 4;
-constexpr int kFirstDecodeWarp = 2;
-constexpr int kFirstEpiWarp = kFirstDecodeWarp + kDecodeWarps;
-constexpr int kThreads = 32 * (kFirstEpiWarp + kEpiWarps);
-constexpr uint32_t kAccCols = TILE_N;           // fp32 columns per accumulator
-constexpr uint32_t kTmemCols = 2 * kAccCols;    // double-buffered
+constexpr int kDecodeWarpsA = kTPR * BM / 32;   // 8
+constexpr int kDecodeWarpsB = kTPR * BNH / 32;  // 8
+constexpr int kEpiWarps = 8;
+constexpr int kFirstDecA = 2;
+constexpr int kFirstDecB = kFirstDecA + kDecodeWarpsA;   // 10
+constexpr int kFirstEpi = kFirstDecB + kDecodeWarpsB;    // 18
+constexpr int kThreads = 32 * (kFirstEpi + kEpiWarps);   // 832
+constexpr int kDecodeWarps = kDecodeWarpsA + kDecodeWarpsB;
+static_assert(kFirstDecA % 4 == 2 && kDecodeWarpsA % 4 == 0, "A decoders cover every TMEM lane quarter");
+
+constexpr uint32_t kAccCols = TILE_N;                 // fp32 accumulator columns
+constexpr uint32_t kAStageCols = BKD / 2;             // f16 pairs per A row per stage
+constexpr uint32_t kTmemCols = 512;
+static_assert(kAccCols + kDecStages * kAStageCols <= kTmemCols, "TMEM budget");
 
 constexpr int A_CODE_BYTES = BM * BKC / 2;
 constexpr int B_CODE_BYTES = BNH * BKC / 2;
 constexpr int A_SCALE_BYTES = BM * BKC / 16;
 constexpr int B_SCALE_BYTES = BNH * BKC / 16;
 constexpr int CODE_STAGE_BYTES = A_CODE_BYTES + B_CODE_BYTES + A_SCALE_BYTES + B_SCALE_BYTES;
-constexpr int A_DEC_BYTES = BM * BKD * 2;
 constexpr int B_DEC_BYTES = BNH * BKD * 2;
-constexpr int DEC_STAGE_BYTES = A_DEC_BYTES + B_DEC_BYTES;
 constexpr int OFF_DEC = kCodeStages * CODE_STAGE_BYTES;
-constexpr int OFF_BAR = OFF_DEC + kDecStages * DEC_STAGE_BYTES;
+constexpr int OFF_BAR = OFF_DEC + kDecStages * B_DEC_BYTES;
 constexpr int SMEM_BYTES = OFF_BAR + 256;
 constexpr int SMEM_ALLOC = SMEM_BYTES + 1024;  // slack to align the base to 1024 B
 
 static_assert(CODE_STAGE_BYTES % 1024 == 0, "code stages must keep 1024-byte alignment");
 static_assert(SMEM_ALLOC <= 232448, "shared memory budget");
 
-// Decoded-operand layout: core matrix (8 rows x 16 B) at
+// Decoded-B layout: core matrix (8 rows x 16 B) at
 //   (row / 8) * SBO + kchunk * LBO + (row % 8) * 16
 constexpr uint32_t kLBO = 128;                  // next 8 K-elements
-constexpr uint32_t kSBO = (BKD / 8) * 128;      // next 8 rows (1024 B)
+constexpr uint32_t kSBO = (BKD / 8) * 128;      // next 8 rows
 constexpr uint32_t kIdesc = idesc_f16_f32(TILE_M, TILE_N);
 
 constexpr uint64_t kWaitLimitNs = 1000000000ull;  // 1 s per pipeline wait
@@ -96,8 +93,8 @@ struct Bars {
   uint64_t code_empty[kCodeStages];
   uint64_t dec_full[kDecStages];    // leader: 2 x kDecodeWarps arrivals
   uint64_t dec_empty[kDecStages];   // MMA commit (multicast to both CTAs)
-  uint64_t acc_full[2];             // MMA commit (multicast)
-  uint64_t acc_empty[2];            // leader: 2 x kEpiWarps arrivals
+  uint64_t acc_full;                // MMA commit (multicast)
+  uint64_t acc_empty;               // leader: 2 x kEpiWarps arrivals
   uint64_t drain;
   uint32_t tmem_base;
   int abort;
@@ -130,7 +127,7 @@ constexpr uint32_t kLutE1M2Lo = 0x46444000u, kLutE1M2Hi = 0x4B4A4948u;
 // nibble sign moved into bit 7 of each byte (prmt + lop3), bytes placed as f16
 // high bytes (prmt), times s8 (exact).
 __device__ __forceinline__ void decode8(uint32_t w, uint32_t lut_lo, uint32_t lut_hi, uint32_t s2,
-                                        uint32_t out[4]) {
+                                        uint32_t* out) {
   const uint32_t wp = w & 0x77777777u;
   const uint32_t ws = w * 16u;
   const uint32_t u0 = prmt(lut_lo, lut_hi, wp);
@@ -143,6 +140,28 @@ __device__ __forceinline__ void decode8(uint32_t w, uint32_t lut_lo, uint32_t lu
   out[1] = hmul2(prmt(v0, 0u, 0x3424u), s2);
   out[2] = hmul2(prmt(v1, 0u, 0x1404u), s2);
   out[3] = hmul2(prmt(v1, 0u, 0x3424u), s2);
+}
+
+// Decode 32 codes (one 16-byte chunk = two 16-element blocks) with their two
+// scale bytes s2b into 16 f16x2 words in K order.
+__device__ __forceinline__ void decode_chunk(const uint4& c, uint32_t s2b, uint32_t* out) {
+  const uint32_t h01 = cvt_f16x2_from_e4m3x2((uint16_t)(s2b & 0x7F7Fu));
+  const uint32_t sv[2] = {prmt(h01, 0u, 0x1010u), prmt(h01, 0u, 0x3232u)};
+  const uint32_t w[4] = {c.x, c.y, c.z, c.w};
+#pragma unroll
+  for (int b = 0; b < 2; ++b) {
+    const bool e1m2 = (s2b >> (8 * b + 7)) & 1u;
+    const uint32_t lut_lo = e1m2 ? kLutE1M2Lo : kLutE2M1Lo;
+    const uint32_t lut_hi = e1m2 ? kLutE1M2Hi : kLutE2M1Hi;
+    decode8(w[2 * b], lut_lo, lut_hi, sv[b], out + 8 * b);
+    decode8(w[2 * b + 1], lut_lo, lut_hi, sv[b], out + 8 * b + 4);
+  }
+}
+
+__device__ __forceinline__ uint32_t scale_pair(const uint4& sc, int chunk) {
+  const int sw = chunk >> 1;  // scale word holding blocks 2*chunk, 2*chunk+1
+  const uint32_t s4 = sw == 0 ? sc.x : sw == 1 ? sc.y : sw == 2 ? sc.z : sc.w;
+  return (s4 >> (16 * (chunk & 1))) & 0xFFFFu;
 }
 
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
@@ -173,10 +192,8 @@ mixfp4_gemm_kernel(const __grid_constant__ CUtensorMap tm_ac, const __grid_const
       mbar_init(smem_u32(&bars->dec_full[s]), 2 * kDecodeWarps);
       mbar_init(smem_u32(&bars->dec_empty[s]), 1);
     }
-    for (int s = 0; s < 2; ++s) {
-      mbar_init(smem_u32(&bars->acc_full[s]), 1);
-      mbar_init(smem_u32(&bars->acc_empty[s]), 2 * kEpiWarps);
-    }
+    mbar_init(smem_u32(&bars->acc_full), 1);
+    mbar_init(smem_u32(&bars->acc_empty), 2 * kEpiWarps);
     mbar_init(smem_u32(&bars->drain), 1);
     bars->abort = 0;
     fence_mbar_init();
@@ -189,6 +206,7 @@ mixfp4_gemm_kernel(const __grid_constant__ CUtensorMap tm_ac, const __grid_const
   cluster_sync();  // barriers of both CTAs initialised, TMEM allocated in both
   tc_fence_after();
   const uint32_t tmem_base = bars->tmem_base;
+  const uint32_t tmem_a0 = tmem_base + kAccCols;  // first A stage column
 
   auto fail = [&](uint32_t code) {
     *abort_flag = 1;
@@ -243,14 +261,11 @@ mixfp4_gemm_kernel(const __grid_constant__ CUtensorMap tm_ac, const __grid_const
       bool ok = true;
       int i = 0;
       for (int t = cluster_id; t < ntiles && ok; t += nclusters, ++i) {
-        const int ab = i & 1;
-        const uint32_t aph = (i >> 1) & 1;
-        if (!mbar_wait_cluster(smem_u32(&bars->acc_empty[ab]), aph ^ 1, abort_flag, kWaitLimitNs)) {
+        if (!mbar_wait_cluster(smem_u32(&bars->acc_empty), (i & 1) ^ 1, abort_flag, kWaitLimitNs)) {
           fail(2u);
           break;
         }
         tc_fence_after();
-        const uint32_t dtm = tmem_base + (uint32_t)ab * kAccCols;
         for (int kc = 0; kc < num_kc && ok; ++kc) {
           for (int sub = 0; sub < kSub; ++sub) {
             if (!mbar_wait_cluster(smem_u32(&bars->dec_full[d]), dph, abort_flag, kWaitLimitNs)) {
@@ -259,34 +274,35 @@ mixfp4_gemm_kernel(const __grid_constant__ CUtensorMap tm_ac, const __grid_const
               break;
             }
             tc_fence_after();
-            const uint32_t abase = sbase + OFF_DEC + d * DEC_STAGE_BYTES;
-            const uint32_t bbase = abase + A_DEC_BYTES;
+            const uint32_t bbase = sbase + OFF_DEC + d * B_DEC_BYTES;
+            const uint32_t abase = tmem_a0 + (uint32_t)d * kAStageCols;
 #pragma unroll
             for (int j = 0; j < BKD / 16; ++j) {
-              const uint64_t ad = smem_desc_noswizzle(abase + j * 256, kLBO, kSBO);
               const uint64_t bd = smem_desc_noswizzle(bbase + j * 256, kLBO, kSBO);
-              mma_f16_pair(dtm, ad, bd, kIdesc, (kc | sub | j) != 0 ? 1u : 0u);
+              mma_f16_pair_tmem_a(tmem_base, abase + j * 8, bd, kIdesc, (kc | sub | j) != 0 ? 1u : 0u);
             }
             mma_commit_pair(smem_u32(&bars->dec_empty[d]), 3);
             if (++d == kDecStages) { d = 0; dph ^= 1; }
           }
         }
-        if (ok) mma_commit_pair(smem_u32(&bars->acc_full[ab]), 3);
+        if (ok) mma_commit_pair(smem_u32(&bars->acc_full), 3);
       }
       // Every MMA issued above completes before the drain barrier fires; wait
       // for it (ignoring the abort flag) so TMEM is never freed under an MMA.
       mma_commit_pair(smem_u32(&bars->drain), 1);
       if (!mbar_wait_cluster(smem_u32(&bars->drain), 0, nullptr, kWaitLimitNs)) fail(8u);
     }
-  } else if (warp < kFirstEpiWarp) {
-    // ---------------- decoders (kTPR threads per operand row) ----------------
-    const int dt = threadIdx.x - 32 * kFirstDecodeWarp;
-    const int row = dt & 255, part = dt >> 8;  // part: which share of a sub-stage's chunks
-    const bool is_a = row < BM;
-    const int rl = is_a ? row : row - BM;
+  } else if (warp < kFirstEpi) {
+    // ---------------- decoders ----------------
+    const bool is_a = warp < kFirstDecB;
+    const int dw = warp - (is_a ? kFirstDecA : kFirstDecB);
+    const int part = dw >> 2;                      // which half of a stage's chunks
+    // A decoders: rows follow the warp's TMEM lane quarter (warp % 4).
+    const int rl = is_a ? ((warp & 3) * 32 + lane) : (dw & 3) * 32 + lane;
     const uint32_t code_off = (is_a ? 0 : A_CODE_BYTES) + rl * (BKC / 2);
     const uint32_t scale_off = A_CODE_BYTES + B_CODE_BYTES + (is_a ? 0 : A_SCALE_BYTES) + rl * (BKC / 16);
-    const uint32_t dec_off = OFF_DEC + (is_a ? 0 : A_DEC_BYTES) + (rl >> 3) * kSBO + (rl & 7) * 16;
+    const uint32_t b_off = OFF_DEC + (rl >> 3) * kSBO + (rl & 7) * 16;
+    const uint32_t a_lane = (uint32_t)((warp & 3) * 32) << 16;
     const uint32_t swz = rl & 7;
     const uint32_t dec_full_leader0 = mapa_shared(smem_u32(&bars->dec_full[0]), 0);
     int d = 0;
@@ -317,31 +333,29 @@ mixfp4_gemm_kernel(const __grid_constant__ CUtensorMap tm_ac, const __grid_const
             ok = false;
             break;
           }
-          const uint32_t dst = sbase + dec_off + d * DEC_STAGE_BYTES;
+          if (is_a) {
+            // 64 K of the row = 32 f16 pairs -> TMEM columns [part * 32, +32) of stage d
+            uint32_t o[32];
 #pragma unroll
-          for (int j = 0; j < kChunksPerThread; ++j) {
-            const int chunk = sub * kChunksPerSub + part * kChunksPerThread + j;  // 32 codes, 2 blocks
-            const int sw = chunk >> 1;  // scale word holding blocks 2*chunk, 2*chunk+1
-            const uint32_t s4 = sw == 0 ? sc.x : sw == 1 ? sc.y : sw == 2 ? sc.z : sc.w;
-            const uint32_t s2b = (s4 >> (16 * (chunk & 1))) & 0xFFFFu;
-            const uint32_t h01 = cvt_f16x2_from_e4m3x2((uint16_t)(s2b & 0x7F7Fu));
-            const uint32_t sv[2] = {prmt(h01, 0u, 0x1010u), prmt(h01, 0u, 0x3232u)};
-            const uint32_t w[4] = {c[j].x, c[j].y, c[j].z, c[j].w};
-            const int kchunk0 = (chunk - sub * kChunksPerSub) * 4;  // first 8-element K chunk
+            for (int j = 0; j < kChunksPerThread; ++j)
+              decode_chunk(c[j], scale_pair(sc, sub * kChunksPerSub + part * kChunksPerThread + j), o + 16 * j);
+            tmem_st_32x32b_x32(tmem_a0 + a_lane + (uint32_t)d * kAStageCols + (uint32_t)part * 32u, o);
+            tmem_st_wait();
+            tc_fence_before();
+          } else {
+            const uint32_t dst = sbase + b_off + d * B_DEC_BYTES;
 #pragma unroll
-            for (int b = 0; b < 2; ++b) {
-              const bool e1m2 = (s2b >> (8 * b + 7)) & 1u;
-              const uint32_t lut_lo = e1m2 ? kLutE1M2Lo : kLutE2M1Lo;
-              const uint32_t lut_hi = e1m2 ? kLutE1M2Hi : kLutE2M1Hi;
+            for (int j = 0; j < kChunksPerThread; ++j) {
+              const int chunk = sub * kChunksPerSub + part * kChunksPerThread + j;
+              uint32_t o[16];
+              decode_chunk(c[j], scale_pair(sc, chunk), o);
+              const int kchunk0 = (chunk - sub * kChunksPerSub) * 4;  // first 8-element K chunk
 #pragma unroll
-              for (int i = 0; i < 2; ++i) {
-                uint32_t o[4];
-                decode8(w[2 * b + i], lut_lo, lut_hi, sv[b], o);
-                sts128(dst + (kchunk0 + 2 * b + i) * kLBO, o[0], o[1], o[2], o[3]);
-              }
+              for (int q = 0; q < 4; ++q)
+                sts128(dst + (kchunk0 + q) * kLBO, o[4 * q], o[4 * q + 1], o[4 * q + 2], o[4 * q + 3]);
             }
+            fence_proxy_async_smem();
           }
-          fence_proxy_async_smem();
           __syncwarp();
           if (lane == 0) {
             if (leader) mbar_arrive(smem_u32(&bars->dec_full[d]));
@@ -359,16 +373,15 @@ mixfp4_gemm_kernel(const __grid_constant__ CUtensorMap tm_ac, const __grid_const
       }
     }
   } else {
-    // ---------------- epilogue ----------------
-    const int q = warp & 3;  // TMEM lane quarter of this warp
+    // ---------------- epilogue (two warps per TMEM lane quarter) ----------------
+    const int q = warp & 3;                  // TMEM lane quarter of this warp
+    const int chalf = (warp - kFirstEpi) >> 2;  // column half
     const float sa = 0.25f * __ldg(a_ts), sb = __ldg(b_ts);
     const bool vec_ok = ((ldc & 3) == 0) && ((reinterpret_cast<uintptr_t>(C) & 15) == 0);
-    const uint32_t acc_empty_leader0 = mapa_shared(smem_u32(&bars->acc_empty[0]), 0);
+    const uint32_t acc_empty_leader = mapa_shared(smem_u32(&bars->acc_empty), 0);
     int i = 0;
     for (int t = cluster_id; t < ntiles; t += nclusters, ++i) {
-      const int ab = i & 1;
-      const uint32_t aph = (i >> 1) & 1;
-      const bool acc_ok = mbar_wait_cluster(smem_u32(&bars->acc_full[ab]), aph, abort_flag, kWaitLimitNs);
+      const bool acc_ok = mbar_wait_cluster(smem_u32(&bars->acc_full), i & 1, abort_flag, kWaitLimitNs);
       tc_fence_after();
       // tcgen05.ld is warp-collective: decide for the whole warp.
       const bool go = __all_sync(0xffffffffu, acc_ok && !*abort_flag);
@@ -378,14 +391,21 @@ mixfp4_gemm_kernel(const __grid_constant__ CUtensorMap tm_ac, const __grid_const
       }
       const int mt = t % mtiles, nt = t / mtiles;
       const int r = mt * TILE_M + (int)rank * BM + q * 32 + lane;
-      const int n0 = nt * TILE_N;
-      const uint32_t tbase = tmem_base + (uint32_t)ab * kAccCols + ((uint32_t)(q * 32) << 16);
+      const int n0 = nt * TILE_N + chalf * (TILE_N / 2);
+      const uint32_t tbase = tmem_base + (uint32_t)(chalf * (TILE_N / 2)) + ((uint32_t)(q * 32) << 16);
 #pragma unroll 1
-      for (int col = 0; col < TILE_N; col += 32) {
+      for (int cc = 0; cc < 4; ++cc) {
         uint32_t v[32];
-        tmem_ld_32x32b_x32(tbase + (uint32_t)col, v);
+        tmem_ld_32x32b_x32(tbase + (uint32_t)(cc * 32), v);
         tmem_ld_wait();
+        if (cc == 3) {
+          // The accumulator is free once its last chunk sits in registers.
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive_cluster(acc_empty_leader);
+        }
         if (r < M) {
+          const int col = cc * 32;
           float* crow = C + (long long)r * ldc + n0 + col;
           float o[32];
 #pragma unroll
@@ -400,9 +420,6 @@ mixfp4_gemm_kernel(const __grid_constant__ CUtensorMap tm_ac, const __grid_const
           }
         }
       }
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive_cluster(acc_empty_leader0 + ab * 8);
     }
   }
 
