@@ -15,7 +15,9 @@
 //   warp 0        TMA producer: codes [rows][128 B] (128-byte swizzle) and
 //                 scales [rows][16 B] of a 256-wide K slice into a 2-deep ring;
 //   warp 1        TMEM allocator (both CTAs); in the leader CTA also the single
-//                 MMA-issuing thread;
+//                 MMA-issuing thread; in the peer CTA one thread that forwards
+//                 "stage decoded" to the leader as a single remote arrival (16
+//                 remote arrivals on one barrier word serialise across SMs);
 //   warps 2-9     A decoders, two threads per A row (lane quarter = warp % 4),
 //                 64 K of the row per stage -> f16 pairs in TMEM columns;
 //   warps 10-17   B decoders, two threads per B row, 64 K of the row per stage
@@ -91,7 +93,8 @@ constexpr uint64_t kWaitLimitNs = 1000000000ull;  // 1 s per pipeline wait
 struct Bars {
   uint64_t code_full[kCodeStages];
   uint64_t code_empty[kCodeStages];
-  uint64_t dec_full[kDecStages];    // leader: 2 x kDecodeWarps arrivals
+  uint64_t dec_full[kDecStages];    // leader: its kDecodeWarps + 1 forwarded peer arrival
+  uint64_t peer_ready[kDecStages];  // peer: its kDecodeWarps arrivals, forwarded as one
   uint64_t dec_empty[kDecStages];   // MMA commit (multicast to both CTAs)
   uint64_t acc_full;                // MMA commit (multicast)
   uint64_t acc_empty;               // leader: 2 x kEpiWarps arrivals
@@ -189,7 +192,8 @@ mixfp4_gemm_kernel(const __grid_constant__ CUtensorMap tm_ac, const __grid_const
       mbar_init(smem_u32(&bars->code_empty[s]), kDecodeWarps);
     }
     for (int s = 0; s < kDecStages; ++s) {
-      mbar_init(smem_u32(&bars->dec_full[s]), 2 * kDecodeWarps);
+      mbar_init(smem_u32(&bars->dec_full[s]), kDecodeWarps + 1);
+      mbar_init(smem_u32(&bars->peer_ready[s]), kDecodeWarps);
       mbar_init(smem_u32(&bars->dec_empty[s]), 1);
     }
     mbar_init(smem_u32(&bars->acc_full), 1);
@@ -291,6 +295,23 @@ mixfp4_gemm_kernel(const __grid_constant__ CUtensorMap tm_ac, const __grid_const
       // for it (ignoring the abort flag) so TMEM is never freed under an MMA.
       mma_commit_pair(smem_u32(&bars->drain), 1);
       if (!mbar_wait_cluster(smem_u32(&bars->drain), 0, nullptr, kWaitLimitNs)) fail(8u);
+    } else if (!leader && lane == 0) {
+      // ---------------- forwarder (peer CTA) ----------------
+      const uint32_t dec_full_leader0 = mapa_shared(smem_u32(&bars->dec_full[0]), 0);
+      int d = 0;
+      uint32_t dph = 0;
+      bool ok = true;
+      for (int t = cluster_id; t < ntiles && ok; t += nclusters) {
+        for (int st = 0; st < num_kc * kSub; ++st) {
+          if (!mbar_wait(smem_u32(&bars->peer_ready[d]), dph, abort_flag, kWaitLimitNs)) {
+            fail(128u);
+            ok = false;
+            break;
+          }
+          mbar_arrive_cluster(dec_full_leader0 + d * 8);
+          if (++d == kDecStages) { d = 0; dph ^= 1; }
+        }
+      }
     }
   } else if (warp < kFirstEpi) {
     // ---------------- decoders ----------------
@@ -304,7 +325,6 @@ mixfp4_gemm_kernel(const __grid_constant__ CUtensorMap tm_ac, const __grid_const
     const uint32_t b_off = OFF_DEC + (rl >> 3) * kSBO + (rl & 7) * 16;
     const uint32_t a_lane = (uint32_t)((warp & 3) * 32) << 16;
     const uint32_t swz = rl & 7;
-    const uint32_t dec_full_leader0 = mapa_shared(smem_u32(&bars->dec_full[0]), 0);
     int d = 0;
     uint32_t dph = 0;
     int it = 0;
@@ -357,10 +377,7 @@ mixfp4_gemm_kernel(const __grid_constant__ CUtensorMap tm_ac, const __grid_const
             fence_proxy_async_smem();
           }
           __syncwarp();
-          if (lane == 0) {
-            if (leader) mbar_arrive(smem_u32(&bars->dec_full[d]));
-            else mbar_arrive_cluster(dec_full_leader0 + d * 8);
-          }
+          if (lane == 0) mbar_arrive(smem_u32(leader ? &bars->dec_full[d] : &bars->peer_ready[d]));
           if (++d == kDecStages) { d = 0; dph ^= 1; }
           if (sub == kSub - 1) {
             // Release the code stage only now: every value loaded from it has
