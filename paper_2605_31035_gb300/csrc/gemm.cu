@@ -448,6 +448,303 @@ mixfp4_gemm_kernel(const __grid_constant__ CUtensorMap tm_ac, const __grid_const
   }
 }
 
+// ============================================================================
+// Skinny-M path (M <= 64 activation rows, e.g. decoding): the roles of the
+// operands are swapped so the weight rows fill the 128-row MMA dimension and
+// every weight element is decoded exactly once:
+//   D^T[n][m] = sum_k W[n][k] X[m][k],  M_mma = 128 weight rows (A operand,
+//   decoded into TMEM), N_mma = X rows rounded up to 16 (B operand, decoded
+//   into shared memory), cta_group::1.
+// Work = (weight tile, 256-wide K slice) units, split evenly over all CTAs
+// (stream-K), so no SM idles; each CTA adds its partial tiles into C with
+// red.global.add (C is zeroed first), so bits depend on the summation order
+// but every result is within the fp32-accumulation bound.
+// Per CTA: warp 0 TMA, warp 1 TMEM allocator + MMA thread, warps 2-17 weight
+// decoders (four threads per row, lane quarter = warp % 4), warps 18-21 X
+// decoders (two threads per row), warps 22-25 epilogue.
+// ============================================================================
+namespace skinny {
+
+constexpr int BW = 128;                        // weight rows per tile (MMA M)
+constexpr int MXMAX = 64;                      // max activation rows (MMA N)
+constexpr int BKC = 256, BKD = 128, kSub = BKC / BKD;
+constexpr int kCodeStages = 4, kDecStages = 4;
+constexpr int kTPRW = 4, kTPRX = 2;
+constexpr int kWarpsW = kTPRW * BW / 32;       // 16
+constexpr int kWarpsX = kTPRX * MXMAX / 32;    // 4
+constexpr int kFirstW = 2, kFirstX = kFirstW + kWarpsW, kFirstEpi = kFirstX + kWarpsX;  // 2, 18, 22
+constexpr int kEpiWarps = 4;
+constexpr int kThreads = 32 * (kFirstEpi + kEpiWarps);  // 832
+static_assert(kFirstW % 4 == 2, "weight decoders start at lane quarter 2");
+constexpr int W_CODE = BW * BKC / 2, X_CODE = MXMAX * BKC / 2;
+constexpr int W_SCALE = BW * BKC / 16, X_SCALE = MXMAX * BKC / 16;
+constexpr int OFF_XC = W_CODE, OFF_WS = OFF_XC + X_CODE, OFF_XS = OFF_WS + W_SCALE;
+constexpr int CODE_STAGE = OFF_XS + X_SCALE;
+constexpr int X_DEC = MXMAX * BKD * 2;
+constexpr int OFF_DEC = kCodeStages * CODE_STAGE;
+constexpr int OFF_BAR = OFF_DEC + kDecStages * X_DEC;
+constexpr int SMEM_ALLOC = OFF_BAR + 256 + 1024;
+static_assert(CODE_STAGE % 1024 == 0 && OFF_XC % 1024 == 0, "swizzled TMA tiles need 1024-byte alignment");
+static_assert(SMEM_ALLOC <= 232448, "shared memory budget");
+constexpr uint32_t kAccCols = MXMAX;            // accumulator columns (N_mma <= 64)
+constexpr uint32_t kWStageCols = BKD / 2;
+constexpr uint32_t kTmemCols = 512;
+static_assert(kAccCols + kDecStages * kWStageCols <= kTmemCols, "TMEM budget");
+constexpr uint32_t kLBO = 128, kSBO = (BKD / 8) * 128;
+
+struct Bars {
+  uint64_t code_full[kCodeStages];
+  uint64_t code_empty[kCodeStages];
+  uint64_t dec_full[kDecStages];
+  uint64_t dec_empty[kDecStages];
+  uint64_t acc_full;
+  uint64_t acc_empty;
+  uint64_t drain;
+  uint32_t tmem_base;
+  int abort;
+};
+static_assert(sizeof(Bars) <= 256, "barrier block");
+
+__global__ void __launch_bounds__(kThreads, 1)
+mixfp4_gemm_skinny_kernel(const __grid_constant__ CUtensorMap tm_wc, const __grid_constant__ CUtensorMap tm_xc,
+                          const __grid_constant__ CUtensorMap tm_ws, const __grid_constant__ CUtensorMap tm_xs,
+                          const float* __restrict__ a_ts, const float* __restrict__ b_ts, int Mx, int N, int K,
+                          float* __restrict__ C, long long ldc, uint32_t idesc, uint32_t* status_word) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  Bars* bars = reinterpret_cast<Bars*>(smem + OFF_BAR);
+  volatile int* abort_flag = &bars->abort;
+  const uint32_t sbase = smem_u32(smem);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int num_kc = K / BKC;
+  const int nmma = (Mx + 15) & ~15;
+  const long long units = (long long)((N + BW - 1) / BW) * num_kc;
+  const long long u_begin = units * blockIdx.x / gridDim.x, u_end = units * (blockIdx.x + 1) / gridDim.x;
+  const uint32_t stage_bytes = W_CODE + W_SCALE + (uint32_t)nmma * (BKC / 2 + BKC / 16);
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kCodeStages; ++s) {
+      mbar_init(smem_u32(&bars->code_full[s]), 1);
+      mbar_init(smem_u32(&bars->code_empty[s]), kWarpsW + kWarpsX);
+    }
+    for (int s = 0; s < kDecStages; ++s) {
+      mbar_init(smem_u32(&bars->dec_full[s]), kWarpsW + kWarpsX);
+      mbar_init(smem_u32(&bars->dec_empty[s]), 1);
+    }
+    mbar_init(smem_u32(&bars->acc_full), 1);
+    mbar_init(smem_u32(&bars->acc_empty), kEpiWarps);
+    mbar_init(smem_u32(&bars->drain), 1);
+    bars->abort = 0;
+    fence_mbar_init();
+  }
+  if (warp == 1) {
+    tmem_alloc(smem_u32(&bars->tmem_base), kTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = bars->tmem_base;
+  const uint32_t tmem_w0 = tmem_base + kAccCols;
+
+  auto fail = [&](uint32_t code) {
+    *abort_flag = 1;
+    if (status_word) atomicOr(status_word, code);
+  };
+
+  if (warp == 0) {
+    // ---------------- TMA producer ----------------
+    if (lane == 0) {
+      tma_prefetch(&tm_wc);
+      tma_prefetch(&tm_xc);
+      tma_prefetch(&tm_ws);
+      tma_prefetch(&tm_xs);
+      int it = 0;
+      long long last = -1;
+      for (long long u = u_begin; u < u_end; ++u, ++it) {
+        const int s = it % kCodeStages;
+        const uint32_t ph = (it / kCodeStages) & 1;
+        if (!mbar_wait(smem_u32(&bars->code_empty[s]), ph ^ 1, abort_flag, kWaitLimitNs)) {
+          fail(1u);
+          break;
+        }
+        const int wt = (int)(u / num_kc), kc = (int)(u % num_kc);
+        const uint32_t st = sbase + s * CODE_STAGE;
+        const uint32_t fb = smem_u32(&bars->code_full[s]);
+        mbar_arrive_expect_tx(fb, stage_bytes);
+        const int xk = kc * (BKC / 2), xs = kc * (BKC / 16);
+        tma_load_2d(st, &tm_wc, xk, wt * BW, fb);
+        tma_load_2d(st + OFF_XC, &tm_xc, xk, 0, fb);
+        tma_load_2d(st + OFF_WS, &tm_ws, xs, wt * BW, fb);
+        tma_load_2d(st + OFF_XS, &tm_xs, xs, 0, fb);
+        last = it;
+      }
+      if (*abort_flag)
+        for (long long v = last - kCodeStages + 1; v <= last; ++v)
+          if (v >= 0)
+            mbar_wait(smem_u32(&bars->code_full[v % kCodeStages]), (uint32_t)((v / kCodeStages) & 1), nullptr,
+                      kWaitLimitNs);
+    }
+  } else if (warp == 1) {
+    // ---------------- MMA issuer ----------------
+    if (lane == 0) {
+      int d = 0, ntile = 0;
+      uint32_t dph = 0;
+      bool ok = true;
+      for (long long u = u_begin; u < u_end && ok;) {
+        const int wt = (int)(u / num_kc);
+        const long long run_end = (long long)(wt + 1) * num_kc < u_end ? (long long)(wt + 1) * num_kc : u_end;
+        if (!mbar_wait(smem_u32(&bars->acc_empty), (ntile & 1) ^ 1, abort_flag, kWaitLimitNs)) {
+          fail(2u);
+          break;
+        }
+        tc_fence_after();
+        bool first = true;
+        for (; u < run_end && ok; ++u) {
+          for (int sub = 0; sub < kSub; ++sub) {
+            if (!mbar_wait(smem_u32(&bars->dec_full[d]), dph, abort_flag, kWaitLimitNs)) {
+              fail(4u);
+              ok = false;
+              break;
+            }
+            tc_fence_after();
+            const uint32_t xb = sbase + OFF_DEC + d * X_DEC;
+            const uint32_t wa = tmem_w0 + (uint32_t)d * kWStageCols;
+#pragma unroll
+            for (int j = 0; j < BKD / 16; ++j) {
+              mma_f16_tmem_a(tmem_base, wa + j * 8, smem_desc_noswizzle(xb + j * 256, kLBO, kSBO), idesc,
+                             first ? 0u : 1u);
+              first = false;
+            }
+            mma_commit(smem_u32(&bars->dec_empty[d]));
+            if (++d == kDecStages) { d = 0; dph ^= 1; }
+          }
+        }
+        if (ok) mma_commit(smem_u32(&bars->acc_full));
+        ++ntile;
+      }
+      mma_commit(smem_u32(&bars->drain));
+      if (!mbar_wait(smem_u32(&bars->drain), 0, nullptr, kWaitLimitNs)) fail(8u);
+    }
+  } else if (warp < kFirstEpi) {
+    // ---------------- decoders ----------------
+    const bool is_w = warp < kFirstX;
+    const int dw = warp - (is_w ? kFirstW : kFirstX);
+    const int tpr = is_w ? kTPRW : kTPRX;
+    // weight decoders: rows by TMEM lane quarter (warp % 4), four parts per row;
+    // X decoders: 64 rows x two parts.
+    const int part = is_w ? (dw >> 2) : (dw >> 1);   // share of a stage's four 32-code chunks
+    const int rl = is_w ? ((warp & 3) * 32 + lane) : ((dw & 1) * 32 + lane);
+    const bool active = is_w || (dw & 1) * 32 < nmma;  // X decoders past the padded rows idle
+    const int cpt = 4 / tpr;                         // chunks per thread per stage
+    const uint32_t code_off = (is_w ? 0 : OFF_XC) + rl * (BKC / 2);
+    const uint32_t scale_off = (is_w ? OFF_WS : OFF_XS) + rl * (BKC / 16);
+    const uint32_t x_off = OFF_DEC + (rl >> 3) * kSBO + (rl & 7) * 16;
+    const uint32_t w_lane = (uint32_t)((warp & 3) * 32) << 16;
+    const uint32_t swz = rl & 7;
+    int d = 0, it = 0;
+    uint32_t dph = 0;
+    for (long long u = u_begin; u < u_end; ++u, ++it) {
+      const int s = it % kCodeStages;
+      const uint32_t ph = (it / kCodeStages) & 1;
+      if (!mbar_wait(smem_u32(&bars->code_full[s]), ph, abort_flag, kWaitLimitNs)) {
+        fail(16u);
+        break;
+      }
+      const uint32_t st = sbase + s * CODE_STAGE;
+      uint4 sc = make_uint4(0, 0, 0, 0);
+      if (active) sc = lds128(st + scale_off);
+      bool ok = true;
+#pragma unroll
+      for (int sub = 0; sub < kSub; ++sub) {
+        uint4 c[2];
+        if (active) {
+#pragma unroll
+          for (int j = 0; j < 2; ++j)
+            if (j < cpt) c[j] = lds128(st + code_off + ((uint32_t)((sub * 4 + part * cpt + j) ^ swz) << 4));
+        }
+        if (!mbar_wait(smem_u32(&bars->dec_empty[d]), dph ^ 1, abort_flag, kWaitLimitNs)) {
+          fail(32u);
+          ok = false;
+          break;
+        }
+        if (is_w) {
+          uint32_t o[16];
+          const int chunk = sub * 4 + part;  // one chunk per thread
+          decode_chunk(c[0], scale_pair(sc, chunk), o);
+          tmem_st_32x32b_x16(tmem_w0 + w_lane + (uint32_t)d * kWStageCols + (uint32_t)part * 16u, o);
+          tmem_st_wait();
+          tc_fence_before();
+        } else if (active) {
+          const uint32_t dst = sbase + x_off + d * X_DEC;
+#pragma unroll
+          for (int j = 0; j < 2; ++j) {
+            const int chunk = sub * 4 + part * 2 + j;
+            uint32_t o[16];
+            decode_chunk(c[j], scale_pair(sc, chunk), o);
+            const int kc0 = (part * 2 + j) * 4;
+#pragma unroll
+            for (int q = 0; q < 4; ++q)
+              sts128(dst + (kc0 + q) * kLBO, o[4 * q], o[4 * q + 1], o[4 * q + 2], o[4 * q + 3]);
+          }
+          fence_proxy_async_smem();
+        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(smem_u32(&bars->dec_full[d]));
+        if (++d == kDecStages) { d = 0; dph ^= 1; }
+        if (sub == kSub - 1) {
+          __syncwarp();
+          if (lane == 0) mbar_arrive(smem_u32(&bars->code_empty[s]));
+        }
+      }
+      if (!ok) break;
+    }
+  } else {
+    // ---------------- epilogue: D^T (lane = weight row) -> red.add into C ----------------
+    const int q = warp & 3;
+    const float sa = 0.25f * __ldg(a_ts), sb = __ldg(b_ts);
+    int ntile = 0;
+    for (long long u = u_begin; u < u_end; ++ntile) {
+      const int wt = (int)(u / num_kc);
+      u = (long long)(wt + 1) * num_kc < u_end ? (long long)(wt + 1) * num_kc : u_end;
+      const bool acc_ok = mbar_wait(smem_u32(&bars->acc_full), ntile & 1, abort_flag, kWaitLimitNs);
+      tc_fence_after();
+      const bool go = __all_sync(0xffffffffu, acc_ok && !*abort_flag);
+      if (!go) {
+        if (!acc_ok && !*abort_flag) fail(64u);
+        break;
+      }
+      const int n = wt * BW + q * 32 + lane;
+      const uint32_t tb = tmem_base + ((uint32_t)(q * 32) << 16);
+      uint32_t v[2][32];
+      tmem_ld_32x32b_x32(tb, v[0]);
+      if (nmma > 32) tmem_ld_32x32b_x32(tb + 32, v[1]);
+      tmem_ld_wait();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(smem_u32(&bars->acc_empty));
+      if (n < N) {
+#pragma unroll
+        for (int m = 0; m < MXMAX; ++m) {
+          if (m < Mx) {
+            const float val = __fmul_rn(__fmul_rn(__uint_as_float(v[m >> 5][m & 31]), sa), sb);
+            atomicAdd(C + (long long)m * ldc + n, val);
+          }
+        }
+      }
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem_base, kTmemCols);
+  }
+}
+
+}  // namespace skinny
+
 PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
   static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
   if (!fn) {
@@ -493,6 +790,33 @@ int launch_gemm(const uint8_t* a_codes, const uint8_t* a_scales, const float* a_
                 int64_t N, int64_t K, float* C, int64_t ldc, uint32_t* status_word,
                 cudaStream_t stream) {
   if (M > (1 << 30) || N > (1 << 30) || K > (1 << 30)) return MIXFP4_ERR_SHAPE;
+  if (M <= skinny::MXMAX && N >= 4 * skinny::BW) {
+    // Few activation rows: weight rows on the MMA M dimension, stream-K over all SMs.
+    const int nmma = (int)((M + 15) & ~15);
+    CUtensorMap twc, txc, tws, txs;
+    if (!make_map(&twc, b_codes, (uint64_t)K / 2, (uint64_t)N, BKC / 2, skinny::BW, CU_TENSOR_MAP_SWIZZLE_128B) ||
+        !make_map(&txc, a_codes, (uint64_t)K / 2, (uint64_t)M, BKC / 2, nmma, CU_TENSOR_MAP_SWIZZLE_128B) ||
+        !make_map(&tws, b_scales, (uint64_t)K / 16, (uint64_t)N, BKC / 16, skinny::BW, CU_TENSOR_MAP_SWIZZLE_NONE) ||
+        !make_map(&txs, a_scales, (uint64_t)K / 16, (uint64_t)M, BKC / 16, nmma, CU_TENSOR_MAP_SWIZZLE_NONE))
+      return MIXFP4_ERR_CUDA;
+    static bool skinny_attr = false;
+    if (!skinny_attr) {
+      if (cudaFuncSetAttribute(skinny::mixfp4_gemm_skinny_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                               skinny::SMEM_ALLOC) != cudaSuccess)
+        return MIXFP4_ERR_CUDA;
+      skinny_attr = true;
+    }
+    if (cudaMemset2DAsync(C, (size_t)ldc * sizeof(float), 0, (size_t)N * sizeof(float), (size_t)M, stream) !=
+        cudaSuccess)
+      return MIXFP4_ERR_CUDA;
+    const int64_t units = ((N + skinny::BW - 1) / skinny::BW) * (K / BKC);
+    int64_t grid = num_sms();
+    if (grid > units) grid = units;
+    skinny::mixfp4_gemm_skinny_kernel<<<(unsigned)grid, skinny::kThreads, skinny::SMEM_ALLOC, stream>>>(
+        twc, txc, tws, txs, a_ts, b_ts, (int)M, (int)N, (int)K, C, (long long)ldc,
+        idesc_f16_f32(skinny::BW, nmma), status_word);
+    return MIXFP4_OK;
+  }
   CUtensorMap tac, tbc, tas, tbs;
   if (!make_map(&tac, a_codes, (uint64_t)K / 2, (uint64_t)M, BKC / 2, BM, CU_TENSOR_MAP_SWIZZLE_128B) ||
       !make_map(&tbc, b_codes, (uint64_t)K / 2, (uint64_t)N, BKC / 2, BNH, CU_TENSOR_MAP_SWIZZLE_128B) ||

@@ -60,10 +60,12 @@ def test_tiny_linear(oracle, mode):
 
 
 @pytest.mark.parametrize("M,N,K", [(200, 300, 512), (1, 1, 256), (129, 257, 768), (64, 520, 1280),
-                                   (300, 16, 256)])
+                                   (300, 16, 256), (1, 600, 512), (17, 1024, 768), (48, 700, 256),
+                                   (64, 2048, 4096), (65, 512, 512)])
 def test_ragged_tiles(oracle, M, N, K):
-    """M and N tails (TMA zero fill, masked stores), one code stage, and odd
-    numbers of code stages (ring wrap)."""
+    """M and N tails (TMA zero fill, masked stores), one code stage, odd
+    numbers of code stages (ring wrap), and the few-row (M <= 64) path with its
+    split of weight tiles and K slices across CTAs."""
     x = synth.activations(M, K, 7000 + M, 7100 + M)
     w = synth.weights(N, K, 7200 + N, 0.02, 0.5)
     full_check(oracle, x, w)
