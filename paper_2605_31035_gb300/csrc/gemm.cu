@@ -9,9 +9,13 @@
 //
 // Work decomposition: persistent CTA pairs (clusters of 2, cta_group::2).  A
 // pair owns 256 x 256 output tiles; each CTA holds 128 rows of A and 128 rows
-// (half) of B.  Decoded A never touches shared memory: it is written to tensor
-// memory (tcgen05.st) and the MMA reads it from there; decoded B goes through
-// shared memory.  Per CTA:
+// (half) of B.  Tiles of the full waves are dealt whole; when the tile count
+// leaves a partial last wave, that wave's (tile, K slice) units are split
+// evenly over all pairs (stream-K) and their partial sums are added into C
+// with red.global.add after the host zeroed those tiles.  Tiles are numbered
+// row band by row band (t = mt * ntiles_n + nt).  Decoded A never touches
+// shared memory: it is written to tensor memory (tcgen05.st) and the MMA reads
+// it from there; decoded B goes through shared memory.  Per CTA:
 //   warp 0        TMA producer: codes [rows][128 B] (128-byte swizzle) and
 //                 scales [rows][16 B] of a 256-wide K slice into a 2-deep ring;
 //   warp 1        TMEM allocator (both CTAs); in the leader CTA also the single
@@ -22,7 +26,8 @@
 //                 64 K of the row per stage -> f16 pairs in TMEM columns;
 //   warps 10-17   B decoders, two threads per B row, 64 K of the row per stage
 //                 -> f16 in the canonical K-major no-swizzle UMMA layout;
-//   warps 18-25   epilogue: tcgen05.ld -> x s32A s32B / 4 -> fp32 C.
+//   warps 18-25   epilogue: tcgen05.ld -> x s32A s32B / 4 -> a per-warp shared
+//                 staging tile -> coalesced fp32 stores (or red.add) to C.
 // TMEM per CTA (512 columns): fp32 accumulator 128 lanes x 256 columns, then
 // kDecStages A stages of 64 columns (128 K of f16 pairs).  The leader's MMA
 // waits for both CTAs' decoders (remote mbarrier arrivals).
@@ -75,7 +80,10 @@ constexpr int B_SCALE_BYTES = BNH * BKC / 16;
 constexpr int CODE_STAGE_BYTES = A_CODE_BYTES + B_CODE_BYTES + A_SCALE_BYTES + B_SCALE_BYTES;
 constexpr int B_DEC_BYTES = BNH * BKD * 2;
 constexpr int OFF_DEC = kCodeStages * CODE_STAGE_BYTES;
-constexpr int OFF_BAR = OFF_DEC + kDecStages * B_DEC_BYTES;
+constexpr int EPI_CHUNK = 16;                  // accumulator columns per epilogue step
+constexpr int EPI_BYTES = 32 * EPI_CHUNK * 4;   // one warp's 32 rows x 16 fp32 staging tile
+constexpr int OFF_EPI = OFF_DEC + kDecStages * B_DEC_BYTES;
+constexpr int OFF_BAR = OFF_EPI + kEpiWarps * EPI_BYTES;
 constexpr int SMEM_BYTES = OFF_BAR + 256;
 constexpr int SMEM_ALLOC = SMEM_BYTES + 1024;  // slack to align the base to 1024 B
 
@@ -89,6 +97,7 @@ constexpr uint32_t kSBO = (BKD / 8) * 128;      // next 8 rows
 constexpr uint32_t kIdesc = idesc_f16_f32(TILE_M, TILE_N);
 
 constexpr uint64_t kWaitLimitNs = 1000000000ull;  // 1 s per pipeline wait
+constexpr int kMinStreamKGainSlices = 8;           // stream-K must save this many K slices per pair
 
 struct Bars {
   uint64_t code_full[kCodeStages];
@@ -167,11 +176,51 @@ __device__ __forceinline__ uint32_t scale_pair(const uint4& sc, int chunk) {
   return (s4 >> (16 * (chunk & 1))) & 0xFFFFu;
 }
 
+__device__ __forceinline__ void red_add_v4(float* p, float a, float b, float c, float d) {
+  asm volatile("red.global.add.v4.f32 [%0], {%1,%2,%3,%4};" :: "l"(p), "f"(a), "f"(b), "f"(c), "f"(d)
+               : "memory");
+}
+
+// Work schedule of one CTA pair, walked identically by every role.  Tiles
+// below dp_tiles are whole-tile work, dealt round-robin (tile = cluster,
+// cluster + nclusters, ...).  The (tile, 256-wide K slice) units of the
+// remaining tiles are split evenly over all pairs (stream-K) and cut into
+// segments at tile edges; a segment that is not a whole tile is added into C
+// (which the host zeroed over those tiles).
+struct Sched {
+  int t, dp_tiles, nclusters, num_kc;
+  long long u, u_end;
+  __device__ Sched(int cluster, int ncl, int dp, int ntiles, int nkc)
+      : t(cluster), dp_tiles(dp), nclusters(ncl), num_kc(nkc) {
+    const long long sk_units = (long long)(ntiles - dp) * nkc;
+    u = sk_units * cluster / ncl;
+    u_end = sk_units * (cluster + 1) / ncl;
+  }
+  // Next segment: tile, K slices [k0, k1).  False when the pair is done.
+  __device__ bool next(int& tile, int& k0, int& k1) {
+    if (t < dp_tiles) {
+      tile = t;
+      k0 = 0;
+      k1 = num_kc;
+      t += nclusters;
+      return true;
+    }
+    if (u >= u_end) return false;
+    const long long tt = u / num_kc;
+    const long long end = (tt + 1) * num_kc < u_end ? (tt + 1) * num_kc : u_end;
+    tile = dp_tiles + (int)tt;
+    k0 = (int)(u - tt * num_kc);
+    k1 = k0 + (int)(end - u);
+    u = end;
+    return true;
+  }
+};
+
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
 mixfp4_gemm_kernel(const __grid_constant__ CUtensorMap tm_ac, const __grid_constant__ CUtensorMap tm_bc,
                    const __grid_constant__ CUtensorMap tm_as, const __grid_constant__ CUtensorMap tm_bs,
                    const float* __restrict__ a_ts, const float* __restrict__ b_ts,
-                   int M, int N, int K, float* __restrict__ C, long long ldc,
+                   int M, int N, int K, float* __restrict__ C, long long ldc, int dp_tiles,
                    uint32_t* status_word) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -227,10 +276,12 @@ mixfp4_gemm_kernel(const __grid_constant__ CUtensorMap tm_ac, const __grid_const
       int last_it = -1;  // last code-stage use issued (its copies may be in flight)
       int it = 0;
       bool ok = true;
-      for (int t = cluster_id; t < ntiles && ok; t += nclusters) {
-        const int mt = t % mtiles, nt = t / mtiles;
+      Sched sched(cluster_id, nclusters, dp_tiles, ntiles, num_kc);
+      int t, k0, k1;
+      while (ok && sched.next(t, k0, k1)) {
+        const int mt = t / ntiles_n, nt = t % ntiles_n;
         const int ma = mt * TILE_M + (int)rank * BM, nb = nt * TILE_N + (int)rank * BNH;
-        for (int kc = 0; kc < num_kc; ++kc, ++it) {
+        for (int kc = k0; kc < k1; ++kc, ++it) {
           const int s = it % kCodeStages;
           const uint32_t ph = (it / kCodeStages) & 1;
           if (!mbar_wait(smem_u32(&bars->code_empty[s]), ph ^ 1, abort_flag, kWaitLimitNs)) {
@@ -263,14 +314,15 @@ mixfp4_gemm_kernel(const __grid_constant__ CUtensorMap tm_ac, const __grid_const
       int d = 0;
       uint32_t dph = 0;
       bool ok = true;
-      int i = 0;
-      for (int t = cluster_id; t < ntiles && ok; t += nclusters, ++i) {
+      Sched sched(cluster_id, nclusters, dp_tiles, ntiles, num_kc);
+      int t, k0, k1;
+      for (int i = 0; ok && sched.next(t, k0, k1); ++i) {
         if (!mbar_wait_cluster(smem_u32(&bars->acc_empty), (i & 1) ^ 1, abort_flag, kWaitLimitNs)) {
           fail(2u);
           break;
         }
         tc_fence_after();
-        for (int kc = 0; kc < num_kc && ok; ++kc) {
+        for (int kc = k0; kc < k1 && ok; ++kc) {
           for (int sub = 0; sub < kSub; ++sub) {
             if (!mbar_wait_cluster(smem_u32(&bars->dec_full[d]), dph, abort_flag, kWaitLimitNs)) {
               fail(4u);
@@ -283,7 +335,7 @@ mixfp4_gemm_kernel(const __grid_constant__ CUtensorMap tm_ac, const __grid_const
 #pragma unroll
             for (int j = 0; j < BKD / 16; ++j) {
               const uint64_t bd = smem_desc_noswizzle(bbase + j * 256, kLBO, kSBO);
-              mma_f16_pair_tmem_a(tmem_base, abase + j * 8, bd, kIdesc, (kc | sub | j) != 0 ? 1u : 0u);
+              mma_f16_pair_tmem_a(tmem_base, abase + j * 8, bd, kIdesc, ((kc - k0) | sub | j) != 0 ? 1u : 0u);
             }
             mma_commit_pair(smem_u32(&bars->dec_empty[d]), 3);
             if (++d == kDecStages) { d = 0; dph ^= 1; }
@@ -301,8 +353,10 @@ mixfp4_gemm_kernel(const __grid_constant__ CUtensorMap tm_ac, const __grid_const
       int d = 0;
       uint32_t dph = 0;
       bool ok = true;
-      for (int t = cluster_id; t < ntiles && ok; t += nclusters) {
-        for (int st = 0; st < num_kc * kSub; ++st) {
+      Sched sched(cluster_id, nclusters, dp_tiles, ntiles, num_kc);
+      int t, k0, k1;
+      while (ok && sched.next(t, k0, k1)) {
+        for (int st = 0; st < (k1 - k0) * kSub; ++st) {
           if (!mbar_wait(smem_u32(&bars->peer_ready[d]), dph, abort_flag, kWaitLimitNs)) {
             fail(128u);
             ok = false;
@@ -329,8 +383,10 @@ mixfp4_gemm_kernel(const __grid_constant__ CUtensorMap tm_ac, const __grid_const
     uint32_t dph = 0;
     int it = 0;
     bool ok = true;
-    for (int t = cluster_id; t < ntiles && ok; t += nclusters) {
-      for (int kc = 0; kc < num_kc && ok; ++kc, ++it) {
+    Sched sched(cluster_id, nclusters, dp_tiles, ntiles, num_kc);
+    int t, k0, k1;
+    while (ok && sched.next(t, k0, k1)) {
+      for (int kc = k0; kc < k1 && ok; ++kc, ++it) {
         const int s = it % kCodeStages;
         const uint32_t ph = (it / kCodeStages) & 1;
         if (!mbar_wait(smem_u32(&bars->code_full[s]), ph, abort_flag, kWaitLimitNs)) {
@@ -391,13 +447,22 @@ mixfp4_gemm_kernel(const __grid_constant__ CUtensorMap tm_ac, const __grid_const
     }
   } else {
     // ---------------- epilogue (two warps per TMEM lane quarter) ----------------
+    // Each warp drains 32 rows x 128 columns in 16-column steps: tcgen05.ld
+    // (lane = row) -> scale -> its shared staging tile (row-major, 16-byte
+    // chunks XOR-swizzled by row so writes and reads are conflict-free) ->
+    // read back four lanes per row, so every global store instruction writes
+    // 64 contiguous bytes in each of 8 rows.
     const int q = warp & 3;                  // TMEM lane quarter of this warp
     const int chalf = (warp - kFirstEpi) >> 2;  // column half
     const float sa = 0.25f * __ldg(a_ts), sb = __ldg(b_ts);
     const bool vec_ok = ((ldc & 3) == 0) && ((reinterpret_cast<uintptr_t>(C) & 15) == 0);
     const uint32_t acc_empty_leader = mapa_shared(smem_u32(&bars->acc_empty), 0);
-    int i = 0;
-    for (int t = cluster_id; t < ntiles; t += nclusters, ++i) {
+    const uint32_t stage = sbase + OFF_EPI + (uint32_t)(warp - kFirstEpi) * EPI_BYTES;
+    const uint32_t wr_row = stage + (uint32_t)lane * 64u, wr_swz = (uint32_t)(lane >> 1) & 3u;
+    Sched sched(cluster_id, nclusters, dp_tiles, ntiles, num_kc);
+    int t, k0, k1;
+    for (int i = 0; sched.next(t, k0, k1); ++i) {
+      const bool whole = k0 == 0 && k1 == num_kc;  // else: add into C (zeroed by the host)
       const bool acc_ok = mbar_wait_cluster(smem_u32(&bars->acc_full), i & 1, abort_flag, kWaitLimitNs);
       tc_fence_after();
       // tcgen05.ld is warp-collective: decide for the whole warp.
@@ -406,35 +471,51 @@ mixfp4_gemm_kernel(const __grid_constant__ CUtensorMap tm_ac, const __grid_const
         if (!acc_ok && !*abort_flag) fail(64u);
         break;
       }
-      const int mt = t % mtiles, nt = t / mtiles;
-      const int r = mt * TILE_M + (int)rank * BM + q * 32 + lane;
+      const int mt = t / ntiles_n, nt = t % ntiles_n;
+      const int row0 = mt * TILE_M + (int)rank * BM + q * 32;
       const int n0 = nt * TILE_N + chalf * (TILE_N / 2);
       const uint32_t tbase = tmem_base + (uint32_t)(chalf * (TILE_N / 2)) + ((uint32_t)(q * 32) << 16);
 #pragma unroll 1
-      for (int cc = 0; cc < 4; ++cc) {
-        uint32_t v[32];
-        tmem_ld_32x32b_x32(tbase + (uint32_t)(cc * 32), v);
-        tmem_ld_wait();
-        if (cc == 3) {
+      for (int cc = 0; cc < TILE_N / 2 / EPI_CHUNK; ++cc) {
+        uint32_t o[EPI_CHUNK];
+        tmem_ld_32x32b_x16(tbase + (uint32_t)(cc * EPI_CHUNK), o);
+        tmem_ld_wait_x16(o);
+        if (cc == TILE_N / 2 / EPI_CHUNK - 1) {
           // The accumulator is free once its last chunk sits in registers.
           tc_fence_before();
           __syncwarp();
           if (lane == 0) mbar_arrive_cluster(acc_empty_leader);
         }
-        if (r < M) {
-          const int col = cc * 32;
-          float* crow = C + (long long)r * ldc + n0 + col;
-          float o[32];
 #pragma unroll
-          for (int k = 0; k < 32; ++k) o[k] = __fmul_rn(__fmul_rn(__uint_as_float(v[k]), sa), sb);
-          if (vec_ok && n0 + col + 32 <= N) {
+        for (int k = 0; k < EPI_CHUNK; ++k) o[k] = __float_as_uint(__fmul_rn(__fmul_rn(__uint_as_float(o[k]), sa), sb));
+        const int col = n0 + cc * EPI_CHUNK;
+        if (vec_ok && col + EPI_CHUNK <= N) {
 #pragma unroll
-            for (int k = 0; k < 32; k += 4)
-              *reinterpret_cast<float4*>(crow + k) = make_float4(o[k], o[k + 1], o[k + 2], o[k + 3]);
-          } else {
-            for (int k = 0; k < 32; ++k)
-              if (n0 + col + k < N) crow[k] = o[k];
+          for (int j = 0; j < 4; ++j)
+            sts128(wr_row + (((uint32_t)j ^ wr_swz) << 4), o[4 * j], o[4 * j + 1], o[4 * j + 2], o[4 * j + 3]);
+          __syncwarp();
+          const int cq = lane & 3;
+#pragma unroll
+          for (int p = 0; p < 4; ++p) {
+            const int rr = (lane >> 2) + 8 * p;
+            const uint4 val = lds128(stage + (uint32_t)rr * 64u + (((uint32_t)cq ^ ((uint32_t)(rr >> 1) & 3u)) << 4));
+            if (row0 + rr < M) {
+              float* dst = C + (long long)(row0 + rr) * ldc + col + 4 * cq;
+              if (whole)
+                *reinterpret_cast<uint4*>(dst) = val;
+              else
+                red_add_v4(dst, __uint_as_float(val.x), __uint_as_float(val.y), __uint_as_float(val.z),
+                           __uint_as_float(val.w));
+            }
           }
+          __syncwarp();  // the staging tile is rewritten by the next step
+        } else if (row0 + lane < M) {
+          float* crow = C + (long long)(row0 + lane) * ldc + col;
+          for (int k = 0; k < EPI_CHUNK; ++k)
+            if (col + k < N) {
+              if (whole) crow[k] = __uint_as_float(o[k]);
+              else atomicAdd(crow + k, __uint_as_float(o[k]));
+            }
         }
       }
     }
@@ -719,7 +800,9 @@ mixfp4_gemm_skinny_kernel(const __grid_constant__ CUtensorMap tm_wc, const __gri
       uint32_t v[2][32];
       tmem_ld_32x32b_x32(tb, v[0]);
       if (nmma > 32) tmem_ld_32x32b_x32(tb + 32, v[1]);
-      tmem_ld_wait();
+      tmem_ld_wait_x32(v[0]);
+      reg_fence16(v[1]);
+      reg_fence16(v[1] + 16);
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(smem_u32(&bars->acc_empty));
@@ -830,11 +913,33 @@ int launch_gemm(const uint8_t* a_codes, const uint8_t* a_scales, const float* a_
       return MIXFP4_ERR_CUDA;
     attr_set = true;
   }
-  const int64_t tiles = ((M + TILE_M - 1) / TILE_M) * ((N + TILE_N - 1) / TILE_N);
+  const int64_t mtiles = (M + TILE_M - 1) / TILE_M, ntiles_n = (N + TILE_N - 1) / TILE_N;
+  const int64_t tiles = mtiles * ntiles_n, num_kc = K / BKC;
   int64_t clusters = num_sms() / 2;
   if (clusters > tiles) clusters = tiles;
+  // Whole tiles in full waves.  The last, partial wave's tiles are shared out
+  // as K slices (stream-K) when the idle time that removes, (clusters - rem)
+  // tiles' worth of K slices spread over all pairs, outweighs what stream-K
+  // adds: zeroing those rows of C and one more accumulator drain per pair.
+  int64_t dp_tiles = tiles;
+  const int64_t rem = tiles % clusters;
+  if (tiles > clusters && rem != 0 && (clusters - rem) * num_kc >= kMinStreamKGainSlices * clusters)
+    dp_tiles = tiles - rem;
+  if (dp_tiles < tiles) {
+    // Zero C from the first stream-K tile's row band down (tile t: mt = t / ntiles_n,
+    // nt = t % ntiles_n, so those rows hold every stream-K tile; whole tiles among
+    // them are overwritten by plain stores after this).
+    const int64_t r0 = (dp_tiles / ntiles_n) * TILE_M;
+    cudaError_t e;
+    if (ldc == N)
+      e = cudaMemsetAsync(C + r0 * ldc, 0, (size_t)(M - r0) * (size_t)N * sizeof(float), stream);
+    else
+      e = cudaMemset2DAsync(C + r0 * ldc, (size_t)ldc * sizeof(float), 0, (size_t)N * sizeof(float),
+                            (size_t)(M - r0), stream);
+    if (e != cudaSuccess) return MIXFP4_ERR_CUDA;
+  }
   mixfp4_gemm_kernel<<<(unsigned)(2 * clusters), kThreads, SMEM_ALLOC, stream>>>(
-      tac, tbc, tas, tbs, a_ts, b_ts, (int)M, (int)N, (int)K, C, (long long)ldc, status_word);
+      tac, tbc, tas, tbs, a_ts, b_ts, (int)M, (int)N, (int)K, C, (long long)ldc, (int)dp_tiles, status_word);
   return MIXFP4_OK;
 }
 

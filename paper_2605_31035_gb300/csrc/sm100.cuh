@@ -177,6 +177,25 @@ __device__ __forceinline__ void tmem_ld_32x32b_x16(uint32_t taddr, uint32_t v[16
 __device__ __forceinline__ void tmem_ld_wait() {
   asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
+// Empty volatile asm that "rewrites" 16 registers: placed after a wait, it
+// keeps the compiler from moving their first use above the wait.
+__device__ __forceinline__ void reg_fence16(uint32_t v[16]) {
+  asm volatile(""
+               : "+r"(v[0]), "+r"(v[1]), "+r"(v[2]), "+r"(v[3]), "+r"(v[4]), "+r"(v[5]), "+r"(v[6]), "+r"(v[7]),
+                 "+r"(v[8]), "+r"(v[9]), "+r"(v[10]), "+r"(v[11]), "+r"(v[12]), "+r"(v[13]), "+r"(v[14]),
+                 "+r"(v[15]));
+}
+// tcgen05.wait::ld, then the destination registers of the awaited loads are
+// fenced (a tcgen05.ld writes them asynchronously).
+__device__ __forceinline__ void tmem_ld_wait_x16(uint32_t v[16]) {
+  tmem_ld_wait();
+  reg_fence16(v);
+}
+__device__ __forceinline__ void tmem_ld_wait_x32(uint32_t v[32]) {
+  tmem_ld_wait();
+  reg_fence16(v);
+  reg_fence16(v + 16);
+}
 
 // ---- tcgen05, CTA pairs (cta_group::2) -------------------------------------------
 // Both CTAs of the pair allocate (same column address in each TMEM).

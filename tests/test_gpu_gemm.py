@@ -136,3 +136,32 @@ def test_full_size_workloads(oracle, name):
         qa = o.mixfp4_quantize(lin.make_x().to(DEV))
         qb = o.mixfp4_quantize(lin.make_w().to(DEV))
         sampled_check(oracle, qa, qb, seed=sum(map(ord, lin.name)))
+
+
+def test_stream_k_tail(oracle):
+    """80 tiles of 256 x 256 with K = 4096: on a GPU with 76 CTA pairs the 4
+    tiles past the first wave are split into K slices over all pairs, up to
+    a dozen or more pairs adding into one tile of C.  Ragged M and N; whole
+    rows and whole columns of C are checked."""
+    M, N, K = 2000, 2500, 4096
+    x = synth.activations(M, K, 7301, 7302)
+    w = synth.weights(N, K, 7303, 0.02, 0.5)
+    o = ops()
+    qa = o.mixfp4_quantize(x.to(DEV))
+    qb = o.mixfp4_quantize(w.to(DEV))
+    status = torch.zeros(1, dtype=torch.int32, device=DEV)
+    C = o.mixfp4_gemm(qa, qb, status_word=status)
+    torch.cuda.synchronize()
+    assert status.item() == 0
+    ac, as_, at = qa.codes.cpu().numpy(), qa.scales.cpu().numpy(), qa.tensor_scale.item()
+    bc, bs, bt = qb.codes.cpu().numpy(), qb.scales.cpu().numpy(), qb.tensor_scale.item()
+    rng = np.random.default_rng(5)
+    rows = np.unique(np.concatenate([[0, 255, 256, 1791, 1792, M - 1], rng.integers(0, M, 16)]))
+    cols = np.unique(np.concatenate([[0, 255, 256, 2303, 2304, N - 1], rng.integers(0, N, 16)]))
+    Cn = C.cpu().numpy()
+    A_r = oracle.dequant_rows_f64(ac, as_, at, rows)
+    B_c = oracle.dequant_rows_f64(bc, bs, bt, cols)
+    B_all = oracle.dequant_rows_f64(bc, bs, bt, range(N))
+    assert_close(Cn[rows], A_r @ B_all.T, A_r, B_all)
+    A_all = oracle.dequant_rows_f64(ac, as_, at, range(M))
+    assert_close(Cn[:, cols], A_all @ B_c.T, A_all, B_c)
