@@ -7,15 +7,23 @@
 //     scale-byte store (a warp writes 256 B and 32 B contiguous);
 //   * all per-element fp32 work runs on packed f32x2 instructions;
 //   * every division of Algorithm 1 (x/s32, B/6, B/7, |a|/s8) is evaluated as
-//     IEEE round-to-nearest by Markstein's correction (P. Markstein, "Computation
-//     of elementary functions on the IBM RISC System/6000 processor", 1990;
-//     Muller et al., Handbook of Floating-Point Arithmetic, Sec. 4.9):
-//         q0 = RN(a*r),  e = RN(a - q0*b) (exact via fma),  q = RN(q0 + e*r)
-//     with r = RN(1/b).  It returns RN(a/b) whenever a >= 2^-102 and the
-//     quotient is normal; smaller numerators only occur where their exact
-//     value cannot change a code or an error sum (see the tiny-value note in
-//     quantize_block), and tensors whose s32 lies outside [2^-20, 2^100] are
-//     first rescaled by an exact power of two;
+//     IEEE round-to-nearest with a divisor known in advance, in two packed
+//     instructions (N. Brisebarre, J.-M. Muller, S. K. Raina, "Accelerating
+//     correctly rounded floating-point division when the divisor is known in
+//     advance", IEEE Trans. Computers 53(8), 2004):
+//         q = RN(a*zh + RN(a*zl)),  zh = RN(1/b),  zl = RN(RN(1 - b*zh)/b).
+//     This is not correctly rounded for every divisor, so each use is covered
+//     by a check: exhaustive on the host for the divisors 6, 7 and every E4M3
+//     value (every fp32 significand of a), and, for x/s32, at run time in the
+//     kernel over all 128 bf16 significands of x (2 of the 2^23 fp32
+//     significands of s32 fail; those tensors use Markstein's correction,
+//     P. Markstein 1990; Muller et al., Handbook of Floating-Point Arithmetic,
+//     Sec. 4.9:  q0 = RN(a*r), e = RN(a - q0*b) (exact via fma),
+//     q = RN(q0 + e*r), r = RN(1/b)).  Both return RN(a/b) whenever a >=
+//     2^-102 and the quotient is normal; smaller numerators only occur where
+//     their exact value cannot change a code or an error sum (see the
+//     tiny-value note in quantize_block), and tensors whose s32 lies outside
+//     [2^-20, 2^100] are first rescaled by an exact power of two;
 //   * E2M1 rounding uses cvt.rn.satfinite.e2m1x2 (RNE, saturating) and E4M3
 //     scale rounding cvt.rn.satfinite.e4m3x2; E1M2 rounding adds 1.5*2^23
 //     (RNE to an integer) and clamps the integer to 7.
@@ -32,21 +40,33 @@ namespace {
 
 constexpr int kQuantThreads = 256;
 
-// Correctly rounded a / b (per lane) given nb = -b and r = RN(1/b).
+// Correctly rounded a / b (per lane) given nb = -b and r = RN(1/b) (Markstein).
 __device__ __forceinline__ u64 div_rn2(u64 a, u64 nb, u64 r) {
   u64 q0 = mul2(a, r);
   u64 e = fma2(q0, nb, a);
   return fma2(e, r, q0);
 }
 
+// RN(a*zh + RN(a*zl)) (per lane): a / b for a divisor b whose (zh, zl) pass
+// the checks described above.
+__device__ __forceinline__ u64 div_kd2(u64 a, u64 zh, u64 zl) { return fma2(a, zh, mul2(a, zl)); }
+
+// (zh, zl) of a divisor b: RN(1/b) and RN(RN(1 - b*zh)/b); (0, 0) for b = 0.
+__device__ __forceinline__ float2 kd_consts(float b) {
+  if (!(b > 0.0f)) return make_float2(0.0f, 0.0f);
+  const float zh = __frcp_rn(b);
+  return make_float2(zh, __fdiv_rn(__fmaf_rn(-b, zh, 1.0f), b));
+}
+
 __device__ __forceinline__ uint32_t lo32(u64 v) { return (uint32_t)v; }
 __device__ __forceinline__ uint32_t hi32(u64 v) { return (uint32_t)(v >> 32); }
 
 struct TensorConsts {
-  float s32;     // per-tensor scale, possibly rescaled to [1, 2)
-  float r32;     // RN(1/s32), or 0 when s32 == 0
-  float r6, r7;  // RN(1/6), RN(1/7)
-  int k;         // |x| is multiplied by 2^k when `scaled`
+  float s32;       // per-tensor scale, possibly rescaled to [1, 2)
+  float r32;       // RN(1/s32), or 0 when s32 == 0
+  float2 kd32;     // (zh, zl) of s32
+  float2 kd6, kd7; // (zh, zl) of 6 and 7
+  int k;           // |x| is multiplied by 2^k when `scaled`
   int scaled;
 };
 
@@ -70,8 +90,9 @@ __device__ __forceinline__ TensorConsts tensor_consts(float* tensor_scale, const
   }
   c.s32 = s32;
   c.r32 = (s32 > 0.0f) ? __frcp_rn(s32) : 0.0f;
-  c.r6 = __frcp_rn(6.0f);
-  c.r7 = __frcp_rn(7.0f);
+  c.kd32 = kd_consts(s32);
+  c.kd6 = kd_consts(6.0f);
+  c.kd7 = kd_consts(7.0f);
   return c;
 }
 
@@ -112,13 +133,16 @@ __device__ __forceinline__ uint32_t sign_bits(uint32_t w0, uint32_t w1, uint32_t
 // E1M2 clamp: when s8 = E4M3(b7) is normal (>= 2^-6) and b7 = fl32(B/7) did
 // not saturate, s8 >= b7 / (1 + 2^-4), so |a|/s8 <= 7 * 1.0625 * (1 + 2^-23)
 // < 7.5 and RNE never exceeds 7; only other blocks need the clamp.
-template <int kMode, bool kScaled>
+// kMarkstein selects the x / s32 method (see the header); the other divisions
+// always take the two-instruction form.
+template <int kMode, bool kScaled, bool kMarkstein>
 __device__ __forceinline__ void quantize_block(const uint32_t w[8], const TensorConsts& tc,
-                                               const float2* __restrict__ tab, uint32_t& code_lo,
+                                               const float4* __restrict__ tab, uint32_t& code_lo,
                                                uint32_t& code_hi, uint32_t& scale_byte) {
   // |x| as packed fp32 pairs (element 2j in the low lane).
   u64 a[8];
   const u64 ns32 = pack2(-tc.s32, -tc.s32), r32 = pack2(tc.r32, tc.r32);
+  const u64 zh32 = pack2(tc.kd32.x, tc.kd32.x), zl32 = pack2(tc.kd32.y, tc.kd32.y);
 #pragma unroll
   for (int j = 0; j < 8; ++j) {
     const uint32_t u = w[j] & 0x7FFF7FFFu;
@@ -127,7 +151,8 @@ __device__ __forceinline__ void quantize_block(const uint32_t w[8], const Tensor
       lo = __float_as_uint(scalbnf(__uint_as_float(lo), tc.k));
       hi = __float_as_uint(scalbnf(__uint_as_float(hi), tc.k));
     }
-    a[j] = div_rn2(bits2(lo, hi), ns32, r32);  // X_FP8 = X / s32 (magnitudes)
+    // X_FP8 = X / s32 (magnitudes)
+    a[j] = kMarkstein ? div_rn2(bits2(lo, hi), ns32, r32) : div_kd2(bits2(lo, hi), zh32, zl32);
   }
   // Block max of |X_FP8|.
   float v[16];
@@ -137,7 +162,7 @@ __device__ __forceinline__ void quantize_block(const uint32_t w[8], const Tensor
   B = max3f(B, max3f(v[9], v[10], v[11]), max3f(v[12], v[13], max3f(v[14], v[15], 0.0f)));
 
   // Candidate block scales s8 = E4M3(fl32(B/6)), E4M3(fl32(B/7)) and RN(1/s8).
-  const u64 bq = div_rn2(pack2(B, B), pack2(-6.0f, -7.0f), pack2(tc.r6, tc.r7));
+  const u64 bq = div_kd2(pack2(B, B), pack2(tc.kd6.x, tc.kd7.x), pack2(tc.kd6.y, tc.kd7.y));
   float b6, b7;
   unpack2(bq, b6, b7);
   const uint32_t sc = cvt_e4m3x2(b7, b6);  // low byte: E2M1 scale code, high: E1M2
@@ -147,14 +172,14 @@ __device__ __forceinline__ void quantize_block(const uint32_t w[8], const Tensor
   uint32_t p2lo = 0, p2hi = 0, p1lo = 0, p1hi = 0;
   if (kMode != MIXFP4_MODE_E1M2_ONLY) {
     // E2M1 candidate.
-    const float2 t = tab[c2];
-    const u64 ns8 = pack2(-t.x, -t.x), r8 = pack2(t.y, t.y);
+    const float4 t = tab[c2];
+    const u64 zh8 = pack2(t.y, t.y), zl8 = pack2(t.z, t.z);
     const uint16_t ns8h = __half_as_ushort(__float2half_rn(-t.x));  // exact: E4M3 values are f16 values
     u64 acc = 0;  // (+0, +0): even / odd chains
     uint32_t e[8];
 #pragma unroll
     for (int j = 0; j < 8; ++j) {
-      const u64 y = div_rn2(a[j], ns8, r8);
+      const u64 y = div_kd2(a[j], zh8, zl8);
       float ylo, yhi;
       unpack2(y, ylo, yhi);
       uint32_t h2;
@@ -180,8 +205,8 @@ __device__ __forceinline__ void quantize_block(const uint32_t w[8], const Tensor
   }
   if (kMode != MIXFP4_MODE_E2M1_ONLY) {
     // E1M2 candidate (x2 units: integers 0..7).
-    const float2 t = tab[c1];
-    const u64 ns8 = pack2(-t.x, -t.x), r8 = pack2(t.y, t.y);
+    const float4 t = tab[c1];
+    const u64 ns8 = pack2(-t.x, -t.x), zh8 = pack2(t.y, t.y), zl8 = pack2(t.z, t.z);
     const u64 magic = pack2(12582912.0f, 12582912.0f);    // 1.5 * 2^23
     const u64 nmagic = pack2(-12582912.0f, -12582912.0f);
     const bool clamp = !(t.x >= 0x1p-6f && b7 <= 448.0f);
@@ -189,7 +214,7 @@ __device__ __forceinline__ void quantize_block(const uint32_t w[8], const Tensor
     uint32_t pb[8];
 #pragma unroll
     for (int j = 0; j < 8; ++j) {
-      const u64 y = div_rn2(a[j], ns8, r8);
+      const u64 y = div_kd2(a[j], zh8, zl8);
       const u64 tq = add2(y, magic);  // RNE to an integer in the low mantissa bits
       uint32_t tlo = lo32(tq), thi = hi32(tq);
       if (clamp) {
@@ -236,7 +261,7 @@ __global__ void __launch_bounds__(kQuantThreads, 4)
 quantize_kernel(const uint16_t* __restrict__ x, int64_t nblocks, int64_t kblocks, int64_t ldx,
                 uint8_t* __restrict__ codes, uint8_t* __restrict__ scales, float* tensor_scale,
                 const uint32_t* amax_word, int scale_given) {
-  __shared__ float2 tab[128];  // E4M3 code -> {s8, RN(1/s8)}
+  __shared__ float4 tab[128];  // E4M3 code -> {s8, zh, zl, 0} (zh, zl: see div_kd2)
   const int64_t nthr = (int64_t)gridDim.x * kQuantThreads;
   int64_t b = (int64_t)blockIdx.x * kQuantThreads + threadIdx.x;
   uint32_t wa[8], wb[8];
@@ -245,21 +270,37 @@ quantize_kernel(const uint16_t* __restrict__ x, int64_t nblocks, int64_t kblocks
   if (threadIdx.x < 128) {
     float s8 = 0.0f, unused;
     if (threadIdx.x < 0x7F) f16x2_to_f32(cvt_f16x2_from_e4m3x2((uint16_t)threadIdx.x), s8, unused);
-    tab[threadIdx.x] = make_float2(s8, s8 > 0.0f ? __frcp_rn(s8) : 0.0f);
+    const float2 kd = kd_consts(s8);
+    tab[threadIdx.x] = make_float4(s8, kd.x, kd.y, 0.0f);
   }
   const TensorConsts tc = tensor_consts(tensor_scale, amax_word, scale_given);
-  __syncthreads();
+  // x / s32 may take the two-instruction division when it returns the IEEE
+  // quotient for all 128 bf16 significands (the quotient scales exactly with
+  // x's exponent) and its correction term a*zl stays normal for every
+  // quotient that can matter (|a| >= 2^-82; see the tiny-value note): the
+  // remainder 1 - s32*zh is 0 or at least 2^-44 in magnitude.
+  bool kd_ok = true;
+  if (threadIdx.x < 128 && !tc.scaled) {
+    const float xs = __uint_as_float(0x3F800000u | (threadIdx.x << 16));
+    const u64 q = div_kd2(pack2(xs, xs), pack2(tc.kd32.x, tc.kd32.x), pack2(tc.kd32.y, tc.kd32.y));
+    const float rem = __fmaf_rn(-tc.s32, tc.kd32.x, 1.0f);
+    kd_ok = tc.s32 > 0.0f && lo32(q) == __float_as_uint(__fdiv_rn(xs, tc.s32)) &&
+            (rem == 0.0f || fabsf(rem) >= 0x1p-44f);
+  }
+  const bool markstein = !__syncthreads_and(kd_ok);
   for (; b < nblocks; b += 2 * nthr) {
     uint32_t lo, hi, sb;
-    if (tc.scaled) quantize_block<kMode, true>(wa, tc, tab, lo, hi, sb);
-    else quantize_block<kMode, false>(wa, tc, tab, lo, hi, sb);
+    if (tc.scaled) quantize_block<kMode, true, true>(wa, tc, tab, lo, hi, sb);
+    else if (markstein) quantize_block<kMode, false, true>(wa, tc, tab, lo, hi, sb);
+    else quantize_block<kMode, false, false>(wa, tc, tab, lo, hi, sb);
     stg64(codes + b * 8, lo, hi);
     scales[b] = (uint8_t)sb;
     if (b + 2 * nthr < nblocks) ldg256_stream(block_src<kContig>(x, b + 2 * nthr, kblocks, ldx), wa);
     const int64_t b1 = b + nthr;
     if (b1 < nblocks) {
-      if (tc.scaled) quantize_block<kMode, true>(wb, tc, tab, lo, hi, sb);
-      else quantize_block<kMode, false>(wb, tc, tab, lo, hi, sb);
+      if (tc.scaled) quantize_block<kMode, true, true>(wb, tc, tab, lo, hi, sb);
+      else if (markstein) quantize_block<kMode, false, true>(wb, tc, tab, lo, hi, sb);
+      else quantize_block<kMode, false, false>(wb, tc, tab, lo, hi, sb);
       stg64(codes + b1 * 8, lo, hi);
       scales[b1] = (uint8_t)sb;
       if (b1 + 2 * nthr < nblocks) ldg256_stream(block_src<kContig>(x, b1 + 2 * nthr, kblocks, ldx), wb);

@@ -1,11 +1,14 @@
-"""Host check of the division method inside the CUDA quantizer (CPU only).
+"""Host checks of the division methods inside the CUDA quantizer (CPU only).
 
 The quantizer evaluates every IEEE division of Algorithm 1 (x/s32, B/6, B/7,
-|a|/s8) with Markstein's fma correction instead of a divide instruction.
-tests/native/markstein_check.c enumerates every significand pair the
-quantizer can present (bf16 numerators x all fp32 s32 significands, all fp32
-numerators x all E4M3 significands, B/6 and B/7) plus exponent edges down to
-2^-102 and requires bit equality with C's IEEE '/'.
+|a|/s8) without a divide instruction: with the two-instruction division by a
+known divisor where it is exact, and with Markstein's fma correction for the
+few tensor scales s32 where the former is not.  tests/native/markstein_check.c
+enumerates every significand pair the quantizer can present (bf16 numerators x
+all fp32 s32 significands, all fp32 numerators x all E4M3 significands, B/6
+and B/7) plus exponent edges down to 2^-102 and requires bit equality with C's
+IEEE '/'; tests/native/known_divisor_check.c does the same for the other
+method and its acceptance rule.
 """
 import os
 import shutil
@@ -25,3 +28,22 @@ def test_markstein_division_matches_ieee(tmp_path):
     assert res.returncode == 0, res.stdout + res.stderr
     lines = [l for l in res.stdout.splitlines() if "mismatches=" in l]
     assert len(lines) == 7 and all(l.endswith("mismatches=0") for l in lines), res.stdout
+
+
+@pytest.mark.skipif(shutil.which("gcc") is None, reason="needs gcc")
+def test_known_divisor_division_matches_ieee(tmp_path):
+    """The two-instruction division RN(a*zh + RN(a*zl)) (Brisebarre, Muller,
+    Raina 2004) that the quantizer uses for |a|/s8, B/6, B/7 and, when its
+    run-time check accepts s32, for x/s32.  tests/native/known_divisor_check.c
+    enumerates every significand pair for the fixed divisors, replays the
+    kernel's acceptance rule for every fp32 significand of s32, and requires
+    the IEEE quotient at other exponents for every accepted one."""
+    exe = tmp_path / "known_divisor_check"
+    subprocess.check_call(["gcc", "-O2", "-ffp-contract=off", "-fopenmp", "-std=c11",
+                           os.path.join(HERE, "native", "known_divisor_check.c"), "-o", str(exe), "-lm"])
+    res = subprocess.run([str(exe)], capture_output=True, text=True, timeout=600)
+    assert res.returncode == 0, res.stdout + res.stderr
+    lines = [l for l in res.stdout.splitlines() if "mismatches=" in l]
+    assert len(lines) == 3 and all(l.endswith("mismatches=0") for l in lines), res.stdout
+    rejected = int(res.stdout.split("rejected=")[1].split()[0])
+    assert 0 < rejected < 1000, res.stdout  # a handful of s32 significands fall back to Markstein

@@ -159,6 +159,22 @@ def test_given_scale(oracle, s32):
     check(oracle, x, 0, s32=np.float32(s32).item(), what=f"given {s32}")
 
 
+@pytest.mark.parametrize("s32", [float.fromhex("0x1.a15686p+0"), float.fromhex("0x1.f250c6p-3"),
+                                 float.fromhex("0x1.000002p+0"), float.fromhex("0x1.0b06ecp+5")])
+def test_given_scale_division_fallback(oracle, s32):
+    """Tensor scales whose x / s32 the kernel must not take with the
+    two-instruction division (it is inexact for a bf16 significand of x, or
+    its correction term can leave the normal range), so the quantizer falls
+    back to Markstein's correction; the block data include the significand
+    that fails (0x1.8e for 0x1.a15686, 0x1.e8 for 0x1.f250c6)."""
+    x = synth.activations(8, 512, 93, 94).float()
+    for i, v in enumerate((float.fromhex("0x1.8ep+0"), float.fromhex("0x1.e8p+0"))):
+        cols = x[::2, i::37].shape[1]
+        x[::2, i::37] = torch.from_numpy(v * 2.0 ** np.arange(-3, 4).repeat(3)[:cols]).float()
+        x[1::2, 5 + i::41] = -v
+    check(oracle, x.to(torch.bfloat16), 0, s32=s32, what=f"given {s32!r}")
+
+
 @pytest.mark.parametrize("shape", [(1, 16), (3, 48), (257, 4112), (5, 16 * 999)])
 def test_ragged_shapes(oracle, shape):
     rows, K = shape
