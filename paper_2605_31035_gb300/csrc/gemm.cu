@@ -255,6 +255,7 @@ mixfp4_gemm_kernel(const __grid_constant__ CUtensorMap tm_ac, const __grid_const
     tmem_alloc_pair(smem_u32(&bars->tmem_base), kTmemCols);
     tmem_relinquish_pair();
   }
+  griddep_launch_dependents();
   tc_fence_before();
   cluster_sync();  // barriers of both CTAs initialised, TMEM allocated in both
   tc_fence_after();
@@ -273,6 +274,7 @@ mixfp4_gemm_kernel(const __grid_constant__ CUtensorMap tm_ac, const __grid_const
       tma_prefetch(&tm_bc);
       tma_prefetch(&tm_as);
       tma_prefetch(&tm_bs);
+      griddep_wait();  // the operands may come from the kernel before this one
       int last_it = -1;  // last code-stage use issued (its copies may be in flight)
       int it = 0;
       bool ok = true;
@@ -454,6 +456,7 @@ mixfp4_gemm_kernel(const __grid_constant__ CUtensorMap tm_ac, const __grid_const
     // 64 contiguous bytes in each of 8 rows.
     const int q = warp & 3;                  // TMEM lane quarter of this warp
     const int chalf = (warp - kFirstEpi) >> 2;  // column half
+    griddep_wait();
     const float sa = 0.25f * __ldg(a_ts), sb = __ldg(b_ts);
     const bool vec_ok = ((ldc & 3) == 0) && ((reinterpret_cast<uintptr_t>(C) & 15) == 0);
     const uint32_t acc_empty_leader = mapa_shared(smem_u32(&bars->acc_empty), 0);
@@ -938,8 +941,12 @@ int launch_gemm(const uint8_t* a_codes, const uint8_t* a_scales, const float* a_
                             (size_t)(M - r0), stream);
     if (e != cudaSuccess) return MIXFP4_ERR_CUDA;
   }
-  mixfp4_gemm_kernel<<<(unsigned)(2 * clusters), kThreads, SMEM_ALLOC, stream>>>(
-      tac, tbc, tas, tbs, a_ts, b_ts, (int)M, (int)N, (int)K, C, (long long)ldc, (int)dp_tiles, status_word);
+  // A programmatic dependent: barrier set-up and TMEM allocation overlap the
+  // tail of the kernel before it; the TMA producer and the epilogue wait for
+  // that kernel before they read the operands or the tensor scales.
+  if (launch_pdl(mixfp4_gemm_kernel, (unsigned)(2 * clusters), kThreads, SMEM_ALLOC, stream, tac, tbc, tas, tbs,
+                 a_ts, b_ts, (int)M, (int)N, (int)K, C, (long long)ldc, (int)dp_tiles, status_word) != cudaSuccess)
+    return MIXFP4_ERR_CUDA;
   return MIXFP4_OK;
 }
 

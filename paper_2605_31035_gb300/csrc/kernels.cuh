@@ -20,4 +20,23 @@ int launch_gemm(const uint8_t* a_codes, const uint8_t* a_scales, const float* a_
                 int64_t M, int64_t N, int64_t K, float* C, int64_t ldc, uint32_t* status_word,
                 cudaStream_t stream);
 
+// Launch `kernel` as a programmatic dependent of the previous kernel on the
+// stream (it may start before that kernel completes; the kernel itself waits,
+// with griddepcontrol.wait, before it reads anything that kernel may write).
+template <typename... Params, typename... Args>
+inline cudaError_t launch_pdl(void (*kernel)(Params...), dim3 grid, dim3 block, size_t smem,
+                              cudaStream_t stream, Args... args) {
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, static_cast<Params>(args)...);
+}
+
 }  // namespace mixfp4

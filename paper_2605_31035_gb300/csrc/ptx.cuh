@@ -36,6 +36,17 @@ __device__ __forceinline__ u64 add2(u64 a, u64 b) {
   return d;
 }
 
+// ---- programmatic dependent launch ----------------------------------------
+// Let the next kernel on the stream, if launched as a programmatic dependent,
+// start its prologue now.
+__device__ __forceinline__ void griddep_launch_dependents() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+// Wait until the preceding kernel on the stream has completed and its memory
+// operations are visible (returns at once when this kernel was not launched
+// as a programmatic dependent).
+__device__ __forceinline__ void griddep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
 __device__ __forceinline__ float max3f(float a, float b, float c) {
   float d;
   asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));

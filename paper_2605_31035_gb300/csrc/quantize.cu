@@ -260,8 +260,13 @@ template <int kMode, bool kContig>
 __global__ void __launch_bounds__(kQuantThreads, 4)
 quantize_kernel(const uint16_t* __restrict__ x, int64_t nblocks, int64_t kblocks, int64_t ldx,
                 uint8_t* __restrict__ codes, uint8_t* __restrict__ scales, float* tensor_scale,
-                const uint32_t* amax_word, int scale_given) {
+                const uint32_t* amax_word, int scale_given, int after_amax) {
   __shared__ float4 tab[128];  // E4M3 code -> {s8, zh, zl, 0} (zh, zl: see div_kd2)
+  // Launched as a programmatic dependent of the amax kernel (after_amax), x
+  // is already complete and may be read before that kernel finishes; only
+  // the amax word must wait.  Otherwise wait before touching any input.
+  if (!after_amax) griddep_wait();
+  griddep_launch_dependents();
   const int64_t nthr = (int64_t)gridDim.x * kQuantThreads;
   int64_t b = (int64_t)blockIdx.x * kQuantThreads + threadIdx.x;
   uint32_t wa[8], wb[8];
@@ -273,6 +278,7 @@ quantize_kernel(const uint16_t* __restrict__ x, int64_t nblocks, int64_t kblocks
     const float2 kd = kd_consts(s8);
     tab[threadIdx.x] = make_float4(s8, kd.x, kd.y, 0.0f);
   }
+  if (after_amax) griddep_wait();
   const TensorConsts tc = tensor_consts(tensor_scale, amax_word, scale_given);
   // x / s32 may take the two-instruction division when it returns the IEEE
   // quotient for all 128 bf16 significands (the quotient scales exactly with
@@ -309,25 +315,37 @@ quantize_kernel(const uint16_t* __restrict__ x, int64_t nblocks, int64_t kblocks
 }
 
 // max |x| over the tensor as the bit pattern of a non-negative fp32 (bf16
-// magnitudes order like unsigned 16-bit integers).
+// magnitudes order like unsigned 16-bit integers).  Each thread keeps four
+// 32-byte loads in flight.
+constexpr int kAmaxUnroll = 4;
+
+template <bool kContig>
+__device__ __forceinline__ const uint16_t* amax_src(const uint16_t* x, int64_t b, int64_t kblocks, int64_t ldx) {
+  if (kContig) return x + b * 16;
+  const int64_t row = b / kblocks;
+  return x + row * ldx + (b - row * kblocks) * 16;
+}
+
 template <bool kContig>
 __global__ void __launch_bounds__(256)
 amax_kernel(const uint16_t* __restrict__ x, int64_t nblocks, int64_t kblocks, int64_t ldx,
             uint32_t* amax_word) {
   uint32_t m = 0;
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
-  for (int64_t b = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; b < nblocks; b += stride) {
-    const uint16_t* src;
-    if (kContig) {
-      src = x + b * 16;
-    } else {
-      const int64_t row = b / kblocks;
-      src = x + row * ldx + (b - row * kblocks) * 16;
-    }
-    uint32_t w[8];
-    ldg256_stream(src, w);
+  for (int64_t b = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; b < nblocks; b += kAmaxUnroll * stride) {
+    uint32_t w[kAmaxUnroll][8];
 #pragma unroll
-    for (int j = 0; j < 8; ++j) m = __vmaxu2(m, w[j] & 0x7FFF7FFFu);
+    for (int u = 0; u < kAmaxUnroll; ++u) {
+      const int64_t bu = b + u * stride;
+      if (bu < nblocks) ldg256_stream(amax_src<kContig>(x, bu, kblocks, ldx), w[u]);
+      else
+#pragma unroll
+        for (int j = 0; j < 8; ++j) w[u][j] = 0u;
+    }
+#pragma unroll
+    for (int u = 0; u < kAmaxUnroll; ++u)
+#pragma unroll
+      for (int j = 0; j < 8; ++j) m = __vmaxu2(m, w[u][j] & 0x7FFF7FFFu);
   }
   m = max(m & 0xFFFFu, m >> 16);
 #pragma unroll
@@ -339,6 +357,8 @@ amax_kernel(const uint16_t* __restrict__ x, int64_t nblocks, int64_t kblocks, in
     for (int i = 1; i < (int)(blockDim.x >> 5); ++i) m = max(m, red[i]);
     if (m) atomicMax(amax_word, m << 16);
   }
+  // The quantize kernel that follows may start once every CTA got here.
+  griddep_launch_dependents();
 }
 
 // out = fl32(sign * v * s8 * s32): v * s8 is exact in fp32, one rounding.
@@ -380,8 +400,8 @@ int launch_amax(const uint16_t* x, int64_t rows, int64_t K, int64_t ldx, uint32_
                 cudaStream_t stream) {
   const int64_t kblocks = K / 16, nblocks = rows * kblocks;
   if (nblocks == 0) return 0;
-  int64_t grid = (nblocks + 255) / 256;
-  if (grid > 152 * 16) grid = 152 * 16;
+  int64_t grid = (nblocks + 256 * kAmaxUnroll - 1) / (256 * kAmaxUnroll);
+  if (grid > 152 * 8) grid = 152 * 8;
   if (ldx == K) amax_kernel<true><<<(unsigned)grid, 256, 0, stream>>>(x, nblocks, kblocks, ldx, amax_word);
   else amax_kernel<false><<<(unsigned)grid, 256, 0, stream>>>(x, nblocks, kblocks, ldx, amax_word);
   return 0;
@@ -396,14 +416,17 @@ int launch_quantize(const uint16_t* x, int64_t rows, int64_t K, int64_t ldx, uin
   int64_t grid = (nblocks + 2 * kQuantThreads - 1) / (2 * kQuantThreads);
   if (grid > 152 * 4) grid = 152 * 4;
   if (grid == 0) return 0;
-#define MIXFP4_LAUNCH_Q(MODE)                                                              \
-  do {                                                                                     \
-    if (ldx == K)                                                                          \
-      quantize_kernel<MODE, true><<<(unsigned)grid, kQuantThreads, 0, stream>>>(            \
-          x, nblocks, kblocks, ldx, codes, scales, tensor_scale, amax_word, scale_given);   \
-    else                                                                                   \
-      quantize_kernel<MODE, false><<<(unsigned)grid, kQuantThreads, 0, stream>>>(           \
-          x, nblocks, kblocks, ldx, codes, scales, tensor_scale, amax_word, scale_given);   \
+  // Launched as a programmatic dependent: it overlaps its launch with the tail
+  // of the kernel before it (see the waits at the top of quantize_kernel).
+  const int after_amax = !scale_given;
+#define MIXFP4_LAUNCH_Q(MODE)                                                                           \
+  do {                                                                                                  \
+    if (ldx == K)                                                                                       \
+      launch_pdl(quantize_kernel<MODE, true>, (unsigned)grid, kQuantThreads, 0, stream, x, nblocks,      \
+                 kblocks, ldx, codes, scales, tensor_scale, amax_word, scale_given, after_amax);        \
+    else                                                                                                \
+      launch_pdl(quantize_kernel<MODE, false>, (unsigned)grid, kQuantThreads, 0, stream, x, nblocks,     \
+                 kblocks, ldx, codes, scales, tensor_scale, amax_word, scale_given, after_amax);        \
   } while (0)
   switch (mode) {
     case MIXFP4_MODE_MIX: MIXFP4_LAUNCH_Q(MIXFP4_MODE_MIX); break;
