@@ -324,8 +324,8 @@ def cpu_baseline(lin, x_cpu, budget_s: float = 15.0):
     layer = OracleLayer(lin, x_cpu, lin.make_w()[:cap], cap)
     secs, _ = layer.run(1, 64)
     per_row = secs / 64.0                      # one X row against one W row
-    n_x = 16
-    n_w = max(64, min(cap, int(budget_s / max(per_row * n_x, 1e-9))))
+    n_w = cap
+    n_x = max(4, min(512, int(budget_s / max(per_row * n_w, 1e-9))))
     secs, flops = layer.run(n_x, n_w)
     return {"value": flops / secs / 1e12, "unit": "TFLOP/s", "cores": 1, "kind": "oracle",
             "sample": f"Algorithm 1 on {n_x} rows of X + float64 GEMM vs {n_w} pre-quantized rows of W "
