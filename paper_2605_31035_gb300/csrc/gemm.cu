@@ -675,6 +675,10 @@ mixfp4_gemm_skinny_kernel(const __grid_constant__ CUtensorMap tm_wc, const __gri
       int d = 0, ntile = 0;
       uint32_t dph = 0;
       bool ok = true;
+      // Descriptor of decoded stage 0, first 16-K step; other stages and steps
+      // only move the start address (14-bit field in 16-byte units, no carry:
+      // shared addresses stay below 256 KiB).
+      const uint64_t bdesc0 = smem_desc_noswizzle(sbase + OFF_DEC, kLBO, kSBO);
       for (long long u = u_begin; u < u_end && ok;) {
         const int wt = (int)(u / num_kc);
         const long long run_end = (long long)(wt + 1) * num_kc < u_end ? (long long)(wt + 1) * num_kc : u_end;
@@ -692,14 +696,12 @@ mixfp4_gemm_skinny_kernel(const __grid_constant__ CUtensorMap tm_wc, const __gri
               break;
             }
             tc_fence_after();
-            const uint32_t xb = sbase + OFF_DEC + d * X_DEC;
+            const uint64_t bd = bdesc0 + (uint64_t)((d * X_DEC) >> 4);
             const uint32_t wa = tmem_w0 + (uint32_t)d * kWStageCols;
+            mma_f16_tmem_a(tmem_base, wa, bd, idesc, first ? 0u : 1u);
+            first = false;
 #pragma unroll
-            for (int j = 0; j < BKD / 16; ++j) {
-              mma_f16_tmem_a(tmem_base, wa + j * 8, smem_desc_noswizzle(xb + j * 256, kLBO, kSBO), idesc,
-                             first ? 0u : 1u);
-              first = false;
-            }
+            for (int j = 1; j < BKD / 16; ++j) mma_f16_tmem_a(tmem_base, wa + j * 8, bd + (uint64_t)(j * 16), idesc, 1u);
             mma_commit(smem_u32(&bars->dec_empty[d]));
             if (++d == kDecStages) { d = 0; dph ^= 1; }
           }
@@ -714,18 +716,27 @@ mixfp4_gemm_skinny_kernel(const __grid_constant__ CUtensorMap tm_wc, const __gri
     // ---------------- decoders ----------------
     const bool is_w = warp < kFirstX;
     const int dw = warp - (is_w ? kFirstW : kFirstX);
-    const int tpr = is_w ? kTPRW : kTPRX;
-    // weight decoders: rows by TMEM lane quarter (warp % 4), four parts per row;
-    // X decoders: 64 rows x two parts.
-    const int part = is_w ? (dw >> 2) : (dw >> 1);   // share of a stage's four 32-code chunks
-    const int rl = is_w ? ((warp & 3) * 32 + lane) : ((dw & 1) * 32 + lane);
-    const bool active = is_w || (dw & 1) * 32 < nmma;  // X decoders past the padded rows idle
-    const int cpt = 4 / tpr;                         // chunks per thread per stage
-    const uint32_t code_off = (is_w ? 0 : OFF_XC) + rl * (BKC / 2);
-    const uint32_t scale_off = (is_w ? OFF_WS : OFF_XS) + rl * (BKC / 16);
-    const uint32_t x_off = OFF_DEC + (rl >> 3) * kSBO + (rl & 7) * 16;
+    // Weight decoders: rows by TMEM lane quarter (warp % 4), four parts per
+    // row, one 32-code chunk each per stage.  X decoders: the stage's
+    // nmma x 4 chunks as items i = chunk * nmma + row, thread t taking items t
+    // and t + 128 (8 consecutive lanes read 8 rows of one chunk: no conflicts).
+    const int xt = dw * 32 + lane;                   // X decoder thread 0..127
+    const int nitem = 4 * nmma;
+    int rows[2], parts[2];
+    if (is_w) {
+      rows[0] = (warp & 3) * 32 + lane;
+      parts[0] = dw >> 2;
+    } else {
+#pragma unroll
+      for (int j = 0; j < 2; ++j) {
+        const int item = xt + 128 * j;
+        rows[j] = item < nitem ? item % nmma : 0;
+        parts[j] = item < nitem ? item / nmma : 0;
+      }
+    }
+    const int nmine = is_w ? 1 : (xt < nitem) + (xt + 128 < nitem);  // chunks per stage
+    const bool active = nmine > 0;
     const uint32_t w_lane = (uint32_t)((warp & 3) * 32) << 16;
-    const uint32_t swz = rl & 7;
     int d = 0, it = 0;
     uint32_t dph = 0;
     for (long long u = u_begin; u < u_end; ++u, ++it) {
@@ -736,17 +747,19 @@ mixfp4_gemm_skinny_kernel(const __grid_constant__ CUtensorMap tm_wc, const __gri
         break;
       }
       const uint32_t st = sbase + s * CODE_STAGE;
-      uint4 sc = make_uint4(0, 0, 0, 0);
-      if (active) sc = lds128(st + scale_off);
+      uint4 sc[2] = {make_uint4(0, 0, 0, 0), make_uint4(0, 0, 0, 0)};  // the rows' 16 block scales
+#pragma unroll
+      for (int j = 0; j < 2; ++j)
+        if (j < nmine) sc[j] = lds128(st + (is_w ? OFF_WS : OFF_XS) + rows[j] * (BKC / 16));
       bool ok = true;
 #pragma unroll
       for (int sub = 0; sub < kSub; ++sub) {
         uint4 c[2];
-        if (active) {
 #pragma unroll
-          for (int j = 0; j < 2; ++j)
-            if (j < cpt) c[j] = lds128(st + code_off + ((uint32_t)((sub * 4 + part * cpt + j) ^ swz) << 4));
-        }
+        for (int j = 0; j < 2; ++j)
+          if (j < nmine)
+            c[j] = lds128(st + (is_w ? 0 : OFF_XC) + rows[j] * (BKC / 2) +
+                          ((uint32_t)((sub * 4 + parts[j]) ^ (rows[j] & 7)) << 4));
         if (!mbar_wait(smem_u32(&bars->dec_empty[d]), dph ^ 1, abort_flag, kWaitLimitNs)) {
           fail(32u);
           ok = false;
@@ -754,22 +767,21 @@ mixfp4_gemm_skinny_kernel(const __grid_constant__ CUtensorMap tm_wc, const __gri
         }
         if (is_w) {
           uint32_t o[16];
-          const int chunk = sub * 4 + part;  // one chunk per thread
-          decode_chunk(c[0], scale_pair(sc, chunk), o);
-          tmem_st_32x32b_x16(tmem_w0 + w_lane + (uint32_t)d * kWStageCols + (uint32_t)part * 16u, o);
+          decode_chunk(c[0], scale_pair(sc[0], sub * 4 + parts[0]), o);
+          tmem_st_32x32b_x16(tmem_w0 + w_lane + (uint32_t)d * kWStageCols + (uint32_t)parts[0] * 16u, o);
           tmem_st_wait();
           tc_fence_before();
         } else if (active) {
-          const uint32_t dst = sbase + x_off + d * X_DEC;
 #pragma unroll
           for (int j = 0; j < 2; ++j) {
-            const int chunk = sub * 4 + part * 2 + j;
-            uint32_t o[16];
-            decode_chunk(c[j], scale_pair(sc, chunk), o);
-            const int kc0 = (part * 2 + j) * 4;
+            if (j < nmine) {
+              uint32_t o[16];
+              decode_chunk(c[j], scale_pair(sc[j], sub * 4 + parts[j]), o);
+              const uint32_t dst = sbase + OFF_DEC + d * X_DEC + (rows[j] >> 3) * kSBO + (rows[j] & 7) * 16;
 #pragma unroll
-            for (int q = 0; q < 4; ++q)
-              sts128(dst + (kc0 + q) * kLBO, o[4 * q], o[4 * q + 1], o[4 * q + 2], o[4 * q + 3]);
+              for (int q = 0; q < 4; ++q)
+                sts128(dst + (parts[j] * 4 + q) * kLBO, o[4 * q], o[4 * q + 1], o[4 * q + 2], o[4 * q + 3]);
+            }
           }
           fence_proxy_async_smem();
         }
