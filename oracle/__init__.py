@@ -61,6 +61,10 @@ def _L():
         lib.oracle_fp4_rne.argtypes = [ctypes.c_int, ctypes.c_float]
         lib.oracle_quantize.restype = ctypes.c_int
         lib.oracle_quantize.argtypes = [P, I64, I64, I64, ctypes.c_int, ctypes.c_int, P, P, P, P, P]
+        lib.oracle_quantize_f32.restype = ctypes.c_int
+        lib.oracle_quantize_f32.argtypes = [P, I64, I64, I64, ctypes.c_int, ctypes.c_int, P, P, P, P, P]
+        lib.oracle_rht.restype = ctypes.c_int
+        lib.oracle_rht.argtypes = [P, I64, I64, I64, P, P]
         lib.oracle_dequantize.restype = None
         lib.oracle_dequantize.argtypes = [P, P, ctypes.c_float, I64, I64, P]
         lib.oracle_gemm_f64.restype = None
@@ -120,6 +124,38 @@ def quantize(x_bf16_bits: np.ndarray, mode: int = MODE_MIX, s32: float | None = 
     if want_errors:
         return codes, scales, float(s[0]), e2, e1
     return codes, scales, float(s[0])
+
+
+def quantize_f32(x: np.ndarray, mode: int = MODE_MIX, s32: float | None = None, want_errors: bool = False):
+    """Algorithm 1 on a [rows, K] float32 tensor (same steps as quantize)."""
+    x = np.ascontiguousarray(x, dtype=np.float32)
+    rows, K = x.shape
+    codes = np.zeros((rows, K // 2), np.uint8)
+    scales = np.zeros((rows, K // 16), np.uint8)
+    s = np.array([0.0 if s32 is None else s32], np.float32)
+    e2 = np.zeros((rows, K // 16), np.float32)
+    e1 = np.zeros((rows, K // 16), np.float32)
+    rc = _L().oracle_quantize_f32(_p(x), rows, K, K, int(mode), 0 if s32 is None else 1, _p(s),
+                                  _p(codes), _p(scales), _p(e2), _p(e1))
+    if rc != 0:
+        raise ValueError("oracle_quantize_f32 rejected the input (non-finite value or K % 16 != 0)")
+    if want_errors:
+        return codes, scales, float(s[0]), e2, e1
+    return codes, scales, float(s[0])
+
+
+def rht(x_bf16_bits: np.ndarray, signs: np.ndarray | None = None) -> np.ndarray:
+    """The 128-point rotation (reading R11) of a [rows, K] bf16 tensor, K % 128 == 0.
+    signs: 16 uint8 (bit i negates element i of every chunk) or None.  Returns fp32."""
+    x = np.ascontiguousarray(x_bf16_bits, dtype=np.uint16)
+    rows, K = x.shape
+    y = np.zeros((rows, K), np.float32)
+    sg = None if signs is None else np.ascontiguousarray(signs, np.uint8)
+    if sg is not None and sg.size != 16:
+        raise ValueError("signs must hold 16 bytes")
+    if _L().oracle_rht(_p(x), rows, K, K, None if sg is None else _p(sg), _p(y)) != 0:
+        raise ValueError("oracle_rht needs K % 128 == 0")
+    return y
 
 
 def dequantize(codes: np.ndarray, scales: np.ndarray, s32: float) -> np.ndarray:

@@ -16,7 +16,12 @@
  *   fp4_*              Table 1 (Sec. 3.1) and App. B.2 codebooks; the x2 E1M2
  *                      remap of Sec. 3.1 / App. B.2
  *   oracle_quantize    Algorithm 1 (MixFP4 quantization), with the type bit of
- *                      App. B.3 (type-in-scale packing)
+ *                      App. B.3 (type-in-scale packing); oracle_quantize_f32
+ *                      is the same steps on an fp32 tensor
+ *   oracle_rht         the random Hadamard transform applied before
+ *                      quantization (Sec. 4 "+RHT", Sec. 3.4 training flow):
+ *                      128-point Sylvester Walsh-Hadamard per chunk (reading
+ *                      R11)
  *   oracle_dequantize  App. B.2/B.3 decode (scale_ue4m3 = scale with bit 7
  *                      cleared) times the per-tensor scale
  *   oracle_gemm_f64    C = A_deq . B_deq^T in float64 (plain definition)
@@ -38,9 +43,17 @@
  *   R7 s8 == 0 gives all-zero magnitudes and d_i = -|a_i|; s32 == 0 gives a_i = 0.
  *   R9 element 2j in the low nibble of byte j; codes [rows][K/2], scales
  *      [rows][K/16], both K-major.
+ *   R11 RHT: every 128-element chunk of a row along K is rotated on its own:
+ *      v_i = -x_i where sign bit i (of a 128-bit vector shared by all chunks)
+ *      is set, else x_i; the Sylvester Hadamard product H_128 v by the radix-2
+ *      butterfly in fp32, strides h = 1, 2, 4, ..., 64 in that order, each
+ *      pair (i, i+h) with i & h == 0 becoming (fl32(v_i + v_{i+h}),
+ *      fl32(v_i - v_{i+h})); then y_i = fl32(v_i * c), c = RN(1/sqrt(128)).
+ *      Algorithm 1 then runs on the fp32 y (X = y).
  */
 #include <math.h>
 #include <stdint.h>
+#include <stdlib.h>
 #include <string.h>
 
 /* ---------------------------------------------------------------------------
@@ -139,20 +152,20 @@ static void candidate(int type, const float a[16], float B, int* s8code,
   *s8code = code;
 }
 
-/* Algorithm 1 over a [rows][K] bf16 tensor (row stride ldx elements).
+/* Algorithm 1 over a [rows][K] fp32 tensor (row stride ldx elements).
  *   mode 0 = MixFP4, 1 = E2M1 only (NVFP4), 2 = E1M2 only (NVINT4)
  *   scale_given 0: s32 = fl32(max|X| / 2688) is computed and written to *s32;
  *   scale_given 1: *s32 is read.
  * Optional err_e2m1 / err_e1m2 ([rows][K/16]) receive each block's S.
  * Returns 0, or -1 on a non-finite input or K % 16 != 0. */
-int oracle_quantize(const uint16_t* x, int64_t rows, int64_t K, int64_t ldx,
-                    int mode, int scale_given, float* s32, uint8_t* codes,
-                    uint8_t* scales, float* err_e2m1, float* err_e1m2) {
+int oracle_quantize_f32(const float* x, int64_t rows, int64_t K, int64_t ldx,
+                        int mode, int scale_given, float* s32, uint8_t* codes,
+                        uint8_t* scales, float* err_e2m1, float* err_e1m2) {
   if (K % 16 != 0) return -1;
   float amax = 0.0f;
   for (int64_t r = 0; r < rows; ++r)
     for (int64_t k = 0; k < K; ++k) {
-      float v = bf16_to_float(x[r * ldx + k]);
+      float v = x[r * ldx + k];
       if (!isfinite(v)) return -1;
       if (fabsf(v) > amax) amax = fabsf(v);
     }
@@ -165,7 +178,7 @@ int oracle_quantize(const uint16_t* x, int64_t rows, int64_t K, int64_t ldx,
       float a[16], B = 0.0f;
       int sign[16];
       for (int i = 0; i < 16; ++i) {
-        float v = bf16_to_float(x[r * ldx + b * 16 + i]);
+        float v = x[r * ldx + b * 16 + i];
         sign[i] = signbit(v) ? 1 : 0;
         a[i] = (s > 0.0f) ? v / s : 0.0f;           /* X_FP8 = X / s32, R1, R7 */
         if (fabsf(a[i]) > B) B = fabsf(a[i]);       /* block-max(|X_FP8|) */
@@ -191,6 +204,46 @@ int oracle_quantize(const uint16_t* x, int64_t rows, int64_t K, int64_t ldx,
       if (err_e1m2) err_e1m2[r * nb + b] = S1;
     }
   }
+  return 0;
+}
+
+/* Algorithm 1 over a [rows][K] bf16 tensor (row stride ldx elements): the
+ * bf16 values are exact in fp32, so this is oracle_quantize_f32 on them. */
+int oracle_quantize(const uint16_t* x, int64_t rows, int64_t K, int64_t ldx,
+                    int mode, int scale_given, float* s32, uint8_t* codes,
+                    uint8_t* scales, float* err_e2m1, float* err_e1m2) {
+  if (K % 16 != 0) return -1;
+  float* xf = (float*)malloc((size_t)(rows > 0 ? rows : 1) * (size_t)(K > 0 ? K : 1) * sizeof(float));
+  if (!xf) return -1;
+  for (int64_t r = 0; r < rows; ++r)
+    for (int64_t k = 0; k < K; ++k) xf[r * K + k] = bf16_to_float(x[r * ldx + k]);
+  int rc = oracle_quantize_f32(xf, rows, K, K, mode, scale_given, s32, codes, scales, err_e2m1, err_e1m2);
+  free(xf);
+  return rc;
+}
+
+/* R11: the 128-point rotation of every chunk of a bf16 [rows][K] tensor
+ * (K % 128 == 0) into fp32 y [rows][K].  signs: 16 bytes, bit i (byte i/8,
+ * bit i%8) negates element i of every chunk; NULL for none. */
+int oracle_rht(const uint16_t* x, int64_t rows, int64_t K, int64_t ldx, const uint8_t* signs, float* y) {
+  if (K % 128 != 0) return -1;
+  const float c = (float)(1.0 / sqrt(128.0));     /* RN(1/sqrt(128)) = 0x3DB504F3 */
+  for (int64_t r = 0; r < rows; ++r)
+    for (int64_t k0 = 0; k0 < K; k0 += 128) {
+      float v[128];
+      for (int i = 0; i < 128; ++i) {
+        float xi = bf16_to_float(x[r * ldx + k0 + i]);
+        v[i] = (signs && ((signs[i >> 3] >> (i & 7)) & 1)) ? -xi : xi;
+      }
+      for (int h = 1; h < 128; h <<= 1)
+        for (int i = 0; i < 128; ++i)
+          if ((i & h) == 0) {
+            float a = v[i], b = v[i + h];
+            v[i] = a + b;
+            v[i + h] = a - b;
+          }
+      for (int i = 0; i < 128; ++i) y[r * K + k0 + i] = v[i] * c;
+    }
   return 0;
 }
 
