@@ -217,9 +217,14 @@ def run_ours(args):
 
     given_ms = time_quant(lambda: ops.mixfp4_quantize(xs, out=qs, tensor_scale=given))
     sweep_ms = time_quant(lambda: ops.mixfp4_quantize(xs, out=qs, workspace=ws))
+    ops.mixfp4_quantize_rht(xs, out=qs, workspace=ws)
+    given_rht = qs.tensor_scale.clone()
+    rht_given_ms = time_quant(lambda: ops.mixfp4_quantize_rht(xs, out=qs, tensor_scale=given_rht))
+    rht_ms = time_quant(lambda: ops.mixfp4_quantize_rht(xs, out=qs, workspace=ws))
     given_gbs = xs.numel() * QUANT_BYTES_PER_ELEM / (given_ms * 1e-3) / 1e9
     sweep_alg_gbs = xs.numel() * QUANT_BYTES_PER_ELEM / (sweep_ms * 1e-3) / 1e9
     sweep_read_gbs = xs.numel() * (QUANT_BYTES_PER_ELEM + 2.0) / (sweep_ms * 1e-3) / 1e9
+    xs_numel = xs.numel()
     del xs, qs
 
     # End to end through the public API with host buffers: pinned X in, C out.
@@ -275,7 +280,14 @@ def run_ours(args):
                 "with_amax_pass": {"ms": round(sweep_ms, 4), "alg_gbs": round(sweep_alg_gbs, 1),
                                    "alg_frac_of_hbm": round(sweep_alg_gbs / pk["hbm_gbs"], 4),
                                    "bytes_incl_amax_read_gbs": round(sweep_read_gbs, 1)},
-                "alg_bytes_per_element": QUANT_BYTES_PER_ELEM, "hbm_peak_gbs": pk["hbm_gbs"]}},
+                "alg_bytes_per_element": QUANT_BYTES_PER_ELEM, "hbm_peak_gbs": pk["hbm_gbs"]},
+            "rht_quantizer_2^28": {
+                "fused_rotation_quantize_given_scale": {
+                    "ms": round(rht_given_ms, 4),
+                    "alg_gbs": round(xs_numel * QUANT_BYTES_PER_ELEM / (rht_given_ms * 1e-3) / 1e9, 1)},
+                "with_amax_pass": {
+                    "ms": round(rht_ms, 4),
+                    "alg_gbs": round(xs_numel * QUANT_BYTES_PER_ELEM / (rht_ms * 1e-3) / 1e9, 1)}}},
         "clocks": clocks,
         "e2e": {"value": round(e2e_value, 2), "unit": "TFLOP/s",
                 "h2d_bytes_per_step": x_host.numel() * 2, "d2h_bytes_per_step": c_host.numel() * 4,
@@ -389,6 +401,9 @@ def run_kernel_only(args):
     elif args.kernel == "quantize":
         fn = lambda: ops.mixfp4_quantize(x, out=qx, workspace=ws)
         work = x.numel() * QUANT_BYTES_PER_ELEM
+    elif args.kernel == "quantize_rht":
+        fn = lambda: ops.mixfp4_quantize_rht(x, out=qx, workspace=ws)
+        work = x.numel() * QUANT_BYTES_PER_ELEM
     else:
         out = torch.empty(x.shape, dtype=torch.float32, device=dev)
         fn = lambda: ops.mixfp4_dequantize(qx, out=out)
@@ -417,7 +432,7 @@ def main(argv=None):
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--cpu-budget", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--kernel", choices=["gemm", "quantize", "dequantize"], default=None,
+    ap.add_argument("--kernel", choices=["gemm", "quantize", "quantize_rht", "dequantize"], default=None,
                     help="profiling mode: launch only this kernel")
     ap.add_argument("--workload", default=WORKLOAD,
                     help="tiny|attn|mlp|decode|hadamard|sweepNN (kernel-only mode)")

@@ -85,6 +85,31 @@ int mixfp4_quantize(const void* x, int dtype, int64_t rows, int64_t K, int64_t l
                     uint32_t* workspace, int mode, int scale_flag, void* stream);
 
 /*
+ * mixfp4_quantize_rht -- the 128-point Walsh-Hadamard rotation applied before
+ * quantization (the random Hadamard transform of Sec. 4 "+RHT" and the
+ * Sec. 3.4 training flow), fused with Algorithm 1 (as mixfp4_quantize).
+ *
+ *   every 128-element chunk of a row along K, on its own:
+ *     v_i = -x_i if bit i of `signs` is set, else x_i        (i = 0..127)
+ *     v   = H_128 v   (Sylvester order) by the radix-2 butterfly in fp32,
+ *                     strides 1, 2, 4, ..., 64 in that order, (a, b) -> (a+b, a-b)
+ *     y_i = fl32(v_i * c),  c = RN(1/sqrt(128))
+ *   then Algorithm 1 on the fp32 tensor y (s32 = fl32(max|y| / 2688) with
+ *   SCALE_COMPUTE; x_i / s32 is the IEEE quotient of the fp32 y_i).
+ * The paper fixes no arithmetic for the rotation; this order is the one used
+ * (and checked bit for bit) here.
+ *
+ * signs        device, 16 bytes (bit i = byte i/8, bit i%8: negate chunk
+ *              element i), the same for every chunk; NULL for no negation
+ *              (the plain normalised Walsh-Hadamard transform).
+ * rows, K      as mixfp4_quantize, and K % 128 == 0 (else MIXFP4_ERR_SHAPE).
+ * Other arguments and the error behaviour are those of mixfp4_quantize.
+ */
+int mixfp4_quantize_rht(const void* x, int dtype, int64_t rows, int64_t K, int64_t ldx, const uint8_t* signs,
+                        uint8_t* codes, uint8_t* scales, float* tensor_scale, uint32_t* workspace, int mode,
+                        int scale_flag, void* stream);
+
+/*
  * mixfp4_dequantize -- App. B.2/B.3 decode:
  *   out[r][k] = fl32((-1)^s * v(T, p) * ue4m3(scale & 0x7F) * s32),
  * one rounding of the exact product.

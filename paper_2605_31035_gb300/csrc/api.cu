@@ -63,6 +63,36 @@ int mixfp4_quantize(const void* x, int dtype, int64_t rows, int64_t K, int64_t l
   return launch_status();
 }
 
+int mixfp4_quantize_rht(const void* x, int dtype, int64_t rows, int64_t K, int64_t ldx, const uint8_t* signs,
+                        uint8_t* codes, uint8_t* scales, float* tensor_scale, uint32_t* workspace, int mode,
+                        int scale_flag, void* stream) {
+  if (dtype != MIXFP4_DTYPE_BF16) return MIXFP4_ERR_DTYPE;
+  if (mode < MIXFP4_MODE_MIX || mode > MIXFP4_MODE_E1M2_ONLY) return MIXFP4_ERR_ARG;
+  if (scale_flag != MIXFP4_SCALE_COMPUTE && scale_flag != MIXFP4_SCALE_GIVEN) return MIXFP4_ERR_ARG;
+  if (rows < 0 || K < 0 || K % 128 != 0 || ldx < K) return MIXFP4_ERR_SHAPE;
+  if (!tensor_scale) return MIXFP4_ERR_NULL;
+  if (scale_flag == MIXFP4_SCALE_COMPUTE && !workspace) return MIXFP4_ERR_NULL;
+  const bool empty = (rows == 0 || K == 0);
+  if (!empty && (!x || !codes || !scales)) return MIXFP4_ERR_NULL;
+  if (!empty && (!aligned(x, 32) || ldx % 16 != 0 || !aligned(codes, 8))) return MIXFP4_ERR_ALIGN;
+  if (!aligned(tensor_scale, 4) || (workspace && !aligned(workspace, 4))) return MIXFP4_ERR_ALIGN;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const int given = scale_flag == MIXFP4_SCALE_GIVEN;
+  if (empty) {
+    if (!given && cudaMemsetAsync(tensor_scale, 0, sizeof(float), s) != cudaSuccess)
+      return MIXFP4_ERR_CUDA;
+    return MIXFP4_OK;
+  }
+  const uint16_t* xb = static_cast<const uint16_t*>(x);
+  if (!given) {
+    if (cudaMemsetAsync(workspace, 0, sizeof(uint32_t), s) != cudaSuccess) return MIXFP4_ERR_CUDA;
+    mixfp4::launch_rht_amax(xb, rows, K, ldx, signs, workspace, s);
+    if (int st = launch_status()) return st;
+  }
+  mixfp4::launch_rht_quantize(xb, rows, K, ldx, signs, codes, scales, tensor_scale, workspace, mode, given, s);
+  return launch_status();
+}
+
 int mixfp4_dequantize(const uint8_t* codes, const uint8_t* scales, const float* tensor_scale,
                       int64_t rows, int64_t K, float* out, void* stream) {
   if (rows < 0 || K < 0 || K % 16 != 0) return MIXFP4_ERR_SHAPE;

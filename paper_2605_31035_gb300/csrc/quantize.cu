@@ -135,6 +135,13 @@ __device__ __forceinline__ uint32_t sign_bits(uint32_t w0, uint32_t w1, uint32_t
 // < 7.5 and RNE never exceeds 7; only other blocks need the clamp.
 // kMarkstein selects the x / s32 method (see the header); the other divisions
 // always take the two-instruction form.
+// Algorithm 1 from X_FP8 on, for one 16-element block: a holds |X_FP8| =
+// |x| / s32 as packed pairs (element 2j in the low lane).  Returns the code
+// words without their sign bits and the scale byte.
+template <int kMode>
+__device__ __forceinline__ void block_core(const u64 a[8], const TensorConsts& tc, const float4* __restrict__ tab,
+                                           uint32_t& mag_lo, uint32_t& mag_hi, uint32_t& scale_byte);
+
 template <int kMode, bool kScaled, bool kMarkstein>
 __device__ __forceinline__ void quantize_block(const uint32_t w[8], const TensorConsts& tc,
                                                const float4* __restrict__ tab, uint32_t& code_lo,
@@ -154,6 +161,15 @@ __device__ __forceinline__ void quantize_block(const uint32_t w[8], const Tensor
     // X_FP8 = X / s32 (magnitudes)
     a[j] = kMarkstein ? div_rn2(bits2(lo, hi), ns32, r32) : div_kd2(bits2(lo, hi), zh32, zl32);
   }
+  uint32_t mlo, mhi;
+  block_core<kMode>(a, tc, tab, mlo, mhi, scale_byte);
+  code_lo = mlo | sign_bits(w[0], w[1], w[2], w[3]);
+  code_hi = mhi | sign_bits(w[4], w[5], w[6], w[7]);
+}
+
+template <int kMode>
+__device__ __forceinline__ void block_core(const u64 a[8], const TensorConsts& tc, const float4* __restrict__ tab,
+                                           uint32_t& mag_lo, uint32_t& mag_hi, uint32_t& scale_byte) {
   // Block max of |X_FP8|.
   float v[16];
 #pragma unroll
@@ -241,8 +257,8 @@ __device__ __forceinline__ void quantize_block(const uint32_t w[8], const Tensor
   else if (kMode == MIXFP4_MODE_E1M2_ONLY) T = 1;
   else T = (S2 < S1) ? 0 : 1;  // strict "<" of Algorithm 1
 
-  code_lo = (T ? p1lo : p2lo) | sign_bits(w[0], w[1], w[2], w[3]);
-  code_hi = (T ? p1hi : p2hi) | sign_bits(w[4], w[5], w[6], w[7]);
+  mag_lo = T ? p1lo : p2lo;
+  mag_hi = T ? p1hi : p2hi;
   scale_byte = T ? (0x80u | c1) : c2;
 }
 
@@ -312,6 +328,166 @@ quantize_kernel(const uint16_t* __restrict__ x, int64_t nblocks, int64_t kblocks
       if (b1 + 2 * nthr < nblocks) ldg256_stream(block_src<kContig>(x, b1 + 2 * nthr, kblocks, ldx), wb);
     }
   }
+}
+
+// ---- 128-point Walsh-Hadamard rotation before quantization ----------------
+// Reading R11 of the random Hadamard transform (Sec. 4 "+RHT", Sec. 3.4): each
+// 128-element chunk of a row along K is rotated on its own: elements whose bit
+// in the caller's 128-bit sign vector is set are negated, the Sylvester
+// product H_128 v is formed by the radix-2 butterfly in fp32 with strides
+// 1, 2, 4, ..., 64 in that order ((a, b) -> (a + b, a - b)), and every value
+// is multiplied by c = RN(1/sqrt(128)).  Algorithm 1 then runs on the fp32
+// values.  Threads hold one 16-element block each, so the 8 lanes 8g..8g+7 of
+// a warp hold one chunk (block t of the chunk on lane 8g + t): strides 1-8 run
+// inside a thread, strides 16, 32, 64 between lanes by shuffles.
+constexpr uint32_t kRhtScaleBits = 0x3DB504F3u;  // RN(1/sqrt(128))
+
+// Sign masks of this thread's 16 chunk positions 16 * (lane & 7) + e, as bf16
+// word masks (bit 15: element 2j, bit 31: element 2j + 1).
+__device__ __forceinline__ void rht_sign_words(const uint8_t* __restrict__ signs, int lane, uint32_t sw[8]) {
+  uint32_t bits = 0;
+  if (signs) {
+    const int pos = lane & 7;
+    bits = (uint32_t)__ldg(signs + 2 * pos) | ((uint32_t)__ldg(signs + 2 * pos + 1) << 8);
+  }
+#pragma unroll
+  for (int j = 0; j < 8; ++j) sw[j] = (((bits >> (2 * j)) & 1u) << 15) | (((bits >> (2 * j + 1)) & 1u) << 31);
+}
+
+// The rotated block of this thread as packed fp32 pairs (element 2j low).
+// Every lane of the 8-lane group must call this together.
+__device__ __forceinline__ void rht_rotate(const uint32_t w[8], const uint32_t sw[8], int lane, u64 y[8]) {
+#pragma unroll
+  for (int j = 0; j < 8; ++j) {
+    const uint32_t u = w[j] ^ sw[j];
+    const float lo = __uint_as_float(u << 16), hi = __uint_as_float(u & 0xFFFF0000u);
+    y[j] = pack2(__fadd_rn(lo, hi), __fsub_rn(lo, hi));  // stride 1
+  }
+#pragma unroll
+  for (int h = 1; h < 8; h <<= 1)  // strides 2, 4, 8 (h pairs apart)
+#pragma unroll
+    for (int j = 0; j < 8; ++j)
+      if ((j & h) == 0) {
+        const u64 a = y[j], b = y[j + h];
+        y[j] = add2(a, b);
+        y[j + h] = sub2(a, b);
+      }
+  const unsigned gmask = 0xFFu << (lane & 24);
+#pragma unroll
+  for (int m = 1; m < 8; m <<= 1) {  // strides 16, 32, 64: partner lane ^ m
+    // lower lane: own + other; upper lane: other - own (fma with -1 rounds the same)
+    const float k = (lane & m) ? -1.0f : 1.0f;
+    const u64 kk = pack2(k, k);
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      const uint32_t olo = __shfl_xor_sync(gmask, lo32(y[j]), m);
+      const uint32_t ohi = __shfl_xor_sync(gmask, hi32(y[j]), m);
+      y[j] = fma2(y[j], kk, bits2(olo, ohi));
+    }
+  }
+  const float c = __uint_as_float(kRhtScaleBits);
+  const u64 cc = pack2(c, c);
+#pragma unroll
+  for (int j = 0; j < 8; ++j) y[j] = mul2(y[j], cc);
+}
+
+// Sign nibble bits of 8 fp32 values held in 4 pairs: element 2j -> bit 3 of
+// byte j, element 2j + 1 -> bit 7.
+__device__ __forceinline__ uint32_t f32_sign_bits(const u64 y[4]) {
+  const uint32_t e = prmt(prmt(lo32(y[0]), lo32(y[1]), 0x0073u), prmt(lo32(y[2]), lo32(y[3]), 0x0073u), 0x5410u);
+  const uint32_t o = prmt(prmt(hi32(y[0]), hi32(y[1]), 0x0073u), prmt(hi32(y[2]), hi32(y[3]), 0x0073u), 0x5410u);
+  return (o & 0x80808080u) | ((e >> 4) & 0x08080808u);
+}
+
+// Algorithm 1 on one rotated block: x / s32 for fp32 numerators by
+// Markstein's correction (correctly rounded for every fp32 numerator down to
+// the tiny-value bound, see the header), then the common core.
+template <int kMode, bool kScaled>
+__device__ __forceinline__ void rht_block(const u64 y[8], const TensorConsts& tc, const float4* __restrict__ tab,
+                                          uint32_t& code_lo, uint32_t& code_hi, uint32_t& scale_byte) {
+  u64 a[8];
+  const u64 ns32 = pack2(-tc.s32, -tc.s32), r32 = pack2(tc.r32, tc.r32);
+#pragma unroll
+  for (int j = 0; j < 8; ++j) {
+    uint32_t lo = lo32(y[j]) & 0x7FFFFFFFu, hi = hi32(y[j]) & 0x7FFFFFFFu;
+    if (kScaled) {
+      lo = __float_as_uint(scalbnf(__uint_as_float(lo), tc.k));
+      hi = __float_as_uint(scalbnf(__uint_as_float(hi), tc.k));
+    }
+    a[j] = div_rn2(bits2(lo, hi), ns32, r32);
+  }
+  uint32_t mlo, mhi;
+  block_core<kMode>(a, tc, tab, mlo, mhi, scale_byte);
+  code_lo = mlo | f32_sign_bits(y);
+  code_hi = mhi | f32_sign_bits(y + 4);
+}
+
+// Rotation + Algorithm 1.  One block per thread per iteration; the grid
+// stride is a multiple of 8 blocks, so the 8 lanes of a chunk stay together.
+template <int kMode, bool kContig>
+__global__ void __launch_bounds__(kQuantThreads, 3)
+rht_quantize_kernel(const uint16_t* __restrict__ x, int64_t nblocks, int64_t kblocks, int64_t ldx,
+                    const uint8_t* __restrict__ signs, uint8_t* __restrict__ codes, uint8_t* __restrict__ scales,
+                    float* tensor_scale, const uint32_t* amax_word, int scale_given, int after_amax) {
+  __shared__ float4 tab[128];
+  if (!after_amax) griddep_wait();
+  griddep_launch_dependents();
+  const int lane = threadIdx.x & 31;
+  const int64_t nthr = (int64_t)gridDim.x * kQuantThreads;
+  int64_t b = (int64_t)blockIdx.x * kQuantThreads + threadIdx.x;
+  uint32_t w[8];
+  if (b < nblocks) ldg256_stream(block_src<kContig>(x, b, kblocks, ldx), w);
+  if (threadIdx.x < 128) {
+    float s8 = 0.0f, unused;
+    if (threadIdx.x < 0x7F) f16x2_to_f32(cvt_f16x2_from_e4m3x2((uint16_t)threadIdx.x), s8, unused);
+    const float2 kd = kd_consts(s8);
+    tab[threadIdx.x] = make_float4(s8, kd.x, kd.y, 0.0f);
+  }
+  uint32_t sw[8];
+  rht_sign_words(signs, lane, sw);
+  if (after_amax) griddep_wait();
+  const TensorConsts tc = tensor_consts(tensor_scale, amax_word, scale_given);
+  __syncthreads();
+  for (; b < nblocks; b += nthr) {
+    u64 y[8];
+    rht_rotate(w, sw, lane, y);
+    if (b + nthr < nblocks) ldg256_stream(block_src<kContig>(x, b + nthr, kblocks, ldx), w);
+    uint32_t lo, hi, sb;
+    if (tc.scaled) rht_block<kMode, true>(y, tc, tab, lo, hi, sb);
+    else rht_block<kMode, false>(y, tc, tab, lo, hi, sb);
+    stg64(codes + b * 8, lo, hi);
+    scales[b] = (uint8_t)sb;
+  }
+}
+
+// max |y| of the rotated tensor as the bit pattern of a non-negative fp32.
+template <bool kContig>
+__global__ void __launch_bounds__(256)
+rht_amax_kernel(const uint16_t* __restrict__ x, int64_t nblocks, int64_t kblocks, int64_t ldx,
+                const uint8_t* __restrict__ signs, uint32_t* amax_word) {
+  const int lane = threadIdx.x & 31;
+  uint32_t sw[8];
+  rht_sign_words(signs, lane, sw);
+  uint32_t m = 0;
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t b = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; b < nblocks; b += stride) {
+    uint32_t w[8];
+    ldg256_stream(block_src<kContig>(x, b, kblocks, ldx), w);
+    u64 y[8];
+    rht_rotate(w, sw, lane, y);
+#pragma unroll
+    for (int j = 0; j < 8; ++j) m = max(m, max(lo32(y[j]) & 0x7FFFFFFFu, hi32(y[j]) & 0x7FFFFFFFu));
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) m = max(m, __shfl_xor_sync(0xffffffffu, m, o));
+  __shared__ uint32_t red[8];
+  if (lane == 0) red[threadIdx.x >> 5] = m;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    for (int i = 1; i < (int)(blockDim.x >> 5); ++i) m = max(m, red[i]);
+    if (m) atomicMax(amax_word, m);
+  }
+  griddep_launch_dependents();
 }
 
 // max |x| over the tensor as the bit pattern of a non-negative fp32 (bf16
@@ -434,6 +610,43 @@ int launch_quantize(const uint16_t* x, int64_t rows, int64_t K, int64_t ldx, uin
     default: MIXFP4_LAUNCH_Q(MIXFP4_MODE_E1M2_ONLY); break;
   }
 #undef MIXFP4_LAUNCH_Q
+  return 0;
+}
+
+int launch_rht_amax(const uint16_t* x, int64_t rows, int64_t K, int64_t ldx, const uint8_t* signs,
+                    uint32_t* amax_word, cudaStream_t stream) {
+  const int64_t kblocks = K / 16, nblocks = rows * kblocks;
+  if (nblocks == 0) return 0;
+  int64_t grid = (nblocks + 255) / 256;
+  if (grid > 152 * 8) grid = 152 * 8;
+  if (ldx == K) rht_amax_kernel<true><<<(unsigned)grid, 256, 0, stream>>>(x, nblocks, kblocks, ldx, signs, amax_word);
+  else rht_amax_kernel<false><<<(unsigned)grid, 256, 0, stream>>>(x, nblocks, kblocks, ldx, signs, amax_word);
+  return 0;
+}
+
+int launch_rht_quantize(const uint16_t* x, int64_t rows, int64_t K, int64_t ldx, const uint8_t* signs,
+                        uint8_t* codes, uint8_t* scales, float* tensor_scale, const uint32_t* amax_word, int mode,
+                        int scale_given, cudaStream_t stream) {
+  const int64_t kblocks = K / 16, nblocks = rows * kblocks;
+  int64_t grid = (nblocks + kQuantThreads - 1) / kQuantThreads;
+  if (grid > 152 * 3) grid = 152 * 3;
+  if (grid == 0) return 0;
+  const int after_amax = !scale_given;
+#define MIXFP4_LAUNCH_R(MODE)                                                                            \
+  do {                                                                                                   \
+    if (ldx == K)                                                                                        \
+      launch_pdl(rht_quantize_kernel<MODE, true>, (unsigned)grid, kQuantThreads, 0, stream, x, nblocks,   \
+                 kblocks, ldx, signs, codes, scales, tensor_scale, amax_word, scale_given, after_amax);  \
+    else                                                                                                 \
+      launch_pdl(rht_quantize_kernel<MODE, false>, (unsigned)grid, kQuantThreads, 0, stream, x, nblocks,  \
+                 kblocks, ldx, signs, codes, scales, tensor_scale, amax_word, scale_given, after_amax);  \
+  } while (0)
+  switch (mode) {
+    case MIXFP4_MODE_MIX: MIXFP4_LAUNCH_R(MIXFP4_MODE_MIX); break;
+    case MIXFP4_MODE_E2M1_ONLY: MIXFP4_LAUNCH_R(MIXFP4_MODE_E2M1_ONLY); break;
+    default: MIXFP4_LAUNCH_R(MIXFP4_MODE_E1M2_ONLY); break;
+  }
+#undef MIXFP4_LAUNCH_R
   return 0;
 }
 

@@ -40,6 +40,8 @@ def lib() -> ctypes.CDLL:
         P, I64, I = ctypes.c_void_p, ctypes.c_int64, ctypes.c_int
         L.mixfp4_quantize.restype = I
         L.mixfp4_quantize.argtypes = [P, I, I64, I64, I64, P, P, P, P, I, I, P]
+        L.mixfp4_quantize_rht.restype = I
+        L.mixfp4_quantize_rht.argtypes = [P, I, I64, I64, I64, P, P, P, P, P, I, I, P]
         L.mixfp4_dequantize.restype = I
         L.mixfp4_dequantize.argtypes = [P, P, P, I64, I64, P, P]
         L.mixfp4_gemm.restype = I
@@ -109,6 +111,29 @@ def mixfp4_quantize(x: torch.Tensor, mode: int = MODE_MIX, tensor_scale: torch.T
                                _ptr(q.tensor_scale), _ptr(ws), int(mode),
                                SCALE_GIVEN if given else SCALE_COMPUTE, _stream(stream))
     _check("mixfp4_quantize", st)
+    return q
+
+
+def mixfp4_quantize_rht(x: torch.Tensor, signs: torch.Tensor | None = None, mode: int = MODE_MIX,
+                        tensor_scale: torch.Tensor | None = None, out: QTensor | None = None,
+                        workspace: torch.Tensor | None = None, stream=None) -> QTensor:
+    """Rotate every 128-element chunk of each row of a bf16 [rows, K] CUDA tensor
+    (sign flips from the 16-byte `signs`, then the normalised Walsh-Hadamard
+    transform) and quantize the result; K % 128 == 0."""
+    assert x.dtype == torch.bfloat16 and x.dim() == 2 and x.stride(1) == 1
+    assert signs is None or (signs.dtype == torch.uint8 and signs.numel() == 16 and signs.is_contiguous())
+    rows, K = x.shape
+    q = out if out is not None else empty_qtensor(rows, K, x.device)
+    given = tensor_scale is not None
+    if given:
+        q.tensor_scale.copy_(tensor_scale.reshape(1))
+    ws = None
+    if not given:
+        ws = workspace if workspace is not None else torch.empty(1, dtype=torch.int32, device=x.device)
+    st = lib().mixfp4_quantize_rht(_ptr(x), DTYPE_BF16, rows, K, x.stride(0), _ptr(signs), _ptr(q.codes),
+                                   _ptr(q.scales), _ptr(q.tensor_scale), _ptr(ws), int(mode),
+                                   SCALE_GIVEN if given else SCALE_COMPUTE, _stream(stream))
+    _check("mixfp4_quantize_rht", st)
     return q
 
 

@@ -53,6 +53,17 @@ def test_quantize_validation(lib):
     assert q(fake, 0, 4, 32, 40, fake, fake, fake, ws, 0, 1, None) == -3        # ldx % 16
 
 
+def test_quantize_rht_validation(lib):
+    fake = ctypes.c_void_p(1 << 20)
+    ws = ctypes.c_void_p(1 << 21)
+    q = lib.mixfp4_quantize_rht
+    assert q(fake, 0, 4, 64, 64, None, fake, fake, fake, ws, 0, 0, None) == -2       # K % 128
+    assert q(fake, 7, 4, 128, 128, None, fake, fake, fake, ws, 0, 0, None) == -4     # dtype
+    assert q(fake, 0, 4, 128, 128, None, fake, fake, fake, None, 0, 0, None) == -1   # workspace
+    assert q(fake, 0, 4, 128, 128, None, fake, fake, fake, ws, 5, 0, None) == -7     # mode
+    assert q(ctypes.c_void_p((1 << 20) + 2), 0, 4, 128, 128, None, fake, fake, fake, ws, 0, 0, None) == -3
+
+
 def test_dequantize_and_gemm_validation(lib):
     fake = ctypes.c_void_p(1 << 20)
     assert lib.mixfp4_dequantize(fake, fake, fake, 4, 24, fake, None) == -2
