@@ -178,6 +178,21 @@ const char* mixfp4_status_string(int status);
 /* ABI version of this library (major * 100 + minor). */
 int mixfp4_version(void);
 
+/*
+ * mixfp4_selftest_bounded_wait -- check of the failure detection in the GEMM
+ * pipelines (no counterpart in the paper): one CTA waits with the same
+ * bounded mbarrier wait the GEMM kernels use on (a) a barrier whose phase
+ * completes, (b) a barrier nothing arrives on (an injected missed arrival)
+ * and (c) that barrier with its abort flag raised, and ORs into *status_word:
+ * bit 0 if (a) failed, bit 1 if (b) gave up, bit 2 if (b) gave up only after
+ * limit_ns, bit 3 if (c) gave up.  A healthy device reports 0xE.
+ *
+ * status_word  device, one uint32, 4-byte aligned (the caller zeroes it).
+ * limit_ns     1 .. 2e9 (else MIXFP4_ERR_ARG).  The call occupies one SM for
+ *              about limit_ns; it does not fault or trap.
+ */
+int mixfp4_selftest_bounded_wait(uint32_t* status_word, uint64_t limit_ns, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

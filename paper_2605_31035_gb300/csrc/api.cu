@@ -132,3 +132,11 @@ int mixfp4_gemm(const uint8_t* a_codes, const uint8_t* a_scales, const float* a_
 }
 
 }  // extern "C"
+
+int mixfp4_selftest_bounded_wait(uint32_t* status_word, uint64_t limit_ns, void* stream) {
+  if (!status_word) return MIXFP4_ERR_NULL;
+  if (!aligned(status_word, 4)) return MIXFP4_ERR_ALIGN;
+  if (limit_ns == 0 || limit_ns > 2000000000ull) return MIXFP4_ERR_ARG;
+  mixfp4::launch_bounded_wait_selftest(status_word, limit_ns, static_cast<cudaStream_t>(stream));
+  return launch_status();
+}

@@ -533,48 +533,48 @@ mixfp4_gemm_kernel(const __grid_constant__ CUtensorMap tm_ac, const __grid_const
 }
 
 // ============================================================================
-// Skinny-M path (M <= 64 activation rows, e.g. decoding): the roles of the
-// operands are swapped so the weight rows fill the 128-row MMA dimension and
-// every weight element is decoded exactly once:
-//   D^T[n][m] = sum_k W[n][k] X[m][k],  M_mma = 128 weight rows (A operand,
-//   decoded into TMEM), N_mma = X rows rounded up to 16 (B operand, decoded
-//   into shared memory), cta_group::1.
-// Work = (weight tile, 256-wide K slice) units, split evenly over all CTAs
-// (stream-K), so no SM idles; each CTA adds its partial tiles into C with
-// red.global.add (C is zeroed first), so bits depend on the summation order
-// but every result is within the fp32-accumulation bound.
+// Few-row path (M <= 64 activation rows, e.g. decoding).  A tcgen05.mma of
+// M = 128, K = 16 costs a fixed ~65 ns whatever its N, so the weight rows go
+// on the wide side: D[m][n] = sum_k X[m][k] W[n][k] with M_mma = 128 (the X
+// rows, A operand decoded into TMEM; lanes past the X rows hold values that
+// are never stored) and N_mma = 256 weight rows (B operand decoded into
+// shared memory), cta_group::1.  Every weight element is decoded once.
+// Work = (weight tile of 256 rows, 256-wide K slice) units split evenly over
+// all CTAs (stream-K); each CTA adds its partial tiles into C (zeroed first)
+// with red.global.add, so bits depend on the summation order but every result
+// is within the fp32-accumulation bound.
 // Per CTA: warp 0 TMA, warp 1 TMEM allocator + MMA thread, warps 2-17 weight
-// decoders (four threads per row, lane quarter = warp % 4), warps 18-21 X
-// decoders (two threads per row), warps 22-25 epilogue.
+// decoders (two threads per weight row, one 32-code chunk each per stage),
+// warps 18-21 X decoders (warp % 4 = TMEM lane quarter = 32 X rows), warps
+// 22-25 epilogue.
 // ============================================================================
 namespace skinny {
 
-constexpr int BW = 128;                        // weight rows per tile (MMA M)
-constexpr int MXMAX = 64;                      // max activation rows (MMA N)
-constexpr int BKC = 256, BKD = 128, kSub = BKC / BKD;
-constexpr int kCodeStages = 4, kDecStages = 4;
-constexpr int kTPRW = 4, kTPRX = 2;
-constexpr int kWarpsW = kTPRW * BW / 32;       // 16
-constexpr int kWarpsX = kTPRX * MXMAX / 32;    // 4
+constexpr int BN = 256;                          // weight rows per tile (MMA N)
+constexpr int MXMAX = 64;                        // max activation rows (MMA M is 128)
+constexpr int BKC = 256, BKD = 64, kSub = BKC / BKD;
+constexpr int kCodeStages = 2, kDecStages = 4;
+constexpr int kWarpsW = 2 * BN / 32;             // 16
+constexpr int kWarpsX = 4;
 constexpr int kFirstW = 2, kFirstX = kFirstW + kWarpsW, kFirstEpi = kFirstX + kWarpsX;  // 2, 18, 22
 constexpr int kEpiWarps = 4;
 constexpr int kThreads = 32 * (kFirstEpi + kEpiWarps);  // 832
-static_assert(kFirstW % 4 == 2, "weight decoders start at lane quarter 2");
-constexpr int W_CODE = BW * BKC / 2, X_CODE = MXMAX * BKC / 2;
-constexpr int W_SCALE = BW * BKC / 16, X_SCALE = MXMAX * BKC / 16;
+static_assert(kFirstX % 4 == 2 && kFirstEpi % 4 == 2, "warp w covers TMEM lane quarter w % 4");
+constexpr int W_CODE = BN * BKC / 2, X_CODE = MXMAX * BKC / 2;
+constexpr int W_SCALE = BN * BKC / 16, X_SCALE = MXMAX * BKC / 16;
 constexpr int OFF_XC = W_CODE, OFF_WS = OFF_XC + X_CODE, OFF_XS = OFF_WS + W_SCALE;
 constexpr int CODE_STAGE = OFF_XS + X_SCALE;
-constexpr int X_DEC = MXMAX * BKD * 2;
+constexpr int W_DEC = BN * BKD * 2;
 constexpr int OFF_DEC = kCodeStages * CODE_STAGE;
-constexpr int OFF_BAR = OFF_DEC + kDecStages * X_DEC;
+constexpr int OFF_BAR = OFF_DEC + kDecStages * W_DEC;
 constexpr int SMEM_ALLOC = OFF_BAR + 256 + 1024;
 static_assert(CODE_STAGE % 1024 == 0 && OFF_XC % 1024 == 0, "swizzled TMA tiles need 1024-byte alignment");
 static_assert(SMEM_ALLOC <= 232448, "shared memory budget");
-constexpr uint32_t kAccCols = MXMAX;            // accumulator columns (N_mma <= 64)
-constexpr uint32_t kWStageCols = BKD / 2;
+constexpr uint32_t kAccCols = BN;                // fp32 accumulator (lanes = X rows)
+constexpr uint32_t kXStageCols = BKD / 2;        // f16 pairs per X row per stage
 constexpr uint32_t kTmemCols = 512;
-static_assert(kAccCols + kDecStages * kWStageCols <= kTmemCols, "TMEM budget");
-constexpr uint32_t kLBO = 128, kSBO = (BKD / 8) * 128;
+static_assert(kAccCols + kDecStages * kXStageCols <= kTmemCols, "TMEM budget");
+constexpr uint32_t kLBO = 128, kSBO = (BKD / 8) * 128;  // decoded W: next 8 K / next 8 rows
 
 struct Bars {
   uint64_t code_full[kCodeStages];
@@ -601,10 +601,10 @@ mixfp4_gemm_skinny_kernel(const __grid_constant__ CUtensorMap tm_wc, const __gri
   const uint32_t sbase = smem_u32(smem);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int num_kc = K / BKC;
-  const int nmma = (Mx + 15) & ~15;
-  const long long units = (long long)((N + BW - 1) / BW) * num_kc;
+  const int nx = (Mx + 15) & ~15;  // X rows fetched
+  const long long units = (long long)((N + BN - 1) / BN) * num_kc;
   const long long u_begin = units * blockIdx.x / gridDim.x, u_end = units * (blockIdx.x + 1) / gridDim.x;
-  const uint32_t stage_bytes = W_CODE + W_SCALE + (uint32_t)nmma * (BKC / 2 + BKC / 16);
+  const uint32_t stage_bytes = W_CODE + W_SCALE + (uint32_t)nx * (BKC / 2 + BKC / 16);
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kCodeStages; ++s) {
@@ -629,7 +629,7 @@ mixfp4_gemm_skinny_kernel(const __grid_constant__ CUtensorMap tm_wc, const __gri
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = bars->tmem_base;
-  const uint32_t tmem_w0 = tmem_base + kAccCols;
+  const uint32_t tmem_x0 = tmem_base + kAccCols;
 
   auto fail = [&](uint32_t code) {
     *abort_flag = 1;
@@ -657,9 +657,9 @@ mixfp4_gemm_skinny_kernel(const __grid_constant__ CUtensorMap tm_wc, const __gri
         const uint32_t fb = smem_u32(&bars->code_full[s]);
         mbar_arrive_expect_tx(fb, stage_bytes);
         const int xk = kc * (BKC / 2), xs = kc * (BKC / 16);
-        tma_load_2d(st, &tm_wc, xk, wt * BW, fb);
+        tma_load_2d(st, &tm_wc, xk, wt * BN, fb);
         tma_load_2d(st + OFF_XC, &tm_xc, xk, 0, fb);
-        tma_load_2d(st + OFF_WS, &tm_ws, xs, wt * BW, fb);
+        tma_load_2d(st + OFF_WS, &tm_ws, xs, wt * BN, fb);
         tma_load_2d(st + OFF_XS, &tm_xs, xs, 0, fb);
         last = it;
       }
@@ -675,9 +675,9 @@ mixfp4_gemm_skinny_kernel(const __grid_constant__ CUtensorMap tm_wc, const __gri
       int d = 0, ntile = 0;
       uint32_t dph = 0;
       bool ok = true;
-      // Descriptor of decoded stage 0, first 16-K step; other stages and steps
-      // only move the start address (14-bit field in 16-byte units, no carry:
-      // shared addresses stay below 256 KiB).
+      // Descriptor of decoded-W stage 0, first 16-K step; other stages and
+      // steps only move the start address (14-bit field in 16-byte units, no
+      // carry: shared addresses stay below 256 KiB).
       const uint64_t bdesc0 = smem_desc_noswizzle(sbase + OFF_DEC, kLBO, kSBO);
       for (long long u = u_begin; u < u_end && ok;) {
         const int wt = (int)(u / num_kc);
@@ -696,12 +696,12 @@ mixfp4_gemm_skinny_kernel(const __grid_constant__ CUtensorMap tm_wc, const __gri
               break;
             }
             tc_fence_after();
-            const uint64_t bd = bdesc0 + (uint64_t)((d * X_DEC) >> 4);
-            const uint32_t wa = tmem_w0 + (uint32_t)d * kWStageCols;
-            mma_f16_tmem_a(tmem_base, wa, bd, idesc, first ? 0u : 1u);
+            const uint64_t bd = bdesc0 + (uint64_t)((d * W_DEC) >> 4);
+            const uint32_t xa = tmem_x0 + (uint32_t)d * kXStageCols;
+            mma_f16_tmem_a(tmem_base, xa, bd, idesc, first ? 0u : 1u);
             first = false;
 #pragma unroll
-            for (int j = 1; j < BKD / 16; ++j) mma_f16_tmem_a(tmem_base, wa + j * 8, bd + (uint64_t)(j * 16), idesc, 1u);
+            for (int j = 1; j < BKD / 16; ++j) mma_f16_tmem_a(tmem_base, xa + j * 8, bd + (uint64_t)(j * 16), idesc, 1u);
             mma_commit(smem_u32(&bars->dec_empty[d]));
             if (++d == kDecStages) { d = 0; dph ^= 1; }
           }
@@ -715,28 +715,17 @@ mixfp4_gemm_skinny_kernel(const __grid_constant__ CUtensorMap tm_wc, const __gri
   } else if (warp < kFirstEpi) {
     // ---------------- decoders ----------------
     const bool is_w = warp < kFirstX;
-    const int dw = warp - (is_w ? kFirstW : kFirstX);
-    // Weight decoders: rows by TMEM lane quarter (warp % 4), four parts per
-    // row, one 32-code chunk each per stage.  X decoders: the stage's
-    // nmma x 4 chunks as items i = chunk * nmma + row, thread t taking items t
-    // and t + 128 (8 consecutive lanes read 8 rows of one chunk: no conflicts).
-    const int xt = dw * 32 + lane;                   // X decoder thread 0..127
-    const int nitem = 4 * nmma;
-    int rows[2], parts[2];
-    if (is_w) {
-      rows[0] = (warp & 3) * 32 + lane;
-      parts[0] = dw >> 2;
-    } else {
-#pragma unroll
-      for (int j = 0; j < 2; ++j) {
-        const int item = xt + 128 * j;
-        rows[j] = item < nitem ? item % nmma : 0;
-        parts[j] = item < nitem ? item / nmma : 0;
-      }
-    }
-    const int nmine = is_w ? 1 : (xt < nitem) + (xt + 128 < nitem);  // chunks per stage
-    const bool active = nmine > 0;
-    const uint32_t w_lane = (uint32_t)((warp & 3) * 32) << 16;
+    // W: row = (dw % 8) * 32 + lane, chunk part = dw / 8 of each 64-K stage.
+    // X: row = (warp % 4) * 32 + lane = its TMEM lane; both chunks of a stage.
+    const int dw = warp - kFirstW;
+    const int row = is_w ? ((dw & 7) * 32 + lane) : ((warp & 3) * 32 + lane);
+    const int part = is_w ? (dw >> 3) : 0;
+    const bool active = is_w || (warp & 3) * 32 < nx;  // X warps past the fetched rows idle
+    const uint32_t code_row = (is_w ? 0u : (uint32_t)OFF_XC) + (uint32_t)row * (BKC / 2);
+    const uint32_t scale_row = (is_w ? (uint32_t)OFF_WS : (uint32_t)OFF_XS) + (uint32_t)row * (BKC / 16);
+    const uint32_t w_dst = OFF_DEC + (uint32_t)(row >> 3) * kSBO + (uint32_t)(row & 7) * 16;
+    const uint32_t x_lane = (uint32_t)((warp & 3) * 32) << 16;
+    const uint32_t swz = (uint32_t)(row & 7);
     int d = 0, it = 0;
     uint32_t dph = 0;
     for (long long u = u_begin; u < u_end; ++u, ++it) {
@@ -747,19 +736,20 @@ mixfp4_gemm_skinny_kernel(const __grid_constant__ CUtensorMap tm_wc, const __gri
         break;
       }
       const uint32_t st = sbase + s * CODE_STAGE;
-      uint4 sc[2] = {make_uint4(0, 0, 0, 0), make_uint4(0, 0, 0, 0)};  // the rows' 16 block scales
-#pragma unroll
-      for (int j = 0; j < 2; ++j)
-        if (j < nmine) sc[j] = lds128(st + (is_w ? OFF_WS : OFF_XS) + rows[j] * (BKC / 16));
+      uint4 sc = make_uint4(0, 0, 0, 0);  // the row's 16 block scales of this K slice
+      if (active) sc = lds128(st + scale_row);
       bool ok = true;
 #pragma unroll
       for (int sub = 0; sub < kSub; ++sub) {
         uint4 c[2];
-#pragma unroll
-        for (int j = 0; j < 2; ++j)
-          if (j < nmine)
-            c[j] = lds128(st + (is_w ? 0 : OFF_XC) + rows[j] * (BKC / 2) +
-                          ((uint32_t)((sub * 4 + parts[j]) ^ (rows[j] & 7)) << 4));
+        if (active) {
+          if (is_w) {
+            c[0] = lds128(st + code_row + ((((uint32_t)(sub * 2 + part)) ^ swz) << 4));
+          } else {
+            c[0] = lds128(st + code_row + ((((uint32_t)(sub * 2)) ^ swz) << 4));
+            c[1] = lds128(st + code_row + ((((uint32_t)(sub * 2 + 1)) ^ swz) << 4));
+          }
+        }
         if (!mbar_wait(smem_u32(&bars->dec_empty[d]), dph ^ 1, abort_flag, kWaitLimitNs)) {
           fail(32u);
           ok = false;
@@ -767,23 +757,19 @@ mixfp4_gemm_skinny_kernel(const __grid_constant__ CUtensorMap tm_wc, const __gri
         }
         if (is_w) {
           uint32_t o[16];
-          decode_chunk(c[0], scale_pair(sc[0], sub * 4 + parts[0]), o);
-          tmem_st_32x32b_x16(tmem_w0 + w_lane + (uint32_t)d * kWStageCols + (uint32_t)parts[0] * 16u, o);
+          decode_chunk(c[0], scale_pair(sc, sub * 2 + part), o);
+          const uint32_t dst = sbase + w_dst + (uint32_t)d * W_DEC;
+#pragma unroll
+          for (int q = 0; q < 4; ++q)
+            sts128(dst + (uint32_t)(part * 4 + q) * kLBO, o[4 * q], o[4 * q + 1], o[4 * q + 2], o[4 * q + 3]);
+          fence_proxy_async_smem();
+        } else if (active) {
+          uint32_t o[32];
+          decode_chunk(c[0], scale_pair(sc, sub * 2), o);
+          decode_chunk(c[1], scale_pair(sc, sub * 2 + 1), o + 16);
+          tmem_st_32x32b_x32(tmem_x0 + x_lane + (uint32_t)d * kXStageCols, o);
           tmem_st_wait();
           tc_fence_before();
-        } else if (active) {
-#pragma unroll
-          for (int j = 0; j < 2; ++j) {
-            if (j < nmine) {
-              uint32_t o[16];
-              decode_chunk(c[j], scale_pair(sc[j], sub * 4 + parts[j]), o);
-              const uint32_t dst = sbase + OFF_DEC + d * X_DEC + (rows[j] >> 3) * kSBO + (rows[j] & 7) * 16;
-#pragma unroll
-              for (int q = 0; q < 4; ++q)
-                sts128(dst + (parts[j] * 4 + q) * kLBO, o[4 * q], o[4 * q + 1], o[4 * q + 2], o[4 * q + 3]);
-            }
-          }
-          fence_proxy_async_smem();
         }
         __syncwarp();
         if (lane == 0) mbar_arrive(smem_u32(&bars->dec_full[d]));
@@ -796,9 +782,12 @@ mixfp4_gemm_skinny_kernel(const __grid_constant__ CUtensorMap tm_wc, const __gri
       if (!ok) break;
     }
   } else {
-    // ---------------- epilogue: D^T (lane = weight row) -> red.add into C ----------------
+    // ---------------- epilogue: lane = X row m, 256 weight columns -> red.add into C ----------------
     const int q = warp & 3;
+    const int m = q * 32 + lane;
     const float sa = 0.25f * __ldg(a_ts), sb = __ldg(b_ts);
+    const bool vec_ok = ((ldc & 3) == 0) && ((reinterpret_cast<uintptr_t>(C) & 15) == 0);
+    const bool mine = q * 32 < Mx;  // warps whose lane quarter holds X rows
     int ntile = 0;
     for (long long u = u_begin; u < u_end; ++ntile) {
       const int wt = (int)(u / num_kc);
@@ -810,23 +799,33 @@ mixfp4_gemm_skinny_kernel(const __grid_constant__ CUtensorMap tm_wc, const __gri
         if (!acc_ok && !*abort_flag) fail(64u);
         break;
       }
-      const int n = wt * BW + q * 32 + lane;
       const uint32_t tb = tmem_base + ((uint32_t)(q * 32) << 16);
-      uint32_t v[2][32];
-      tmem_ld_32x32b_x32(tb, v[0]);
-      if (nmma > 32) tmem_ld_32x32b_x32(tb + 32, v[1]);
-      tmem_ld_wait_x32(v[0]);
-      reg_fence16(v[1]);
-      reg_fence16(v[1] + 16);
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(smem_u32(&bars->acc_empty));
-      if (n < N) {
+#pragma unroll 1
+      for (int cc = 0; cc < BN / 32; ++cc) {
+        uint32_t v[32];
+        if (mine) {
+          tmem_ld_32x32b_x32(tb + (uint32_t)(cc * 32), v);
+          tmem_ld_wait_x32(v);
+        }
+        if (cc == BN / 32 - 1) {
+          // The accumulator is free once its last chunk sits in registers.
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(smem_u32(&bars->acc_empty));
+        }
+        const int n0 = wt * BN + cc * 32;
+        if (mine && m < Mx) {
+          float* crow = C + (long long)m * ldc + n0;
+          if (vec_ok && n0 + 32 <= N) {
 #pragma unroll
-        for (int m = 0; m < MXMAX; ++m) {
-          if (m < Mx) {
-            const float val = __fmul_rn(__fmul_rn(__uint_as_float(v[m >> 5][m & 31]), sa), sb);
-            atomicAdd(C + (long long)m * ldc + n, val);
+            for (int k = 0; k < 32; k += 4)
+              red_add_v4(crow + k, __fmul_rn(__fmul_rn(__uint_as_float(v[k]), sa), sb),
+                         __fmul_rn(__fmul_rn(__uint_as_float(v[k + 1]), sa), sb),
+                         __fmul_rn(__fmul_rn(__uint_as_float(v[k + 2]), sa), sb),
+                         __fmul_rn(__fmul_rn(__uint_as_float(v[k + 3]), sa), sb));
+          } else {
+            for (int k = 0; k < 32; ++k)
+              if (n0 + k < N) atomicAdd(crow + k, __fmul_rn(__fmul_rn(__uint_as_float(v[k]), sa), sb));
           }
         }
       }
@@ -888,14 +887,14 @@ int launch_gemm(const uint8_t* a_codes, const uint8_t* a_scales, const float* a_
                 int64_t N, int64_t K, float* C, int64_t ldc, uint32_t* status_word,
                 cudaStream_t stream) {
   if (M > (1 << 30) || N > (1 << 30) || K > (1 << 30)) return MIXFP4_ERR_SHAPE;
-  if (M <= skinny::MXMAX && N >= 4 * skinny::BW) {
-    // Few activation rows: weight rows on the MMA M dimension, stream-K over all SMs.
-    const int nmma = (int)((M + 15) & ~15);
+  if (M <= skinny::MXMAX && N >= 2 * skinny::BN) {
+    // Few activation rows: weight rows on the wide MMA N side, stream-K over all SMs.
+    const int nx = (int)((M + 15) & ~15);
     CUtensorMap twc, txc, tws, txs;
-    if (!make_map(&twc, b_codes, (uint64_t)K / 2, (uint64_t)N, BKC / 2, skinny::BW, CU_TENSOR_MAP_SWIZZLE_128B) ||
-        !make_map(&txc, a_codes, (uint64_t)K / 2, (uint64_t)M, BKC / 2, nmma, CU_TENSOR_MAP_SWIZZLE_128B) ||
-        !make_map(&tws, b_scales, (uint64_t)K / 16, (uint64_t)N, BKC / 16, skinny::BW, CU_TENSOR_MAP_SWIZZLE_NONE) ||
-        !make_map(&txs, a_scales, (uint64_t)K / 16, (uint64_t)M, BKC / 16, nmma, CU_TENSOR_MAP_SWIZZLE_NONE))
+    if (!make_map(&twc, b_codes, (uint64_t)K / 2, (uint64_t)N, BKC / 2, skinny::BN, CU_TENSOR_MAP_SWIZZLE_128B) ||
+        !make_map(&txc, a_codes, (uint64_t)K / 2, (uint64_t)M, BKC / 2, nx, CU_TENSOR_MAP_SWIZZLE_128B) ||
+        !make_map(&tws, b_scales, (uint64_t)K / 16, (uint64_t)N, BKC / 16, skinny::BN, CU_TENSOR_MAP_SWIZZLE_NONE) ||
+        !make_map(&txs, a_scales, (uint64_t)K / 16, (uint64_t)M, BKC / 16, nx, CU_TENSOR_MAP_SWIZZLE_NONE))
       return MIXFP4_ERR_CUDA;
     static bool skinny_attr = false;
     if (!skinny_attr) {
@@ -907,12 +906,12 @@ int launch_gemm(const uint8_t* a_codes, const uint8_t* a_scales, const float* a_
     if (cudaMemset2DAsync(C, (size_t)ldc * sizeof(float), 0, (size_t)N * sizeof(float), (size_t)M, stream) !=
         cudaSuccess)
       return MIXFP4_ERR_CUDA;
-    const int64_t units = ((N + skinny::BW - 1) / skinny::BW) * (K / BKC);
+    const int64_t units = ((N + skinny::BN - 1) / skinny::BN) * (K / BKC);
     int64_t grid = num_sms();
     if (grid > units) grid = units;
     skinny::mixfp4_gemm_skinny_kernel<<<(unsigned)grid, skinny::kThreads, skinny::SMEM_ALLOC, stream>>>(
         twc, txc, tws, txs, a_ts, b_ts, (int)M, (int)N, (int)K, C, (long long)ldc,
-        idesc_f16_f32(skinny::BW, nmma), status_word);
+        idesc_f16_f32(128, skinny::BN), status_word);
     return MIXFP4_OK;
   }
   CUtensorMap tac, tbc, tas, tbs;

@@ -46,6 +46,8 @@ def lib() -> ctypes.CDLL:
         L.mixfp4_dequantize.argtypes = [P, P, P, I64, I64, P, P]
         L.mixfp4_gemm.restype = I
         L.mixfp4_gemm.argtypes = [P, P, P, P, P, P, I64, I64, I64, P, I64, P, P]
+        L.mixfp4_selftest_bounded_wait.restype = I
+        L.mixfp4_selftest_bounded_wait.argtypes = [P, ctypes.c_uint64, P]
         L.mixfp4_status_string.restype = ctypes.c_char_p
         L.mixfp4_status_string.argtypes = [I]
         L.mixfp4_version.restype = I
@@ -156,6 +158,15 @@ def mixfp4_gemm(a: QTensor, b: QTensor, out: torch.Tensor | None = None,
                            M, N, K, _ptr(C), C.stride(0), _ptr(status_word), _stream(stream))
     _check("mixfp4_gemm", st)
     return C
+
+
+def selftest_bounded_wait(limit_ns: int = 20_000_000, stream=None) -> int:
+    """Run the bounded-wait self-test; returns the status bits (0xE when healthy)."""
+    status = torch.zeros(1, dtype=torch.int32, device="cuda")
+    _check("mixfp4_selftest_bounded_wait",
+           lib().mixfp4_selftest_bounded_wait(_ptr(status), int(limit_ns), _stream(stream)))
+    torch.cuda.synchronize()
+    return int(status.item())
 
 
 def linear(x: torch.Tensor, w_q: QTensor, mode: int = MODE_MIX, stream=None) -> torch.Tensor:
