@@ -58,6 +58,7 @@ constexpr int kDecStages = 4;
 constexpr int kTPR = 2;                       // decode threads per operand row
 constexpr int kChunksPerSub = BKD / 32;       // 16-byte code chunks (32 codes) per row per stage
 constexpr int kChunksPerThread = kChunksPerSub / kTPR;
+static_assert(kChunksPerThread % 2 == 0, "A decoders store two chunks (32 TMEM columns) at a time");
 constexpr int kDecodeWarpsA = kTPR * BM / 32;   // 8
 constexpr int kDecodeWarpsB = kTPR * BNH / 32;  // 8
 constexpr int kEpiWarps = 8;
@@ -94,7 +95,6 @@ static_assert(SMEM_ALLOC <= 232448, "shared memory budget");
 //   (row / 8) * SBO + kchunk * LBO + (row % 8) * 16
 constexpr uint32_t kLBO = 128;                  // next 8 K-elements
 constexpr uint32_t kSBO = (BKD / 8) * 128;      // next 8 rows
-constexpr uint32_t kIdesc = idesc_f16_f32(TILE_M, TILE_N);
 
 constexpr uint64_t kWaitLimitNs = 1000000000ull;  // 1 s per pipeline wait
 constexpr int kMinStreamKGainSlices = 8;           // stream-K must save this many K slices per pair
@@ -216,6 +216,11 @@ struct Sched {
   }
 };
 
+// kTileN: pair tile width (256, 224 or 192; each CTA holds kTileN / 2 rows of
+// B).  Shared and tensor memory are laid out for 256; narrower tiles leave the
+// tail of the B regions unused (decoders may write those rows; the MMA never
+// reads them).
+template <int kTileN>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
 mixfp4_gemm_kernel(const __grid_constant__ CUtensorMap tm_ac, const __grid_constant__ CUtensorMap tm_bc,
                    const __grid_constant__ CUtensorMap tm_as, const __grid_constant__ CUtensorMap tm_bs,
@@ -231,7 +236,11 @@ mixfp4_gemm_kernel(const __grid_constant__ CUtensorMap tm_ac, const __grid_const
   const uint32_t rank = cluster_ctarank();
   const bool leader = rank == 0;
   const int num_kc = K / BKC;
-  const int mtiles = (M + TILE_M - 1) / TILE_M, ntiles_n = (N + TILE_N - 1) / TILE_N;
+  static_assert(kTileN % 32 == 0 && kTileN >= 64 && kTileN <= TILE_N, "tile width");
+  constexpr int kBRows = kTileN / 2;  // B rows per CTA
+  constexpr uint32_t kStageTx = A_CODE_BYTES + A_SCALE_BYTES + kBRows * (BKC / 2 + BKC / 16);
+  constexpr uint32_t kIdescT = idesc_f16_f32(TILE_M, kTileN);
+  const int mtiles = (M + TILE_M - 1) / TILE_M, ntiles_n = (N + kTileN - 1) / kTileN;
   const int ntiles = mtiles * ntiles_n;
   const int cluster_id = blockIdx.x >> 1, nclusters = gridDim.x >> 1;
 
@@ -282,7 +291,7 @@ mixfp4_gemm_kernel(const __grid_constant__ CUtensorMap tm_ac, const __grid_const
       int t, k0, k1;
       while (ok && sched.next(t, k0, k1)) {
         const int mt = t / ntiles_n, nt = t % ntiles_n;
-        const int ma = mt * TILE_M + (int)rank * BM, nb = nt * TILE_N + (int)rank * BNH;
+        const int ma = mt * TILE_M + (int)rank * BM, nb = nt * kTileN + (int)rank * kBRows;
         for (int kc = k0; kc < k1; ++kc, ++it) {
           const int s = it % kCodeStages;
           const uint32_t ph = (it / kCodeStages) & 1;
@@ -293,7 +302,7 @@ mixfp4_gemm_kernel(const __grid_constant__ CUtensorMap tm_ac, const __grid_const
           }
           const uint32_t st = sbase + s * CODE_STAGE_BYTES;
           const uint32_t fb = smem_u32(&bars->code_full[s]);
-          mbar_arrive_expect_tx(fb, CODE_STAGE_BYTES);
+          mbar_arrive_expect_tx(fb, kStageTx);
           const int xk = kc * (BKC / 2), xs = kc * (BKC / 16);
           tma_load_2d(st, &tm_ac, xk, ma, fb);
           tma_load_2d(st + A_CODE_BYTES, &tm_bc, xk, nb, fb);
@@ -337,7 +346,7 @@ mixfp4_gemm_kernel(const __grid_constant__ CUtensorMap tm_ac, const __grid_const
 #pragma unroll
             for (int j = 0; j < BKD / 16; ++j) {
               const uint64_t bd = smem_desc_noswizzle(bbase + j * 256, kLBO, kSBO);
-              mma_f16_pair_tmem_a(tmem_base, abase + j * 8, bd, kIdesc, ((kc - k0) | sub | j) != 0 ? 1u : 0u);
+              mma_f16_pair_tmem_a(tmem_base, abase + j * 8, bd, kIdescT, ((kc - k0) | sub | j) != 0 ? 1u : 0u);
             }
             mma_commit_pair(smem_u32(&bars->dec_empty[d]), 3);
             if (++d == kDecStages) { d = 0; dph ^= 1; }
@@ -412,12 +421,17 @@ mixfp4_gemm_kernel(const __grid_constant__ CUtensorMap tm_ac, const __grid_const
             break;
           }
           if (is_a) {
-            // 64 K of the row = 32 f16 pairs -> TMEM columns [part * 32, +32) of stage d
-            uint32_t o[32];
+            // The thread's kChunksPerThread * 32 K of the row = 16 f16 pairs per
+            // chunk -> TMEM columns [part * 16 * kChunksPerThread, ...) of stage d,
+            // stored two chunks (32 columns) at a time.
 #pragma unroll
-            for (int j = 0; j < kChunksPerThread; ++j)
-              decode_chunk(c[j], scale_pair(sc, sub * kChunksPerSub + part * kChunksPerThread + j), o + 16 * j);
-            tmem_st_32x32b_x32(tmem_a0 + a_lane + (uint32_t)d * kAStageCols + (uint32_t)part * 32u, o);
+            for (int j = 0; j < kChunksPerThread; j += 2) {
+              uint32_t o[32];
+              decode_chunk(c[j], scale_pair(sc, sub * kChunksPerSub + part * kChunksPerThread + j), o);
+              decode_chunk(c[j + 1], scale_pair(sc, sub * kChunksPerSub + part * kChunksPerThread + j + 1), o + 16);
+              tmem_st_32x32b_x32(tmem_a0 + a_lane + (uint32_t)d * kAStageCols +
+                                     (uint32_t)(part * 16 * kChunksPerThread + 16 * j), o);
+            }
             tmem_st_wait();
             tc_fence_before();
           } else {
@@ -476,14 +490,14 @@ mixfp4_gemm_kernel(const __grid_constant__ CUtensorMap tm_ac, const __grid_const
       }
       const int mt = t / ntiles_n, nt = t % ntiles_n;
       const int row0 = mt * TILE_M + (int)rank * BM + q * 32;
-      const int n0 = nt * TILE_N + chalf * (TILE_N / 2);
-      const uint32_t tbase = tmem_base + (uint32_t)(chalf * (TILE_N / 2)) + ((uint32_t)(q * 32) << 16);
+      const int n0 = nt * kTileN + chalf * kBRows;
+      const uint32_t tbase = tmem_base + (uint32_t)(chalf * kBRows) + ((uint32_t)(q * 32) << 16);
 #pragma unroll 1
-      for (int cc = 0; cc < TILE_N / 2 / EPI_CHUNK; ++cc) {
+      for (int cc = 0; cc < kBRows / EPI_CHUNK; ++cc) {
         uint32_t o[EPI_CHUNK];
         tmem_ld_32x32b_x16(tbase + (uint32_t)(cc * EPI_CHUNK), o);
         tmem_ld_wait_x16(o);
-        if (cc == TILE_N / 2 / EPI_CHUNK - 1) {
+        if (cc == kBRows / EPI_CHUNK - 1) {
           // The accumulator is free once its last chunk sits in registers.
           tc_fence_before();
           __syncwarp();
@@ -882,6 +896,49 @@ int num_sms() {
 
 }  // namespace
 
+// Launch the pair kernel with tile width kTileN over `tiles` tiles, the first
+// dp_tiles whole and the rest split into K slices (stream-K).
+template <int kTileN>
+int launch_pair(const uint8_t* a_codes, const uint8_t* a_scales, const float* a_ts, const uint8_t* b_codes,
+                const uint8_t* b_scales, const float* b_ts, int64_t M, int64_t N, int64_t K, float* C, int64_t ldc,
+                uint32_t* status_word, int64_t clusters, int64_t tiles, int64_t dp_tiles, cudaStream_t stream) {
+  CUtensorMap tac, tbc, tas, tbs;
+  if (!make_map(&tac, a_codes, (uint64_t)K / 2, (uint64_t)M, BKC / 2, BM, CU_TENSOR_MAP_SWIZZLE_128B) ||
+      !make_map(&tbc, b_codes, (uint64_t)K / 2, (uint64_t)N, BKC / 2, kTileN / 2, CU_TENSOR_MAP_SWIZZLE_128B) ||
+      !make_map(&tas, a_scales, (uint64_t)K / 16, (uint64_t)M, BKC / 16, BM, CU_TENSOR_MAP_SWIZZLE_NONE) ||
+      !make_map(&tbs, b_scales, (uint64_t)K / 16, (uint64_t)N, BKC / 16, kTileN / 2, CU_TENSOR_MAP_SWIZZLE_NONE))
+    return MIXFP4_ERR_CUDA;
+  static bool attr_set = false;
+  if (!attr_set) {
+    if (cudaFuncSetAttribute(mixfp4_gemm_kernel<kTileN>, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_ALLOC) !=
+        cudaSuccess)
+      return MIXFP4_ERR_CUDA;
+    attr_set = true;
+  }
+  const int64_t ntiles_n = (N + kTileN - 1) / kTileN;
+  if (dp_tiles < tiles) {
+    // Zero C from the first stream-K tile's row band down (tile t: mt = t / ntiles_n,
+    // nt = t % ntiles_n, so those rows hold every stream-K tile; whole tiles among
+    // them are overwritten by plain stores after this).
+    const int64_t r0 = (dp_tiles / ntiles_n) * TILE_M;
+    cudaError_t e;
+    if (ldc == N)
+      e = cudaMemsetAsync(C + r0 * ldc, 0, (size_t)(M - r0) * (size_t)N * sizeof(float), stream);
+    else
+      e = cudaMemset2DAsync(C + r0 * ldc, (size_t)ldc * sizeof(float), 0, (size_t)N * sizeof(float),
+                            (size_t)(M - r0), stream);
+    if (e != cudaSuccess) return MIXFP4_ERR_CUDA;
+  }
+  // A programmatic dependent: barrier set-up and TMEM allocation overlap the
+  // tail of the kernel before it; the TMA producer and the epilogue wait for
+  // that kernel before they read the operands or the tensor scales.
+  if (launch_pdl(mixfp4_gemm_kernel<kTileN>, (unsigned)(2 * clusters), kThreads, SMEM_ALLOC, stream, tac, tbc, tas,
+                 tbs, a_ts, b_ts, (int)M, (int)N, (int)K, C, (long long)ldc, (int)dp_tiles, status_word) !=
+      cudaSuccess)
+    return MIXFP4_ERR_CUDA;
+  return MIXFP4_OK;
+}
+
 int launch_gemm(const uint8_t* a_codes, const uint8_t* a_scales, const float* a_ts,
                 const uint8_t* b_codes, const uint8_t* b_scales, const float* b_ts, int64_t M,
                 int64_t N, int64_t K, float* C, int64_t ldc, uint32_t* status_word,
@@ -914,23 +971,22 @@ int launch_gemm(const uint8_t* a_codes, const uint8_t* a_scales, const float* a_
         idesc_f16_f32(128, skinny::BN), status_word);
     return MIXFP4_OK;
   }
-  CUtensorMap tac, tbc, tas, tbs;
-  if (!make_map(&tac, a_codes, (uint64_t)K / 2, (uint64_t)M, BKC / 2, BM, CU_TENSOR_MAP_SWIZZLE_128B) ||
-      !make_map(&tbc, b_codes, (uint64_t)K / 2, (uint64_t)N, BKC / 2, BNH, CU_TENSOR_MAP_SWIZZLE_128B) ||
-      !make_map(&tas, a_scales, (uint64_t)K / 16, (uint64_t)M, BKC / 16, BM, CU_TENSOR_MAP_SWIZZLE_NONE) ||
-      !make_map(&tbs, b_scales, (uint64_t)K / 16, (uint64_t)N, BKC / 16, BNH, CU_TENSOR_MAP_SWIZZLE_NONE))
-    return MIXFP4_ERR_CUDA;
-  static bool attr_set = false;
-  if (!attr_set) {
-    if (cudaFuncSetAttribute(mixfp4_gemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_ALLOC) !=
-        cudaSuccess)
-      return MIXFP4_ERR_CUDA;
-    attr_set = true;
-  }
-  const int64_t mtiles = (M + TILE_M - 1) / TILE_M, ntiles_n = (N + TILE_N - 1) / TILE_N;
-  const int64_t tiles = mtiles * ntiles_n, num_kc = K / BKC;
-  int64_t clusters = num_sms() / 2;
-  if (clusters > tiles) clusters = tiles;
+  // Tile width: the pair tiles are 256 rows of A by kTileN rows of B.  With
+  // few tiles per pair a narrower tile can remove a partly idle last wave;
+  // the main loop is bound by decoding A and B (256 + kTileN rows per K
+  // step), so the cost of a width is waves * (256 + kTileN).  Stream-K (for
+  // 256) is preferred when it applies.
+  const int64_t mtiles = (M + TILE_M - 1) / TILE_M, num_kc = K / BKC;
+  auto waves = [&](int64_t n, int64_t* tiles_out, int64_t* clusters_out) {
+    const int64_t t = mtiles * ((N + n - 1) / n);
+    int64_t c = num_sms() / 2;
+    if (c > t) c = t;
+    *tiles_out = t;
+    *clusters_out = c;
+    return (t + c - 1) / c;
+  };
+  int64_t tiles, clusters;
+  const int64_t w256 = waves(256, &tiles, &clusters);
   // Whole tiles in full waves.  The last, partial wave's tiles are shared out
   // as K slices (stream-K) when the idle time that removes, (clusters - rem)
   // tiles' worth of K slices spread over all pairs, outweighs what stream-K
@@ -939,26 +995,32 @@ int launch_gemm(const uint8_t* a_codes, const uint8_t* a_scales, const float* a_
   const int64_t rem = tiles % clusters;
   if (tiles > clusters && rem != 0 && (clusters - rem) * num_kc >= kMinStreamKGainSlices * clusters)
     dp_tiles = tiles - rem;
-  if (dp_tiles < tiles) {
-    // Zero C from the first stream-K tile's row band down (tile t: mt = t / ntiles_n,
-    // nt = t % ntiles_n, so those rows hold every stream-K tile; whole tiles among
-    // them are overwritten by plain stores after this).
-    const int64_t r0 = (dp_tiles / ntiles_n) * TILE_M;
-    cudaError_t e;
-    if (ldc == N)
-      e = cudaMemsetAsync(C + r0 * ldc, 0, (size_t)(M - r0) * (size_t)N * sizeof(float), stream);
-    else
-      e = cudaMemset2DAsync(C + r0 * ldc, (size_t)ldc * sizeof(float), 0, (size_t)N * sizeof(float),
-                            (size_t)(M - r0), stream);
-    if (e != cudaSuccess) return MIXFP4_ERR_CUDA;
+  int tile_n = 256;
+  if (dp_tiles == tiles) {
+    int64_t best = w256 * (256 + 256);
+    for (int n : {224, 192}) {
+      int64_t t, c;
+      const int64_t cost = waves(n, &t, &c) * (256 + n);
+      if (cost < best) {
+        best = cost;
+        tile_n = n;
+        tiles = t;
+        clusters = c;
+        dp_tiles = t;
+      }
+    }
   }
-  // A programmatic dependent: barrier set-up and TMEM allocation overlap the
-  // tail of the kernel before it; the TMA producer and the epilogue wait for
-  // that kernel before they read the operands or the tensor scales.
-  if (launch_pdl(mixfp4_gemm_kernel, (unsigned)(2 * clusters), kThreads, SMEM_ALLOC, stream, tac, tbc, tas, tbs,
-                 a_ts, b_ts, (int)M, (int)N, (int)K, C, (long long)ldc, (int)dp_tiles, status_word) != cudaSuccess)
-    return MIXFP4_ERR_CUDA;
-  return MIXFP4_OK;
+  switch (tile_n) {
+    case 224:
+      return launch_pair<224>(a_codes, a_scales, a_ts, b_codes, b_scales, b_ts, M, N, K, C, ldc, status_word,
+                              clusters, tiles, dp_tiles, stream);
+    case 192:
+      return launch_pair<192>(a_codes, a_scales, a_ts, b_codes, b_scales, b_ts, M, N, K, C, ldc, status_word,
+                              clusters, tiles, dp_tiles, stream);
+    default:
+      return launch_pair<256>(a_codes, a_scales, a_ts, b_codes, b_scales, b_ts, M, N, K, C, ldc, status_word,
+                              clusters, tiles, dp_tiles, stream);
+  }
 }
 
 }  // namespace mixfp4

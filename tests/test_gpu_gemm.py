@@ -165,3 +165,21 @@ def test_stream_k_tail(oracle):
     assert_close(Cn[rows], A_r @ B_all.T, A_r, B_all)
     A_all = oracle.dequant_rows_f64(ac, as_, at, range(M))
     assert_close(Cn[:, cols], A_all @ B_c.T, A_all, B_c)
+
+
+@pytest.mark.parametrize("M,N,K", [(2048, 4000, 512), (256, 1000, 512), (300, 600, 1024)])
+def test_narrow_tile_widths(oracle, M, N, K):
+    """Shapes for which the launcher picks 224- or 192-wide pair tiles (so the
+    last wave is full): every element of C against float64 from the oracle's
+    dequantized operands."""
+    x = synth.activations(M, K, 7401 + M, 7402)
+    w = synth.weights(N, K, 7403 + N, 0.02, 0.5)
+    o = ops()
+    qa, qb = o.mixfp4_quantize(x.to(DEV)), o.mixfp4_quantize(w.to(DEV))
+    status = torch.zeros(1, dtype=torch.int32, device=DEV)
+    C = o.mixfp4_gemm(qa, qb, status_word=status)
+    torch.cuda.synchronize()
+    assert status.item() == 0
+    A = oracle.dequant_rows_f64(qa.codes.cpu().numpy(), qa.scales.cpu().numpy(), qa.tensor_scale.item(), range(M))
+    B = oracle.dequant_rows_f64(qb.codes.cpu().numpy(), qb.scales.cpu().numpy(), qb.tensor_scale.item(), range(N))
+    assert_close(C.cpu().numpy(), A @ B.T, A, B)
