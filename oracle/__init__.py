@@ -13,6 +13,9 @@ Function map (paper passages are cited in ``mixfp4_oracle.c``):
   dequantize                App. B.2/B.3 decode times the tensor scale
   gemm_f64                  C = A_deq B_deq^T in float64
   gemm_exact                App. B.1 Eq. (factor), exact integer accumulation
+  split_native              MixFP4 operand as the sum of two E2M1 operands with
+                            shared scales, plus the tensor core's tiled scale
+                            layout (the native FP4 GEMM variant)
 """
 from __future__ import annotations
 
@@ -73,6 +76,8 @@ def _L():
         lib.oracle_gemm_exact.argtypes = [P, P, ctypes.c_float, P, P, ctypes.c_float, I64, I64, I64, P]
         lib.oracle_dequant_row_f64.restype = None
         lib.oracle_dequant_row_f64.argtypes = [P, P, ctypes.c_float, I64, I64, P]
+        lib.oracle_split_native.argtypes = [P, P, I64, I64, P, P, P]
+        lib.oracle_split_native.restype = ctypes.c_int
         _lib = lib
     return _lib
 
@@ -200,3 +205,23 @@ def gemm_exact(a, b) -> np.ndarray:
     C = np.zeros((M, N), np.longdouble)
     _L().oracle_gemm_exact(_p(ac), _p(as_), float(as32), _p(bc), _p(bs), float(bs32), M, N, K, _p(C))
     return C.astype(np.float64)
+
+
+def sf_tiled_bytes(rows: int, K: int) -> int:
+    """Size of the tiled block-scale array: rows rounded up to 256, K/16 bytes each."""
+    return ((rows + 255) // 256) * 256 * (K // 16)
+
+
+def split_native(codes: np.ndarray, scales: np.ndarray):
+    """Native E2M1 operands of a MixFP4 tensor: (main codes, residual codes,
+    tiled ue4m3 scales); see oracle_split_native in mixfp4_oracle.c."""
+    codes = np.ascontiguousarray(codes, np.uint8)
+    scales = np.ascontiguousarray(scales, np.uint8)
+    rows, K = codes.shape[0], codes.shape[1] * 2
+    main = np.zeros_like(codes)
+    res = np.zeros_like(codes)
+    sf = np.zeros(sf_tiled_bytes(rows, K), np.uint8)
+    rc = _L().oracle_split_native(_p(codes), _p(scales), rows, K, _p(main), _p(res), _p(sf))
+    if rc != 0:
+        raise ValueError(f"oracle_split_native failed ({rc})")
+    return main, res, sf

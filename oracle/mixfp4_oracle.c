@@ -27,6 +27,9 @@
  *   oracle_gemm_f64    C = A_deq . B_deq^T in float64 (plain definition)
  *   oracle_gemm_exact  App. B.1 Eq. (factor): per-block integer dot times the
  *                      scale product, accumulated exactly in __int128
+ *   oracle_split_native  the MixFP4 operand as main + residual E2M1 operands
+ *                      sharing its scales (Table 1 codebooks; 5 = 4 + 1,
+ *                      7 = 6 + 1), scales in the tensor core's tiled layout
  *
  * Readings where the paper is silent (the same list is kept in the design doc):
  *   R1 X_FP8 = fl32(X / s32) is an fp32 value (no FP8 cast).
@@ -346,4 +349,67 @@ void oracle_gemm_exact(const uint8_t* ac, const uint8_t* as, float as32,
       long double t = (long double)total;
       C[m * N + n] = ldexpl(t, -22) * (long double)as32 * (long double)bs32;
     }
+}
+
+/* ---------------------------------------------------------------------------
+ * Native block-scaled FP4 operands (the split behind the E2M1 x E2M1
+ * tensor-core variant of the MixFP4 GEMM).  A MixFP4 operand is written as
+ * the sum of two E2M1 operands that share its block scales:
+ *   E2M1 block (T = 0): main = the stored nibble, residual = +0.
+ *   E1M2 block (T = 1): the magnitude v = p (Sec. 3.1 remap) is split as
+ *     v = e + r, e the largest E2M1 codebook value <= v, r = v - e (which is
+ *     0 or 1, both E2M1 values); main = sign | code(e), residual = sign |
+ *     code(r), sign = the stored sign bit.
+ * Scales: the E4M3 magnitude (bits 6..0; the type bit is dropped because the
+ * split codes carry the values) in the tensor core's block-16 scale layout:
+ * tiles of 128 rows x 4 blocks (64 K), 512 bytes each, tile (rt, kt) at
+ * ((rt * (K / 64)) + kt) * 512, row r of the tile and block b at
+ * (r % 32) * 16 + (r / 32) * 4 + b.  Row tiles cover rows rounded up to a
+ * multiple of 256; padding bytes are 0.
+ * Parity of the value split is pinned on the CPU (the parts' decoded values
+ * sum to the MixFP4 value for every nibble and type); the scale layout is a
+ * hardware format, parity unpinned on the CPU and checked by the GPU product.
+ * ------------------------------------------------------------------------- */
+static int e2m1_code_of(double v) {
+  for (int q = 0; q < 8; ++q)
+    if (oracle_fp4_value(0, q) == v) return q;
+  return -1;
+}
+
+static void split_nibble(int nib, int T, int* main_nib, int* res_nib) {
+  if (!T) {
+    *main_nib = nib;
+    *res_nib = 0;
+    return;
+  }
+  double v = oracle_fp4_value(1, nib & 7), e = 0.0;
+  for (int q = 0; q < 8; ++q) {
+    double c = oracle_fp4_value(0, q);
+    if (c <= v && c > e) e = c;
+  }
+  *main_nib = (nib & 8) | e2m1_code_of(e);
+  *res_nib = (nib & 8) | e2m1_code_of(v - e);
+}
+
+int oracle_split_native(const uint8_t* codes, const uint8_t* scales, int64_t rows, int64_t K,
+                        uint8_t* main_codes, uint8_t* res_codes, uint8_t* sf) {
+  if (K % 64 != 0) return -1;
+  int64_t nb = K / 16, kt_n = K / 64, rt_n = 2 * ((rows + 255) / 256);
+  for (int64_t r = 0; r < rows; ++r)
+    for (int64_t j = 0; j < K / 2; ++j) {
+      int T = scales[r * nb + (2 * j) / 16] >> 7;
+      int lo_m, lo_r, hi_m, hi_r;
+      split_nibble(codes[r * (K / 2) + j] & 0xF, T, &lo_m, &lo_r);
+      split_nibble(codes[r * (K / 2) + j] >> 4, T, &hi_m, &hi_r);
+      if (lo_m < 0 || lo_r < 0 || hi_m < 0 || hi_r < 0) return -2;
+      main_codes[r * (K / 2) + j] = (uint8_t)(lo_m | (hi_m << 4));
+      res_codes[r * (K / 2) + j] = (uint8_t)(lo_r | (hi_r << 4));
+    }
+  memset(sf, 0, (size_t)(rt_n * kt_n * 512));
+  for (int64_t r = 0; r < rows; ++r)
+    for (int64_t b = 0; b < nb; ++b) {
+      int64_t rt = r / 128, rr = r % 128, kt = b / 4;
+      sf[(rt * kt_n + kt) * 512 + (rr % 32) * 16 + (rr / 32) * 4 + (b % 4)] = scales[r * nb + b] & 0x7F;
+    }
+  return 0;
 }
