@@ -146,6 +146,50 @@ int mixfp4_gemm(const uint8_t* a_codes, const uint8_t* a_scales, const float* a_
                 uint32_t* status_word, void* stream);
 
 /*
+ * mixfp4_split_native -- the operands of the native FP4 GEMM variant.  A
+ * MixFP4 tensor is rewritten as the sum of two E2M1 tensors that share its
+ * block scales (no counterpart in the paper; every value is exact):
+ *   E2M1 block (T = 0): main = the stored codes, residual = 0;
+ *   E1M2 block (T = 1): each magnitude v = p (Sec. 3.1 remap, v in 0..7) is
+ *     e + r with e the largest E2M1 value <= v (0,1,2,3,4,4,6,6) and r = v - e
+ *     (1 for v = 5 and 7, else 0); both parts carry the element's sign bit.
+ * The block scales are written as ue4m3 (bits 6..0 of the scale byte) in the
+ * tensor core's tiled block-16 layout: tiles of 128 rows x 4 blocks (64 K),
+ * 512 bytes each; tile (rt, kt) starts at byte (rt * K/64 + kt) * 512; row r
+ * of the tile, block b of the tile at (r % 32) * 16 + (r / 32) * 4 + b.  Rows
+ * are padded to a multiple of 256 with zero bytes.
+ *
+ * codes, scales  device, a MixFP4 tensor [rows][K/2], [rows][K/16] (16- and
+ *                4-byte aligned).
+ * rows, K        rows >= 0, K % 64 == 0 (else MIXFP4_ERR_SHAPE).
+ * main_codes, res_codes  device, uint8 [rows][K/2] each, 16-byte aligned.  (output)
+ * sf_tiled       device, uint8 [ceil(rows/256) * 256 * K/16], 16-byte aligned.
+ *                                                                         (output)
+ */
+int mixfp4_split_native(const uint8_t* codes, const uint8_t* scales, int64_t rows, int64_t K,
+                        uint8_t* main_codes, uint8_t* res_codes, uint8_t* sf_tiled, void* stream);
+
+/*
+ * mixfp4_gemm_native -- the MixFP4 GEMM on the block-scaled FP4 tensor path:
+ *   C = s32A * s32B * (A_main + A_res) . (B_main + B_res)^T,
+ * the four products of E2M1 operands with ue4m3 block-16 scales contracted by
+ * tcgen05.mma kind::mxf4nvf4 with fp32 accumulation.  It computes the same C
+ * as mixfp4_gemm (App. B.1 Eq. (factor)) up to fp32 summation order.
+ *
+ * a_main/a_res/a_sf  A (activations, M x K) as written by mixfp4_split_native;
+ *                    a_res may be NULL when A has no E1M2 block (an E2M1-only
+ *                    tensor), which drops the products with it.
+ * a_ts               device, one float s32A.
+ * b_main/b_res/b_sf/b_ts  the same for B (weights, N x K).
+ * M, N, K, C, ldc, status_word  as mixfp4_gemm (K % 256 == 0).
+ * Code and scale pointers must be 16-byte aligned.
+ */
+int mixfp4_gemm_native(const uint8_t* a_main, const uint8_t* a_res, const uint8_t* a_sf, const float* a_ts,
+                       const uint8_t* b_main, const uint8_t* b_res, const uint8_t* b_sf, const float* b_ts,
+                       int64_t M, int64_t N, int64_t K, float* C, int64_t ldc, uint32_t* status_word,
+                       void* stream);
+
+/*
  * mixfp4_quantize_noalloc -- mixfp4_quantize with MIXFP4_SCALE_COMPUTE for
  * callers that cannot allocate device memory.  The paper has no counterpart;
  * this is a deployment convenience.

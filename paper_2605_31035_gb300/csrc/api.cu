@@ -131,6 +131,48 @@ int mixfp4_gemm(const uint8_t* a_codes, const uint8_t* a_scales, const float* a_
   return launch_status();
 }
 
+int mixfp4_split_native(const uint8_t* codes, const uint8_t* scales, int64_t rows, int64_t K,
+                        uint8_t* main_codes, uint8_t* res_codes, uint8_t* sf_tiled, void* stream) {
+  if (rows < 0 || K < 0 || K % 64 != 0) return MIXFP4_ERR_SHAPE;
+  if (rows == 0 || K == 0) return MIXFP4_OK;
+  if (!codes || !scales || !main_codes || !res_codes || !sf_tiled) return MIXFP4_ERR_NULL;
+  if (!aligned(codes, 16) || !aligned(scales, 4) || !aligned(main_codes, 16) || !aligned(res_codes, 16) ||
+      !aligned(sf_tiled, 16))
+    return MIXFP4_ERR_ALIGN;
+  int st = mixfp4::launch_split_native(codes, scales, rows, K, main_codes, res_codes, sf_tiled,
+                                       static_cast<cudaStream_t>(stream));
+  if (st) return st;
+  return launch_status();
+}
+
+int mixfp4_gemm_native(const uint8_t* a_main, const uint8_t* a_res, const uint8_t* a_sf, const float* a_ts,
+                       const uint8_t* b_main, const uint8_t* b_res, const uint8_t* b_sf, const float* b_ts,
+                       int64_t M, int64_t N, int64_t K, float* C, int64_t ldc, uint32_t* status_word,
+                       void* stream) {
+  if (M < 0 || N < 0 || K < 0 || K % 256 != 0 || ldc < N) return MIXFP4_ERR_SHAPE;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (status_word) {
+    if (!aligned(status_word, 4)) return MIXFP4_ERR_ALIGN;
+    if (cudaMemsetAsync(status_word, 0, sizeof(uint32_t), s) != cudaSuccess) return MIXFP4_ERR_CUDA;
+  }
+  if (M == 0 || N == 0) return MIXFP4_OK;
+  if (!C) return MIXFP4_ERR_NULL;
+  if (!aligned(C, 4)) return MIXFP4_ERR_ALIGN;
+  if (K == 0) {
+    if (cudaMemset2DAsync(C, (size_t)ldc * sizeof(float), 0, (size_t)N * sizeof(float), (size_t)M, s) != cudaSuccess)
+      return MIXFP4_ERR_CUDA;
+    return MIXFP4_OK;
+  }
+  if (!a_main || !a_sf || !a_ts || !b_main || !b_sf || !b_ts) return MIXFP4_ERR_NULL;
+  if (!aligned(a_main, 16) || !aligned(a_sf, 16) || !aligned(b_main, 16) || !aligned(b_sf, 16) ||
+      (a_res && !aligned(a_res, 16)) || (b_res && !aligned(b_res, 16)) || !aligned(a_ts, 4) || !aligned(b_ts, 4))
+    return MIXFP4_ERR_ALIGN;
+  int st = mixfp4::launch_gemm_native(a_main, a_res, a_sf, a_ts, b_main, b_res, b_sf, b_ts, M, N, K, C, ldc,
+                                      status_word, s);
+  if (st) return st;
+  return launch_status();
+}
+
 }  // extern "C"
 
 int mixfp4_selftest_bounded_wait(uint32_t* status_word, uint64_t limit_ns, void* stream) {

@@ -38,7 +38,9 @@
 #include <cuda_runtime.h>
 #include <cstdint>
 
+#include "host_util.cuh"
 #include "kernels.cuh"
+#include "pipeline.cuh"
 #include "ptx.cuh"
 #include "sm100.cuh"
 
@@ -113,14 +115,6 @@ struct Bars {
 };
 static_assert(sizeof(Bars) <= 256, "barrier block");
 
-__device__ __forceinline__ void sts128(uint32_t addr, uint32_t a, uint32_t b, uint32_t c, uint32_t d) {
-  asm volatile("st.shared.v4.b32 [%0], {%1,%2,%3,%4};" :: "r"(addr), "r"(a), "r"(b), "r"(c), "r"(d) : "memory");
-}
-__device__ __forceinline__ uint4 lds128(uint32_t addr) {
-  uint4 v;
-  asm volatile("ld.shared.v4.b32 {%0,%1,%2,%3}, [%4];" : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(addr) : "memory");
-  return v;
-}
 __device__ __forceinline__ uint32_t hmul2(uint32_t a, uint32_t b) {
   uint32_t d;
   asm("mul.rn.f16x2 %0, %1, %2;" : "=r"(d) : "r"(a), "r"(b));
@@ -175,46 +169,6 @@ __device__ __forceinline__ uint32_t scale_pair(const uint4& sc, int chunk) {
   const uint32_t s4 = sw == 0 ? sc.x : sw == 1 ? sc.y : sw == 2 ? sc.z : sc.w;
   return (s4 >> (16 * (chunk & 1))) & 0xFFFFu;
 }
-
-__device__ __forceinline__ void red_add_v4(float* p, float a, float b, float c, float d) {
-  asm volatile("red.global.add.v4.f32 [%0], {%1,%2,%3,%4};" :: "l"(p), "f"(a), "f"(b), "f"(c), "f"(d)
-               : "memory");
-}
-
-// Work schedule of one CTA pair, walked identically by every role.  Tiles
-// below dp_tiles are whole-tile work, dealt round-robin (tile = cluster,
-// cluster + nclusters, ...).  The (tile, 256-wide K slice) units of the
-// remaining tiles are split evenly over all pairs (stream-K) and cut into
-// segments at tile edges; a segment that is not a whole tile is added into C
-// (which the host zeroed over those tiles).
-struct Sched {
-  int t, dp_tiles, nclusters, num_kc;
-  long long u, u_end;
-  __device__ Sched(int cluster, int ncl, int dp, int ntiles, int nkc)
-      : t(cluster), dp_tiles(dp), nclusters(ncl), num_kc(nkc) {
-    const long long sk_units = (long long)(ntiles - dp) * nkc;
-    u = sk_units * cluster / ncl;
-    u_end = sk_units * (cluster + 1) / ncl;
-  }
-  // Next segment: tile, K slices [k0, k1).  False when the pair is done.
-  __device__ bool next(int& tile, int& k0, int& k1) {
-    if (t < dp_tiles) {
-      tile = t;
-      k0 = 0;
-      k1 = num_kc;
-      t += nclusters;
-      return true;
-    }
-    if (u >= u_end) return false;
-    const long long tt = u / num_kc;
-    const long long end = (tt + 1) * num_kc < u_end ? (tt + 1) * num_kc : u_end;
-    tile = dp_tiles + (int)tt;
-    k0 = (int)(u - tt * num_kc);
-    k1 = k0 + (int)(end - u);
-    u = end;
-    return true;
-  }
-};
 
 // kTileN: pair tile width (256, 224 or 192; each CTA holds kTileN / 2 rows of
 // B).  Shared and tensor memory are laid out for 256; narrower tiles leave the
@@ -855,44 +809,6 @@ mixfp4_gemm_skinny_kernel(const __grid_constant__ CUtensorMap tm_wc, const __gri
 }
 
 }  // namespace skinny
-
-PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
-  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
-  if (!fn) {
-    void* p = nullptr;
-    cudaDriverEntryPointQueryResult q;
-    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
-            cudaSuccess &&
-        q == cudaDriverEntryPointSuccess)
-      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
-  }
-  return fn;
-}
-
-// 2D uint8 tensor [rows][row_bytes] (dense), box [box_rows][box_bytes].
-bool make_map(CUtensorMap* m, const void* base, uint64_t row_bytes, uint64_t rows, uint32_t box_bytes,
-              uint32_t box_rows, CUtensorMapSwizzle swz) {
-  auto fn = encode_fn();
-  if (!fn) return false;
-  cuuint64_t dims[2] = {row_bytes, rows};
-  cuuint64_t strides[1] = {row_bytes};
-  cuuint32_t box[2] = {box_bytes, box_rows};
-  cuuint32_t estr[2] = {1, 1};
-  return fn(m, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<void*>(base), dims, strides, box, estr,
-            CU_TENSOR_MAP_INTERLEAVE_NONE, swz, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
-}
-
-int num_sms() {
-  static int n = 0;
-  if (!n) {
-    int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess ||
-        cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0)
-      n = 148;
-  }
-  return n;
-}
 
 }  // namespace
 

@@ -114,6 +114,13 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* m, 
       :: "r"(dst), "l"(reinterpret_cast<uint64_t>(m)), "r"(x), "r"(y), "r"(bar) : "memory");
 }
 
+// 1D bulk copy global -> shared (both addresses 16-byte aligned, bytes a
+// multiple of 16), completing `bytes` of transaction count on `bar`.
+__device__ __forceinline__ void bulk_load(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar) {
+  asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+               :: "r"(dst), "l"(reinterpret_cast<uint64_t>(src)), "r"(bytes), "r"(bar) : "memory");
+}
+
 // Order this thread's generic-proxy shared-memory writes before later
 // async-proxy (tensor core) reads.
 __device__ __forceinline__ void fence_proxy_async_smem() {
@@ -230,6 +237,18 @@ __device__ __forceinline__ void mma_f16_pair_tmem_a(uint32_t d_tmem, uint32_t a_
 }
 // 32 lanes x 32 consecutive 32-bit columns from registers: thread i of the
 // warp writes lane (base lane + i), columns [col, col + 32).
+// Block-scaled E2M1 x E2M1 MMA over a CTA pair (K = 64 per instruction):
+// D[tmem] (+)= (A . B^T) with every 16-element block of A and B multiplied by
+// its ue4m3 scale, read from tensor memory at sfa_tmem / sfb_tmem.
+__device__ __forceinline__ void mma_nvf4_pair(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
+                                              uint32_t sfa_tmem, uint32_t sfb_tmem, uint32_t accumulate) {
+  asm volatile(
+      "{\n.reg .pred p;\nsetp.ne.b32 p, %6, 0;\n"
+      "tcgen05.mma.cta_group::2.kind::mxf4nvf4.block_scale.scale_vec::4X [%0], %1, %2, %3, [%4], [%5], p;\n}"
+      :: "r"(d_tmem), "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(sfa_tmem), "r"(sfb_tmem), "r"(accumulate)
+      : "memory");
+}
+
 __device__ __forceinline__ void tmem_st_32x32b_x32(uint32_t taddr, const uint32_t v[32]) {
   asm volatile(
       "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,"
@@ -273,6 +292,34 @@ __device__ __forceinline__ uint64_t smem_desc_noswizzle(uint32_t saddr, uint32_t
   d |= (uint64_t)1 << 46;  // descriptor version for tcgen05
   // base offset 0, absolute-LBO mode off, layout type 0 = no swizzle
   return d;
+}
+
+// Shared-memory matrix descriptor for a K-major operand stored as the TMA
+// writes it with 128-byte swizzling: rows of 128 bytes, 8-row atoms of 1024
+// bytes (the atom base 1024-byte aligned), 16-byte chunks XOR-ed with the row
+// within the atom.  `saddr` may point 32 * j bytes into the atom's rows (the
+// K step j of an instruction that reads 32 bytes per row); the swizzle is
+// applied to the absolute address.  SBO = 1024 (next 8 rows); LBO is unused
+// for swizzled K-major layouts.
+__device__ __forceinline__ uint64_t smem_desc_sw128(uint32_t saddr) {
+  uint64_t d = 0;
+  d |= (uint64_t)((saddr >> 4) & 0x3FFFu);
+  d |= (uint64_t)1 << 16;             // LBO (ignored)
+  d |= (uint64_t)(1024 >> 4) << 32;   // SBO
+  d |= (uint64_t)1 << 46;             // descriptor version for tcgen05
+  d |= (uint64_t)2 << 61;             // layout type 2: 128-byte swizzle
+  return d;
+}
+
+// Instruction descriptor of the block-scaled tcgen05.mma kind::mxf4nvf4: A and
+// B E2M1 (packed, K-major), scale factors ue4m3 (block 16, scale_vec::4X, so
+// both scale-factor ids 0), D fp32, dense, M x N.
+__host__ __device__ constexpr uint32_t idesc_nvf4_f32(int M, int N) {
+  return (1u << 7)                      // A format: E2M1
+         | (1u << 10)                   // B format: E2M1
+         | ((uint32_t)(N >> 3) << 17)   // N / 8
+         | (0u << 23)                   // scale format: ue4m3
+         | ((uint32_t)(M >> 4) << 24);  // M / 16
 }
 
 // Instruction descriptor of tcgen05.mma kind::f16: D fp32, A and B f16, both

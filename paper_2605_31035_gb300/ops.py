@@ -46,6 +46,10 @@ def lib() -> ctypes.CDLL:
         L.mixfp4_dequantize.argtypes = [P, P, P, I64, I64, P, P]
         L.mixfp4_gemm.restype = I
         L.mixfp4_gemm.argtypes = [P, P, P, P, P, P, I64, I64, I64, P, I64, P, P]
+        L.mixfp4_split_native.restype = I
+        L.mixfp4_split_native.argtypes = [P, P, I64, I64, P, P, P, P]
+        L.mixfp4_gemm_native.restype = I
+        L.mixfp4_gemm_native.argtypes = [P, P, P, P, P, P, P, P, I64, I64, I64, P, I64, P, P]
         L.mixfp4_selftest_bounded_wait.restype = I
         L.mixfp4_selftest_bounded_wait.argtypes = [P, ctypes.c_uint64, P]
         L.mixfp4_status_string.restype = ctypes.c_char_p
@@ -157,6 +161,56 @@ def mixfp4_gemm(a: QTensor, b: QTensor, out: torch.Tensor | None = None,
                            _ptr(b.codes), _ptr(b.scales), _ptr(b.tensor_scale),
                            M, N, K, _ptr(C), C.stride(0), _ptr(status_word), _stream(stream))
     _check("mixfp4_gemm", st)
+    return C
+
+
+@dataclass
+class NativeTensor:
+    """A MixFP4 tensor as native E2M1 operands: main and residual codes
+    [rows, K/2] (residual None when the tensor has no E1M2 block), ue4m3 block
+    scales in the tensor core's tiled layout, and s32."""
+    main: torch.Tensor
+    res: torch.Tensor | None
+    sf: torch.Tensor
+    tensor_scale: torch.Tensor
+
+    @property
+    def rows(self) -> int:
+        return self.main.shape[0]
+
+    @property
+    def K(self) -> int:
+        return self.main.shape[1] * 2
+
+
+def sf_tiled_bytes(rows: int, K: int) -> int:
+    return ((rows + 255) // 256) * 256 * (K // 16)
+
+
+def mixfp4_split_native(q: QTensor, keep_residual: bool = True, stream=None) -> NativeTensor:
+    """Split a MixFP4 tensor into native E2M1 operands.  keep_residual=False
+    drops the residual, which is exact only for tensors without E1M2 blocks
+    (MODE_E2M1_ONLY)."""
+    dev = q.codes.device
+    main = torch.empty_like(q.codes)
+    res = torch.empty_like(q.codes)
+    sf = torch.empty(sf_tiled_bytes(q.rows, q.K), dtype=torch.uint8, device=dev)
+    st = lib().mixfp4_split_native(_ptr(q.codes), _ptr(q.scales), q.rows, q.K, _ptr(main), _ptr(res), _ptr(sf),
+                                   _stream(stream))
+    _check("mixfp4_split_native", st)
+    return NativeTensor(main, res if keep_residual else None, sf, q.tensor_scale)
+
+
+def mixfp4_gemm_native(a: NativeTensor, b: NativeTensor, out: torch.Tensor | None = None,
+                       status_word: torch.Tensor | None = None, stream=None) -> torch.Tensor:
+    """C = A . B^T on the block-scaled FP4 tensor path; a is M x K, b is N x K."""
+    assert a.K == b.K
+    M, N, K = a.rows, b.rows, a.K
+    C = out if out is not None else torch.empty(M, N, dtype=torch.float32, device=a.main.device)
+    st = lib().mixfp4_gemm_native(_ptr(a.main), _ptr(a.res), _ptr(a.sf), _ptr(a.tensor_scale),
+                                  _ptr(b.main), _ptr(b.res), _ptr(b.sf), _ptr(b.tensor_scale),
+                                  M, N, K, _ptr(C), C.stride(0), _ptr(status_word), _stream(stream))
+    _check("mixfp4_gemm_native", st)
     return C
 
 

@@ -95,3 +95,23 @@ def test_product_path_has_no_oracle_or_cpu_fallback():
                 src = open(os.path.join(dirpath, f)).read()
                 assert "import oracle" not in src and "from oracle" not in src, f
                 assert "liboracle" not in src, f
+
+
+def test_native_variant_validation(lib):
+    fake = ctypes.c_void_p(1 << 20)
+    odd = ctypes.c_void_p((1 << 20) + 8)
+    s = lib.mixfp4_split_native
+    assert s(fake, fake, 4, 96, fake, fake, fake, None) == -2          # K % 64
+    assert s(fake, fake, -1, 64, fake, fake, fake, None) == -2
+    assert s(fake, fake, 4, 64, fake, None, fake, None) == -1          # residual output
+    assert s(fake, fake, 4, 64, fake, fake, odd, None) == -3           # tiled scales alignment
+    assert s(fake, fake, 0, 64, None, None, None, None) == 0           # empty: nothing to do
+    g = lib.mixfp4_gemm_native
+    args = lambda **kw: [kw.get(k, fake) for k in ("am", "ar", "asf", "ats", "bm", "br", "bsf", "bts")]
+    assert g(*args(), 4, 4, 128, fake, 4, None, None) == -2                      # K % 256
+    assert g(*args(), 4, 8, 256, fake, 4, None, None) == -2                      # ldc < N
+    assert g(*args(), 4, 4, 256, None, 4, None, None) == -1                      # C
+    assert g(*args(am=None), 4, 4, 256, fake, 4, None, None) == -1               # A main codes
+    assert g(*args(bsf=None), 4, 4, 256, fake, 4, None, None) == -1              # B scales
+    assert g(*args(ar=odd), 4, 4, 256, fake, 4, None, None) == -3                # residual alignment
+    assert g(*args(), 0, 4, 256, fake, 4, None, None) == 0                       # empty M
