@@ -426,6 +426,15 @@ def run_kernel_only(args):
         C = torch.empty(x.shape[0], w.shape[0], dtype=torch.float32, device=dev)
         fn = lambda: ops.mixfp4_gemm(qx, qw, out=C)
         work = 2.0 * x.shape[0] * w.shape[0] * x.shape[1]
+    elif args.kernel == "gemm_native":
+        nx = ops.mixfp4_split_native(qx)
+        nw = ops.mixfp4_split_native(ops.mixfp4_quantize(w, workspace=ws))
+        C = torch.empty(x.shape[0], w.shape[0], dtype=torch.float32, device=dev)
+        fn = lambda: ops.mixfp4_gemm_native(nx, nw, out=C)
+        work = 2.0 * x.shape[0] * w.shape[0] * x.shape[1]
+    elif args.kernel == "split_native":
+        fn = lambda: ops.mixfp4_split_native(qx)
+        work = x.numel() * (0.5 + 1.0 / 16 + 1.0 + 1.0 / 16)
     elif args.kernel == "quantize":
         fn = lambda: ops.mixfp4_quantize(x, out=qx, workspace=ws)
         work = x.numel() * QUANT_BYTES_PER_ELEM
@@ -446,8 +455,9 @@ def run_kernel_only(args):
     e1.record()
     torch.cuda.synchronize()
     ms = e0.elapsed_time(e1) / args.steps
-    unit = "TFLOP/s" if args.kernel == "gemm" else "GB/s"
-    rate = work / (ms * 1e-3) / (1e12 if args.kernel == "gemm" else 1e9)
+    is_gemm = args.kernel.startswith("gemm")
+    unit = "TFLOP/s" if is_gemm else "GB/s"
+    rate = work / (ms * 1e-3) / (1e12 if is_gemm else 1e9)
     print(json.dumps({"kernel": args.kernel, "workload": args.workload, "ms": round(ms, 5),
                       "rate": round(rate, 1), "unit": unit}))
 
@@ -460,7 +470,7 @@ def main(argv=None):
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--cpu-budget", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--kernel", choices=["gemm", "quantize", "quantize_rht", "dequantize"], default=None,
+    ap.add_argument("--kernel", choices=["gemm", "gemm_native", "split_native", "quantize", "quantize_rht", "dequantize"], default=None,
                     help="profiling mode: launch only this kernel")
     ap.add_argument("--workload", default=WORKLOAD,
                     help="tiny|attn|mlp|decode|hadamard|sweepNN (kernel-only mode)")

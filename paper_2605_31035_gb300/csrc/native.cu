@@ -26,17 +26,17 @@
 //               rows of A and 128 rows of B for a 256-wide K slice (128-byte
 //               swizzle, the layout the MMA reads directly), and the scale
 //               tiles of its A rows and of all 256 B rows (1D bulk copies);
-//   warp 1      TMEM allocator; in the leader the MMA-issuing thread, in the
-//               peer the thread that forwards "stage ready" to the leader;
-//   warps 2-5   scale writers: shared -> tensor memory (tcgen05.st), one warp
-//               per TMEM lane quarter; the tiled layout puts row 32c + l's
-//               four scales of a K step in lane l's word c, written to every
-//               lane quarter, so the scale columns of a K step are 4 (A) + 8
-//               (B);
-//   warps 6-21  epilogue: 4 warps per lane quarter, 64 accumulator columns
-//               each in two 32-column rounds (tcgen05.ld -> x s32A s32B ->
-//               fp32 stores or adds to C); the accumulator is released as
-//               soon as the second round is in registers.
+//   warp 1      TMEM allocator; in the leader the MMA-issuing thread, which
+//               also copies each K step's scale tiles from shared to tensor
+//               memory (tcgen05.cp 32x128b.warpx4: the tiled layout puts row
+//               32c + l's four scales of a K step in lane l's word c, and the
+//               copy replicates the 32 lines to every lane quarter, so a K
+//               step takes 4 (A) + 8 (B) scale columns) ahead of its MMAs in
+//               the same tensor-core stream; in the peer the thread that
+//               forwards "stage landed" to the leader;
+//   warps 2-17  epilogue: 4 warps per lane quarter, 64 accumulator columns
+//               each (two 32-column tcgen05.ld, then the accumulator is
+//               released, then x s32A s32B -> fp32 stores or adds to C).
 // TMEM per CTA: 256 fp32 accumulator columns, then 48 scale columns per stage.
 // Every pipeline wait is bounded; a wait that gives up records a status bit
 // and the CTA drains and exits without writing C.
@@ -129,15 +129,15 @@ constexpr uint32_t kSfCols = 12;                  // TMEM columns per K step: 4 
 constexpr uint32_t kStageSfCols = kKSteps * kSfCols;
 constexpr uint32_t kAccCols = TILE_N;
 constexpr uint32_t kTmemCols = 512;
-constexpr int kSfWarps = 4, kEpiWarps = 16;
-constexpr int kFirstSf = 2, kFirstEpi = kFirstSf + kSfWarps;
-constexpr int kThreads = 32 * (kFirstEpi + kEpiWarps);  // 704
+constexpr int kEpiWarps = 16;
+constexpr int kFirstEpi = 2;
+constexpr int kThreads = 32 * (kFirstEpi + kEpiWarps);  // 576
 constexpr int kEpiCols = 64;                             // accumulator columns per epilogue warp
 constexpr int kSmemBudget = 232448 - 1024 - 256;
 constexpr uint64_t kWaitLimitNs = 1000000000ull;
 constexpr int kMaxStages = 5;
 static_assert(kAccCols + kMaxStages * kStageSfCols <= kTmemCols, "TMEM budget");
-static_assert(kFirstSf % 4 == 2 && kFirstEpi % 4 == 2, "warps cover every TMEM lane quarter");
+static_assert(kFirstEpi % 4 == 2, "epilogue warps cover every TMEM lane quarter");
 static_assert(kEpiWarps * kEpiCols == 4 * TILE_N, "epilogue covers the accumulator");
 
 template <bool kARes, bool kBRes>
@@ -160,8 +160,7 @@ struct Layout {
 
 struct Bars {
   uint64_t full[kMaxStages];        // TMA bytes of the stage landed (local)
-  uint64_t ready[kMaxStages];       // leader: kSfWarps local + 1 forwarded arrival
-  uint64_t peer_ready[kMaxStages];  // peer: its kSfWarps arrivals
+  uint64_t ready[kMaxStages];       // leader: the peer's stage landed (forwarded)
   uint64_t empty[kMaxStages];       // MMA commit (multicast to both CTAs)
   uint64_t acc_full;                // MMA commit (multicast)
   uint64_t acc_empty;               // leader: 2 x kEpiWarps arrivals
@@ -196,8 +195,7 @@ nvf4_gemm_kernel(const __grid_constant__ CUtensorMap tm_am, const __grid_constan
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
       mbar_init(smem_u32(&bars->full[s]), 1);
-      mbar_init(smem_u32(&bars->ready[s]), kSfWarps + 1);
-      mbar_init(smem_u32(&bars->peer_ready[s]), kSfWarps);
+      mbar_init(smem_u32(&bars->ready[s]), 1);
       mbar_init(smem_u32(&bars->empty[s]), 1);
     }
     mbar_init(smem_u32(&bars->acc_full), 1);
@@ -285,7 +283,13 @@ nvf4_gemm_kernel(const __grid_constant__ CUtensorMap tm_am, const __grid_constan
         tc_fence_after();
         for (int kc = k0; kc < k1; ++kc, ++it) {
           const int s = it % S;
-          if (!mbar_wait_cluster(smem_u32(&bars->ready[s]), (uint32_t)((it / S) & 1), abort_flag, kWaitLimitNs)) {
+          const uint32_t ph = (uint32_t)((it / S) & 1);
+          if (!mbar_wait(smem_u32(&bars->full[s]), ph, abort_flag, kWaitLimitNs)) {
+            fail(16u);
+            ok = false;
+            break;
+          }
+          if (!mbar_wait_cluster(smem_u32(&bars->ready[s]), ph, abort_flag, kWaitLimitNs)) {
             fail(4u);
             ok = false;
             break;
@@ -296,6 +300,11 @@ nvf4_gemm_kernel(const __grid_constant__ CUtensorMap tm_am, const __grid_constan
           for (int j = 0; j < kKSteps; ++j) {
             const uint32_t sfa = tmem_sf0 + (uint32_t)s * kStageSfCols + (uint32_t)j * kSfCols;
             const uint32_t sfb = sfa + 4;
+            // Scale tiles of this K step (32 lines of 16 bytes each, contiguous).
+            tmem_cp_32x128b_x4_pair(sfa, smem_desc_noswizzle(st + L::OFF_SFA + j * SF_TILE, 128, 128));
+            tmem_cp_32x128b_x4_pair(sfb, smem_desc_noswizzle(st + L::OFF_SFB + j * SF_TILE, 128, 128));
+            tmem_cp_32x128b_x4_pair(sfb + 4,
+                                    smem_desc_noswizzle(st + L::OFF_SFB + SFB_BYTES / 2 + j * SF_TILE, 128, 128));
             const uint64_t am = smem_desc_sw128(st + L::OFF_AM + j * 32);
             const uint64_t bm = smem_desc_sw128(st + L::OFF_BM + j * 32);
             mma_nvf4_pair(tmem_base, am, bm, kIdesc, sfa, sfb, (kc > k0 || j > 0) ? 1u : 0u);
@@ -315,6 +324,8 @@ nvf4_gemm_kernel(const __grid_constant__ CUtensorMap tm_am, const __grid_constan
       if (!mbar_wait_cluster(smem_u32(&bars->drain), 0, nullptr, kWaitLimitNs)) fail(8u);
     } else if (!leader && lane == 0) {
       // ---------------- forwarder (peer CTA) ----------------
+      // The leader's MMAs read this CTA's half of every stage: pass on each
+      // landed stage as one remote arrival.
       const uint32_t ready_leader0 = mapa_shared(smem_u32(&bars->ready[0]), 0);
       int it = 0;
       bool ok = true;
@@ -323,54 +334,13 @@ nvf4_gemm_kernel(const __grid_constant__ CUtensorMap tm_am, const __grid_constan
       while (ok && sched.next(t, k0, k1)) {
         for (int kc = k0; kc < k1; ++kc, ++it) {
           const int s = it % S;
-          if (!mbar_wait(smem_u32(&bars->peer_ready[s]), (uint32_t)((it / S) & 1), abort_flag, kWaitLimitNs)) {
+          if (!mbar_wait(smem_u32(&bars->full[s]), (uint32_t)((it / S) & 1), abort_flag, kWaitLimitNs)) {
             fail(128u);
             ok = false;
             break;
           }
           mbar_arrive_cluster(ready_leader0 + s * 8);
         }
-      }
-    }
-  } else if (warp < kFirstEpi) {
-    // ---------------- scale writers ----------------
-    // Lane l of the warp for lane quarter q writes TMEM lane 32q + l: per K
-    // step j, columns 12j + c (c = 0..3) = 16-byte line l of the A scale tile,
-    // 12j + 4 + c and 12j + 8 + c = line l of the two B scale tiles.
-    const uint32_t q = (uint32_t)(warp & 3);
-    const uint32_t taddr0 = tmem_sf0 + ((q * 32) << 16);
-    int it = 0;
-    bool ok = true;
-    Sched sched(cluster_id, nclusters, dp_tiles, ntiles, num_kc);
-    int t, k0, k1;
-    while (ok && sched.next(t, k0, k1)) {
-      for (int kc = k0; kc < k1; ++kc, ++it) {
-        const int s = it % S;
-        if (!mbar_wait(smem_u32(&bars->full[s]), (uint32_t)((it / S) & 1), abort_flag, kWaitLimitNs)) {
-          fail(16u);
-          ok = false;
-          break;
-        }
-        const uint32_t st = sbase + s * L::STAGE;
-        uint32_t v[kStageSfCols];
-#pragma unroll
-        for (int j = 0; j < kKSteps; ++j) {
-          const uint4 a = lds128(st + L::OFF_SFA + j * SF_TILE + lane * 16);
-          const uint4 b0 = lds128(st + L::OFF_SFB + j * SF_TILE + lane * 16);
-          const uint4 b1 = lds128(st + L::OFF_SFB + SFB_BYTES / 2 + j * SF_TILE + lane * 16);
-          uint32_t* w = v + j * kSfCols;
-          w[0] = a.x; w[1] = a.y; w[2] = a.z; w[3] = a.w;
-          w[4] = b0.x; w[5] = b0.y; w[6] = b0.z; w[7] = b0.w;
-          w[8] = b1.x; w[9] = b1.y; w[10] = b1.z; w[11] = b1.w;
-        }
-        const uint32_t ta = taddr0 + (uint32_t)s * kStageSfCols;
-        tmem_st_32x32b_x16(ta, v);
-        tmem_st_32x32b_x16(ta + 16, v + 16);
-        tmem_st_32x32b_x16(ta + 32, v + 32);
-        tmem_st_wait();
-        tc_fence_before();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(smem_u32(leader ? &bars->ready[s] : &bars->peer_ready[s]));
       }
     }
   } else {
@@ -397,37 +367,34 @@ nvf4_gemm_kernel(const __grid_constant__ CUtensorMap tm_am, const __grid_constan
       const int row = mt * TILE_M + (int)rank * BM + q * 32 + lane;
       const int col0 = nt * TILE_N + cg * kEpiCols;
       float* crow = C + (long long)row * ldc + col0;
+      uint32_t v[kEpiCols];
+      tmem_ld_32x32b_x32(tbase, v);
+      tmem_ld_32x32b_x32(tbase + 32, v + 32);
+      tmem_ld_wait_x32(v);
+      reg_fence16(v + 32);
+      reg_fence16(v + 48);
+      // The accumulator is free once all its columns sit in registers.
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive_cluster(acc_empty_leader);
+      if (row < M) {
 #pragma unroll
-      for (int h = 0; h < kEpiCols / 32; ++h) {
-        uint32_t v[32];
-        tmem_ld_32x32b_x32(tbase + (uint32_t)(32 * h), v);
-        tmem_ld_wait_x32(v);
-        if (h == kEpiCols / 32 - 1) {
-          // The accumulator is free once its last columns sit in registers.
-          tc_fence_before();
-          __syncwarp();
-          if (lane == 0) mbar_arrive_cluster(acc_empty_leader);
-        }
-        if (row < M) {
+        for (int c = 0; c < kEpiCols; c += 4) {
+          float o[4];
 #pragma unroll
-          for (int c = 0; c < 32; c += 4) {
-            const int cc = 32 * h + c;
-            float o[4];
+          for (int e = 0; e < 4; ++e) o[e] = __fmul_rn(__fmul_rn(__uint_as_float(v[c + e]), sa), sb);
+          if (vec_ok && col0 + c + 4 <= N) {
+            if (whole)
+              *reinterpret_cast<float4*>(crow + c) = make_float4(o[0], o[1], o[2], o[3]);
+            else
+              red_add_v4(crow + c, o[0], o[1], o[2], o[3]);
+          } else {
 #pragma unroll
-            for (int e = 0; e < 4; ++e) o[e] = __fmul_rn(__fmul_rn(__uint_as_float(v[c + e]), sa), sb);
-            if (vec_ok && col0 + cc + 4 <= N) {
-              if (whole)
-                *reinterpret_cast<float4*>(crow + cc) = make_float4(o[0], o[1], o[2], o[3]);
-              else
-                red_add_v4(crow + cc, o[0], o[1], o[2], o[3]);
-            } else {
-#pragma unroll
-              for (int e = 0; e < 4; ++e)
-                if (col0 + cc + e < N) {
-                  if (whole) crow[cc + e] = o[e];
-                  else atomicAdd(crow + cc + e, o[e]);
-                }
-            }
+            for (int e = 0; e < 4; ++e)
+              if (col0 + c + e < N) {
+                if (whole) crow[c + e] = o[e];
+                else atomicAdd(crow + c + e, o[e]);
+              }
           }
         }
       }

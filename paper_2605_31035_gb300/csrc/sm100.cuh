@@ -249,6 +249,16 @@ __device__ __forceinline__ void mma_nvf4_pair(uint32_t d_tmem, uint64_t a_desc, 
       : "memory");
 }
 
+// Issued by one thread of the pair's leader CTA: copy 32 rows x 16 bytes from
+// shared memory (matrix descriptor `sdesc`, same shared offset in both CTAs)
+// into the tensor memory of both CTAs, replicated to the four 32-lane
+// quarters: lane 32q + r receives row r as 4 consecutive 32-bit columns from
+// `taddr`.  Ordered with the tcgen05.mma issued after it by the same thread,
+// and tracked by tcgen05.commit like them.
+__device__ __forceinline__ void tmem_cp_32x128b_x4_pair(uint32_t taddr, uint64_t sdesc) {
+  asm volatile("tcgen05.cp.cta_group::2.32x128b.warpx4 [%0], %1;" :: "r"(taddr), "l"(sdesc) : "memory");
+}
+
 __device__ __forceinline__ void tmem_st_32x32b_x32(uint32_t taddr, const uint32_t v[32]) {
   asm volatile(
       "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,"
