@@ -221,6 +221,31 @@ def run_ours(args):
     given_rht = qs.tensor_scale.clone()
     rht_given_ms = time_quant(lambda: ops.mixfp4_quantize_rht(xs, out=qs, tensor_scale=given_rht))
     rht_ms = time_quant(lambda: ops.mixfp4_quantize_rht(xs, out=qs, workspace=ws))
+    # Native block-scaled FP4 variant on the same workload: the weights are
+    # split once (like their quantization), the activations every call.
+    nw = ops.mixfp4_split_native(w_q)
+    nx = ops.mixfp4_split_native(q_x)
+    Cn = torch.empty_like(C)
+
+    def time_flushed(fn, reps=50):
+        for _ in range(3):
+            fn()
+        evs = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(reps)]
+        for e in evs:
+            flush.zero_()
+            e[0].record(stream)
+            fn()
+            e[1].record(stream)
+        torch.cuda.synchronize(dev)
+        return statistics.median(a.elapsed_time(b) for a, b in evs)
+
+    native_gemm_ms = time_flushed(lambda: ops.mixfp4_gemm_native(nx, nw, out=Cn))
+    native_split_ms = time_flushed(lambda: ops.mixfp4_split_native(q_x, out=nx))
+    native_layer_ms = time_flushed(lambda: (ops.mixfp4_quantize(x, out=q_x, workspace=ws),
+                                            ops.mixfp4_split_native(q_x, out=nx),
+                                            ops.mixfp4_gemm_native(nx, nw, out=Cn)))
+    del nw, nx, Cn
+
     given_gbs = xs.numel() * QUANT_BYTES_PER_ELEM / (given_ms * 1e-3) / 1e9
     sweep_alg_gbs = xs.numel() * QUANT_BYTES_PER_ELEM / (sweep_ms * 1e-3) / 1e9
     sweep_read_gbs = xs.numel() * (QUANT_BYTES_PER_ELEM + 2.0) / (sweep_ms * 1e-3) / 1e9
@@ -309,6 +334,13 @@ def run_ours(args):
                                    "alg_frac_of_hbm": round(sweep_alg_gbs / pk["hbm_gbs"], 4),
                                    "bytes_incl_amax_read_gbs": round(sweep_read_gbs, 1)},
                 "alg_bytes_per_element": QUANT_BYTES_PER_ELEM, "hbm_peak_gbs": pk["hbm_gbs"]},
+            "native_fp4_variant": {
+                "gemm_native_ms": round(native_gemm_ms, 5),
+                "gemm_native_tflops": round(flops / (native_gemm_ms * 1e-3) / 1e12, 2),
+                "split_x_ms": round(native_split_ms, 5),
+                "layer_ms_quantize_split_gemm": round(native_layer_ms, 5),
+                "layer_tflops": round(flops / (native_layer_ms * 1e-3) / 1e12, 2),
+                "note": "E1M2 blocks split into E2M1 main + residual, kind::mxf4nvf4 products; weights split once"},
             "rht_quantizer_2^28": {
                 "fused_rotation_quantize_given_scale": {
                     "ms": round(rht_given_ms, 4),

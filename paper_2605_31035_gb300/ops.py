@@ -187,14 +187,19 @@ def sf_tiled_bytes(rows: int, K: int) -> int:
     return ((rows + 255) // 256) * 256 * (K // 16)
 
 
-def mixfp4_split_native(q: QTensor, keep_residual: bool = True, stream=None) -> NativeTensor:
+def mixfp4_split_native(q: QTensor, keep_residual: bool = True, out: NativeTensor | None = None,
+                        stream=None) -> NativeTensor:
     """Split a MixFP4 tensor into native E2M1 operands.  keep_residual=False
     drops the residual, which is exact only for tensors without E1M2 blocks
-    (MODE_E2M1_ONLY)."""
+    (MODE_E2M1_ONLY).  `out` (with a residual buffer) is reused when given."""
     dev = q.codes.device
-    main = torch.empty_like(q.codes)
-    res = torch.empty_like(q.codes)
-    sf = torch.empty(sf_tiled_bytes(q.rows, q.K), dtype=torch.uint8, device=dev)
+    if out is not None:
+        assert out.res is not None and out.main.shape == q.codes.shape
+        main, res, sf = out.main, out.res, out.sf
+    else:
+        main = torch.empty_like(q.codes)
+        res = torch.empty_like(q.codes)
+        sf = torch.empty(sf_tiled_bytes(q.rows, q.K), dtype=torch.uint8, device=dev)
     st = lib().mixfp4_split_native(_ptr(q.codes), _ptr(q.scales), q.rows, q.K, _ptr(main), _ptr(res), _ptr(sf),
                                    _stream(stream))
     _check("mixfp4_split_native", st)
