@@ -16,6 +16,12 @@ Function map (paper passages are cited in ``mixfp4_oracle.c``):
   split_native              MixFP4 operand as the sum of two E2M1 operands with
                             shared scales, plus the tensor core's tiled scale
                             layout (the native FP4 GEMM variant)
+  quantize_colwise          Algorithm 1 along the other dimension (blocks of 16
+                            rows in one column): quantize of the transpose, the
+                            WGRAD / DGRAD operand orientation (Sec. 3.4)
+  quantize_2d               Algorithm 1 with 16 x 16 tiles (2D weight blocks of
+                            the training flow, Sec. 3.4), reading R12
+  transpose_2d              the transposed operand of a 2D-quantized tensor
 """
 from __future__ import annotations
 
@@ -78,6 +84,12 @@ def _L():
         lib.oracle_dequant_row_f64.argtypes = [P, P, ctypes.c_float, I64, I64, P]
         lib.oracle_split_native.argtypes = [P, P, I64, I64, P, P, P]
         lib.oracle_split_native.restype = ctypes.c_int
+        lib.oracle_quantize_2d.restype = ctypes.c_int
+        lib.oracle_quantize_2d.argtypes = [P, I64, I64, I64, ctypes.c_int, ctypes.c_int, P, P, P]
+        lib.oracle_quantize_2d_f32.restype = ctypes.c_int
+        lib.oracle_quantize_2d_f32.argtypes = [P, I64, I64, I64, ctypes.c_int, ctypes.c_int, P, P, P]
+        lib.oracle_transpose_2d.restype = ctypes.c_int
+        lib.oracle_transpose_2d.argtypes = [P, P, I64, I64, P, P]
         _lib = lib
     return _lib
 
@@ -225,3 +237,54 @@ def split_native(codes: np.ndarray, scales: np.ndarray):
     if rc != 0:
         raise ValueError(f"oracle_split_native failed ({rc})")
     return main, res, sf
+
+
+def quantize_colwise(x_bf16_bits: np.ndarray, mode: int = MODE_MIX, s32: float | None = None):
+    """Algorithm 1 with each block running down a column (16 consecutive rows):
+    by definition the row-wise quantization of the transpose.  Returns codes
+    [C, R/2], scales [C, R/16] and s32 for an [R, C] input."""
+    return quantize(np.ascontiguousarray(np.asarray(x_bf16_bits, np.uint16).T), mode, s32)
+
+
+def quantize_2d(x_bf16_bits: np.ndarray, mode: int = MODE_MIX, s32: float | None = None):
+    """Algorithm 1 with 16 x 16 blocks (reading R12) on a [rows, K] bf16 tensor;
+    codes [rows, K/2] and scales [rows, K/16] (each tile's scale byte repeated
+    on its rows), s32."""
+    x = np.ascontiguousarray(x_bf16_bits, dtype=np.uint16)
+    rows, K = x.shape
+    codes = np.zeros((rows, K // 2), np.uint8)
+    scales = np.zeros((rows, K // 16), np.uint8)
+    s = np.array([0.0 if s32 is None else s32], np.float32)
+    rc = _L().oracle_quantize_2d(_p(x), rows, K, K, int(mode), 0 if s32 is None else 1, _p(s),
+                                 _p(codes), _p(scales))
+    if rc != 0:
+        raise ValueError("oracle_quantize_2d rejected the input (non-finite value or K % 16 != 0)")
+    return codes, scales, float(s[0])
+
+
+def quantize_2d_f32(x: np.ndarray, mode: int = MODE_MIX, s32: float | None = None):
+    """quantize_2d on a [rows, K] float32 tensor."""
+    x = np.ascontiguousarray(x, dtype=np.float32)
+    rows, K = x.shape
+    codes = np.zeros((rows, K // 2), np.uint8)
+    scales = np.zeros((rows, K // 16), np.uint8)
+    s = np.array([0.0 if s32 is None else s32], np.float32)
+    rc = _L().oracle_quantize_2d_f32(_p(x), rows, K, K, int(mode), 0 if s32 is None else 1, _p(s),
+                                     _p(codes), _p(scales))
+    if rc != 0:
+        raise ValueError("oracle_quantize_2d_f32 rejected the input")
+    return codes, scales, float(s[0])
+
+
+def transpose_2d(codes: np.ndarray, scales: np.ndarray):
+    """Codes and scales of the transpose of a 2D-quantized tensor (rows % 16 == 0,
+    K % 16 == 0): codes_t [K, rows/2], scales_t [K, rows/16]."""
+    codes = np.ascontiguousarray(codes, np.uint8)
+    scales = np.ascontiguousarray(scales, np.uint8)
+    rows, K = codes.shape[0], codes.shape[1] * 2
+    ct = np.zeros((K, rows // 2), np.uint8)
+    st = np.zeros((K, rows // 16), np.uint8)
+    rc = _L().oracle_transpose_2d(_p(codes), _p(scales), rows, K, _p(ct), _p(st))
+    if rc != 0:
+        raise ValueError(f"oracle_transpose_2d failed ({rc})")
+    return ct, st

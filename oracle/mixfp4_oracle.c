@@ -30,6 +30,11 @@
  *   oracle_split_native  the MixFP4 operand as main + residual E2M1 operands
  *                      sharing its scales (Table 1 codebooks; 5 = 4 + 1,
  *                      7 = 6 + 1), scales in the tensor core's tiled layout
+ *   oracle_quantize_2d Algorithm 1 with 2D 16 x 16 blocks, the weight
+ *                      quantization of the training flow (Sec. 3.4, Sec. 4
+ *                      pre-training recipe); reading R12
+ *   oracle_transpose_2d  the transposed operand (DGRAD orientation) of a
+ *                      2D-quantized tensor: codes and tile scales transposed
  *
  * Readings where the paper is silent (the same list is kept in the design doc):
  *   R1 X_FP8 = fl32(X / s32) is an fp32 value (no FP8 cast).
@@ -53,6 +58,13 @@
  *      pair (i, i+h) with i & h == 0 becoming (fl32(v_i + v_{i+h}),
  *      fl32(v_i - v_{i+h})); then y_i = fl32(v_i * c), c = RN(1/sqrt(128)).
  *      Algorithm 1 then runs on the fp32 y (X = y).
+ *   R12 2D blocks: a block is the 16 x 16 tile of rows 16t..16t+15 and
+ *      columns 16b..16b+15 (a ragged last tile has fewer rows; its missing
+ *      rows count as zeros).  B is the tile max; each candidate has one s8
+ *      from B; each row's 16 elements give the R5 sum S_r; the tile's S is
+ *      the pairwise tree ((S_0+S_1)+(S_2+S_3))+((S_4+S_5)+(S_6+S_7)) + ...
+ *      over the 16 row slots; T is chosen by R6 for the whole tile, and every
+ *      row of the tile stores the tile's scale byte.
  */
 #include <math.h>
 #include <stdint.h>
@@ -411,5 +423,107 @@ int oracle_split_native(const uint8_t* codes, const uint8_t* scales, int64_t row
       int64_t rt = r / 128, rr = r % 128, kt = b / 4;
       sf[(rt * kt_n + kt) * 512 + (rr % 32) * 16 + (rr / 32) * 4 + (b % 4)] = scales[r * nb + b] & 0x7F;
     }
+  return 0;
+}
+
+/* ---------------------------------------------------------------------------
+ * 2D block quantization (Sec. 3.4: weights are quantized in 2D blocks in the
+ * training flow; Sec. 4 pre-training recipe), reading R12: Algorithm 1 with
+ * the block taken as a 16 x 16 tile.
+ * ------------------------------------------------------------------------- */
+static float tree16(const float s[16]) {
+  float l1[8], l2[4], l3[2];
+  for (int i = 0; i < 8; ++i) l1[i] = s[2 * i] + s[2 * i + 1];
+  for (int i = 0; i < 4; ++i) l2[i] = l1[2 * i] + l1[2 * i + 1];
+  for (int i = 0; i < 2; ++i) l3[i] = l2[2 * i] + l2[2 * i + 1];
+  return l3[0] + l3[1];
+}
+
+int oracle_quantize_2d_f32(const float* x, int64_t rows, int64_t K, int64_t ldx, int mode, int scale_given,
+                           float* s32, uint8_t* codes, uint8_t* scales) {
+  if (K % 16 != 0) return -1;
+  float amax = 0.0f;
+  for (int64_t r = 0; r < rows; ++r)
+    for (int64_t k = 0; k < K; ++k) {
+      float v = x[r * ldx + k];
+      if (!isfinite(v)) return -1;
+      if (fabsf(v) > amax) amax = fabsf(v);
+    }
+  float s = scale_given ? *s32 : amax / 2688.0f;   /* Alg. 1 tensor scale */
+  if (!scale_given) *s32 = s;
+  int64_t nb = K / 16;
+  for (int64_t r0 = 0; r0 < rows; r0 += 16) {
+    for (int64_t b = 0; b < nb; ++b) {
+      float a[16][16], B = 0.0f;
+      int sign[16][16];
+      for (int i = 0; i < 16; ++i)
+        for (int k = 0; k < 16; ++k) {
+          float v = (r0 + i < rows) ? x[(r0 + i) * ldx + b * 16 + k] : 0.0f;  /* missing rows: zeros */
+          sign[i][k] = signbit(v) ? 1 : 0;
+          a[i][k] = (s > 0.0f) ? v / s : 0.0f;     /* X_FP8 = X / s32, R1, R7 */
+          if (fabsf(a[i][k]) > B) B = fabsf(a[i][k]);  /* tile max */
+        }
+      int c2 = 0, c1 = 0, p2[16][16], p1[16][16];
+      float S2r[16], S1r[16], S2 = 0.0f, S1 = 0.0f;
+      for (int i = 0; i < 16; ++i) {
+        S2r[i] = S1r[i] = 0.0f;
+        if (mode != 2) candidate(0, a[i], B, &c2, p2[i], &S2r[i]);
+        if (mode != 1) candidate(1, a[i], B, &c1, p1[i], &S1r[i]);
+      }
+      if (mode != 2) S2 = tree16(S2r);
+      if (mode != 1) S1 = tree16(S1r);
+      int T;
+      if (mode == 1) T = 0;
+      else if (mode == 2) T = 1;
+      else T = (S2 < S1) ? 0 : 1;                   /* R6 on the tile */
+      int code = T ? c1 : c2;
+      for (int i = 0; i < 16 && r0 + i < rows; ++i) {
+        const int* p = T ? p1[i] : p2[i];
+        uint8_t* crow = codes + (r0 + i) * (K / 2) + b * 8;
+        for (int j = 0; j < 8; ++j) {
+          int lo = (sign[i][2 * j] << 3) | p[2 * j];
+          int hi = (sign[i][2 * j + 1] << 3) | p[2 * j + 1];
+          crow[j] = (uint8_t)(lo | (hi << 4));      /* R9 */
+        }
+        scales[(r0 + i) * nb + b] = (uint8_t)((T << 7) | code);
+      }
+    }
+  }
+  return 0;
+}
+
+int oracle_quantize_2d(const uint16_t* x, int64_t rows, int64_t K, int64_t ldx, int mode, int scale_given,
+                       float* s32, uint8_t* codes, uint8_t* scales) {
+  if (K % 16 != 0) return -1;
+  float* xf = (float*)malloc((size_t)(rows > 0 ? rows : 1) * (size_t)(K > 0 ? K : 1) * sizeof(float));
+  if (!xf) return -1;
+  for (int64_t r = 0; r < rows; ++r)
+    for (int64_t k = 0; k < K; ++k) xf[r * K + k] = bf16_to_float(x[r * ldx + k]);
+  int rc = oracle_quantize_2d_f32(xf, rows, K, K, mode, scale_given, s32, codes, scales);
+  free(xf);
+  return rc;
+}
+
+/* The transposed operand of a 2D-quantized [rows][K] tensor (rows % 16 == 0,
+ * K % 16 == 0): element (r, k) of the input is element (k, r) of the output
+ * (codes_t [K][rows/2], scales_t [K][rows/16]); the scale of output block
+ * (k, r/16) is the scale byte shared by tile (r/16, k/16).  Returns -2 if a
+ * tile's rows do not share one scale byte (not a 2D-quantized tensor). */
+int oracle_transpose_2d(const uint8_t* codes, const uint8_t* scales, int64_t rows, int64_t K, uint8_t* codes_t,
+                        uint8_t* scales_t) {
+  if (rows % 16 != 0 || K % 16 != 0) return -1;
+  int64_t nb = K / 16, nbt = rows / 16;
+  for (int64_t r = 0; r < rows; ++r)
+    for (int64_t b = 0; b < nb; ++b)
+      if (scales[r * nb + b] != scales[(r / 16) * 16 * nb + b]) return -2;
+  for (int64_t k = 0; k < K; ++k) {
+    for (int64_t j = 0; j < rows / 2; ++j) {
+      int r = (int)(2 * j);
+      int lo = (codes[r * (K / 2) + k / 2] >> (4 * (k % 2))) & 0xF;
+      int hi = (codes[(r + 1) * (K / 2) + k / 2] >> (4 * (k % 2))) & 0xF;
+      codes_t[k * (rows / 2) + j] = (uint8_t)(lo | (hi << 4));
+    }
+    for (int64_t t = 0; t < nbt; ++t) scales_t[k * nbt + t] = scales[(t * 16) * nb + k / 16];
+  }
   return 0;
 }
