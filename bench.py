@@ -246,6 +246,18 @@ def run_ours(args):
                                             ops.mixfp4_gemm_native(nx, nw, out=Cn)))
     del nw, nx, Cn
 
+    # Training-flow orientations on the same 2^28-element tensor: 16-row
+    # blocks down the columns (WGRAD operand) and 16 x 16 blocks (weights),
+    # each with the tensor scale given (the same bytes as the row-wise kernel).
+    qc = ops.empty_qtensor(xs.shape[1], xs.shape[0], dev)
+    colwise_ms = time_quant(lambda: ops.mixfp4_quantize_colwise(xs, out=qc, tensor_scale=given))
+    del qc
+    q2d_ms = time_quant(lambda: ops.mixfp4_quantize_2d(xs, out=qs, tensor_scale=given))
+    qt = ops.QTensor(torch.empty(xs.shape[1], xs.shape[0] // 2, dtype=torch.uint8, device=dev),
+                     torch.empty(xs.shape[1], xs.shape[0] // 16, dtype=torch.uint8, device=dev), qs.tensor_scale)
+    transpose_ms = time_quant(lambda: ops.mixfp4_transpose_2d(qs, out=qt))
+    del qt
+
     given_gbs = xs.numel() * QUANT_BYTES_PER_ELEM / (given_ms * 1e-3) / 1e9
     sweep_alg_gbs = xs.numel() * QUANT_BYTES_PER_ELEM / (sweep_ms * 1e-3) / 1e9
     sweep_read_gbs = xs.numel() * (QUANT_BYTES_PER_ELEM + 2.0) / (sweep_ms * 1e-3) / 1e9
@@ -341,6 +353,13 @@ def run_ours(args):
                 "layer_ms_quantize_split_gemm": round(native_layer_ms, 5),
                 "layer_tflops": round(flops / (native_layer_ms * 1e-3) / 1e12, 2),
                 "note": "E1M2 blocks split into E2M1 main + residual, kind::mxf4nvf4 products; weights split once"},
+            "training_orientations_2^28": {
+                "colwise_given_scale": {"ms": round(colwise_ms, 4),
+                                        "alg_gbs": round(xs_numel * QUANT_BYTES_PER_ELEM / (colwise_ms * 1e-3) / 1e9, 1)},
+                "2d_blocks_given_scale": {"ms": round(q2d_ms, 4),
+                                          "alg_gbs": round(xs_numel * QUANT_BYTES_PER_ELEM / (q2d_ms * 1e-3) / 1e9, 1)},
+                "transpose_2d": {"ms": round(transpose_ms, 4),
+                                 "alg_gbs": round(xs_numel * 2 * (0.5 + 1.0 / 16) / (transpose_ms * 1e-3) / 1e9, 1)}},
             "rht_quantizer_2^28": {
                 "fused_rotation_quantize_given_scale": {
                     "ms": round(rht_given_ms, 4),
@@ -470,6 +489,17 @@ def run_kernel_only(args):
     elif args.kernel == "quantize":
         fn = lambda: ops.mixfp4_quantize(x, out=qx, workspace=ws)
         work = x.numel() * QUANT_BYTES_PER_ELEM
+    elif args.kernel == "quantize_colwise":
+        qc = ops.empty_qtensor(x.shape[1], x.shape[0], dev)
+        fn = lambda: ops.mixfp4_quantize_colwise(x, out=qc, workspace=ws)
+        work = x.numel() * QUANT_BYTES_PER_ELEM
+    elif args.kernel == "quantize_2d":
+        fn = lambda: ops.mixfp4_quantize_2d(x, out=qx, workspace=ws)
+        work = x.numel() * QUANT_BYTES_PER_ELEM
+    elif args.kernel == "transpose_2d":
+        q2 = ops.mixfp4_quantize_2d(x, workspace=ws)
+        fn = lambda: ops.mixfp4_transpose_2d(q2)
+        work = x.numel() * 2 * (0.5 + 1.0 / 16)
     elif args.kernel == "quantize_rht":
         fn = lambda: ops.mixfp4_quantize_rht(x, out=qx, workspace=ws)
         work = x.numel() * QUANT_BYTES_PER_ELEM
@@ -502,7 +532,8 @@ def main(argv=None):
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--cpu-budget", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--kernel", choices=["gemm", "gemm_native", "split_native", "quantize", "quantize_rht", "dequantize"], default=None,
+    ap.add_argument("--kernel", choices=["gemm", "gemm_native", "split_native", "quantize", "quantize_rht", "quantize_colwise",
+                             "quantize_2d", "transpose_2d", "dequantize"], default=None,
                     help="profiling mode: launch only this kernel")
     ap.add_argument("--workload", default=WORKLOAD,
                     help="tiny|attn|mlp|decode|hadamard|sweepNN (kernel-only mode)")

@@ -110,6 +110,61 @@ int mixfp4_quantize_rht(const void* x, int dtype, int64_t rows, int64_t K, int64
                         int scale_flag, void* stream);
 
 /*
+ * mixfp4_quantize_colwise -- Algorithm 1 with every 16-element block running
+ * down a column: the operand orientation of a GEMM that reduces over the rows
+ * of X, as in the weight-gradient GEMM of the training flow (Sec. 3.4, WGRAD
+ * reduces over tokens; DGRAD over the weights' output dimension).  The
+ * result is bit for bit mixfp4_quantize of the transpose X^T:
+ *   codes  [C][R/2]   element r of column c in nibble r % 2 of byte r / 2
+ *   scales [C][R/16]  one byte per 16 rows of a column
+ * s32 = fl32(max|X| / 2688) as for mixfp4_quantize.
+ *
+ * x            device, bf16 [R][ldx]; 32-byte aligned; ldx % 16 == 0, ldx >= C.
+ * R, C         R % 16 == 0, C % 16 == 0 (else MIXFP4_ERR_SHAPE); 0 is a no-op
+ *              (with SCALE_COMPUTE *tensor_scale is set to 0).
+ * codes        device, uint8 [C][R/2], 8-byte aligned.                  (output)
+ * scales       device, uint8 [C][R/16].                                 (output)
+ * tensor_scale, workspace, mode, scale_flag, stream: as mixfp4_quantize.
+ */
+int mixfp4_quantize_colwise(const void* x, int dtype, int64_t R, int64_t C, int64_t ldx, uint8_t* codes,
+                            uint8_t* scales, float* tensor_scale, uint32_t* workspace, int mode, int scale_flag,
+                            void* stream);
+
+/*
+ * mixfp4_quantize_2d -- Algorithm 1 with 16 x 16 blocks, the weight
+ * quantization of the training flow (Sec. 3.4: weights in 2D blocks).  The
+ * tile of rows 16t..16t+15 and columns 16b..16b+15 has one block max (the
+ * tile's), one E4M3 scale per candidate and one type bit; each candidate's
+ * error is the per-row sum of mixfp4_quantize, combined over the tile's 16
+ * rows by the pairwise tree ((S0+S1)+(S2+S3)) + ... in fp32 (rows past the
+ * tensor count as zeros).  Output in the row-wise layout of mixfp4_quantize,
+ * every row of a tile storing the tile's scale byte, so mixfp4_gemm takes it
+ * as is and mixfp4_transpose_2d gives the transposed operand exactly.
+ * Arguments, alignment and errors: as mixfp4_quantize (rows need not be a
+ * multiple of 16).
+ */
+int mixfp4_quantize_2d(const void* x, int dtype, int64_t rows, int64_t K, int64_t ldx, uint8_t* codes,
+                       uint8_t* scales, float* tensor_scale, uint32_t* workspace, int mode, int scale_flag,
+                       void* stream);
+
+/*
+ * mixfp4_transpose_2d -- the MixFP4 tensor W^T of a tensor W quantized with
+ * 2D blocks (mixfp4_quantize_2d): element (r, k) of W is element (k, r) of
+ * the output, and each tile's shared scale byte becomes the scale of the
+ * transposed tile's rows.  It needs no arithmetic: W^T decodes to the
+ * transpose of W's decoded values exactly (the DGRAD operand of the weights).
+ * The scale of a tile is read from its first row, so the input must come
+ * from mixfp4_quantize_2d (or share one scale byte per tile otherwise).
+ *
+ * codes, scales      device, uint8 [rows][K/2] (8-byte aligned), [rows][K/16].
+ * rows, K            rows % 16 == 0, K % 16 == 0 (else MIXFP4_ERR_SHAPE).
+ * codes_t, scales_t  device, uint8 [K][rows/2] (8-byte aligned), [K][rows/16]. (output)
+ * s32 is unchanged (the caller reuses the tensor scale).
+ */
+int mixfp4_transpose_2d(const uint8_t* codes, const uint8_t* scales, int64_t rows, int64_t K, uint8_t* codes_t,
+                        uint8_t* scales_t, void* stream);
+
+/*
  * mixfp4_dequantize -- App. B.2/B.3 decode:
  *   out[r][k] = fl32((-1)^s * v(T, p) * ue4m3(scale & 0x7F) * s32),
  * one rounding of the exact product.

@@ -93,6 +93,77 @@ int mixfp4_quantize_rht(const void* x, int dtype, int64_t rows, int64_t K, int64
   return launch_status();
 }
 
+int mixfp4_quantize_colwise(const void* x, int dtype, int64_t R, int64_t C, int64_t ldx, uint8_t* codes,
+                            uint8_t* scales, float* tensor_scale, uint32_t* workspace, int mode, int scale_flag,
+                            void* stream) {
+  if (dtype != MIXFP4_DTYPE_BF16) return MIXFP4_ERR_DTYPE;
+  if (mode < MIXFP4_MODE_MIX || mode > MIXFP4_MODE_E1M2_ONLY) return MIXFP4_ERR_ARG;
+  if (scale_flag != MIXFP4_SCALE_COMPUTE && scale_flag != MIXFP4_SCALE_GIVEN) return MIXFP4_ERR_ARG;
+  if (R < 0 || C < 0 || R % 16 != 0 || C % 16 != 0 || ldx < C) return MIXFP4_ERR_SHAPE;
+  if (!tensor_scale) return MIXFP4_ERR_NULL;
+  if (scale_flag == MIXFP4_SCALE_COMPUTE && !workspace) return MIXFP4_ERR_NULL;
+  const bool empty = (R == 0 || C == 0);
+  if (!empty && (!x || !codes || !scales)) return MIXFP4_ERR_NULL;
+  if (!empty && (!aligned(x, 32) || ldx % 16 != 0 || !aligned(codes, 8))) return MIXFP4_ERR_ALIGN;
+  if (!aligned(tensor_scale, 4) || (workspace && !aligned(workspace, 4))) return MIXFP4_ERR_ALIGN;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const int given = scale_flag == MIXFP4_SCALE_GIVEN;
+  if (empty) {
+    if (!given && cudaMemsetAsync(tensor_scale, 0, sizeof(float), s) != cudaSuccess) return MIXFP4_ERR_CUDA;
+    return MIXFP4_OK;
+  }
+  const uint16_t* xb = static_cast<const uint16_t*>(x);
+  if (!given) {
+    if (cudaMemsetAsync(workspace, 0, sizeof(uint32_t), s) != cudaSuccess) return MIXFP4_ERR_CUDA;
+    mixfp4::launch_amax(xb, R, C, ldx, workspace, s);  // max |x| does not depend on the orientation
+    if (int st = launch_status()) return st;
+  }
+  if (mixfp4::launch_quantize_colwise(xb, R, C, ldx, codes, scales, tensor_scale, workspace, mode, given, s) != 0)
+    return MIXFP4_ERR_CUDA;
+  return launch_status();
+}
+
+int mixfp4_quantize_2d(const void* x, int dtype, int64_t rows, int64_t K, int64_t ldx, uint8_t* codes,
+                       uint8_t* scales, float* tensor_scale, uint32_t* workspace, int mode, int scale_flag,
+                       void* stream) {
+  if (dtype != MIXFP4_DTYPE_BF16) return MIXFP4_ERR_DTYPE;
+  if (mode < MIXFP4_MODE_MIX || mode > MIXFP4_MODE_E1M2_ONLY) return MIXFP4_ERR_ARG;
+  if (scale_flag != MIXFP4_SCALE_COMPUTE && scale_flag != MIXFP4_SCALE_GIVEN) return MIXFP4_ERR_ARG;
+  if (rows < 0 || K < 0 || K % 16 != 0 || ldx < K) return MIXFP4_ERR_SHAPE;
+  if (!tensor_scale) return MIXFP4_ERR_NULL;
+  if (scale_flag == MIXFP4_SCALE_COMPUTE && !workspace) return MIXFP4_ERR_NULL;
+  const bool empty = (rows == 0 || K == 0);
+  if (!empty && (!x || !codes || !scales)) return MIXFP4_ERR_NULL;
+  if (!empty && (!aligned(x, 32) || ldx % 16 != 0 || !aligned(codes, 8))) return MIXFP4_ERR_ALIGN;
+  if (!aligned(tensor_scale, 4) || (workspace && !aligned(workspace, 4))) return MIXFP4_ERR_ALIGN;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const int given = scale_flag == MIXFP4_SCALE_GIVEN;
+  if (empty) {
+    if (!given && cudaMemsetAsync(tensor_scale, 0, sizeof(float), s) != cudaSuccess) return MIXFP4_ERR_CUDA;
+    return MIXFP4_OK;
+  }
+  const uint16_t* xb = static_cast<const uint16_t*>(x);
+  if (!given) {
+    if (cudaMemsetAsync(workspace, 0, sizeof(uint32_t), s) != cudaSuccess) return MIXFP4_ERR_CUDA;
+    mixfp4::launch_amax(xb, rows, K, ldx, workspace, s);
+    if (int st = launch_status()) return st;
+  }
+  if (mixfp4::launch_quantize_2d(xb, rows, K, ldx, codes, scales, tensor_scale, workspace, mode, given, s) != 0)
+    return MIXFP4_ERR_CUDA;
+  return launch_status();
+}
+
+int mixfp4_transpose_2d(const uint8_t* codes, const uint8_t* scales, int64_t rows, int64_t K, uint8_t* codes_t,
+                        uint8_t* scales_t, void* stream) {
+  if (rows < 0 || K < 0 || rows % 16 != 0 || K % 16 != 0) return MIXFP4_ERR_SHAPE;
+  if (rows == 0 || K == 0) return MIXFP4_OK;
+  if (!codes || !scales || !codes_t || !scales_t) return MIXFP4_ERR_NULL;
+  if (!aligned(codes, 8) || !aligned(codes_t, 8)) return MIXFP4_ERR_ALIGN;
+  if (mixfp4::launch_transpose_2d(codes, scales, rows, K, codes_t, scales_t, static_cast<cudaStream_t>(stream)) != 0)
+    return MIXFP4_ERR_CUDA;
+  return MIXFP4_OK;
+}
+
 int mixfp4_dequantize(const uint8_t* codes, const uint8_t* scales, const float* tensor_scale,
                       int64_t rows, int64_t K, float* out, void* stream) {
   if (rows < 0 || K < 0 || K % 16 != 0) return MIXFP4_ERR_SHAPE;

@@ -18,6 +18,14 @@ int launch_rht_amax(const uint16_t* x, int64_t rows, int64_t K, int64_t ldx, con
 int launch_rht_quantize(const uint16_t* x, int64_t rows, int64_t K, int64_t ldx, const uint8_t* signs,
                         uint8_t* codes, uint8_t* scales, float* tensor_scale, const uint32_t* amax_word, int mode,
                         int scale_given, cudaStream_t stream);
+int launch_quantize_colwise(const uint16_t* x, int64_t R, int64_t C, int64_t ldx, uint8_t* codes, uint8_t* scales,
+                            float* tensor_scale, const uint32_t* amax_word, int mode, int scale_given,
+                            cudaStream_t stream);
+int launch_quantize_2d(const uint16_t* x, int64_t rows, int64_t K, int64_t ldx, uint8_t* codes, uint8_t* scales,
+                       float* tensor_scale, const uint32_t* amax_word, int mode, int scale_given,
+                       cudaStream_t stream);
+int launch_transpose_2d(const uint8_t* codes, const uint8_t* scales, int64_t rows, int64_t K, uint8_t* codes_t,
+                        uint8_t* scales_t, cudaStream_t stream);
 int launch_bounded_wait_selftest(uint32_t* status, uint64_t limit_ns, cudaStream_t stream);
 int launch_dequantize(const uint8_t* codes, const uint8_t* scales, const float* tensor_scale,
                       int64_t rows, int64_t K, float* out, cudaStream_t stream);

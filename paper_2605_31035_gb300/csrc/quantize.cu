@@ -31,243 +31,13 @@
 #include <cuda_runtime.h>
 #include <cstdint>
 
-#include "ptx.cuh"
 #include "kernels.cuh"
+#include "ptx.cuh"
+#include "quant_core.cuh"
 
 namespace mixfp4 {
 
 namespace {
-
-constexpr int kQuantThreads = 256;
-
-// Correctly rounded a / b (per lane) given nb = -b and r = RN(1/b) (Markstein).
-__device__ __forceinline__ u64 div_rn2(u64 a, u64 nb, u64 r) {
-  u64 q0 = mul2(a, r);
-  u64 e = fma2(q0, nb, a);
-  return fma2(e, r, q0);
-}
-
-// RN(a*zh + RN(a*zl)) (per lane): a / b for a divisor b whose (zh, zl) pass
-// the checks described above.
-__device__ __forceinline__ u64 div_kd2(u64 a, u64 zh, u64 zl) { return fma2(a, zh, mul2(a, zl)); }
-
-// (zh, zl) of a divisor b: RN(1/b) and RN(RN(1 - b*zh)/b); (0, 0) for b = 0.
-__device__ __forceinline__ float2 kd_consts(float b) {
-  if (!(b > 0.0f)) return make_float2(0.0f, 0.0f);
-  const float zh = __frcp_rn(b);
-  return make_float2(zh, __fdiv_rn(__fmaf_rn(-b, zh, 1.0f), b));
-}
-
-__device__ __forceinline__ uint32_t lo32(u64 v) { return (uint32_t)v; }
-__device__ __forceinline__ uint32_t hi32(u64 v) { return (uint32_t)(v >> 32); }
-
-struct TensorConsts {
-  float s32;       // per-tensor scale, possibly rescaled to [1, 2)
-  float r32;       // RN(1/s32), or 0 when s32 == 0
-  float2 kd32;     // (zh, zl) of s32
-  float2 kd6, kd7; // (zh, zl) of 6 and 7
-  int k;           // |x| is multiplied by 2^k when `scaled`
-  int scaled;
-};
-
-// Per-tensor constants, derived by every thread (a persistent thread handles
-// many blocks, so this costs a few instructions per block at most).
-__device__ __forceinline__ TensorConsts tensor_consts(float* tensor_scale, const uint32_t* amax_word,
-                                                      int scale_given) {
-  float s32;
-  if (scale_given) {
-    s32 = *tensor_scale;
-  } else {
-    s32 = __fdiv_rn(__uint_as_float(*amax_word), 2688.0f);  // 6*448 = 7*384
-    if (blockIdx.x == 0 && threadIdx.x == 0) *tensor_scale = s32;
-  }
-  TensorConsts c;
-  c.scaled = !(s32 == 0.0f || (s32 >= 0x1p-20f && s32 <= 0x1p100f));
-  c.k = 0;
-  if (c.scaled) {
-    c.k = -ilogbf(s32);
-    s32 = scalbnf(s32, c.k);  // exact, now in [1, 2)
-  }
-  c.s32 = s32;
-  c.r32 = (s32 > 0.0f) ? __frcp_rn(s32) : 0.0f;
-  c.kd32 = kd_consts(s32);
-  c.kd6 = kd_consts(6.0f);
-  c.kd7 = kd_consts(7.0f);
-  return c;
-}
-
-// E2M1 quantization of a pair (RNE, saturating): returns the byte of the two
-// nibbles (first element low) and the dequantized pair as f16x2.
-__device__ __forceinline__ uint32_t e2m1_pair(float lo, float hi, uint32_t& h2) {
-  uint32_t byte;
-  asm("{ .reg .b8 t; cvt.rn.satfinite.e2m1x2.f32 t, %2, %3; cvt.rn.f16x2.e2m1x2 %1, t; cvt.u32.u8 %0, t; }"
-      : "=r"(byte), "=r"(h2) : "f"(hi), "f"(lo));
-  return byte;
-}
-
-// Four byte values (each in the low byte of a word) packed into one word.
-__device__ __forceinline__ uint32_t pack_low_bytes(uint32_t b0, uint32_t b1, uint32_t b2, uint32_t b3) {
-  return prmt(prmt(b0, b1, 0x0040u), prmt(b2, b3, 0x0040u), 0x5410u);
-}
-
-// Sign nibble bits of 8 elements held in 4 bf16 pairs: element 2j -> bit 3 of
-// byte j, element 2j+1 -> bit 7 (the sign bits of the code word).
-__device__ __forceinline__ uint32_t sign_bits(uint32_t w0, uint32_t w1, uint32_t w2, uint32_t w3) {
-  const uint32_t x = prmt(w0, w1, 0x7351u);   // [w0.b1, w1.b1, w0.b3, w1.b3]
-  const uint32_t y = prmt(w2, w3, 0x7351u);
-  const uint32_t even = prmt(x, y, 0x5410u);  // byte j bit 7 = sign of element 2j
-  const uint32_t odd = prmt(x, y, 0x7632u);   // byte j bit 7 = sign of element 2j+1
-  return (odd & 0x80808080u) | ((even >> 4) & 0x08080808u);
-}
-
-// Algorithm 1 for one 16-element block held as 8 bf16 pairs.
-//
-// Tiny-value note: with s32 in [2^-20, 2^100], an element with |x| < 2^-102
-// has |a| < 2^-82.  Its code magnitude is 0 under either candidate (every
-// nonzero block scale is >= 2^-9, and a zero block scale forces 0), and its
-// squared error is below 2^-160, which cannot change a binary32 sum.  So
-// whether its quotient is correctly rounded does not affect any output.  The
-// same holds for |a| < 2^-102 in the |a|/s8 step and for B < 2^-102, where
-// both block scales round to E4M3 zero anyway.
-//
-// E1M2 clamp: when s8 = E4M3(b7) is normal (>= 2^-6) and b7 = fl32(B/7) did
-// not saturate, s8 >= b7 / (1 + 2^-4), so |a|/s8 <= 7 * 1.0625 * (1 + 2^-23)
-// < 7.5 and RNE never exceeds 7; only other blocks need the clamp.
-// kMarkstein selects the x / s32 method (see the header); the other divisions
-// always take the two-instruction form.
-// Algorithm 1 from X_FP8 on, for one 16-element block: a holds |X_FP8| =
-// |x| / s32 as packed pairs (element 2j in the low lane).  Returns the code
-// words without their sign bits and the scale byte.
-template <int kMode>
-__device__ __forceinline__ void block_core(const u64 a[8], const TensorConsts& tc, const float4* __restrict__ tab,
-                                           uint32_t& mag_lo, uint32_t& mag_hi, uint32_t& scale_byte);
-
-template <int kMode, bool kScaled, bool kMarkstein>
-__device__ __forceinline__ void quantize_block(const uint32_t w[8], const TensorConsts& tc,
-                                               const float4* __restrict__ tab, uint32_t& code_lo,
-                                               uint32_t& code_hi, uint32_t& scale_byte) {
-  // |x| as packed fp32 pairs (element 2j in the low lane).
-  u64 a[8];
-  const u64 ns32 = pack2(-tc.s32, -tc.s32), r32 = pack2(tc.r32, tc.r32);
-  const u64 zh32 = pack2(tc.kd32.x, tc.kd32.x), zl32 = pack2(tc.kd32.y, tc.kd32.y);
-#pragma unroll
-  for (int j = 0; j < 8; ++j) {
-    const uint32_t u = w[j] & 0x7FFF7FFFu;
-    uint32_t lo = u << 16, hi = u & 0xFFFF0000u;
-    if (kScaled) {
-      lo = __float_as_uint(scalbnf(__uint_as_float(lo), tc.k));
-      hi = __float_as_uint(scalbnf(__uint_as_float(hi), tc.k));
-    }
-    // X_FP8 = X / s32 (magnitudes)
-    a[j] = kMarkstein ? div_rn2(bits2(lo, hi), ns32, r32) : div_kd2(bits2(lo, hi), zh32, zl32);
-  }
-  uint32_t mlo, mhi;
-  block_core<kMode>(a, tc, tab, mlo, mhi, scale_byte);
-  code_lo = mlo | sign_bits(w[0], w[1], w[2], w[3]);
-  code_hi = mhi | sign_bits(w[4], w[5], w[6], w[7]);
-}
-
-template <int kMode>
-__device__ __forceinline__ void block_core(const u64 a[8], const TensorConsts& tc, const float4* __restrict__ tab,
-                                           uint32_t& mag_lo, uint32_t& mag_hi, uint32_t& scale_byte) {
-  // Block max of |X_FP8|.
-  float v[16];
-#pragma unroll
-  for (int j = 0; j < 8; ++j) unpack2(a[j], v[2 * j], v[2 * j + 1]);
-  float B = max3f(max3f(v[0], v[1], v[2]), max3f(v[3], v[4], v[5]), max3f(v[6], v[7], v[8]));
-  B = max3f(B, max3f(v[9], v[10], v[11]), max3f(v[12], v[13], max3f(v[14], v[15], 0.0f)));
-
-  // Candidate block scales s8 = E4M3(fl32(B/6)), E4M3(fl32(B/7)) and RN(1/s8).
-  const u64 bq = div_kd2(pack2(B, B), pack2(tc.kd6.x, tc.kd7.x), pack2(tc.kd6.y, tc.kd7.y));
-  float b6, b7;
-  unpack2(bq, b6, b7);
-  const uint32_t sc = cvt_e4m3x2(b7, b6);  // low byte: E2M1 scale code, high: E1M2
-  const uint32_t c2 = sc & 0x7Fu, c1 = (sc >> 8) & 0x7Fu;
-
-  float S2 = 0.0f, S1 = 0.0f;
-  uint32_t p2lo = 0, p2hi = 0, p1lo = 0, p1hi = 0;
-  if (kMode != MIXFP4_MODE_E1M2_ONLY) {
-    // E2M1 candidate.
-    const float4 t = tab[c2];
-    const u64 zh8 = pack2(t.y, t.y), zl8 = pack2(t.z, t.z);
-    const uint16_t ns8h = __half_as_ushort(__float2half_rn(-t.x));  // exact: E4M3 values are f16 values
-    u64 acc = 0;  // (+0, +0): even / odd chains
-    uint32_t e[8];
-#pragma unroll
-    for (int j = 0; j < 8; ++j) {
-      const u64 y = div_kd2(a[j], zh8, zl8);
-      float ylo, yhi;
-      unpack2(y, ylo, yhi);
-      uint32_t h2;
-      e[j] = e2m1_pair(ylo, yhi, h2);
-      if (kMode == MIXFP4_MODE_MIX) {
-        float alo, ahi, dlo, dhi;
-        unpack2(a[j], alo, ahi);
-        // d = |a| - q s8 (exact), with q taken straight from its f16 decode
-        asm("{ .reg .f16 ql, qh; mov.b32 {ql, qh}, %2;\n"
-            " fma.rn.f32.f16 %0, ql, %3, %4;\n fma.rn.f32.f16 %1, qh, %3, %5; }"
-            : "=f"(dlo), "=f"(dhi) : "r"(h2), "h"(ns8h), "f"(alo), "f"(ahi));
-        const u64 d = pack2(dlo, dhi);
-        acc = fma2(d, d, acc);
-      }
-    }
-    p2lo = pack_low_bytes(e[0], e[1], e[2], e[3]);
-    p2hi = pack_low_bytes(e[4], e[5], e[6], e[7]);
-    if (kMode == MIXFP4_MODE_MIX) {
-      float se, so;
-      unpack2(acc, se, so);
-      S2 = se + so;
-    }
-  }
-  if (kMode != MIXFP4_MODE_E2M1_ONLY) {
-    // E1M2 candidate (x2 units: integers 0..7).
-    const float4 t = tab[c1];
-    const u64 ns8 = pack2(-t.x, -t.x), zh8 = pack2(t.y, t.y), zl8 = pack2(t.z, t.z);
-    const u64 magic = pack2(12582912.0f, 12582912.0f);    // 1.5 * 2^23
-    const u64 nmagic = pack2(-12582912.0f, -12582912.0f);
-    const bool clamp = !(t.x >= 0x1p-6f && b7 <= 448.0f);
-    u64 acc = 0;
-    uint32_t pb[8];
-#pragma unroll
-    for (int j = 0; j < 8; ++j) {
-      const u64 y = div_kd2(a[j], zh8, zl8);
-      const u64 tq = add2(y, magic);  // RNE to an integer in the low mantissa bits
-      uint32_t tlo = lo32(tq), thi = hi32(tq);
-      if (clamp) {
-        tlo = min(tlo, 0x4B400007u);
-        thi = min(thi, 0x4B400007u);
-      }
-      pb[j] = tlo + (thi << 4);  // low byte: payload pair (first element low)
-      if (kMode == MIXFP4_MODE_MIX) {
-        const u64 q = add2(bits2(tlo, thi), nmagic);
-        const u64 d = fma2(q, ns8, a[j]);
-        acc = fma2(d, d, acc);
-      }
-    }
-    p1lo = pack_low_bytes(pb[0], pb[1], pb[2], pb[3]);
-    p1hi = pack_low_bytes(pb[4], pb[5], pb[6], pb[7]);
-    if (kMode == MIXFP4_MODE_MIX) {
-      float se, so;
-      unpack2(acc, se, so);
-      S1 = se + so;
-    }
-  }
-  int T;
-  if (kMode == MIXFP4_MODE_E2M1_ONLY) T = 0;
-  else if (kMode == MIXFP4_MODE_E1M2_ONLY) T = 1;
-  else T = (S2 < S1) ? 0 : 1;  // strict "<" of Algorithm 1
-
-  mag_lo = T ? p1lo : p2lo;
-  mag_hi = T ? p1hi : p2hi;
-  scale_byte = T ? (0x80u | c1) : c2;
-}
-
-template <bool kContig>
-__device__ __forceinline__ const uint16_t* block_src(const uint16_t* x, int64_t b, int64_t kblocks, int64_t ldx) {
-  if (kContig) return x + b * 16;
-  const int64_t row = b / kblocks;
-  return x + row * ldx + (b - row * kblocks) * 16;
-}
 
 // Persistent grid: each thread walks blocks b, b + nthr, b + 2 nthr, ... and
 // keeps the next block's 32-byte load in flight while it quantizes the
@@ -288,28 +58,10 @@ quantize_kernel(const uint16_t* __restrict__ x, int64_t nblocks, int64_t kblocks
   uint32_t wa[8], wb[8];
   if (b < nblocks) ldg256_stream(block_src<kContig>(x, b, kblocks, ldx), wa);
   if (b + nthr < nblocks) ldg256_stream(block_src<kContig>(x, b + nthr, kblocks, ldx), wb);
-  if (threadIdx.x < 128) {
-    float s8 = 0.0f, unused;
-    if (threadIdx.x < 0x7F) f16x2_to_f32(cvt_f16x2_from_e4m3x2((uint16_t)threadIdx.x), s8, unused);
-    const float2 kd = kd_consts(s8);
-    tab[threadIdx.x] = make_float4(s8, kd.x, kd.y, 0.0f);
-  }
+  fill_scale_table(tab);
   if (after_amax) griddep_wait();
   const TensorConsts tc = tensor_consts(tensor_scale, amax_word, scale_given);
-  // x / s32 may take the two-instruction division when it returns the IEEE
-  // quotient for all 128 bf16 significands (the quotient scales exactly with
-  // x's exponent) and its correction term a*zl stays normal for every
-  // quotient that can matter (|a| >= 2^-82; see the tiny-value note): the
-  // remainder 1 - s32*zh is 0 or at least 2^-44 in magnitude.
-  bool kd_ok = true;
-  if (threadIdx.x < 128 && !tc.scaled) {
-    const float xs = __uint_as_float(0x3F800000u | (threadIdx.x << 16));
-    const u64 q = div_kd2(pack2(xs, xs), pack2(tc.kd32.x, tc.kd32.x), pack2(tc.kd32.y, tc.kd32.y));
-    const float rem = __fmaf_rn(-tc.s32, tc.kd32.x, 1.0f);
-    kd_ok = tc.s32 > 0.0f && lo32(q) == __float_as_uint(__fdiv_rn(xs, tc.s32)) &&
-            (rem == 0.0f || fabsf(rem) >= 0x1p-44f);
-  }
-  const bool markstein = !__syncthreads_and(kd_ok);
+  const bool markstein = markstein_needed(tc);
   for (; b < nblocks; b += 2 * nthr) {
     uint32_t lo, hi, sb;
     if (tc.scaled) quantize_block<kMode, true, true>(wa, tc, tab, lo, hi, sb);

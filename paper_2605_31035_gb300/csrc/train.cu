@@ -1,0 +1,227 @@
+// Quantizer orientations of the MixFP4 training flow (Sec. 3.4: FPROP, DGRAD
+// and WGRAD all run on MixFP4 operands; weights use 2D blocks) for sm_103a.
+//
+//   quantize_colwise_kernel  Algorithm 1 with each 16-element block running
+//       down a column of an [R][C] bf16 tensor: the operand of a GEMM that
+//       reduces over R (WGRAD reduces over tokens).  Output as the row-wise
+//       quantization of the transpose: codes [C][R/2], scales [C][R/16].
+//       A CTA stages a 64-row x 256-column tile in shared memory with
+//       coalesced 16-byte loads; thread t then owns column t, reads its four
+//       16-row blocks (2-byte shared loads, consecutive threads on consecutive
+//       columns, no bank conflicts) and writes 32 contiguous code bytes.
+//   quantize_2d_kernel  Algorithm 1 with 16 x 16 blocks (reading R12): a
+//       half-warp holds one tile, lane i one 16-element row of it, so the
+//       tile max and the tree of the rows' error sums are warp shuffles
+//       (block_core<kMode, true>); the two half-warps of a warp take
+//       horizontally adjacent tiles (64 contiguous bytes per row).  Output in
+//       the row-wise layout, every row of a tile repeating its scale byte, so
+//       mixfp4_gemm consumes it unchanged.
+//   transpose_2d_kernel  codes and tile scales of the transpose of a
+//       2D-quantized tensor (the DGRAD operand of the weights): 64 x 64
+//       element tiles through shared memory, one 8-byte store per thread.
+// Every kernel shares quantize.cu's per-block arithmetic (quant_core.cuh), so
+// its codes are those of Algorithm 1 on the same values bit for bit.
+#include <cuda_runtime.h>
+#include <cstdint>
+
+#include "kernels.cuh"
+#include "ptx.cuh"
+#include "quant_core.cuh"
+
+namespace mixfp4 {
+namespace {
+
+constexpr int kColThreads = 256;        // columns per tile
+constexpr int kColRows = 64;            // rows per tile (four 16-row blocks)
+
+template <int kMode>
+__global__ void __launch_bounds__(kColThreads, 4)
+quantize_colwise_kernel(const uint16_t* __restrict__ x, int64_t R, int64_t C, int64_t ldx,
+                        uint8_t* __restrict__ codes, uint8_t* __restrict__ scales, float* tensor_scale,
+                        const uint32_t* amax_word, int scale_given) {
+  __shared__ float4 tab[128];
+  __shared__ __align__(16) uint16_t tile[kColRows][kColThreads];
+  griddep_wait();
+  griddep_launch_dependents();
+  fill_scale_table(tab);
+  const TensorConsts tc = tensor_consts(tensor_scale, amax_word, scale_given);
+  const bool markstein = markstein_needed(tc);
+  const int tid = threadIdx.x;
+  const int64_t ct_n = (C + kColThreads - 1) / kColThreads, rt_n = (R + kColRows - 1) / kColRows;
+  const int64_t nblk_t = R / 16;  // blocks per output row
+  for (int64_t t = blockIdx.x; t < ct_n * rt_n; t += gridDim.x) {
+    const int64_t r0 = (t / ct_n) * kColRows, c0 = (t % ct_n) * kColThreads;
+    // Stage the tile: 64 rows x 32 chunks of 8 columns (16 bytes).
+#pragma unroll
+    for (int k = 0; k < kColRows * (kColThreads / 8) / kColThreads; ++k) {
+      const int q = tid + k * kColThreads;
+      const int row = q / (kColThreads / 8), ch = q % (kColThreads / 8);
+      uint4 v = make_uint4(0u, 0u, 0u, 0u);
+      if (r0 + row < R && c0 + ch * 8 < C)
+        v = __ldg(reinterpret_cast<const uint4*>(x + (r0 + row) * ldx + c0 + ch * 8));
+      *reinterpret_cast<uint4*>(&tile[row][ch * 8]) = v;
+    }
+    __syncthreads();
+    const int64_t c = c0 + tid;
+    if (c < C) {
+#pragma unroll 1
+      for (int rb = 0; rb < kColRows / 16 && r0 + rb * 16 < R; ++rb) {
+        uint32_t w[8];
+#pragma unroll
+        for (int j = 0; j < 8; ++j)
+          w[j] = (uint32_t)tile[rb * 16 + 2 * j][tid] | ((uint32_t)tile[rb * 16 + 2 * j + 1][tid] << 16);
+        uint32_t lo, hi, sb;
+        if (tc.scaled) quantize_block<kMode, true, true>(w, tc, tab, lo, hi, sb);
+        else if (markstein) quantize_block<kMode, false, true>(w, tc, tab, lo, hi, sb);
+        else quantize_block<kMode, false, false>(w, tc, tab, lo, hi, sb);
+        const int64_t ob = r0 / 16 + rb;  // block index along R
+        stg64(codes + c * (R / 2) + ob * 8, lo, hi);
+        scales[c * nblk_t + ob] = (uint8_t)sb;
+      }
+    }
+    __syncthreads();  // the tile is restaged next
+  }
+}
+
+constexpr int k2dThreads = 256;
+
+template <int kMode>
+__global__ void __launch_bounds__(k2dThreads, 4)
+quantize_2d_kernel(const uint16_t* __restrict__ x, int64_t rows, int64_t K, int64_t ldx,
+                   uint8_t* __restrict__ codes, uint8_t* __restrict__ scales, float* tensor_scale,
+                   const uint32_t* amax_word, int scale_given) {
+  __shared__ float4 tab[128];
+  griddep_wait();
+  griddep_launch_dependents();
+  fill_scale_table(tab);
+  const TensorConsts tc = tensor_consts(tensor_scale, amax_word, scale_given);
+  const bool markstein = markstein_needed(tc);
+  const int lane = threadIdx.x & 31, i = lane & 15, h = lane >> 4;
+  const int64_t nb = K / 16, pairs = (nb + 1) / 2, rt_n = (rows + 15) / 16;
+  const int64_t units = rt_n * pairs;  // (row tile, pair of block columns), one per warp
+  const int64_t warp0 = ((int64_t)blockIdx.x * k2dThreads + threadIdx.x) >> 5;
+  const int64_t nwarps = ((int64_t)gridDim.x * k2dThreads) >> 5;
+  for (int64_t u = warp0; u < units; u += nwarps) {
+    const int64_t r = (u / pairs) * 16 + i, b = (u % pairs) * 2 + h;
+    const bool live = r < rows && b < nb;
+    uint32_t w[8];
+    if (live) {
+      ldg256_stream(x + r * ldx + b * 16, w);
+    } else {
+#pragma unroll
+      for (int j = 0; j < 8; ++j) w[j] = 0u;  // missing rows of a ragged tile count as zeros (R12)
+    }
+    uint32_t lo, hi, sb;
+    if (tc.scaled) quantize_block<kMode, true, true, true>(w, tc, tab, lo, hi, sb);
+    else if (markstein) quantize_block<kMode, false, true, true>(w, tc, tab, lo, hi, sb);
+    else quantize_block<kMode, false, false, true>(w, tc, tab, lo, hi, sb);
+    if (live) {
+      stg64(codes + r * (K / 2) + b * 8, lo, hi);
+      scales[r * nb + b] = (uint8_t)sb;
+    }
+  }
+}
+
+constexpr int kTrTile = 64;  // elements per side of a transpose tile
+
+__global__ void __launch_bounds__(256)
+transpose_2d_kernel(const uint8_t* __restrict__ codes, const uint8_t* __restrict__ scales, int64_t rows, int64_t K,
+                    uint8_t* __restrict__ codes_t, uint8_t* __restrict__ scales_t) {
+  __shared__ uint8_t in[kTrTile][kTrTile / 2 + 4];  // padded rows: fewer bank conflicts on the column reads
+  const int tid = threadIdx.x;
+  const int64_t ct_n = (K + kTrTile - 1) / kTrTile, rt_n = (rows + kTrTile - 1) / kTrTile;
+  for (int64_t t = blockIdx.x; t < ct_n * rt_n; t += gridDim.x) {
+    const int64_t r0 = (t / ct_n) * kTrTile, k0 = (t % ct_n) * kTrTile;
+    // 64 rows x 32 code bytes: one 8-byte load per thread.
+    {
+      const int row = tid >> 2, q = tid & 3;
+      uint2 v = make_uint2(0u, 0u);
+      if (r0 + row < rows && k0 + q * 16 < K)
+        v = *reinterpret_cast<const uint2*>(codes + (r0 + row) * (K / 2) + k0 / 2 + q * 8);
+      *reinterpret_cast<uint32_t*>(&in[row][q * 8]) = v.x;
+      *reinterpret_cast<uint32_t*>(&in[row][q * 8 + 4]) = v.y;
+    }
+    __syncthreads();
+    // Output row k0 + kk (input column), bytes 8 q .. 8 q + 7 = input rows 16 q .. 16 q + 15.
+    {
+      const int kk = tid >> 2, q = tid & 3;
+      const int64_t k = k0 + kk;
+      if (k < K && r0 + q * 16 < rows) {
+        const int sh = 4 * (kk & 1);
+        uint32_t o[2] = {0u, 0u};
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          const uint32_t lo = (in[q * 16 + 2 * j][kk >> 1] >> sh) & 0xFu;
+          const uint32_t hi = (in[q * 16 + 2 * j + 1][kk >> 1] >> sh) & 0xFu;
+          o[j >> 2] |= (lo | (hi << 4)) << (8 * (j & 3));
+        }
+        stg64(codes_t + k * (rows / 2) + r0 / 2 + q * 8, o[0], o[1]);
+        // The tile (r0/16 + q, k/16) scale, shared by the tile's rows.
+        scales_t[k * (rows / 16) + r0 / 16 + q] = scales[(r0 + q * 16) * (K / 16) + k / 16];
+      }
+    }
+    __syncthreads();
+  }
+}
+
+}  // namespace
+
+int launch_quantize_colwise(const uint16_t* x, int64_t R, int64_t C, int64_t ldx, uint8_t* codes, uint8_t* scales,
+                            float* tensor_scale, const uint32_t* amax_word, int mode, int scale_given,
+                            cudaStream_t stream) {
+  const int64_t tiles = ((C + kColThreads - 1) / kColThreads) * ((R + kColRows - 1) / kColRows);
+  if (tiles == 0) return 0;
+  int64_t grid = tiles < 152 * 4 ? tiles : 152 * 4;
+  cudaError_t e;
+  switch (mode) {
+    case MIXFP4_MODE_MIX:
+      e = launch_pdl(quantize_colwise_kernel<MIXFP4_MODE_MIX>, (unsigned)grid, kColThreads, 0, stream, x, R, C, ldx,
+                     codes, scales, tensor_scale, amax_word, scale_given);
+      break;
+    case MIXFP4_MODE_E2M1_ONLY:
+      e = launch_pdl(quantize_colwise_kernel<MIXFP4_MODE_E2M1_ONLY>, (unsigned)grid, kColThreads, 0, stream, x, R, C,
+                     ldx, codes, scales, tensor_scale, amax_word, scale_given);
+      break;
+    default:
+      e = launch_pdl(quantize_colwise_kernel<MIXFP4_MODE_E1M2_ONLY>, (unsigned)grid, kColThreads, 0, stream, x, R, C,
+                     ldx, codes, scales, tensor_scale, amax_word, scale_given);
+      break;
+  }
+  return e == cudaSuccess ? 0 : -1;
+}
+
+int launch_quantize_2d(const uint16_t* x, int64_t rows, int64_t K, int64_t ldx, uint8_t* codes, uint8_t* scales,
+                       float* tensor_scale, const uint32_t* amax_word, int mode, int scale_given,
+                       cudaStream_t stream) {
+  const int64_t units = ((rows + 15) / 16) * ((K / 16 + 1) / 2);
+  if (units == 0) return 0;
+  int64_t grid = (units + k2dThreads / 32 - 1) / (k2dThreads / 32);
+  if (grid > 152 * 4) grid = 152 * 4;
+  cudaError_t e;
+  switch (mode) {
+    case MIXFP4_MODE_MIX:
+      e = launch_pdl(quantize_2d_kernel<MIXFP4_MODE_MIX>, (unsigned)grid, k2dThreads, 0, stream, x, rows, K, ldx,
+                     codes, scales, tensor_scale, amax_word, scale_given);
+      break;
+    case MIXFP4_MODE_E2M1_ONLY:
+      e = launch_pdl(quantize_2d_kernel<MIXFP4_MODE_E2M1_ONLY>, (unsigned)grid, k2dThreads, 0, stream, x, rows, K,
+                     ldx, codes, scales, tensor_scale, amax_word, scale_given);
+      break;
+    default:
+      e = launch_pdl(quantize_2d_kernel<MIXFP4_MODE_E1M2_ONLY>, (unsigned)grid, k2dThreads, 0, stream, x, rows, K,
+                     ldx, codes, scales, tensor_scale, amax_word, scale_given);
+      break;
+  }
+  return e == cudaSuccess ? 0 : -1;
+}
+
+int launch_transpose_2d(const uint8_t* codes, const uint8_t* scales, int64_t rows, int64_t K, uint8_t* codes_t,
+                        uint8_t* scales_t, cudaStream_t stream) {
+  const int64_t tiles = ((K + kTrTile - 1) / kTrTile) * ((rows + kTrTile - 1) / kTrTile);
+  if (tiles == 0) return 0;
+  const int64_t grid = tiles < 152 * 8 ? tiles : 152 * 8;
+  transpose_2d_kernel<<<(unsigned)grid, 256, 0, stream>>>(codes, scales, rows, K, codes_t, scales_t);
+  return cudaGetLastError() == cudaSuccess ? 0 : -1;
+}
+
+}  // namespace mixfp4

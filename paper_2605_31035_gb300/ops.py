@@ -42,6 +42,12 @@ def lib() -> ctypes.CDLL:
         L.mixfp4_quantize.argtypes = [P, I, I64, I64, I64, P, P, P, P, I, I, P]
         L.mixfp4_quantize_rht.restype = I
         L.mixfp4_quantize_rht.argtypes = [P, I, I64, I64, I64, P, P, P, P, P, I, I, P]
+        L.mixfp4_quantize_colwise.restype = I
+        L.mixfp4_quantize_colwise.argtypes = [P, I, I64, I64, I64, P, P, P, P, I, I, P]
+        L.mixfp4_quantize_2d.restype = I
+        L.mixfp4_quantize_2d.argtypes = [P, I, I64, I64, I64, P, P, P, P, I, I, P]
+        L.mixfp4_transpose_2d.restype = I
+        L.mixfp4_transpose_2d.argtypes = [P, P, I64, I64, P, P, P]
         L.mixfp4_dequantize.restype = I
         L.mixfp4_dequantize.argtypes = [P, P, P, I64, I64, P, P]
         L.mixfp4_gemm.restype = I
@@ -141,6 +147,61 @@ def mixfp4_quantize_rht(x: torch.Tensor, signs: torch.Tensor | None = None, mode
                                    SCALE_GIVEN if given else SCALE_COMPUTE, _stream(stream))
     _check("mixfp4_quantize_rht", st)
     return q
+
+
+def mixfp4_quantize_colwise(x: torch.Tensor, mode: int = MODE_MIX, tensor_scale: torch.Tensor | None = None,
+                            out: QTensor | None = None, workspace: torch.Tensor | None = None,
+                            stream=None) -> QTensor:
+    """Quantize a bf16 [R, C] CUDA tensor with 16-row blocks down each column
+    (the orientation of a GEMM reducing over R): returns the MixFP4 tensor of
+    X^T, codes [C, R/2], scales [C, R/16]."""
+    assert x.dtype == torch.bfloat16 and x.dim() == 2 and x.stride(1) == 1
+    R, C = x.shape
+    q = out if out is not None else empty_qtensor(C, R, x.device)
+    given = tensor_scale is not None
+    if given:
+        q.tensor_scale.copy_(tensor_scale.reshape(1))
+    ws = None
+    if not given:
+        ws = workspace if workspace is not None else torch.empty(1, dtype=torch.int32, device=x.device)
+    st = lib().mixfp4_quantize_colwise(_ptr(x), DTYPE_BF16, R, C, x.stride(0), _ptr(q.codes), _ptr(q.scales),
+                                       _ptr(q.tensor_scale), _ptr(ws), int(mode),
+                                       SCALE_GIVEN if given else SCALE_COMPUTE, _stream(stream))
+    _check("mixfp4_quantize_colwise", st)
+    return q
+
+
+def mixfp4_quantize_2d(x: torch.Tensor, mode: int = MODE_MIX, tensor_scale: torch.Tensor | None = None,
+                       out: QTensor | None = None, workspace: torch.Tensor | None = None,
+                       stream=None) -> QTensor:
+    """Quantize a bf16 [rows, K] CUDA tensor with 16 x 16 blocks (one scale
+    and format per tile, repeated on the tile's rows)."""
+    assert x.dtype == torch.bfloat16 and x.dim() == 2 and x.stride(1) == 1
+    rows, K = x.shape
+    q = out if out is not None else empty_qtensor(rows, K, x.device)
+    given = tensor_scale is not None
+    if given:
+        q.tensor_scale.copy_(tensor_scale.reshape(1))
+    ws = None
+    if not given:
+        ws = workspace if workspace is not None else torch.empty(1, dtype=torch.int32, device=x.device)
+    st = lib().mixfp4_quantize_2d(_ptr(x), DTYPE_BF16, rows, K, x.stride(0), _ptr(q.codes), _ptr(q.scales),
+                                  _ptr(q.tensor_scale), _ptr(ws), int(mode),
+                                  SCALE_GIVEN if given else SCALE_COMPUTE, _stream(stream))
+    _check("mixfp4_quantize_2d", st)
+    return q
+
+
+def mixfp4_transpose_2d(q: QTensor, out: QTensor | None = None, stream=None) -> QTensor:
+    """The transpose of a 2D-quantized tensor (rows and K multiples of 16);
+    the tensor scale is shared with the input."""
+    t = out if out is not None else QTensor(
+        torch.empty(q.K, q.rows // 2, dtype=torch.uint8, device=q.codes.device),
+        torch.empty(q.K, q.rows // 16, dtype=torch.uint8, device=q.codes.device), q.tensor_scale)
+    st = lib().mixfp4_transpose_2d(_ptr(q.codes), _ptr(q.scales), q.rows, q.K, _ptr(t.codes), _ptr(t.scales),
+                                   _stream(stream))
+    _check("mixfp4_transpose_2d", st)
+    return t
 
 
 def mixfp4_dequantize(q: QTensor, out: torch.Tensor | None = None, stream=None) -> torch.Tensor:

@@ -115,3 +115,27 @@ def test_native_variant_validation(lib):
     assert g(*args(bsf=None), 4, 4, 256, fake, 4, None, None) == -1              # B scales
     assert g(*args(ar=odd), 4, 4, 256, fake, 4, None, None) == -3                # residual alignment
     assert g(*args(), 0, 4, 256, fake, 4, None, None) == 0                       # empty M
+
+
+def test_training_orientation_validation(lib):
+    fake = ctypes.c_void_p(1 << 20)
+    ws = ctypes.c_void_p(1 << 21)
+    c = lib.mixfp4_quantize_colwise
+    assert c(fake, 0, 24, 32, 32, fake, fake, fake, ws, 0, 0, None) == -2       # R % 16
+    assert c(fake, 0, 32, 24, 32, fake, fake, fake, ws, 0, 0, None) == -2       # C % 16
+    assert c(fake, 0, 32, 32, 16, fake, fake, fake, ws, 0, 0, None) == -2       # ldx < C
+    assert c(fake, 7, 32, 32, 32, fake, fake, fake, ws, 0, 0, None) == -4       # dtype
+    assert c(fake, 0, 32, 32, 32, fake, fake, fake, None, 0, 0, None) == -1     # workspace
+    assert c(fake, 0, 32, 32, 32, fake, fake, fake, ws, 4, 0, None) == -7       # mode
+    assert c(ctypes.c_void_p((1 << 20) + 16), 0, 32, 32, 32, fake, fake, fake, ws, 0, 0, None) == -3
+    q = lib.mixfp4_quantize_2d
+    assert q(fake, 0, 5, 24, 24, fake, fake, fake, ws, 0, 0, None) == -2        # K % 16
+    assert q(fake, 0, 5, 32, 32, None, fake, fake, ws, 0, 0, None) == -1        # codes
+    assert q(fake, 0, 5, 32, 40, fake, fake, fake, ws, 0, 1, None) == -3        # ldx % 16
+    assert q(fake, 0, 5, 32, 32, fake, fake, fake, ws, 0, 3, None) == -7        # scale flag
+    t = lib.mixfp4_transpose_2d
+    assert t(fake, fake, 24, 32, fake, fake, None) == -2                        # rows % 16
+    assert t(fake, fake, 32, 24, fake, fake, None) == -2                        # K % 16
+    assert t(fake, None, 32, 32, fake, fake, None) == -1
+    assert t(fake, fake, 32, 32, ctypes.c_void_p((1 << 20) + 4), fake, None) == -3
+    assert t(fake, fake, 0, 32, None, None, None) == 0                          # empty
