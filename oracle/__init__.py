@@ -22,6 +22,10 @@ Function map (paper passages are cited in ``mixfp4_oracle.c``):
   quantize_2d               Algorithm 1 with 16 x 16 tiles (2D weight blocks of
                             the training flow, Sec. 3.4), reading R12
   transpose_2d              the transposed operand of a 2D-quantized tensor
+  philox4x32_10             Salmon et al.'s counter-based generator (SC'11)
+  quantize_sr               Algorithm 1 with stochastic rounding of the chosen
+                            format's codes (reading R13); quantize_colwise_sr
+                            the same down the columns
 """
 from __future__ import annotations
 
@@ -88,6 +92,15 @@ def _L():
         lib.oracle_quantize_2d.argtypes = [P, I64, I64, I64, ctypes.c_int, ctypes.c_int, P, P, P]
         lib.oracle_quantize_2d_f32.restype = ctypes.c_int
         lib.oracle_quantize_2d_f32.argtypes = [P, I64, I64, I64, ctypes.c_int, ctypes.c_int, P, P, P]
+        lib.oracle_philox4x32_10.restype = None
+        lib.oracle_philox4x32_10.argtypes = [P, P, P]
+        lib.oracle_sr_uniform.restype = ctypes.c_float
+        lib.oracle_sr_uniform.argtypes = [ctypes.c_uint64, ctypes.c_uint64, ctypes.c_uint64]
+        lib.oracle_sr_payload.restype = ctypes.c_int
+        lib.oracle_sr_payload.argtypes = [ctypes.c_int, ctypes.c_float, ctypes.c_float]
+        lib.oracle_quantize_sr.restype = ctypes.c_int
+        lib.oracle_quantize_sr.argtypes = [P, I64, I64, I64, ctypes.c_int, ctypes.c_int, P, ctypes.c_uint64,
+                                           ctypes.c_uint64, P, P]
         lib.oracle_transpose_2d.restype = ctypes.c_int
         lib.oracle_transpose_2d.argtypes = [P, P, I64, I64, P, P]
         _lib = lib
@@ -288,3 +301,41 @@ def transpose_2d(codes: np.ndarray, scales: np.ndarray):
     if rc != 0:
         raise ValueError(f"oracle_transpose_2d failed ({rc})")
     return ct, st
+
+
+def philox4x32_10(ctr, key):
+    """The four output words of Philox4x32-10 for a 4-word counter and 2-word key."""
+    c = np.ascontiguousarray(np.asarray(ctr, np.uint32))
+    k = np.ascontiguousarray(np.asarray(key, np.uint32))
+    out = np.zeros(4, np.uint32)
+    _L().oracle_philox4x32_10(_p(c), _p(k), _p(out))
+    return out
+
+
+def sr_uniform(seed: int, offset: int, e: int) -> float:
+    return _L().oracle_sr_uniform(int(seed), int(offset), int(e))
+
+
+def sr_payload(fmt: int, m: float, eps: float) -> int:
+    return _L().oracle_sr_payload(int(fmt), float(m), float(eps))
+
+
+def quantize_sr(x_bf16_bits: np.ndarray, seed: int, offset: int = 0, mode: int = MODE_MIX,
+                s32: float | None = None):
+    """Algorithm 1 with stochastic rounding (reading R13) on a [rows, K] bf16 tensor."""
+    x = np.ascontiguousarray(x_bf16_bits, dtype=np.uint16)
+    rows, K = x.shape
+    codes = np.zeros((rows, K // 2), np.uint8)
+    scales = np.zeros((rows, K // 16), np.uint8)
+    s = np.array([0.0 if s32 is None else s32], np.float32)
+    rc = _L().oracle_quantize_sr(_p(x), rows, K, K, int(mode), 0 if s32 is None else 1, _p(s), int(seed),
+                                 int(offset), _p(codes), _p(scales))
+    if rc != 0:
+        raise ValueError("oracle_quantize_sr rejected the input")
+    return codes, scales, float(s[0])
+
+
+def quantize_colwise_sr(x_bf16_bits: np.ndarray, seed: int, offset: int = 0, mode: int = MODE_MIX,
+                        s32: float | None = None):
+    """quantize_sr of the transpose (element index c * R + r of an [R, C] input)."""
+    return quantize_sr(np.ascontiguousarray(np.asarray(x_bf16_bits, np.uint16).T), seed, offset, mode, s32)

@@ -35,6 +35,12 @@
  *                      pre-training recipe); reading R12
  *   oracle_transpose_2d  the transposed operand (DGRAD orientation) of a
  *                      2D-quantized tensor: codes and tile scales transposed
+ *   oracle_philox4x32_10  the counter-based generator of J. K. Salmon et al.,
+ *                      "Parallel random numbers: as easy as 1, 2, 3" (SC'11),
+ *                      source of the stochastic-rounding uniforms
+ *   oracle_quantize_sr Algorithm 1 with stochastic rounding of the codes
+ *                      (App. "Ablation Study of Stochastic Rounding", Sec. 4
+ *                      pre-training recipe: SR on gradients); reading R13
  *
  * Readings where the paper is silent (the same list is kept in the design doc):
  *   R1 X_FP8 = fl32(X / s32) is an fp32 value (no FP8 cast).
@@ -65,6 +71,18 @@
  *      the pairwise tree ((S_0+S_1)+(S_2+S_3))+((S_4+S_5)+(S_6+S_7)) + ...
  *      over the 16 row slots; T is chosen by R6 for the whole tile, and every
  *      row of the tile stores the tile's scale byte.
+ *   R13 stochastic rounding: the format and block scale are chosen exactly as
+ *      in Algorithm 1 (round-to-nearest candidates, R4-R6); the chosen
+ *      format's codes are then rounded stochastically: with m = fl32(|a|/s8)
+ *      and l <= m < u its two neighbours in the codebook (m at or above the
+ *      largest value saturates), the code is u iff eps < (m - l) / (u - l)
+ *      (both exact fp32 values), else l, so P(u) = (m - l) / (u - l): the
+ *      probability falls with the distance, as the paper states; its integer
+ *      formula clamp(round(q + eps - 0.5)) is the same distribution on the
+ *      E1M2 grid.  eps = (w >> 8) * 2^-24 for the word w of Philox4x32-10
+ *      with key (seed low, seed high) and counter (e / 4 low, e / 4 high,
+ *      offset low, offset high), word e % 4, e = the element's row-major index
+ *      (r * K + k).  The sign bit stays signbit(x).
  */
 #include <math.h>
 #include <stdint.h>
@@ -525,5 +543,80 @@ int oracle_transpose_2d(const uint8_t* codes, const uint8_t* scales, int64_t row
     }
     for (int64_t t = 0; t < nbt; ++t) scales_t[k * nbt + t] = scales[(t * 16) * nb + k / 16];
   }
+  return 0;
+}
+
+/* ---------------------------------------------------------------------------
+ * Philox4x32-10 (Salmon, Moraes, Dror, Shaw, SC'11): ten rounds of two 32x32
+ * -> 64-bit products with the multipliers 0xD2511F53 and 0xCD9E8D57, the key
+ * bumped by (0x9E3779B9, 0xBB67AE85) between rounds.
+ * ------------------------------------------------------------------------- */
+void oracle_philox4x32_10(const uint32_t ctr[4], const uint32_t key[2], uint32_t out[4]) {
+  uint32_t c0 = ctr[0], c1 = ctr[1], c2 = ctr[2], c3 = ctr[3], k0 = key[0], k1 = key[1];
+  for (int round = 0; round < 10; ++round) {
+    if (round > 0) {
+      k0 += 0x9E3779B9u;
+      k1 += 0xBB67AE85u;
+    }
+    uint64_t p0 = (uint64_t)0xD2511F53u * c0;
+    uint64_t p1 = (uint64_t)0xCD9E8D57u * c2;
+    uint32_t n0 = (uint32_t)(p1 >> 32) ^ c1 ^ k0;
+    uint32_t n1 = (uint32_t)p1;
+    uint32_t n2 = (uint32_t)(p0 >> 32) ^ c3 ^ k1;
+    uint32_t n3 = (uint32_t)p0;
+    c0 = n0; c1 = n1; c2 = n2; c3 = n3;
+  }
+  out[0] = c0; out[1] = c1; out[2] = c2; out[3] = c3;
+}
+
+/* The R13 uniform of element e: a multiple of 2^-24 in [0, 1). */
+float oracle_sr_uniform(uint64_t seed, uint64_t offset, uint64_t e) {
+  uint32_t ctr[4] = {(uint32_t)(e / 4), (uint32_t)((e / 4) >> 32), (uint32_t)offset, (uint32_t)(offset >> 32)};
+  uint32_t key[2] = {(uint32_t)seed, (uint32_t)(seed >> 32)};
+  uint32_t w[4];
+  oracle_philox4x32_10(ctr, key, w);
+  return (float)(w[e % 4] >> 8) * 0x1p-24f;
+}
+
+/* R13: the stochastic payload of magnitude m in format `type`, by search over
+ * the codebook for the neighbours l <= m < u. */
+int oracle_sr_payload(int type, float m, float eps) {
+  double lo = -1.0, hi = INFINITY;
+  int plo = 0, phi = -1;
+  for (int p = 0; p < 8; ++p) {
+    double v = oracle_fp4_value(type, p);
+    if (v <= m && v > lo) { lo = v; plo = p; }
+    if (v > m && v < hi) { hi = v; phi = p; }
+  }
+  if (phi < 0) return plo;                          /* at or above the maximum */
+  double f = ((double)m - lo) / (hi - lo);          /* exact: an fp32 value */
+  return ((double)eps < f) ? phi : plo;
+}
+
+/* Algorithm 1 with stochastic rounding of the chosen format (R13) on a
+ * [rows][K] bf16 tensor; arguments as oracle_quantize plus seed and offset. */
+int oracle_quantize_sr(const uint16_t* x, int64_t rows, int64_t K, int64_t ldx, int mode, int scale_given,
+                       float* s32, uint64_t seed, uint64_t offset, uint8_t* codes, uint8_t* scales) {
+  if (K % 16 != 0) return -1;
+  int rc = oracle_quantize(x, rows, K, ldx, mode, scale_given, s32, codes, scales, NULL, NULL);
+  if (rc != 0) return rc;
+  float s = *s32;
+  int64_t nb = K / 16;
+  for (int64_t r = 0; r < rows; ++r)
+    for (int64_t b = 0; b < nb; ++b) {
+      int T = scales[r * nb + b] >> 7;
+      float s8 = (float)oracle_e4m3_value(scales[r * nb + b] & 0x7F);
+      for (int i = 0; i < 16; ++i) {
+        int64_t k = b * 16 + i;
+        float v = bf16_to_float(x[r * ldx + k]);
+        float a = (s > 0.0f) ? v / s : 0.0f;                    /* R1, R7 */
+        float m = (s8 > 0.0f) ? fabsf(a) / s8 : 0.0f;           /* R4's quotient */
+        float eps = oracle_sr_uniform(seed, offset, (uint64_t)(r * K + k));
+        int p = oracle_sr_payload(T, m, eps);
+        int nib = ((signbit(v) ? 1 : 0) << 3) | p;
+        uint8_t* byte = codes + r * (K / 2) + k / 2;
+        *byte = (uint8_t)((k % 2) ? ((*byte & 0x0F) | (nib << 4)) : ((*byte & 0xF0) | nib));
+      }
+    }
   return 0;
 }
