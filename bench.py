@@ -257,6 +257,7 @@ def run_ours(args):
                      torch.empty(xs.shape[1], xs.shape[0] // 16, dtype=torch.uint8, device=dev), qs.tensor_scale)
     transpose_ms = time_quant(lambda: ops.mixfp4_transpose_2d(qs, out=qt))
     del qt
+    sr_ms = time_quant(lambda: ops.mixfp4_quantize_sr(xs, 1234, 0, out=qs, tensor_scale=given))
 
     given_gbs = xs.numel() * QUANT_BYTES_PER_ELEM / (given_ms * 1e-3) / 1e9
     sweep_alg_gbs = xs.numel() * QUANT_BYTES_PER_ELEM / (sweep_ms * 1e-3) / 1e9
@@ -358,6 +359,8 @@ def run_ours(args):
                                         "alg_gbs": round(xs_numel * QUANT_BYTES_PER_ELEM / (colwise_ms * 1e-3) / 1e9, 1)},
                 "2d_blocks_given_scale": {"ms": round(q2d_ms, 4),
                                           "alg_gbs": round(xs_numel * QUANT_BYTES_PER_ELEM / (q2d_ms * 1e-3) / 1e9, 1)},
+                "stochastic_rounding_given_scale": {
+                    "ms": round(sr_ms, 4), "alg_gbs": round(xs_numel * QUANT_BYTES_PER_ELEM / (sr_ms * 1e-3) / 1e9, 1)},
                 "transpose_2d": {"ms": round(transpose_ms, 4),
                                  "alg_gbs": round(xs_numel * 2 * (0.5 + 1.0 / 16) / (transpose_ms * 1e-3) / 1e9, 1)}},
             "rht_quantizer_2^28": {

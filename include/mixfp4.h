@@ -131,6 +131,35 @@ int mixfp4_quantize_colwise(const void* x, int dtype, int64_t R, int64_t C, int6
                             void* stream);
 
 /*
+ * mixfp4_quantize_sr, mixfp4_quantize_colwise_sr -- mixfp4_quantize and
+ * mixfp4_quantize_colwise with stochastic rounding of the codes, the
+ * gradient quantization of the training flow (Sec. 4 pre-training recipe;
+ * the paper's stochastic-rounding ablation).  Format and block scale are
+ * chosen exactly as Algorithm 1 chooses them (round-to-nearest candidates, so
+ * scale bytes and s32 equal those of the rounding-to-nearest entry point);
+ * then each code of the chosen format is rounded stochastically: with
+ * m = fl32(|x / s32| / s8) and l <= m < u its neighbours in the codebook,
+ * the magnitude is u iff eps < (m - l) / (u - l), else l (m at or above the
+ * largest value saturates), so the value rounds up with probability
+ * (m - l) / (u - l).  The sign bit is signbit(x).
+ *   eps = (w >> 8) * 2^-24, w = word e % 4 of Philox4x32-10 (Salmon et al.,
+ *   SC'11) with key (seed & 0xFFFFFFFF, seed >> 32) and counter
+ *   (e / 4 low word, e / 4 high word, offset low word, offset high word),
+ *   e = the element's index in the output tensor's row-major order (r * K + k
+ *   for mixfp4_quantize_sr; c * R + r, i.e. in X^T, for the column-wise one).
+ * A fresh (seed, offset) per call gives independent draws; the same pair
+ * reproduces the same codes.
+ * Other arguments, layouts and errors: as mixfp4_quantize and
+ * mixfp4_quantize_colwise.
+ */
+int mixfp4_quantize_sr(const void* x, int dtype, int64_t rows, int64_t K, int64_t ldx, uint8_t* codes,
+                       uint8_t* scales, float* tensor_scale, uint32_t* workspace, int mode, int scale_flag,
+                       uint64_t seed, uint64_t offset, void* stream);
+int mixfp4_quantize_colwise_sr(const void* x, int dtype, int64_t R, int64_t C, int64_t ldx, uint8_t* codes,
+                               uint8_t* scales, float* tensor_scale, uint32_t* workspace, int mode, int scale_flag,
+                               uint64_t seed, uint64_t offset, void* stream);
+
+/*
  * mixfp4_quantize_2d -- Algorithm 1 with 16 x 16 blocks, the weight
  * quantization of the training flow (Sec. 3.4: weights in 2D blocks).  The
  * tile of rows 16t..16t+15 and columns 16b..16b+15 has one block max (the

@@ -93,9 +93,12 @@ int mixfp4_quantize_rht(const void* x, int dtype, int64_t rows, int64_t K, int64
   return launch_status();
 }
 
-int mixfp4_quantize_colwise(const void* x, int dtype, int64_t R, int64_t C, int64_t ldx, uint8_t* codes,
-                            uint8_t* scales, float* tensor_scale, uint32_t* workspace, int mode, int scale_flag,
-                            void* stream) {
+namespace {
+
+// Shared body of the column-wise entry points (sr = 0: round to nearest).
+int quantize_colwise_impl(const void* x, int dtype, int64_t R, int64_t C, int64_t ldx, uint8_t* codes,
+                          uint8_t* scales, float* tensor_scale, uint32_t* workspace, int mode, int scale_flag,
+                          int sr, uint64_t seed, uint64_t offset, void* stream) {
   if (dtype != MIXFP4_DTYPE_BF16) return MIXFP4_ERR_DTYPE;
   if (mode < MIXFP4_MODE_MIX || mode > MIXFP4_MODE_E1M2_ONLY) return MIXFP4_ERR_ARG;
   if (scale_flag != MIXFP4_SCALE_COMPUTE && scale_flag != MIXFP4_SCALE_GIVEN) return MIXFP4_ERR_ARG;
@@ -118,7 +121,55 @@ int mixfp4_quantize_colwise(const void* x, int dtype, int64_t R, int64_t C, int6
     mixfp4::launch_amax(xb, R, C, ldx, workspace, s);  // max |x| does not depend on the orientation
     if (int st = launch_status()) return st;
   }
-  if (mixfp4::launch_quantize_colwise(xb, R, C, ldx, codes, scales, tensor_scale, workspace, mode, given, s) != 0)
+  if (mixfp4::launch_quantize_colwise(xb, R, C, ldx, codes, scales, tensor_scale, workspace, mode, given, sr, seed,
+                                      offset, s) != 0)
+    return MIXFP4_ERR_CUDA;
+  return launch_status();
+}
+
+}  // namespace
+
+int mixfp4_quantize_colwise(const void* x, int dtype, int64_t R, int64_t C, int64_t ldx, uint8_t* codes,
+                            uint8_t* scales, float* tensor_scale, uint32_t* workspace, int mode, int scale_flag,
+                            void* stream) {
+  return quantize_colwise_impl(x, dtype, R, C, ldx, codes, scales, tensor_scale, workspace, mode, scale_flag, 0, 0, 0,
+                               stream);
+}
+
+int mixfp4_quantize_colwise_sr(const void* x, int dtype, int64_t R, int64_t C, int64_t ldx, uint8_t* codes,
+                               uint8_t* scales, float* tensor_scale, uint32_t* workspace, int mode, int scale_flag,
+                               uint64_t seed, uint64_t offset, void* stream) {
+  return quantize_colwise_impl(x, dtype, R, C, ldx, codes, scales, tensor_scale, workspace, mode, scale_flag, 1, seed,
+                               offset, stream);
+}
+
+int mixfp4_quantize_sr(const void* x, int dtype, int64_t rows, int64_t K, int64_t ldx, uint8_t* codes,
+                       uint8_t* scales, float* tensor_scale, uint32_t* workspace, int mode, int scale_flag,
+                       uint64_t seed, uint64_t offset, void* stream) {
+  if (dtype != MIXFP4_DTYPE_BF16) return MIXFP4_ERR_DTYPE;
+  if (mode < MIXFP4_MODE_MIX || mode > MIXFP4_MODE_E1M2_ONLY) return MIXFP4_ERR_ARG;
+  if (scale_flag != MIXFP4_SCALE_COMPUTE && scale_flag != MIXFP4_SCALE_GIVEN) return MIXFP4_ERR_ARG;
+  if (rows < 0 || K < 0 || K % 16 != 0 || ldx < K) return MIXFP4_ERR_SHAPE;
+  if (!tensor_scale) return MIXFP4_ERR_NULL;
+  if (scale_flag == MIXFP4_SCALE_COMPUTE && !workspace) return MIXFP4_ERR_NULL;
+  const bool empty = (rows == 0 || K == 0);
+  if (!empty && (!x || !codes || !scales)) return MIXFP4_ERR_NULL;
+  if (!empty && (!aligned(x, 32) || ldx % 16 != 0 || !aligned(codes, 8))) return MIXFP4_ERR_ALIGN;
+  if (!aligned(tensor_scale, 4) || (workspace && !aligned(workspace, 4))) return MIXFP4_ERR_ALIGN;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const int given = scale_flag == MIXFP4_SCALE_GIVEN;
+  if (empty) {
+    if (!given && cudaMemsetAsync(tensor_scale, 0, sizeof(float), s) != cudaSuccess) return MIXFP4_ERR_CUDA;
+    return MIXFP4_OK;
+  }
+  const uint16_t* xb = static_cast<const uint16_t*>(x);
+  if (!given) {
+    if (cudaMemsetAsync(workspace, 0, sizeof(uint32_t), s) != cudaSuccess) return MIXFP4_ERR_CUDA;
+    mixfp4::launch_amax(xb, rows, K, ldx, workspace, s);
+    if (int st = launch_status()) return st;
+  }
+  if (mixfp4::launch_quantize_sr(xb, rows, K, ldx, codes, scales, tensor_scale, workspace, mode, given, seed, offset,
+                                 s) != 0)
     return MIXFP4_ERR_CUDA;
   return launch_status();
 }

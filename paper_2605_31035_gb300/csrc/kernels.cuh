@@ -19,8 +19,11 @@ int launch_rht_quantize(const uint16_t* x, int64_t rows, int64_t K, int64_t ldx,
                         uint8_t* codes, uint8_t* scales, float* tensor_scale, const uint32_t* amax_word, int mode,
                         int scale_given, cudaStream_t stream);
 int launch_quantize_colwise(const uint16_t* x, int64_t R, int64_t C, int64_t ldx, uint8_t* codes, uint8_t* scales,
-                            float* tensor_scale, const uint32_t* amax_word, int mode, int scale_given,
-                            cudaStream_t stream);
+                            float* tensor_scale, const uint32_t* amax_word, int mode, int scale_given, int sr,
+                            uint64_t seed, uint64_t offset, cudaStream_t stream);
+int launch_quantize_sr(const uint16_t* x, int64_t rows, int64_t K, int64_t ldx, uint8_t* codes, uint8_t* scales,
+                       float* tensor_scale, const uint32_t* amax_word, int mode, int scale_given, uint64_t seed,
+                       uint64_t offset, cudaStream_t stream);
 int launch_quantize_2d(const uint16_t* x, int64_t rows, int64_t K, int64_t ldx, uint8_t* codes, uint8_t* scales,
                        float* tensor_scale, const uint32_t* amax_word, int mode, int scale_given,
                        cudaStream_t stream);

@@ -260,6 +260,96 @@ __device__ __forceinline__ void block_core(const u64 a[8], const TensorConsts& t
   scale_byte = T ? (0x80u | c1) : c2;
 }
 
+// ---- stochastic rounding (reading R13) --------------------------------------
+// Philox4x32-10 (J. K. Salmon, M. A. Moraes, R. O. Dror, D. E. Shaw, "Parallel
+// random numbers: as easy as 1, 2, 3", SC'11): ten rounds of two 32 x 32-bit
+// products (multipliers 0xD2511F53, 0xCD9E8D57), key bumped by
+// (0x9E3779B9, 0xBB67AE85) between rounds.
+__device__ __forceinline__ uint4 philox4x32_10(uint4 c, uint32_t k0, uint32_t k1) {
+#pragma unroll
+  for (int round = 0; round < 10; ++round) {
+    if (round > 0) {
+      k0 += 0x9E3779B9u;
+      k1 += 0xBB67AE85u;
+    }
+    const uint32_t lo0 = 0xD2511F53u * c.x, hi0 = __umulhi(0xD2511F53u, c.x);
+    const uint32_t lo1 = 0xCD9E8D57u * c.z, hi1 = __umulhi(0xCD9E8D57u, c.z);
+    c = make_uint4(hi1 ^ c.y ^ k0, lo1, hi0 ^ c.w ^ k1, lo0);
+  }
+  return c;
+}
+
+// Stochastic payloads of a magnitude m = |a| / s8 (exact fp32 arithmetic
+// throughout): with l <= m < u the codebook neighbours, u iff eps < (m - l) /
+// (u - l); m at or above the largest value saturates.
+__device__ __forceinline__ uint32_t sr_payload_e1m2(float m, float eps) {
+  if (!(m < 7.0f)) return 7u;
+  const float l = floorf(m);
+  return (uint32_t)l + (eps < m - l ? 1u : 0u);
+}
+__device__ __forceinline__ uint32_t sr_payload_e2m1(float m, float eps) {
+  if (!(m < 6.0f)) return 7u;                                   // 6
+  if (m >= 4.0f) return 6u + (eps < (m - 4.0f) * 0.5f ? 1u : 0u);  // 4 or 6
+  if (m >= 2.0f) {
+    const float l = floorf(m);                                  // 2 or 3: payloads 4, 5
+    return (uint32_t)l + 2u + (eps < m - l ? 1u : 0u);
+  }
+  const float u = m * 2.0f, l = floorf(u);                      // 0, .5, 1, 1.5: payloads 0..3
+  return (uint32_t)l + (eps < u - l ? 1u : 0u);
+}
+
+// Algorithm 1 for one block (format and scale exactly as quantize_block
+// chooses them), then the chosen format's codes rounded stochastically.  e0 is
+// the logical index of the block's first element (a multiple of 16): element
+// e0 + i draws word i % 4 of Philox4x32-10 with counter (e0 / 4 + i / 4,
+// offset) and key seed, eps = (word >> 8) * 2^-24.
+template <int kMode, bool kScaled, bool kMarkstein>
+__device__ __forceinline__ void quantize_block_sr(const uint32_t w[8], const TensorConsts& tc,
+                                                  const float4* __restrict__ tab, uint64_t seed, uint64_t offset,
+                                                  uint64_t e0, uint32_t& code_lo, uint32_t& code_hi,
+                                                  uint32_t& scale_byte) {
+  u64 a[8];
+  const u64 ns32 = pack2(-tc.s32, -tc.s32), r32 = pack2(tc.r32, tc.r32);
+  const u64 zh32 = pack2(tc.kd32.x, tc.kd32.x), zl32 = pack2(tc.kd32.y, tc.kd32.y);
+#pragma unroll
+  for (int j = 0; j < 8; ++j) {
+    const uint32_t u = w[j] & 0x7FFF7FFFu;
+    uint32_t lo = u << 16, hi = u & 0xFFFF0000u;
+    if (kScaled) {
+      lo = __float_as_uint(scalbnf(__uint_as_float(lo), tc.k));
+      hi = __float_as_uint(scalbnf(__uint_as_float(hi), tc.k));
+    }
+    a[j] = kMarkstein ? div_rn2(bits2(lo, hi), ns32, r32) : div_kd2(bits2(lo, hi), zh32, zl32);
+  }
+  uint32_t unused_lo, unused_hi;
+  block_core<kMode>(a, tc, tab, unused_lo, unused_hi, scale_byte);
+  const float4 t = tab[scale_byte & 0x7Fu];
+  const bool e1m2 = (scale_byte >> 7) != 0;
+  const u64 zh8 = pack2(t.y, t.y), zl8 = pack2(t.z, t.z);
+  uint32_t bytes[8];
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    const uint64_t c = e0 / 4 + (uint64_t)q;
+    const uint4 r = philox4x32_10(make_uint4((uint32_t)c, (uint32_t)(c >> 32), (uint32_t)offset,
+                                             (uint32_t)(offset >> 32)),
+                                  (uint32_t)seed, (uint32_t)(seed >> 32));
+    const uint32_t rw[4] = {r.x, r.y, r.z, r.w};
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {  // pair j = 2q + h holds elements 4q + 2h, 4q + 2h + 1
+      const int j = 2 * q + h;
+      float mlo, mhi;
+      unpack2(div_kd2(a[j], zh8, zl8), mlo, mhi);  // fl32(|a| / s8), as Algorithm 1's quotient
+      const float elo = __uint2float_rn(rw[2 * h] >> 8) * 0x1p-24f;
+      const float ehi = __uint2float_rn(rw[2 * h + 1] >> 8) * 0x1p-24f;
+      const uint32_t plo = e1m2 ? sr_payload_e1m2(mlo, elo) : sr_payload_e2m1(mlo, elo);
+      const uint32_t phi = e1m2 ? sr_payload_e1m2(mhi, ehi) : sr_payload_e2m1(mhi, ehi);
+      bytes[j] = plo | (phi << 4);
+    }
+  }
+  code_lo = pack_low_bytes(bytes[0], bytes[1], bytes[2], bytes[3]) | sign_bits(w[0], w[1], w[2], w[3]);
+  code_hi = pack_low_bytes(bytes[4], bytes[5], bytes[6], bytes[7]) | sign_bits(w[4], w[5], w[6], w[7]);
+}
+
 // E4M3 code -> {s8, zh, zl, 0} table of the block scales (zh, zl: see div_kd2),
 // filled by the CTA's first 128 threads.
 __device__ __forceinline__ void fill_scale_table(float4* tab) {

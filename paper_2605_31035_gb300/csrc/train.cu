@@ -16,6 +16,9 @@
 //       horizontally adjacent tiles (64 contiguous bytes per row).  Output in
 //       the row-wise layout, every row of a tile repeating its scale byte, so
 //       mixfp4_gemm consumes it unchanged.
+//   quantize_sr_kernel  row-wise quantization with stochastic rounding of the
+//       chosen format's codes (reading R13, the gradients of the training
+//       flow); quantize_colwise_kernel<.., true> the same down the columns.
 //   transpose_2d_kernel  codes and tile scales of the transpose of a
 //       2D-quantized tensor (the DGRAD operand of the weights): 64 x 64
 //       element tiles through shared memory, one 8-byte store per thread.
@@ -34,11 +37,11 @@ namespace {
 constexpr int kColThreads = 256;        // columns per tile
 constexpr int kColRows = 64;            // rows per tile (four 16-row blocks)
 
-template <int kMode>
+template <int kMode, bool kSR>
 __global__ void __launch_bounds__(kColThreads, 4)
 quantize_colwise_kernel(const uint16_t* __restrict__ x, int64_t R, int64_t C, int64_t ldx,
                         uint8_t* __restrict__ codes, uint8_t* __restrict__ scales, float* tensor_scale,
-                        const uint32_t* amax_word, int scale_given) {
+                        const uint32_t* amax_word, int scale_given, uint64_t seed, uint64_t offset) {
   __shared__ float4 tab[128];
   __shared__ __align__(16) uint16_t tile[kColRows][kColThreads];
   griddep_wait();
@@ -71,15 +74,50 @@ quantize_colwise_kernel(const uint16_t* __restrict__ x, int64_t R, int64_t C, in
         for (int j = 0; j < 8; ++j)
           w[j] = (uint32_t)tile[rb * 16 + 2 * j][tid] | ((uint32_t)tile[rb * 16 + 2 * j + 1][tid] << 16);
         uint32_t lo, hi, sb;
-        if (tc.scaled) quantize_block<kMode, true, true>(w, tc, tab, lo, hi, sb);
-        else if (markstein) quantize_block<kMode, false, true>(w, tc, tab, lo, hi, sb);
-        else quantize_block<kMode, false, false>(w, tc, tab, lo, hi, sb);
         const int64_t ob = r0 / 16 + rb;  // block index along R
+        if (kSR) {
+          const uint64_t e0 = (uint64_t)c * (uint64_t)R + (uint64_t)ob * 16;  // element index in X^T
+          if (tc.scaled) quantize_block_sr<kMode, true, true>(w, tc, tab, seed, offset, e0, lo, hi, sb);
+          else if (markstein) quantize_block_sr<kMode, false, true>(w, tc, tab, seed, offset, e0, lo, hi, sb);
+          else quantize_block_sr<kMode, false, false>(w, tc, tab, seed, offset, e0, lo, hi, sb);
+        } else {
+          if (tc.scaled) quantize_block<kMode, true, true>(w, tc, tab, lo, hi, sb);
+          else if (markstein) quantize_block<kMode, false, true>(w, tc, tab, lo, hi, sb);
+          else quantize_block<kMode, false, false>(w, tc, tab, lo, hi, sb);
+        }
         stg64(codes + c * (R / 2) + ob * 8, lo, hi);
         scales[c * nblk_t + ob] = (uint8_t)sb;
       }
     }
     __syncthreads();  // the tile is restaged next
+  }
+}
+
+// Row-wise quantization with stochastic rounding (R13): one thread per
+// 16-element block, grid-stride; the element index of block b's first element
+// is 16 b (row-major over [rows][K]).
+template <int kMode, bool kContig>
+__global__ void __launch_bounds__(256, 3)
+quantize_sr_kernel(const uint16_t* __restrict__ x, int64_t nblocks, int64_t kblocks, int64_t ldx,
+                   uint8_t* __restrict__ codes, uint8_t* __restrict__ scales, float* tensor_scale,
+                   const uint32_t* amax_word, int scale_given, uint64_t seed, uint64_t offset) {
+  __shared__ float4 tab[128];
+  griddep_wait();
+  griddep_launch_dependents();
+  fill_scale_table(tab);
+  const TensorConsts tc = tensor_consts(tensor_scale, amax_word, scale_given);
+  const bool markstein = markstein_needed(tc);
+  const int64_t nthr = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t b = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; b < nblocks; b += nthr) {
+    uint32_t w[8];
+    ldg256_stream(block_src<kContig>(x, b, kblocks, ldx), w);
+    uint32_t lo, hi, sb;
+    const uint64_t e0 = (uint64_t)b * 16;
+    if (tc.scaled) quantize_block_sr<kMode, true, true>(w, tc, tab, seed, offset, e0, lo, hi, sb);
+    else if (markstein) quantize_block_sr<kMode, false, true>(w, tc, tab, seed, offset, e0, lo, hi, sb);
+    else quantize_block_sr<kMode, false, false>(w, tc, tab, seed, offset, e0, lo, hi, sb);
+    stg64(codes + b * 8, lo, hi);
+    scales[b] = (uint8_t)sb;
   }
 }
 
@@ -167,26 +205,49 @@ transpose_2d_kernel(const uint8_t* __restrict__ codes, const uint8_t* __restrict
 }  // namespace
 
 int launch_quantize_colwise(const uint16_t* x, int64_t R, int64_t C, int64_t ldx, uint8_t* codes, uint8_t* scales,
-                            float* tensor_scale, const uint32_t* amax_word, int mode, int scale_given,
-                            cudaStream_t stream) {
+                            float* tensor_scale, const uint32_t* amax_word, int mode, int scale_given, int sr,
+                            uint64_t seed, uint64_t offset, cudaStream_t stream) {
   const int64_t tiles = ((C + kColThreads - 1) / kColThreads) * ((R + kColRows - 1) / kColRows);
   if (tiles == 0) return 0;
   int64_t grid = tiles < 152 * 4 ? tiles : 152 * 4;
   cudaError_t e;
+#define MIXFP4_LAUNCH_C(MODE, SR)                                                                            \
+  e = launch_pdl(quantize_colwise_kernel<MODE, SR>, (unsigned)grid, kColThreads, 0, stream, x, R, C, ldx, codes, \
+                 scales, tensor_scale, amax_word, scale_given, seed, offset)
   switch (mode) {
     case MIXFP4_MODE_MIX:
-      e = launch_pdl(quantize_colwise_kernel<MIXFP4_MODE_MIX>, (unsigned)grid, kColThreads, 0, stream, x, R, C, ldx,
-                     codes, scales, tensor_scale, amax_word, scale_given);
+      if (sr) MIXFP4_LAUNCH_C(MIXFP4_MODE_MIX, true); else MIXFP4_LAUNCH_C(MIXFP4_MODE_MIX, false);
       break;
     case MIXFP4_MODE_E2M1_ONLY:
-      e = launch_pdl(quantize_colwise_kernel<MIXFP4_MODE_E2M1_ONLY>, (unsigned)grid, kColThreads, 0, stream, x, R, C,
-                     ldx, codes, scales, tensor_scale, amax_word, scale_given);
+      if (sr) MIXFP4_LAUNCH_C(MIXFP4_MODE_E2M1_ONLY, true); else MIXFP4_LAUNCH_C(MIXFP4_MODE_E2M1_ONLY, false);
       break;
     default:
-      e = launch_pdl(quantize_colwise_kernel<MIXFP4_MODE_E1M2_ONLY>, (unsigned)grid, kColThreads, 0, stream, x, R, C,
-                     ldx, codes, scales, tensor_scale, amax_word, scale_given);
+      if (sr) MIXFP4_LAUNCH_C(MIXFP4_MODE_E1M2_ONLY, true); else MIXFP4_LAUNCH_C(MIXFP4_MODE_E1M2_ONLY, false);
       break;
   }
+#undef MIXFP4_LAUNCH_C
+  return e == cudaSuccess ? 0 : -1;
+}
+
+int launch_quantize_sr(const uint16_t* x, int64_t rows, int64_t K, int64_t ldx, uint8_t* codes, uint8_t* scales,
+                       float* tensor_scale, const uint32_t* amax_word, int mode, int scale_given, uint64_t seed,
+                       uint64_t offset, cudaStream_t stream) {
+  const int64_t kblocks = K / 16, nblocks = rows * kblocks;
+  if (nblocks == 0) return 0;
+  int64_t grid = (nblocks + 255) / 256;
+  if (grid > 152 * 3) grid = 152 * 3;
+  cudaError_t e;
+#define MIXFP4_LAUNCH_S(MODE)                                                                               \
+  e = (ldx == K) ? launch_pdl(quantize_sr_kernel<MODE, true>, (unsigned)grid, 256, 0, stream, x, nblocks, kblocks, \
+                              ldx, codes, scales, tensor_scale, amax_word, scale_given, seed, offset)          \
+                 : launch_pdl(quantize_sr_kernel<MODE, false>, (unsigned)grid, 256, 0, stream, x, nblocks,       \
+                              kblocks, ldx, codes, scales, tensor_scale, amax_word, scale_given, seed, offset)
+  switch (mode) {
+    case MIXFP4_MODE_MIX: MIXFP4_LAUNCH_S(MIXFP4_MODE_MIX); break;
+    case MIXFP4_MODE_E2M1_ONLY: MIXFP4_LAUNCH_S(MIXFP4_MODE_E2M1_ONLY); break;
+    default: MIXFP4_LAUNCH_S(MIXFP4_MODE_E1M2_ONLY); break;
+  }
+#undef MIXFP4_LAUNCH_S
   return e == cudaSuccess ? 0 : -1;
 }
 

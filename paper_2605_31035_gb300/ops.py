@@ -44,6 +44,11 @@ def lib() -> ctypes.CDLL:
         L.mixfp4_quantize_rht.argtypes = [P, I, I64, I64, I64, P, P, P, P, P, I, I, P]
         L.mixfp4_quantize_colwise.restype = I
         L.mixfp4_quantize_colwise.argtypes = [P, I, I64, I64, I64, P, P, P, P, I, I, P]
+        U64 = ctypes.c_uint64
+        L.mixfp4_quantize_sr.restype = I
+        L.mixfp4_quantize_sr.argtypes = [P, I, I64, I64, I64, P, P, P, P, I, I, U64, U64, P]
+        L.mixfp4_quantize_colwise_sr.restype = I
+        L.mixfp4_quantize_colwise_sr.argtypes = [P, I, I64, I64, I64, P, P, P, P, I, I, U64, U64, P]
         L.mixfp4_quantize_2d.restype = I
         L.mixfp4_quantize_2d.argtypes = [P, I, I64, I64, I64, P, P, P, P, I, I, P]
         L.mixfp4_transpose_2d.restype = I
@@ -168,6 +173,28 @@ def mixfp4_quantize_colwise(x: torch.Tensor, mode: int = MODE_MIX, tensor_scale:
                                        _ptr(q.tensor_scale), _ptr(ws), int(mode),
                                        SCALE_GIVEN if given else SCALE_COMPUTE, _stream(stream))
     _check("mixfp4_quantize_colwise", st)
+    return q
+
+
+def mixfp4_quantize_sr(x: torch.Tensor, seed: int, offset: int = 0, mode: int = MODE_MIX,
+                       tensor_scale: torch.Tensor | None = None, out: QTensor | None = None,
+                       workspace: torch.Tensor | None = None, colwise: bool = False, stream=None) -> QTensor:
+    """mixfp4_quantize (or, with colwise=True, mixfp4_quantize_colwise) with
+    stochastic rounding of the codes drawn from (seed, offset)."""
+    assert x.dtype == torch.bfloat16 and x.dim() == 2 and x.stride(1) == 1
+    rows, K = x.shape
+    q = out if out is not None else (empty_qtensor(K, rows, x.device) if colwise else empty_qtensor(rows, K, x.device))
+    given = tensor_scale is not None
+    if given:
+        q.tensor_scale.copy_(tensor_scale.reshape(1))
+    ws = None
+    if not given:
+        ws = workspace if workspace is not None else torch.empty(1, dtype=torch.int32, device=x.device)
+    fn = lib().mixfp4_quantize_colwise_sr if colwise else lib().mixfp4_quantize_sr
+    st = fn(_ptr(x), DTYPE_BF16, rows, K, x.stride(0), _ptr(q.codes), _ptr(q.scales), _ptr(q.tensor_scale),
+            _ptr(ws), int(mode), SCALE_GIVEN if given else SCALE_COMPUTE, int(seed) & (2 ** 64 - 1),
+            int(offset) & (2 ** 64 - 1), _stream(stream))
+    _check("mixfp4_quantize_colwise_sr" if colwise else "mixfp4_quantize_sr", st)
     return q
 
 

@@ -139,3 +139,16 @@ def test_training_orientation_validation(lib):
     assert t(fake, None, 32, 32, fake, fake, None) == -1
     assert t(fake, fake, 32, 32, ctypes.c_void_p((1 << 20) + 4), fake, None) == -3
     assert t(fake, fake, 0, 32, None, None, None) == 0                          # empty
+
+
+def test_stochastic_rounding_validation(lib):
+    fake = ctypes.c_void_p(1 << 20)
+    ws = ctypes.c_void_p(1 << 21)
+    q = lib.mixfp4_quantize_sr
+    assert q(fake, 0, 4, 24, 24, fake, fake, fake, ws, 0, 0, 1, 0, None) == -2       # K % 16
+    assert q(fake, 0, 4, 32, 32, fake, fake, fake, None, 0, 0, 1, 0, None) == -1     # workspace
+    assert q(fake, 0, 4, 32, 32, fake, fake, fake, ws, 9, 0, 1, 0, None) == -7       # mode
+    assert q(fake, 0, 0, 32, 32, None, None, fake, ws, 0, 1, 1, 0, None) == 0       # empty, scale given
+    c = lib.mixfp4_quantize_colwise_sr
+    assert c(fake, 0, 24, 32, 32, fake, fake, fake, ws, 0, 0, 1, 0, None) == -2      # R % 16
+    assert c(fake, 3, 32, 32, 32, fake, fake, fake, ws, 0, 0, 1, 0, None) == -4      # dtype
