@@ -316,6 +316,8 @@ def run_ours(args):
     e2e_ms = reduce_max(e0.elapsed_time(e1), dev)
     e2e_value = world * e2e_steps * flops / (e2e_ms * 1e-3) / 1e12
 
+    configs = None if args.no_configs else config_gemms(dev, flush, stream, pk["bf16_tflops"])
+
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         cpu = cpu_baseline(lin, x_cpu, budget_s=args.cpu_budget)
@@ -370,6 +372,7 @@ def run_ours(args):
                 "with_amax_pass": {
                     "ms": round(rht_ms, 4),
                     "alg_gbs": round(xs_numel * QUANT_BYTES_PER_ELEM / (rht_ms * 1e-3) / 1e9, 1)}}},
+        "configs_gemm": configs,
         "clocks": clocks,
         "e2e": {"value": round(e2e_value, 2), "unit": "TFLOP/s",
                 "h2d_bytes_per_step": x_host.numel() * 2, "d2h_bytes_per_step": c_host[0].numel() * 4,
@@ -379,6 +382,97 @@ def run_ours(args):
     }
     if rank == 0:
         print(json.dumps(out), flush=True)
+
+
+# ------------------------------------------------------ the other configs' GEMMs
+def config_gemms(dev, flush, stream, peak_t):
+    """GEMM time of the other LLM-shaped configs (the MLP, decode-shaped and
+    Hadamard-rotated linears) on both GEMM paths.  Inputs are drawn on the GPU
+    from a seeded generator with the same distributions as synth.py (Student-t
+    activations with 1 % outlier channels x 50, normal weights with lognormal
+    row scales; the Hadamard case rotates 128-chunks of both by the normalised
+    Sylvester matrix); weights and activations are quantized once, since these
+    lines time the GEMM kernels alone (L2 flushed before each launch)."""
+    import math
+    import torch
+    from paper_2605_31035_gb300 import ops
+
+    g = torch.Generator(device=dev)
+
+    def t3(rows, K, seed, outliers=True):
+        g.manual_seed(seed)
+        out = torch.empty(rows, K, dtype=torch.bfloat16, device=dev)
+        step = max(1, (1 << 25) // K)
+        for r0 in range(0, rows, step):
+            r1 = min(rows, r0 + step)
+            z = torch.randn(4, r1 - r0, K, device=dev, generator=g)
+            v = z[0] / torch.sqrt((z[1] * z[1] + z[2] * z[2] + z[3] * z[3]) / 3.0) * 0.5
+            if outliers:
+                gc = torch.Generator(device="cpu")
+                gc.manual_seed(seed + 1)
+                ch = torch.randperm(K, generator=gc)[:int(math.floor(0.01 * K))].to(dev)
+                v[:, ch] *= 50.0
+            out[r0:r1] = v.to(torch.bfloat16)
+        return out
+
+    def normal(N, K, seed, std, row_sigma, outliers=False):
+        g.manual_seed(seed)
+        w = torch.randn(N, K, device=dev, generator=g) * std
+        if row_sigma:
+            w *= torch.exp(torch.randn(N, 1, device=dev, generator=g) * row_sigma)
+        if outliers:
+            gc = torch.Generator(device="cpu")
+            gc.manual_seed(seed + 1)
+            w[:, torch.randperm(K, generator=gc)[:int(math.floor(0.01 * K))].to(dev)] *= 50.0
+        return w.to(torch.bfloat16)
+
+    def hadamard(x):
+        h = torch.ones(1, 1, dtype=torch.float32, device=dev)
+        while h.shape[0] < 128:
+            h = torch.cat([torch.cat([h, h], 1), torch.cat([h, -h], 1)], 0)
+        h = h / math.sqrt(128.0)
+        rows, K = x.shape
+        return (x.float().reshape(rows, K // 128, 128) @ h.T).reshape(rows, K).to(torch.bfloat16)
+
+    def timed(fn, reps=20):
+        for _ in range(3):
+            fn()
+        evs = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(reps)]
+        for e in evs:
+            flush.zero_()
+            e[0].record(stream)
+            fn()
+            e[1].record(stream)
+        torch.cuda.synchronize(dev)
+        return statistics.median(a.elapsed_time(b) for a, b in evs)
+
+    cases = [("mlp_gate_up", 4096, 14336, 4096, lambda: t3(4096, 4096, 11), lambda: normal(14336, 4096, 12, 0.02, 0.5)),
+             ("mlp_down", 4096, 4096, 14336, lambda: t3(4096, 14336, 13), lambda: normal(4096, 14336, 14, 0.02, 0.5)),
+             ("decode", 16, 28672, 8192, lambda: t3(16, 8192, 15), lambda: normal(28672, 8192, 16, 0.015, None)),
+             ("hadamard_8192", 8192, 8192, 8192, lambda: hadamard(t3(8192, 8192, 17)),
+              lambda: hadamard(normal(8192, 8192, 18, 0.02, None, outliers=True)))]
+    out = {}
+    for name, M, N, K, mx, mw in cases:
+        qx, qw = ops.mixfp4_quantize(mx()), ops.mixfp4_quantize(mw())
+        C = torch.empty(M, N, dtype=torch.float32, device=dev)
+        fl = 2.0 * M * N * K
+        ms = timed(lambda: ops.mixfp4_gemm(qx, qw, out=C))
+        rec = {"M": M, "N": N, "K": K, "gemm_ms": round(ms, 4), "tflops": round(fl / (ms * 1e-3) / 1e12, 1),
+               "frac_of_bf16_peak": round(fl / (ms * 1e-3) / 1e12 / peak_t, 4)}
+        if M <= 64:
+            byts = N * K * (0.5 + 1.0 / 16) + M * K * (0.5 + 1.0 / 16) + M * N * 4
+            rec["gbs"] = round(byts / (ms * 1e-3) / 1e9, 1)
+            rec["hbm_bytes_per_launch"] = int(byts)
+        else:
+            nx, nw = ops.mixfp4_split_native(qx), ops.mixfp4_split_native(qw)
+            ms_n = timed(lambda: ops.mixfp4_gemm_native(nx, nw, out=C))
+            rec["native_ms"] = round(ms_n, 4)
+            rec["native_tflops"] = round(fl / (ms_n * 1e-3) / 1e12, 1)
+            del nx, nw
+        out[name] = rec
+        del qx, qw, C
+        torch.cuda.empty_cache()
+    return out
 
 
 # ------------------------------------------------------------------ CPU oracle legs
@@ -535,6 +629,7 @@ def main(argv=None):
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--cpu-budget", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-configs", action="store_true", help="skip the other configs' GEMM lines")
     ap.add_argument("--kernel", choices=["gemm", "gemm_native", "split_native", "quantize", "quantize_rht", "quantize_colwise",
                              "quantize_2d", "transpose_2d", "dequantize"], default=None,
                     help="profiling mode: launch only this kernel")
