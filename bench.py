@@ -483,6 +483,10 @@ def config_gemms(dev, flush, stream, peak_t):
             byts = N * K * (0.5 + 1.0 / 16) + M * K * (0.5 + 1.0 / 16) + M * N * 4
             rec["gbs"] = round(byts / (ms * 1e-3) / 1e9, 1)
             rec["hbm_bytes_per_launch"] = int(byts)
+            ms_n = timed(lambda: ops.mixfp4_gemm_native_fewrows(qx, qw, out=C))
+            rec["native_fewrows_ms"] = round(ms_n, 4)
+            rec["native_fewrows_gbs"] = round(byts / (ms_n * 1e-3) / 1e9, 1)
+            rec["native_fewrows_frac_of_hbm"] = round(byts / (ms_n * 1e-3) / 1e9 / peaks()["hbm_gbs"], 4)
         else:
             nx, nw = ops.mixfp4_split_native(qx), ops.mixfp4_split_native(qw)
             ms_n = timed(lambda: ops.mixfp4_gemm_native(nx, nw, out=C))
@@ -600,6 +604,11 @@ def run_kernel_only(args):
         C = torch.empty(x.shape[0], w.shape[0], dtype=torch.float32, device=dev)
         fn = lambda: ops.mixfp4_gemm_native(nx, nw, out=C)
         work = 2.0 * x.shape[0] * w.shape[0] * x.shape[1]
+    elif args.kernel == "gemm_native_fewrows":
+        qw = ops.mixfp4_quantize(w, workspace=ws)
+        C = torch.empty(x.shape[0], w.shape[0], dtype=torch.float32, device=dev)
+        fn = lambda: ops.mixfp4_gemm_native_fewrows(qx, qw, out=C)
+        work = 2.0 * x.shape[0] * w.shape[0] * x.shape[1]
     elif args.kernel == "split_native":
         fn = lambda: ops.mixfp4_split_native(qx)
         work = x.numel() * (0.5 + 1.0 / 16 + 1.0 + 1.0 / 16)
@@ -650,7 +659,7 @@ def main(argv=None):
     ap.add_argument("--cpu-budget", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-configs", action="store_true", help="skip the other configs' GEMM lines")
-    ap.add_argument("--kernel", choices=["gemm", "gemm_native", "split_native", "quantize", "quantize_rht", "quantize_colwise",
+    ap.add_argument("--kernel", choices=["gemm", "gemm_native", "gemm_native_fewrows", "split_native", "quantize", "quantize_rht", "quantize_colwise",
                              "quantize_2d", "transpose_2d", "dequantize"], default=None,
                     help="profiling mode: launch only this kernel")
     ap.add_argument("--workload", default=WORKLOAD,

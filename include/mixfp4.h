@@ -274,6 +274,23 @@ int mixfp4_gemm_native(const uint8_t* a_main, const uint8_t* a_res, const uint8_
                        void* stream);
 
 /*
+ * mixfp4_gemm_native_fewrows -- the native block-scaled FP4 variant for few
+ * activation rows (decode-shaped GEMMs, M <= 64), taking the MixFP4 operands
+ * as stored (the arguments of mixfp4_gemm): each 128-row x 256-K unit of B
+ * and the matching slice of A are split into E2M1 main + residual parts in
+ * shared memory (as mixfp4_split_native defines them) and contracted by
+ * tcgen05.mma kind::mxf4nvf4, one instruction per 64-K step covering all four
+ * products (main and residual stacked on the M and N sides).  C is the same
+ * product as mixfp4_gemm's up to fp32 summation order; the host zeroes C
+ * first and the partial sums of the K slices are added into it.
+ * M            0 <= M <= 64 (else MIXFP4_ERR_SHAPE).
+ * Other arguments, alignment and errors: as mixfp4_gemm.
+ */
+int mixfp4_gemm_native_fewrows(const uint8_t* a_codes, const uint8_t* a_scales, const float* a_ts,
+                               const uint8_t* b_codes, const uint8_t* b_scales, const float* b_ts, int64_t M,
+                               int64_t N, int64_t K, float* C, int64_t ldc, uint32_t* status_word, void* stream);
+
+/*
  * mixfp4_quantize_noalloc -- mixfp4_quantize with MIXFP4_SCALE_COMPUTE for
  * callers that cannot allocate device memory.  The paper has no counterpart;
  * this is a deployment convenience.

@@ -253,6 +253,33 @@ int mixfp4_gemm(const uint8_t* a_codes, const uint8_t* a_scales, const float* a_
   return launch_status();
 }
 
+int mixfp4_gemm_native_fewrows(const uint8_t* a_codes, const uint8_t* a_scales, const float* a_ts,
+                               const uint8_t* b_codes, const uint8_t* b_scales, const float* b_ts, int64_t M,
+                               int64_t N, int64_t K, float* C, int64_t ldc, uint32_t* status_word, void* stream) {
+  if (M < 0 || M > 64 || N < 0 || K < 0 || K % 256 != 0 || ldc < N) return MIXFP4_ERR_SHAPE;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (status_word) {
+    if (!aligned(status_word, 4)) return MIXFP4_ERR_ALIGN;
+    if (cudaMemsetAsync(status_word, 0, sizeof(uint32_t), s) != cudaSuccess) return MIXFP4_ERR_CUDA;
+  }
+  if (M == 0 || N == 0) return MIXFP4_OK;
+  if (!C) return MIXFP4_ERR_NULL;
+  if (!aligned(C, 4)) return MIXFP4_ERR_ALIGN;
+  if (K == 0) {
+    if (cudaMemset2DAsync(C, (size_t)ldc * sizeof(float), 0, (size_t)N * sizeof(float), (size_t)M, s) != cudaSuccess)
+      return MIXFP4_ERR_CUDA;
+    return MIXFP4_OK;
+  }
+  if (!a_codes || !a_scales || !a_ts || !b_codes || !b_scales || !b_ts) return MIXFP4_ERR_NULL;
+  if (!aligned(a_codes, 16) || !aligned(a_scales, 16) || !aligned(b_codes, 16) || !aligned(b_scales, 16) ||
+      !aligned(a_ts, 4) || !aligned(b_ts, 4))
+    return MIXFP4_ERR_ALIGN;
+  int st = mixfp4::launch_gemm_native_fewrows(a_codes, a_scales, a_ts, b_codes, b_scales, b_ts, M, N, K, C, ldc,
+                                              status_word, s);
+  if (st) return st;
+  return launch_status();
+}
+
 int mixfp4_split_native(const uint8_t* codes, const uint8_t* scales, int64_t rows, int64_t K,
                         uint8_t* main_codes, uint8_t* res_codes, uint8_t* sf_tiled, void* stream) {
   if (rows < 0 || K < 0 || K % 64 != 0) return MIXFP4_ERR_SHAPE;

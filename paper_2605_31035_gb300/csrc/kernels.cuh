@@ -36,6 +36,10 @@ int launch_gemm(const uint8_t* a_codes, const uint8_t* a_scales, const float* a_
                 const uint8_t* b_codes, const uint8_t* b_scales, const float* b_ts,
                 int64_t M, int64_t N, int64_t K, float* C, int64_t ldc, uint32_t* status_word,
                 cudaStream_t stream);
+int launch_gemm_native_fewrows(const uint8_t* a_codes, const uint8_t* a_scales, const float* a_ts,
+                               const uint8_t* b_codes, const uint8_t* b_scales, const float* b_ts, int64_t M,
+                               int64_t N, int64_t K, float* C, int64_t ldc, uint32_t* status_word,
+                               cudaStream_t stream);
 int launch_split_native(const uint8_t* codes, const uint8_t* scales, int64_t rows, int64_t K, uint8_t* main_codes,
                         uint8_t* res_codes, uint8_t* sf, cudaStream_t stream);
 int launch_gemm_native(const uint8_t* a_main, const uint8_t* a_res, const uint8_t* a_sf, const float* a_ts,

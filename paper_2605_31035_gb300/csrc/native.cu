@@ -456,6 +456,437 @@ int launch(const uint8_t* a_main, const uint8_t* a_res, const uint8_t* a_sf, con
 }
 
 }  // namespace nv
+
+// ============================================================================
+// Few-row native variant (M <= 64 activation rows, the decode shape): the
+// MixFP4 operands are split into E2M1 main + residual parts on the fly, in
+// shared memory, instead of beforehand.  Weight rows go on the MMA N side in
+// units of 128 rows x one 256-wide K slice: the split writes the 128 main rows
+// to rows 0-127 and the 128 residual rows to rows 128-255 of one N = 256
+// operand tile, and the activation rows' main and residual parts to rows
+// 0-63 and 64-127 of the M = 128 operand tile, so ONE kind::mxf4nvf4 MMA per
+// 64-K step forms all four products; the epilogue adds the accumulator's four
+// quadrants: C[m][n] = D[m][n] + D[m][128+n] + D[64+m][n] + D[64+m][128+n].
+// Per CTA (one per SM, units split evenly over all SMs, partial sums added
+// into C which the host zeroed):
+//   warp 0      TMA: 128 x 128-byte weight code tile (128-byte swizzle), its
+//               128 x 16-byte scale tile, the activation rows' code and scale
+//               tiles, into a ring of 2-4 stages (21-27 KB each, by the row
+//               count), ahead of a 3-stage ring of split operand tiles;
+//   warp 1      TMEM allocation; lane 0 issues the MMAs (one per 64-K step);
+//   warps 2-17  split the weight codes (four threads per row, two 16-byte
+//               chunks each: E2M1 blocks copied, E1M2 nibbles p -> main
+//               {0,2,4,5,6,6,7,7}[p] and residual (p in {5,7} ? 2 : 0) by
+//               bit logic on eight nibbles at a time) into the swizzled
+//               operand tile, and the scale bytes into the tensor core's
+//               tiled layout; warps 18-21 the same for the activation rows;
+//   warps 22-25 epilogue, one TMEM lane quarter each;
+//   warps 26-27 copy each split stage's scale tiles into tensor memory
+//               (tcgen05.cp, half of the K steps each) and commit, so that
+//               scale copies and MMAs are issued by three threads in parallel
+//               (each tcgen05 instruction holds its issuing thread ~50 ns).
+// ============================================================================
+namespace nvs {
+
+constexpr int WR = 128;                    // weight rows per unit (MMA N = 2 x 128)
+constexpr int XR = 64;                     // activation rows (MMA M = 2 x 64)
+constexpr int BKC = 256;                   // K per unit
+constexpr int ROWB = BKC / 2;              // 128 code bytes per row per unit
+constexpr int kMaxCodeStages = 4, kSplitStages = 3;
+// Code stage (ring of TMA destinations): weight codes and scales, then the
+// nx activation rows' codes and scales; its size depends on nx (host side).
+constexpr int OFF_WC = 0, OFF_WS = WR * ROWB, OFF_XC = OFF_WS + WR * 16;
+constexpr int S_B = 0, S_A = 2 * WR * ROWB, S_SFA = S_A + 2 * XR * ROWB, S_SFB = S_SFA + 4 * 512;
+constexpr int SPLIT_STAGE = S_SFB + 4 * 512;                     // 52 KB
+constexpr int OFF_RINGS = 1024;                                  // after the barrier block
+constexpr int kSmemBudget = 232448 - 1024;                       // 1024 for the alignment of the base
+static_assert(OFF_XC % 1024 == 0 && SPLIT_STAGE % 1024 == 0 && S_A % 1024 == 0,
+              "swizzled tiles need 1024-byte alignment");
+__host__ __device__ constexpr int code_stage_bytes(int nx) { return ((OFF_XC + nx * (ROWB + 16) + 1023) / 1024) * 1024; }
+__host__ __device__ constexpr int code_stages(int nx) {
+  return (kSmemBudget - OFF_RINGS - kSplitStages * SPLIT_STAGE) / code_stage_bytes(nx) < kMaxCodeStages
+             ? (kSmemBudget - OFF_RINGS - kSplitStages * SPLIT_STAGE) / code_stage_bytes(nx)
+             : kMaxCodeStages;
+}
+static_assert(code_stages(XR) >= 2, "shared memory budget");
+constexpr int kWSplitWarps = 16, kXSplitWarps = 4;
+constexpr int kFirstW = 2, kFirstX = kFirstW + kWSplitWarps, kFirstEpi = kFirstX + kXSplitWarps;  // 2, 18, 22
+constexpr int kCopyWarp = kFirstEpi + 4, kCopyWarps = 2;                                          // 26, 27
+constexpr int kThreads = 32 * (kCopyWarp + kCopyWarps);                                           // 896
+static_assert(kFirstEpi % 4 == 2, "epilogue warps cover the four TMEM lane quarters");
+constexpr uint32_t kAccCols = 2 * WR;                            // 256 fp32 columns
+constexpr uint32_t kSfCols = 12;                                 // per K step: 4 (A) + 8 (B)
+constexpr uint32_t kTmemCols = 512;
+constexpr uint64_t kWaitLimitNs = 1000000000ull;
+static_assert(kAccCols + kSplitStages * 4 * kSfCols <= kTmemCols, "TMEM budget");
+
+struct Bars {
+  uint64_t code_full[kMaxCodeStages];
+  uint64_t code_empty[kMaxCodeStages];
+  uint64_t split_full[kSplitStages];
+  uint64_t sf_full[kSplitStages];   // the stage's scales are in tensor memory (commit of the copy warp)
+  uint64_t split_empty[kSplitStages];
+  uint64_t acc_full;
+  uint64_t acc_empty;
+  uint64_t drain;
+  uint32_t tmem_base;
+  int abort;
+};
+static_assert(sizeof(Bars) <= 256, "barrier block");
+
+// The E2M1 main and residual parts of eight E1M2 nibbles (sign in bit 3 of
+// each, payload p in bits 0-2): main payload bits m0 = p1 (p0 | p2),
+// m1 = p2 | (p0 ~p1), m2 = p2 | p1 (the codes of 0,1,2,3,4,4,6,6), residual
+// payload 2 where p0 p2 (p = 5, 7); both keep the sign bit.  Each line is one
+// three-input logic instruction (lop3; truth-table byte from a = 0xF0,
+// b = 0xCC, c = 0xAA).
+#define MIXFP4_LOP3(d, a, b, c, LUT) asm("lop3.b32 %0, %1, %2, %3, " #LUT ";" : "=r"(d) : "r"(a), "r"(b), "r"(c))
+__device__ __forceinline__ void split_e1m2_word(uint32_t w, uint32_t tmask, uint32_t& main, uint32_t& res) {
+  const uint32_t r1 = w >> 1, r2 = w >> 2, l1 = w << 1;
+  uint32_t m0, m1, t, r;
+  MIXFP4_LOP3(m0, r1, w, r2, 0xE0);                  // p1 & (p0 | p2)          at bit 4i
+  MIXFP4_LOP3(m1, r1, l1, w, 0xF4);                  // p2 | (p0 & ~p1)         at bit 4i+1
+  MIXFP4_LOP3(t, m0, m1, 0x22222222u, 0xD8);         // bit 4i+1 from m1
+  MIXFP4_LOP3(t, t, w | l1, 0x44444444u, 0xD8);      // bit 4i+2: p2 | p1
+  MIXFP4_LOP3(t, t, w, 0x88888888u, 0xD8);           // bit 4i+3: the sign
+  MIXFP4_LOP3(r, l1, r1, 0x22222222u, 0x80);         // p0 & p2                 at bit 4i+1
+  MIXFP4_LOP3(r, r, w, 0x88888888u, 0xF8);           // | the sign
+  MIXFP4_LOP3(main, t, w, tmask, 0xE4);              // tmask ? main : w  (per bit: (a & c) | (b & ~c))
+  res = r & tmask;                                    // E2M1 blocks have no residual
+}
+#undef MIXFP4_LOP3
+
+// Split one 16-byte chunk (two blocks) given the blocks' type bits.
+__device__ __forceinline__ void split_chunk(uint4 c, bool t0, bool t1, uint4& m, uint4& r) {
+  const uint32_t k0 = t0 ? 0xFFFFFFFFu : 0u, k1 = t1 ? 0xFFFFFFFFu : 0u;
+  split_e1m2_word(c.x, k0, m.x, r.x);
+  split_e1m2_word(c.y, k0, m.y, r.y);
+  split_e1m2_word(c.z, k1, m.z, r.z);
+  split_e1m2_word(c.w, k1, m.w, r.w);
+}
+
+// Row r's four ue4m3 scales of K step j in the tiled layout of a 128-row tile.
+__device__ __forceinline__ uint32_t sf_offset(int r) { return (uint32_t)((r & 31) * 16 + (r >> 5) * 4); }
+
+__global__ void __launch_bounds__(kThreads, 1)
+nvf4_fewrows_kernel(const __grid_constant__ CUtensorMap tm_wc, const __grid_constant__ CUtensorMap tm_ws,
+                    const __grid_constant__ CUtensorMap tm_xc, const __grid_constant__ CUtensorMap tm_xs,
+                    const float* __restrict__ a_ts, const float* __restrict__ b_ts, int Mx, int nx, int N, int K,
+                    float* __restrict__ C, long long ldc, uint32_t* status_word) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  Bars* bars = reinterpret_cast<Bars*>(smem);
+  volatile int* abort_flag = &bars->abort;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int num_kc = K / BKC;
+  const long long units = (long long)((N + WR - 1) / WR) * num_kc;
+  const long long u_begin = units * blockIdx.x / gridDim.x, u_end = units * (blockIdx.x + 1) / gridDim.x;
+  const uint32_t stage_bytes = WR * ROWB + WR * 16 + (uint32_t)nx * (ROWB + 16);
+  const int CS = code_stage_bytes(nx), NCS = code_stages(nx);
+  const uint32_t OFF_XS = (uint32_t)(OFF_XC + nx * ROWB);
+  const uint32_t sbase = smem_u32(smem) + OFF_RINGS;          // code ring, then the split ring
+  const uint32_t OFF_SPLIT = (uint32_t)(NCS * CS);
+
+  // Split stages start as zeros: activation rows >= nx (and their residual
+  // rows and scales) are never written, so they stay zero.
+  for (uint32_t i = threadIdx.x; i < (uint32_t)(kSplitStages * SPLIT_STAGE / 16); i += blockDim.x)
+    sts128(sbase + OFF_SPLIT + i * 16, 0u, 0u, 0u, 0u);
+  fence_proxy_async_smem();
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < NCS; ++s) {
+      mbar_init(smem_u32(&bars->code_full[s]), 1);
+      mbar_init(smem_u32(&bars->code_empty[s]), kWSplitWarps + kXSplitWarps);
+    }
+    for (int s = 0; s < kSplitStages; ++s) {
+      mbar_init(smem_u32(&bars->split_full[s]), kWSplitWarps + kXSplitWarps);
+      mbar_init(smem_u32(&bars->sf_full[s]), kCopyWarps);
+      mbar_init(smem_u32(&bars->split_empty[s]), 1);
+    }
+    mbar_init(smem_u32(&bars->acc_full), 1);
+    mbar_init(smem_u32(&bars->acc_empty), 4);
+    mbar_init(smem_u32(&bars->drain), 1);
+    bars->abort = 0;
+    fence_mbar_init();
+  }
+  if (warp == 1) {
+    tmem_alloc(smem_u32(&bars->tmem_base), kTmemCols);
+    tmem_relinquish();
+  }
+  griddep_launch_dependents();
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = bars->tmem_base;
+  const uint32_t tmem_sf0 = tmem_base + kAccCols;
+
+  auto fail = [&](uint32_t code) {
+    *abort_flag = 1;
+    if (status_word) atomicOr(status_word, code);
+  };
+
+  if (warp == 0) {
+    // ---------------- TMA producer ----------------
+    if (lane == 0) {
+      tma_prefetch(&tm_wc);
+      tma_prefetch(&tm_ws);
+      tma_prefetch(&tm_xc);
+      tma_prefetch(&tm_xs);
+      griddep_wait();
+      int it = 0;
+      long long last = -1;
+      for (long long u = u_begin; u < u_end; ++u, ++it) {
+        const int s = it % NCS;
+        if (!mbar_wait(smem_u32(&bars->code_empty[s]), ((it / NCS) & 1) ^ 1, abort_flag, kWaitLimitNs)) {
+          fail(1u);
+          break;
+        }
+        const int g = (int)(u / num_kc), kc = (int)(u % num_kc);
+        const uint32_t st = sbase + s * CS;
+        const uint32_t fb = smem_u32(&bars->code_full[s]);
+        mbar_arrive_expect_tx(fb, stage_bytes);
+        tma_load_2d(st + OFF_WC, &tm_wc, kc * ROWB, g * WR, fb);
+        tma_load_2d(st + OFF_WS, &tm_ws, kc * 16, g * WR, fb);
+        tma_load_2d(st + OFF_XC, &tm_xc, kc * ROWB, 0, fb);
+        tma_load_2d(st + OFF_XS, &tm_xs, kc * 16, 0, fb);
+        last = it;
+      }
+      if (*abort_flag)
+        for (long long v = last - NCS + 1; v <= last; ++v)
+          if (v >= 0)
+            mbar_wait(smem_u32(&bars->code_full[v % NCS]), (uint32_t)((v / NCS) & 1), nullptr,
+                      kWaitLimitNs);
+    }
+  } else if (warp == 1) {
+    // ---------------- MMA issuer ----------------
+    if (lane == 0) {
+      constexpr uint32_t kIdesc = idesc_nvf4_f32(2 * XR, 2 * WR);
+      int it = 0, run = 0;
+      bool ok = true;
+      for (long long u = u_begin; u < u_end && ok; ++run) {
+        const int g = (int)(u / num_kc);
+        const long long run_end = (long long)(g + 1) * num_kc < u_end ? (long long)(g + 1) * num_kc : u_end;
+        if (!mbar_wait(smem_u32(&bars->acc_empty), (run & 1) ^ 1, abort_flag, kWaitLimitNs)) {
+          fail(2u);
+          break;
+        }
+        tc_fence_after();
+        bool first = true;
+        for (; u < run_end; ++u, ++it) {
+          const int s = it % kSplitStages;
+          if (!mbar_wait(smem_u32(&bars->sf_full[s]), (uint32_t)((it / kSplitStages) & 1), abort_flag,
+                         kWaitLimitNs)) {
+            fail(4u);
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t sp = sbase + OFF_SPLIT + s * SPLIT_STAGE;
+#pragma unroll
+          for (int j = 0; j < BKC / 64; ++j) {
+            const uint32_t sfa = tmem_sf0 + (uint32_t)(s * 4 + j) * kSfCols, sfb = sfa + 4;
+            mma_nvf4(tmem_base, smem_desc_sw128(sp + S_A + j * 32), smem_desc_sw128(sp + S_B + j * 32), kIdesc, sfa,
+                     sfb, first ? 0u : 1u);
+            first = false;
+          }
+          mma_commit(smem_u32(&bars->split_empty[s]));
+        }
+        if (ok) mma_commit(smem_u32(&bars->acc_full));
+      }
+      mma_commit(smem_u32(&bars->drain));
+      if (!mbar_wait(smem_u32(&bars->drain), 0, nullptr, kWaitLimitNs)) fail(8u);
+    }
+  } else if (warp >= kCopyWarp) {
+    // ---------------- scale copies ----------------
+    // Once a stage is split, its A and B scale tiles go to tensor memory
+    // (tcgen05.cp, replicated to the four lane quarters; the B tile twice, for
+    // the main and residual halves of N) and the commits tell the MMA thread;
+    // the two copy warps take K steps 0-1 and 2-3.  A stage's columns are
+    // rewritten only after its next split, which waits for the MMAs that
+    // read them.
+    const int j0 = 2 * (warp - kCopyWarp);
+    if (lane == 0) {
+      int it = 0;
+      for (long long u = u_begin; u < u_end; ++u, ++it) {
+        const int s = it % kSplitStages;
+        if (!mbar_wait(smem_u32(&bars->split_full[s]), (uint32_t)((it / kSplitStages) & 1), abort_flag,
+                       kWaitLimitNs)) {
+          fail(128u);
+          break;
+        }
+        tc_fence_after();
+        const uint32_t sp = sbase + OFF_SPLIT + s * SPLIT_STAGE;
+#pragma unroll
+        for (int j = j0; j < j0 + 2; ++j) {
+          const uint32_t sfa = tmem_sf0 + (uint32_t)(s * 4 + j) * kSfCols, sfb = sfa + 4;
+          tmem_cp_32x128b_x4(sfa, smem_desc_noswizzle(sp + S_SFA + j * 512, 128, 128));
+          tmem_cp_32x128b_x4(sfb, smem_desc_noswizzle(sp + S_SFB + j * 512, 128, 128));
+          tmem_cp_32x128b_x4(sfb + 4, smem_desc_noswizzle(sp + S_SFB + j * 512, 128, 128));
+        }
+        mma_commit(smem_u32(&bars->sf_full[s]));
+      }
+    }
+  } else if (warp < kFirstEpi) {
+    // ---------------- splitters ----------------
+    // Weights: thread t of 512 splits row t / 4, chunks 2 (t % 4) and +1
+    // (blocks 4 (t % 4) .. +3, scale word t % 4).  Activations: thread t of
+    // 128 splits chunks q = t + 128 i (row q / 8, chunk q % 8) of rows < nx.
+    const bool is_w = warp < kFirstX;
+    const int t = is_w ? (warp - kFirstW) * 32 + lane : (warp - kFirstX) * 32 + lane;
+    auto pick = [](const uint4& v, int i) {  // v[i] without dynamic indexing
+      return (i & 2) ? ((i & 1) ? v.w : v.z) : ((i & 1) ? v.y : v.x);
+    };
+    int it = 0;
+    for (long long u = u_begin; u < u_end; ++u, ++it) {
+      const int s = it % NCS, sps = it % kSplitStages;
+      if (!mbar_wait(smem_u32(&bars->code_full[s]), (uint32_t)((it / NCS) & 1), abort_flag,
+                     kWaitLimitNs)) {
+        fail(16u);
+        break;
+      }
+      if (!mbar_wait(smem_u32(&bars->split_empty[sps]), (uint32_t)(((it / kSplitStages) & 1) ^ 1), abort_flag,
+                     kWaitLimitNs)) {
+        fail(32u);
+        break;
+      }
+      const uint32_t st = sbase + s * CS, sp = sbase + OFF_SPLIT + sps * SPLIT_STAGE;
+      if (is_w) {
+        const int row = t >> 2, q4 = t & 3;
+        const uint32_t swz = (uint32_t)(row & 7);
+        const uint4 sc = lds128(st + OFF_WS + (uint32_t)row * 16);
+        const uint32_t sw = pick(sc, q4);
+#pragma unroll
+        for (int k = 0; k < 2; ++k) {
+          const uint32_t pc = ((uint32_t)(2 * q4 + k) ^ swz) << 4;
+          const uint32_t tb = sw >> (16 * k);
+          uint4 m, r;
+          split_chunk(lds128(st + OFF_WC + (uint32_t)row * ROWB + pc), (tb & 0x80u) != 0, (tb & 0x8000u) != 0, m, r);
+          sts128(sp + S_B + (uint32_t)row * ROWB + pc, m.x, m.y, m.z, m.w);
+          sts128(sp + S_B + (uint32_t)(row + WR) * ROWB + pc, r.x, r.y, r.z, r.w);
+        }
+        // Scales of K step q4 into the tiled layout (bit 7, the type, cleared).
+        sts32(sp + S_SFB + q4 * 512 + sf_offset(row), sw & 0x7F7F7F7Fu);
+      } else {
+#pragma unroll 1
+        for (int q = t; q < nx * 8; q += kXSplitWarps * 32) {
+          const int row = q >> 3, c = q & 7;
+          const uint32_t pc = ((uint32_t)c ^ (uint32_t)(row & 7)) << 4;
+          const uint4 sc = lds128(st + OFF_XS + (uint32_t)row * 16);
+          const uint32_t sw = pick(sc, c >> 1), tb = sw >> (16 * (c & 1));
+          uint4 m, r;
+          split_chunk(lds128(st + OFF_XC + (uint32_t)row * ROWB + pc), (tb & 0x80u) != 0, (tb & 0x8000u) != 0, m, r);
+          sts128(sp + S_A + (uint32_t)row * ROWB + pc, m.x, m.y, m.z, m.w);
+          sts128(sp + S_A + (uint32_t)(row + XR) * ROWB + pc, r.x, r.y, r.z, r.w);
+          if ((c & 1) == 0) {  // scale word c / 2 = K step c / 2, for the main and residual rows
+            sts32(sp + S_SFA + (c >> 1) * 512 + sf_offset(row), sw & 0x7F7F7F7Fu);
+            sts32(sp + S_SFA + (c >> 1) * 512 + sf_offset(row + XR), sw & 0x7F7F7F7Fu);
+          }
+        }
+      }
+      fence_proxy_async_smem();
+      __syncwarp();
+      if (lane == 0) {
+        mbar_arrive(smem_u32(&bars->split_full[sps]));
+        mbar_arrive(smem_u32(&bars->code_empty[s]));
+      }
+    }
+  } else {
+    // ---------------- epilogue ----------------
+    // Warps for lane quarters 0, 1 hold the activation rows' main products,
+    // quarters 2, 3 their residual products (row m + 64); both add into C.
+    const int q = warp & 3;
+    const int m = (q & 1) * 32 + lane;
+    griddep_wait();
+    const float sa = __ldg(a_ts), sb = __ldg(b_ts);
+    const bool vec_ok = ((ldc & 3) == 0) && ((reinterpret_cast<uintptr_t>(C) & 15) == 0);
+    const bool mine = (q & 1) * 32 < Mx;
+    const uint32_t tb = tmem_base + ((uint32_t)(q * 32) << 16);
+    int run = 0;
+    for (long long u = u_begin; u < u_end; ++run) {
+      const int g = (int)(u / num_kc);
+      u = (long long)(g + 1) * num_kc < u_end ? (long long)(g + 1) * num_kc : u_end;
+      const bool acc_ok = mbar_wait(smem_u32(&bars->acc_full), run & 1, abort_flag, kWaitLimitNs);
+      tc_fence_after();
+      const bool go = __all_sync(0xffffffffu, acc_ok && !*abort_flag);
+      if (!go) {
+        if (!acc_ok && !*abort_flag) fail(64u);
+        break;
+      }
+#pragma unroll 1
+      for (int cc = 0; cc < WR / 16; ++cc) {
+        uint32_t v[16], w[16];
+        if (mine) {
+          tmem_ld_32x32b_x16(tb + (uint32_t)(cc * 16), v);
+          tmem_ld_32x32b_x16(tb + (uint32_t)(WR + cc * 16), w);
+          tmem_ld_wait_x16(v);
+          reg_fence16(w);
+        }
+        if (cc == WR / 16 - 1) {
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(smem_u32(&bars->acc_empty));
+        }
+        const int n0 = g * WR + cc * 16;
+        if (mine && m < Mx) {
+          float* crow = C + (long long)m * ldc + n0;
+          float o[16];
+#pragma unroll
+          for (int k = 0; k < 16; ++k)
+            o[k] = __fmul_rn(__fmul_rn(__fadd_rn(__uint_as_float(v[k]), __uint_as_float(w[k])), sa), sb);
+          if (vec_ok && n0 + 16 <= N) {
+#pragma unroll
+            for (int k = 0; k < 16; k += 4) red_add_v4(crow + k, o[k], o[k + 1], o[k + 2], o[k + 3]);
+          } else {
+            for (int k = 0; k < 16; ++k)
+              if (n0 + k < N) atomicAdd(crow + k, o[k]);
+          }
+        }
+      }
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem_base, kTmemCols);
+  }
+}
+
+int launch(const uint8_t* a_codes, const uint8_t* a_scales, const float* a_ts, const uint8_t* b_codes,
+           const uint8_t* b_scales, const float* b_ts, int64_t M, int64_t N, int64_t K, float* C, int64_t ldc,
+           uint32_t* status_word, cudaStream_t stream) {
+  const int nx = (int)((M + 15) & ~15);
+  CUtensorMap twc, tws, txc, txs;
+  if (!make_map(&twc, b_codes, (uint64_t)K / 2, (uint64_t)N, ROWB, WR, CU_TENSOR_MAP_SWIZZLE_128B) ||
+      !make_map(&tws, b_scales, (uint64_t)K / 16, (uint64_t)N, 16, WR, CU_TENSOR_MAP_SWIZZLE_NONE) ||
+      !make_map(&txc, a_codes, (uint64_t)K / 2, (uint64_t)M, ROWB, (uint32_t)nx, CU_TENSOR_MAP_SWIZZLE_128B) ||
+      !make_map(&txs, a_scales, (uint64_t)K / 16, (uint64_t)M, 16, (uint32_t)nx, CU_TENSOR_MAP_SWIZZLE_NONE))
+    return MIXFP4_ERR_CUDA;
+  const int smem = OFF_RINGS + code_stages(nx) * code_stage_bytes(nx) + kSplitStages * SPLIT_STAGE + 1024;
+  static bool attr_set = false;
+  if (!attr_set) {
+    if (cudaFuncSetAttribute(nvf4_fewrows_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, 232448) !=
+        cudaSuccess)
+      return MIXFP4_ERR_CUDA;
+    attr_set = true;
+  }
+  cudaError_t e;
+  if (ldc == N)
+    e = cudaMemsetAsync(C, 0, (size_t)M * (size_t)N * sizeof(float), stream);
+  else
+    e = cudaMemset2DAsync(C, (size_t)ldc * sizeof(float), 0, (size_t)N * sizeof(float), (size_t)M, stream);
+  if (e != cudaSuccess) return MIXFP4_ERR_CUDA;
+  const int64_t units = ((N + WR - 1) / WR) * (K / BKC);
+  int64_t grid = num_sms();
+  if (grid > units) grid = units;
+  if (launch_pdl(nvf4_fewrows_kernel, (unsigned)grid, kThreads, smem, stream, twc, tws, txc, txs, a_ts, b_ts,
+                 (int)M, nx, (int)N, (int)K, C, (long long)ldc, status_word) != cudaSuccess)
+    return MIXFP4_ERR_CUDA;
+  return MIXFP4_OK;
+}
+
+}  // namespace nvs
+
 }  // namespace
 
 int launch_split_native(const uint8_t* codes, const uint8_t* scales, int64_t rows, int64_t K, uint8_t* main_codes,
@@ -487,4 +918,13 @@ int launch_gemm_native(const uint8_t* a_main, const uint8_t* a_res, const uint8_
                                   stream);
 }
 
+}  // namespace mixfp4
+
+namespace mixfp4 {
+int launch_gemm_native_fewrows(const uint8_t* a_codes, const uint8_t* a_scales, const float* a_ts,
+                               const uint8_t* b_codes, const uint8_t* b_scales, const float* b_ts, int64_t M,
+                               int64_t N, int64_t K, float* C, int64_t ldc, uint32_t* status_word,
+                               cudaStream_t stream) {
+  return nvs::launch(a_codes, a_scales, a_ts, b_codes, b_scales, b_ts, M, N, K, C, ldc, status_word, stream);
+}
 }  // namespace mixfp4

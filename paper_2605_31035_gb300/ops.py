@@ -61,6 +61,8 @@ def lib() -> ctypes.CDLL:
         L.mixfp4_split_native.argtypes = [P, P, I64, I64, P, P, P, P]
         L.mixfp4_gemm_native.restype = I
         L.mixfp4_gemm_native.argtypes = [P, P, P, P, P, P, P, P, I64, I64, I64, P, I64, P, P]
+        L.mixfp4_gemm_native_fewrows.restype = I
+        L.mixfp4_gemm_native_fewrows.argtypes = [P, P, P, P, P, P, I64, I64, I64, P, I64, P, P]
         L.mixfp4_selftest_bounded_wait.restype = I
         L.mixfp4_selftest_bounded_wait.argtypes = [P, ctypes.c_uint64, P]
         L.mixfp4_status_string.restype = ctypes.c_char_p
@@ -304,6 +306,20 @@ def mixfp4_gemm_native(a: NativeTensor, b: NativeTensor, out: torch.Tensor | Non
                                   _ptr(b.main), _ptr(b.res), _ptr(b.sf), _ptr(b.tensor_scale),
                                   M, N, K, _ptr(C), C.stride(0), _ptr(status_word), _stream(stream))
     _check("mixfp4_gemm_native", st)
+    return C
+
+
+def mixfp4_gemm_native_fewrows(a: QTensor, b: QTensor, out: torch.Tensor | None = None,
+                               status_word: torch.Tensor | None = None, stream=None) -> torch.Tensor:
+    """C = A_deq . B_deq^T for a with at most 64 rows, on the block-scaled FP4
+    tensor path with the operands split on the fly."""
+    assert a.K == b.K and a.rows <= 64
+    M, N, K = a.rows, b.rows, a.K
+    C = out if out is not None else torch.empty(M, N, dtype=torch.float32, device=a.codes.device)
+    st = lib().mixfp4_gemm_native_fewrows(_ptr(a.codes), _ptr(a.scales), _ptr(a.tensor_scale),
+                                          _ptr(b.codes), _ptr(b.scales), _ptr(b.tensor_scale),
+                                          M, N, K, _ptr(C), C.stride(0), _ptr(status_word), _stream(stream))
+    _check("mixfp4_gemm_native_fewrows", st)
     return C
 
 

@@ -152,3 +152,13 @@ def test_stochastic_rounding_validation(lib):
     c = lib.mixfp4_quantize_colwise_sr
     assert c(fake, 0, 24, 32, 32, fake, fake, fake, ws, 0, 0, 1, 0, None) == -2      # R % 16
     assert c(fake, 3, 32, 32, 32, fake, fake, fake, ws, 0, 0, 1, 0, None) == -4      # dtype
+
+
+def test_fewrows_native_validation(lib):
+    fake = ctypes.c_void_p(1 << 20)
+    g = lib.mixfp4_gemm_native_fewrows
+    assert g(fake, fake, fake, fake, fake, fake, 65, 128, 256, fake, 128, None, None) == -2   # M > 64
+    assert g(fake, fake, fake, fake, fake, fake, 16, 128, 128, fake, 128, None, None) == -2   # K % 256
+    assert g(fake, fake, fake, None, fake, fake, 16, 128, 256, fake, 128, None, None) == -1   # B codes
+    assert g(fake, fake, fake, fake, fake, fake, 16, 128, 256, ctypes.c_void_p((1 << 20) + 2), 128, None, None) == -3
+    assert g(fake, fake, fake, fake, fake, fake, 0, 128, 256, fake, 128, None, None) == 0     # empty

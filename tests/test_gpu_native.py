@@ -159,3 +159,61 @@ def test_native_full_size_workloads(oracle, name):
         B = oracle.dequant_rows_f64(qb.codes.cpu().numpy(), qb.scales.cpu().numpy(), qb.tensor_scale.item(), ns)
         Cg = C[torch.from_numpy(ms).to(DEV)][:, torch.from_numpy(ns).to(DEV)].cpu().numpy()
         assert_close(Cg, A @ B.T, A, B)
+
+
+@pytest.mark.parametrize("M,N,K", [(1, 128, 256), (16, 300, 768), (33, 1000, 512), (64, 256, 2048), (7, 129, 1280)])
+def test_fewrows_native_gemm(oracle, M, N, K):
+    """The few-row native path splits the stored MixFP4 operands on the fly:
+    one or several 128-row weight groups, a ragged last group, activation
+    rows from 1 to 64, several K slices per CTA."""
+    x = synth.activations(M, K, 8600 + M, 8601)
+    w = synth.weights(N, K, 8602 + N, 0.02, 0.5)
+    qa, ra = quant_both(oracle, x)
+    qb, rb = quant_both(oracle, w)
+    status = torch.zeros(1, dtype=torch.int32, device=DEV)
+    C = ops().mixfp4_gemm_native_fewrows(qa, qb, status_word=status)
+    torch.cuda.synchronize()
+    assert status.item() == 0
+    Cref = oracle.gemm_f64(ra, rb)
+    A = oracle.dequant_rows_f64(ra[0], ra[1], ra[2], range(M))
+    B = oracle.dequant_rows_f64(rb[0], rb[1], rb[2], range(N))
+    assert_close(C.cpu().numpy(), Cref, A, B)
+
+
+def test_fewrows_native_modes_and_ldc(oracle):
+    """E2M1-only and E1M2-only operands (all-main and all-split blocks) and a
+    padded output row stride."""
+    o = ops()
+    for mode_a, mode_b in ((1, 1), (2, 2), (0, 2)):
+        x = synth.activations(16, 512, 8700 + mode_a, 8701)
+        w = synth.weights(256, 512, 8702 + mode_b, 0.02, 0.5)
+        qa, ra = quant_both(oracle, x, mode_a)
+        qb, rb = quant_both(oracle, w, mode_b)
+        Cbuf = torch.full((16, 300), 7.0, dtype=torch.float32, device=DEV)
+        C = o.mixfp4_gemm_native_fewrows(qa, qb, out=Cbuf[:, :256])
+        torch.cuda.synchronize()
+        assert torch.all(Cbuf[:, 256:] == 7.0)
+        A = oracle.dequant_rows_f64(ra[0], ra[1], ra[2], range(16))
+        B = oracle.dequant_rows_f64(rb[0], rb[1], rb[2], range(256))
+        assert_close(C.cpu().numpy(), oracle.gemm_f64(ra, rb), A, B)
+
+
+@pytest.mark.slow
+def test_fewrows_native_decode_shape(oracle):
+    """The decode-shaped linear (16 x 8192 . 28672 x 8192) against sampled
+    weight rows of the float64 oracle."""
+    lin = synth.workloads()["decode"].linears[0]
+    x, w = lin.make_x(), lin.make_w()
+    qa, ra = quant_both(oracle, x)
+    qb = ops().mixfp4_quantize(w.to(DEV))
+    C = ops().mixfp4_gemm_native_fewrows(qa, qb)
+    torch.cuda.synchronize()
+    rng = np.random.default_rng(8)
+    rows = np.unique(np.concatenate([[0, 28671], rng.integers(0, 28672, 40)]))
+    s32 = float(qb.tensor_scale.item())
+    rb = oracle.quantize(synth.bf16_bits(w[torch.from_numpy(rows)]), s32=s32)
+    assert np.array_equal(qb.codes[torch.from_numpy(rows).to(DEV)].cpu().numpy(), rb[0])
+    Cref = oracle.gemm_f64(ra, rb)
+    A = oracle.dequant_rows_f64(ra[0], ra[1], ra[2], range(16))
+    B = oracle.dequant_rows_f64(rb[0], rb[1], rb[2], range(len(rows)))
+    assert_close(C.cpu().numpy()[:, rows], Cref, A, B)
