@@ -115,23 +115,17 @@ class ClockSampler:
 
 
 class L2Flush:
-    """Empties the 129 MB L2 between timed launches: a 256 MiB write evicts
-    everything, then a 256 MiB read replaces the write's dirty lines with clean
-    ones, so the timed kernel starts cold and its reads do not also pay for
-    writing the flush buffer back to HBM."""
-    NOTE = ("flushed before every timed step, outside its events: 256 MiB write, then 256 MiB read "
-            "(cold L2 holding no dirty lines)")
+    """Empties the 129 MB L2 between timed launches by writing a 256 MiB
+    buffer (the timed kernel then starts cold; its first reads also write the
+    flush's dirty lines back to HBM)."""
+    NOTE = "flushed before every timed step, outside its events: 256 MiB write"
 
     def __init__(self, dev):
         import torch
         self.w = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
-        self.r = torch.ones(64 << 20, dtype=torch.float32, device=dev)
-        self.sink = torch.empty((), dtype=torch.float32, device=dev)
 
     def __call__(self):
-        import torch
         self.w.zero_()
-        torch.sum(self.r, dim=0, out=self.sink)
 
 
 def dist_setup(n_gpus: int):
