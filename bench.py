@@ -217,6 +217,9 @@ def run_ours(args):
     qs = ops.empty_qtensor(xs.shape[0], xs.shape[1], dev)
     ops.mixfp4_quantize(xs, out=qs, workspace=ws)
     given = qs.tensor_scale.clone()
+    qc0 = ops.mixfp4_quantize_colwise_rht(xs, workspace=ws)
+    given_rht_col = qc0.tensor_scale.clone()
+    del qc0
 
     def time_quant(fn, reps=10):
         for _ in range(3):
@@ -272,6 +275,9 @@ def run_ours(args):
     transpose_ms = time_quant(lambda: ops.mixfp4_transpose_2d(qs, out=qt))
     del qt
     sr_ms = time_quant(lambda: ops.mixfp4_quantize_sr(xs, 1234, 0, out=qs, tensor_scale=given))
+    qc = ops.empty_qtensor(xs.shape[1], xs.shape[0], dev)
+    crht_ms = time_quant(lambda: ops.mixfp4_quantize_colwise_rht(xs, out=qc, tensor_scale=given_rht_col))
+    del qc
 
     given_gbs = xs.numel() * QUANT_BYTES_PER_ELEM / (given_ms * 1e-3) / 1e9
     sweep_alg_gbs = xs.numel() * QUANT_BYTES_PER_ELEM / (sweep_ms * 1e-3) / 1e9
@@ -375,6 +381,8 @@ def run_ours(args):
                                         "alg_gbs": round(xs_numel * QUANT_BYTES_PER_ELEM / (colwise_ms * 1e-3) / 1e9, 1)},
                 "2d_blocks_given_scale": {"ms": round(q2d_ms, 4),
                                           "alg_gbs": round(xs_numel * QUANT_BYTES_PER_ELEM / (q2d_ms * 1e-3) / 1e9, 1)},
+                "colwise_rotated_given_scale": {
+                    "ms": round(crht_ms, 4), "alg_gbs": round(xs_numel * QUANT_BYTES_PER_ELEM / (crht_ms * 1e-3) / 1e9, 1)},
                 "stochastic_rounding_given_scale": {
                     "ms": round(sr_ms, 4), "alg_gbs": round(xs_numel * QUANT_BYTES_PER_ELEM / (sr_ms * 1e-3) / 1e9, 1)},
                 "transpose_2d": {"ms": round(transpose_ms, 4),

@@ -131,6 +131,22 @@ int mixfp4_quantize_colwise(const void* x, int dtype, int64_t R, int64_t C, int6
                             void* stream);
 
 /*
+ * mixfp4_quantize_colwise_rht -- mixfp4_quantize_colwise with the 128-point
+ * Walsh-Hadamard rotation of mixfp4_quantize_rht applied along the rows first:
+ * the weight-gradient inputs of the training recipe (Sec. 3.4, Sec. 4: the
+ * RHT is applied to both WGRAD operands, whose reduction runs over R).  Every
+ * 128-row chunk of each column is rotated (signs, butterfly order and scaling
+ * as mixfp4_quantize_rht) and the rotated column is quantized down its rows:
+ * bit for bit mixfp4_quantize_rht of X^T, codes [C][R/2], scales [C][R/16].
+ * With SCALE_COMPUTE, s32 = fl32(max|rotated X| / 2688).
+ * R, C         R % 128 == 0, C % 16 == 0 (else MIXFP4_ERR_SHAPE).
+ * Other arguments and errors: as mixfp4_quantize_colwise and mixfp4_quantize_rht.
+ */
+int mixfp4_quantize_colwise_rht(const void* x, int dtype, int64_t R, int64_t C, int64_t ldx, const uint8_t* signs,
+                                uint8_t* codes, uint8_t* scales, float* tensor_scale, uint32_t* workspace, int mode,
+                                int scale_flag, void* stream);
+
+/*
  * mixfp4_quantize_sr, mixfp4_quantize_colwise_sr -- mixfp4_quantize and
  * mixfp4_quantize_colwise with stochastic rounding of the codes, the
  * gradient quantization of the training flow (Sec. 4 pre-training recipe;

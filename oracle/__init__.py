@@ -339,3 +339,12 @@ def quantize_colwise_sr(x_bf16_bits: np.ndarray, seed: int, offset: int = 0, mod
                         s32: float | None = None):
     """quantize_sr of the transpose (element index c * R + r of an [R, C] input)."""
     return quantize_sr(np.ascontiguousarray(np.asarray(x_bf16_bits, np.uint16).T), seed, offset, mode, s32)
+
+
+def quantize_colwise_rht(x_bf16_bits: np.ndarray, signs: np.ndarray | None = None, mode: int = MODE_MIX,
+                         s32: float | None = None):
+    """The 128-point rotation (R11) of every 128-row chunk of each column of an
+    [R, C] tensor, then Algorithm 1 down the columns: by definition
+    quantize_f32(rht(X^T))."""
+    xt = np.ascontiguousarray(np.asarray(x_bf16_bits, np.uint16).T)
+    return quantize_f32(rht(xt, signs), mode, s32)

@@ -174,6 +174,38 @@ int mixfp4_quantize_sr(const void* x, int dtype, int64_t rows, int64_t K, int64_
   return launch_status();
 }
 
+int mixfp4_quantize_colwise_rht(const void* x, int dtype, int64_t R, int64_t C, int64_t ldx, const uint8_t* signs,
+                                uint8_t* codes, uint8_t* scales, float* tensor_scale, uint32_t* workspace, int mode,
+                                int scale_flag, void* stream) {
+  if (dtype != MIXFP4_DTYPE_BF16) return MIXFP4_ERR_DTYPE;
+  if (mode < MIXFP4_MODE_MIX || mode > MIXFP4_MODE_E1M2_ONLY) return MIXFP4_ERR_ARG;
+  if (scale_flag != MIXFP4_SCALE_COMPUTE && scale_flag != MIXFP4_SCALE_GIVEN) return MIXFP4_ERR_ARG;
+  if (R < 0 || C < 0 || R % 128 != 0 || C % 16 != 0 || ldx < C) return MIXFP4_ERR_SHAPE;
+  if (!tensor_scale) return MIXFP4_ERR_NULL;
+  if (scale_flag == MIXFP4_SCALE_COMPUTE && !workspace) return MIXFP4_ERR_NULL;
+  const bool empty = (R == 0 || C == 0);
+  if (!empty && (!x || !codes || !scales)) return MIXFP4_ERR_NULL;
+  if (!empty && (!aligned(x, 32) || ldx % 16 != 0 || !aligned(codes, 8))) return MIXFP4_ERR_ALIGN;
+  if (!aligned(tensor_scale, 4) || (workspace && !aligned(workspace, 4))) return MIXFP4_ERR_ALIGN;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const int given = scale_flag == MIXFP4_SCALE_GIVEN;
+  if (empty) {
+    if (!given && cudaMemsetAsync(tensor_scale, 0, sizeof(float), s) != cudaSuccess) return MIXFP4_ERR_CUDA;
+    return MIXFP4_OK;
+  }
+  const uint16_t* xb = static_cast<const uint16_t*>(x);
+  if (!given) {
+    if (cudaMemsetAsync(workspace, 0, sizeof(uint32_t), s) != cudaSuccess) return MIXFP4_ERR_CUDA;
+    if (mixfp4::launch_quantize_colwise_rht(xb, R, C, ldx, signs, codes, scales, tensor_scale, workspace, mode, 0, 1,
+                                            s) != 0)
+      return MIXFP4_ERR_CUDA;
+  }
+  if (mixfp4::launch_quantize_colwise_rht(xb, R, C, ldx, signs, codes, scales, tensor_scale, workspace, mode, given, 0,
+                                          s) != 0)
+    return MIXFP4_ERR_CUDA;
+  return launch_status();
+}
+
 int mixfp4_quantize_2d(const void* x, int dtype, int64_t rows, int64_t K, int64_t ldx, uint8_t* codes,
                        uint8_t* scales, float* tensor_scale, uint32_t* workspace, int mode, int scale_flag,
                        void* stream) {

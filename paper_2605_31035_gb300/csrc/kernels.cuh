@@ -24,6 +24,9 @@ int launch_quantize_colwise(const uint16_t* x, int64_t R, int64_t C, int64_t ldx
 int launch_quantize_sr(const uint16_t* x, int64_t rows, int64_t K, int64_t ldx, uint8_t* codes, uint8_t* scales,
                        float* tensor_scale, const uint32_t* amax_word, int mode, int scale_given, uint64_t seed,
                        uint64_t offset, cudaStream_t stream);
+int launch_quantize_colwise_rht(const uint16_t* x, int64_t R, int64_t C, int64_t ldx, const uint8_t* signs,
+                                uint8_t* codes, uint8_t* scales, float* tensor_scale, uint32_t* amax_word, int mode,
+                                int scale_given, int amax_pass, cudaStream_t stream);
 int launch_quantize_2d(const uint16_t* x, int64_t rows, int64_t K, int64_t ldx, uint8_t* codes, uint8_t* scales,
                        float* tensor_scale, const uint32_t* amax_word, int mode, int scale_given,
                        cudaStream_t stream);

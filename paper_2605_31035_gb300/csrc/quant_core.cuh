@@ -387,5 +387,99 @@ __device__ __forceinline__ const uint16_t* block_src(const uint16_t* x, int64_t 
   return x + row * ldx + (b - row * kblocks) * 16;
 }
 
+// ---- 128-point Walsh-Hadamard rotation before quantization ----------------
+// Reading R11 of the random Hadamard transform (Sec. 4 "+RHT", Sec. 3.4): each
+// 128-element chunk of a row along K is rotated on its own: elements whose bit
+// in the caller's 128-bit sign vector is set are negated, the Sylvester
+// product H_128 v is formed by the radix-2 butterfly in fp32 with strides
+// 1, 2, 4, ..., 64 in that order ((a, b) -> (a + b, a - b)), and every value
+// is multiplied by c = RN(1/sqrt(128)).  Algorithm 1 then runs on the fp32
+// values.  Threads hold one 16-element block each, so the 8 lanes 8g..8g+7 of
+// a warp hold one chunk (block t of the chunk on lane 8g + t): strides 1-8 run
+// inside a thread, strides 16, 32, 64 between lanes by shuffles.
+constexpr uint32_t kRhtScaleBits = 0x3DB504F3u;  // RN(1/sqrt(128))
+
+// Sign masks of this thread's 16 chunk positions 16 * (lane & 7) + e, as bf16
+// word masks (bit 15: element 2j, bit 31: element 2j + 1).
+__device__ __forceinline__ void rht_sign_words(const uint8_t* __restrict__ signs, int lane, uint32_t sw[8]) {
+  uint32_t bits = 0;
+  if (signs) {
+    const int pos = lane & 7;
+    bits = (uint32_t)__ldg(signs + 2 * pos) | ((uint32_t)__ldg(signs + 2 * pos + 1) << 8);
+  }
+#pragma unroll
+  for (int j = 0; j < 8; ++j) sw[j] = (((bits >> (2 * j)) & 1u) << 15) | (((bits >> (2 * j + 1)) & 1u) << 31);
+}
+
+// The rotated block of this thread as packed fp32 pairs (element 2j low).
+// Every lane of the 8-lane group must call this together.
+__device__ __forceinline__ void rht_rotate(const uint32_t w[8], const uint32_t sw[8], int lane, u64 y[8]) {
+#pragma unroll
+  for (int j = 0; j < 8; ++j) {
+    const uint32_t u = w[j] ^ sw[j];
+    const float lo = __uint_as_float(u << 16), hi = __uint_as_float(u & 0xFFFF0000u);
+    y[j] = pack2(__fadd_rn(lo, hi), __fsub_rn(lo, hi));  // stride 1
+  }
+#pragma unroll
+  for (int h = 1; h < 8; h <<= 1)  // strides 2, 4, 8 (h pairs apart)
+#pragma unroll
+    for (int j = 0; j < 8; ++j)
+      if ((j & h) == 0) {
+        const u64 a = y[j], b = y[j + h];
+        y[j] = add2(a, b);
+        y[j + h] = sub2(a, b);
+      }
+  const unsigned gmask = 0xFFu << (lane & 24);
+#pragma unroll
+  for (int m = 1; m < 8; m <<= 1) {  // strides 16, 32, 64: partner lane ^ m
+    // lower lane: own + other; upper lane: other - own (fma with -1 rounds the same)
+    const float k = (lane & m) ? -1.0f : 1.0f;
+    const u64 kk = pack2(k, k);
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      const uint32_t olo = __shfl_xor_sync(gmask, lo32(y[j]), m);
+      const uint32_t ohi = __shfl_xor_sync(gmask, hi32(y[j]), m);
+      y[j] = fma2(y[j], kk, bits2(olo, ohi));
+    }
+  }
+  const float c = __uint_as_float(kRhtScaleBits);
+  const u64 cc = pack2(c, c);
+#pragma unroll
+  for (int j = 0; j < 8; ++j) y[j] = mul2(y[j], cc);
+}
+
+// Sign nibble bits of 8 fp32 values held in 4 pairs: element 2j -> bit 3 of
+// byte j, element 2j + 1 -> bit 7.
+__device__ __forceinline__ uint32_t f32_sign_bits(const u64 y[4]) {
+  const uint32_t e = prmt(prmt(lo32(y[0]), lo32(y[1]), 0x0073u), prmt(lo32(y[2]), lo32(y[3]), 0x0073u), 0x5410u);
+  const uint32_t o = prmt(prmt(hi32(y[0]), hi32(y[1]), 0x0073u), prmt(hi32(y[2]), hi32(y[3]), 0x0073u), 0x5410u);
+  return (o & 0x80808080u) | ((e >> 4) & 0x08080808u);
+}
+
+// Algorithm 1 on one rotated block: x / s32 for fp32 numerators by
+// Markstein's correction (correctly rounded for every fp32 numerator down to
+// the tiny-value bound, see the header), then the common core.
+template <int kMode, bool kScaled>
+__device__ __forceinline__ void rht_block(const u64 y[8], const TensorConsts& tc, const float4* __restrict__ tab,
+                                          uint32_t& code_lo, uint32_t& code_hi, uint32_t& scale_byte) {
+  u64 a[8];
+  const u64 ns32 = pack2(-tc.s32, -tc.s32), r32 = pack2(tc.r32, tc.r32);
+#pragma unroll
+  for (int j = 0; j < 8; ++j) {
+    uint32_t lo = lo32(y[j]) & 0x7FFFFFFFu, hi = hi32(y[j]) & 0x7FFFFFFFu;
+    if (kScaled) {
+      lo = __float_as_uint(scalbnf(__uint_as_float(lo), tc.k));
+      hi = __float_as_uint(scalbnf(__uint_as_float(hi), tc.k));
+    }
+    a[j] = div_rn2(bits2(lo, hi), ns32, r32);
+  }
+  uint32_t mlo, mhi;
+  block_core<kMode>(a, tc, tab, mlo, mhi, scale_byte);
+  code_lo = mlo | f32_sign_bits(y);
+  code_hi = mhi | f32_sign_bits(y + 4);
+}
+
+// Rotation + Algorithm 1.  One block per thread per iteration; the grid
+// stride is a multiple of 8 blocks, so the 8 lanes of a chunk stay together.
 }  // namespace
 }  // namespace mixfp4

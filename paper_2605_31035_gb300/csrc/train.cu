@@ -19,6 +19,8 @@
 //   quantize_sr_kernel  row-wise quantization with stochastic rounding of the
 //       chosen format's codes (reading R13, the gradients of the training
 //       flow); quantize_colwise_kernel<.., true> the same down the columns.
+//   quantize_colwise_rht_kernel  the column-wise quantizer with the 128-point
+//       rotation applied along the rows first (the WGRAD inputs).
 //   transpose_2d_kernel  codes and tile scales of the transpose of a
 //       2D-quantized tensor (the DGRAD operand of the weights): 64 x 64
 //       element tiles through shared memory, one 8-byte store per thread.
@@ -160,6 +162,94 @@ quantize_2d_kernel(const uint16_t* __restrict__ x, int64_t rows, int64_t K, int6
   }
 }
 
+// Column-wise quantization with the 128-point rotation along the rows (the
+// weight-gradient inputs of the training recipe, Sec. 3.4 / Sec. 4: the RHT
+// is applied to both WGRAD operands, whose reduction runs over tokens): every
+// 128-row chunk of each column is rotated (reading R11: the caller's sign
+// vector, the same butterfly order) and the rotated column is quantized down
+// its rows -- bit for bit mixfp4_quantize_rht of X^T.  A CTA stages a
+// 128-row x 64-column tile TRANSPOSED in shared memory (a column's 128 values
+// contiguous, 272-byte pitch): each warp loads 8 columns of 32 consecutive
+// rows (16-byte loads) and scatters them with 2-byte stores that are
+// consecutive within the warp.  Then each 8-lane group holds one column chunk
+// (lane b: rows 16b..16b+15, one 32-byte shared read) and rotates it with the
+// row-wise kernel's shuffle butterfly.  kAmax: the pass that reduces max |y|
+// of the rotated tensor into the workspace word instead of quantizing.
+constexpr int kCrRows = 128, kCrCols = 64, kCrPitch = kCrRows + 8;  // staged column pitch (u16)
+
+template <int kMode, bool kAmax>
+__global__ void __launch_bounds__(256, 3)
+quantize_colwise_rht_kernel(const uint16_t* __restrict__ x, int64_t R, int64_t C, int64_t ldx,
+                            const uint8_t* __restrict__ signs, uint8_t* __restrict__ codes,
+                            uint8_t* __restrict__ scales, float* tensor_scale, uint32_t* amax_word, int scale_given) {
+  __shared__ float4 tab[128];
+  __shared__ __align__(16) uint16_t tile[kCrCols][kCrPitch];
+  griddep_wait();
+  griddep_launch_dependents();
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  uint32_t sw[8];
+  rht_sign_words(signs, lane, sw);  // lane & 7 = the block of the chunk this lane holds
+  TensorConsts tc{};
+  if (!kAmax) {
+    fill_scale_table(tab);
+    tc = tensor_consts(tensor_scale, amax_word, scale_given);
+  }
+  uint32_t m = 0;
+  const int64_t ct_n = (C + kCrCols - 1) / kCrCols, rt_n = R / kCrRows;
+  for (int64_t t = blockIdx.x; t < ct_n * rt_n; t += gridDim.x) {
+    const int64_t r0 = (t / ct_n) * kCrRows, c0 = (t % ct_n) * kCrCols;
+    // Stage: chunk q = (8 columns from 8 cg, row q % 128).
+#pragma unroll
+    for (int k = 0; k < kCrRows * kCrCols / 8 / 256; ++k) {
+      const int q = tid + 256 * k, row = q & (kCrRows - 1), cg = q >> 7;
+      uint4 v = make_uint4(0u, 0u, 0u, 0u);
+      if (c0 + cg * 8 < C) v = __ldg(reinterpret_cast<const uint4*>(x + (r0 + row) * ldx + c0 + cg * 8));
+      const uint32_t e[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        tile[cg * 8 + 2 * i][row] = (uint16_t)(e[i] & 0xFFFFu);
+        tile[cg * 8 + 2 * i + 1][row] = (uint16_t)(e[i] >> 16);
+      }
+    }
+    __syncthreads();
+#pragma unroll 1
+    for (int pass = 0; pass < kCrCols / 32; ++pass) {
+      const int cl = pass * 32 + warp * 4 + (lane >> 3), b = lane & 7;
+      const int64_t c = c0 + cl;
+      const uint4 lo4 = *reinterpret_cast<const uint4*>(&tile[cl][16 * b]);
+      const uint4 hi4 = *reinterpret_cast<const uint4*>(&tile[cl][16 * b + 8]);
+      const uint32_t w[8] = {lo4.x, lo4.y, lo4.z, lo4.w, hi4.x, hi4.y, hi4.z, hi4.w};
+      u64 y[8];
+      rht_rotate(w, sw, lane, y);  // all 32 lanes: shuffles within 8-lane groups
+      if (kAmax) {
+#pragma unroll
+        for (int j = 0; j < 8; ++j) m = max(m, max(lo32(y[j]) & 0x7FFFFFFFu, hi32(y[j]) & 0x7FFFFFFFu));
+      } else {
+        uint32_t lo, hi, sb;
+        if (tc.scaled) rht_block<kMode, true>(y, tc, tab, lo, hi, sb);
+        else rht_block<kMode, false>(y, tc, tab, lo, hi, sb);
+        if (c < C) {
+          const int64_t ob = r0 / 16 + b;
+          stg64(codes + c * (R / 2) + ob * 8, lo, hi);
+          scales[c * (R / 16) + ob] = (uint8_t)sb;
+        }
+      }
+    }
+    __syncthreads();  // the tile is restaged next
+  }
+  if (kAmax) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) m = max(m, __shfl_xor_sync(0xffffffffu, m, o));
+    __shared__ uint32_t red[8];
+    if (lane == 0) red[warp] = m;
+    __syncthreads();
+    if (tid == 0) {
+      for (int i = 1; i < 8; ++i) m = max(m, red[i]);
+      if (m) atomicMax(amax_word, m);
+    }
+  }
+}
+
 constexpr int kTrTile = 64;  // elements per side of a transpose tile
 
 __global__ void __launch_bounds__(256)
@@ -273,6 +363,29 @@ int launch_quantize_2d(const uint16_t* x, int64_t rows, int64_t K, int64_t ldx, 
                      ldx, codes, scales, tensor_scale, amax_word, scale_given);
       break;
   }
+  return e == cudaSuccess ? 0 : -1;
+}
+
+int launch_quantize_colwise_rht(const uint16_t* x, int64_t R, int64_t C, int64_t ldx, const uint8_t* signs,
+                                uint8_t* codes, uint8_t* scales, float* tensor_scale, uint32_t* amax_word, int mode,
+                                int scale_given, int amax_pass, cudaStream_t stream) {
+  const int64_t tiles = ((C + kCrCols - 1) / kCrCols) * (R / kCrRows);
+  if (tiles == 0) return 0;
+  const int64_t grid = tiles < 152 * 3 ? tiles : 152 * 3;
+  cudaError_t e;
+#define MIXFP4_LAUNCH_CR(MODE, AMAX)                                                                           \
+  e = launch_pdl(quantize_colwise_rht_kernel<MODE, AMAX>, (unsigned)grid, 256, 0, stream, x, R, C, ldx, signs, codes, \
+                 scales, tensor_scale, amax_word, scale_given)
+  if (amax_pass) {
+    MIXFP4_LAUNCH_CR(MIXFP4_MODE_MIX, true);
+  } else {
+    switch (mode) {
+      case MIXFP4_MODE_MIX: MIXFP4_LAUNCH_CR(MIXFP4_MODE_MIX, false); break;
+      case MIXFP4_MODE_E2M1_ONLY: MIXFP4_LAUNCH_CR(MIXFP4_MODE_E2M1_ONLY, false); break;
+      default: MIXFP4_LAUNCH_CR(MIXFP4_MODE_E1M2_ONLY, false); break;
+    }
+  }
+#undef MIXFP4_LAUNCH_CR
   return e == cudaSuccess ? 0 : -1;
 }
 

@@ -44,6 +44,8 @@ def lib() -> ctypes.CDLL:
         L.mixfp4_quantize_rht.argtypes = [P, I, I64, I64, I64, P, P, P, P, P, I, I, P]
         L.mixfp4_quantize_colwise.restype = I
         L.mixfp4_quantize_colwise.argtypes = [P, I, I64, I64, I64, P, P, P, P, I, I, P]
+        L.mixfp4_quantize_colwise_rht.restype = I
+        L.mixfp4_quantize_colwise_rht.argtypes = [P, I, I64, I64, I64, P, P, P, P, P, I, I, P]
         U64 = ctypes.c_uint64
         L.mixfp4_quantize_sr.restype = I
         L.mixfp4_quantize_sr.argtypes = [P, I, I64, I64, I64, P, P, P, P, I, I, U64, U64, P]
@@ -175,6 +177,28 @@ def mixfp4_quantize_colwise(x: torch.Tensor, mode: int = MODE_MIX, tensor_scale:
                                        _ptr(q.tensor_scale), _ptr(ws), int(mode),
                                        SCALE_GIVEN if given else SCALE_COMPUTE, _stream(stream))
     _check("mixfp4_quantize_colwise", st)
+    return q
+
+
+def mixfp4_quantize_colwise_rht(x: torch.Tensor, signs: torch.Tensor | None = None, mode: int = MODE_MIX,
+                                tensor_scale: torch.Tensor | None = None, out: QTensor | None = None,
+                                workspace: torch.Tensor | None = None, stream=None) -> QTensor:
+    """Rotate every 128-row chunk of each column of a bf16 [R, C] CUDA tensor and
+    quantize down the columns: the MixFP4 tensor of the rotated X^T."""
+    assert x.dtype == torch.bfloat16 and x.dim() == 2 and x.stride(1) == 1
+    assert signs is None or (signs.dtype == torch.uint8 and signs.numel() == 16 and signs.is_contiguous())
+    R, C = x.shape
+    q = out if out is not None else empty_qtensor(C, R, x.device)
+    given = tensor_scale is not None
+    if given:
+        q.tensor_scale.copy_(tensor_scale.reshape(1))
+    ws = None
+    if not given:
+        ws = workspace if workspace is not None else torch.empty(1, dtype=torch.int32, device=x.device)
+    st = lib().mixfp4_quantize_colwise_rht(_ptr(x), DTYPE_BF16, R, C, x.stride(0), _ptr(signs), _ptr(q.codes),
+                                           _ptr(q.scales), _ptr(q.tensor_scale), _ptr(ws), int(mode),
+                                           SCALE_GIVEN if given else SCALE_COMPUTE, _stream(stream))
+    _check("mixfp4_quantize_colwise_rht", st)
     return q
 
 

@@ -162,3 +162,13 @@ def test_fewrows_native_validation(lib):
     assert g(fake, fake, fake, None, fake, fake, 16, 128, 256, fake, 128, None, None) == -1   # B codes
     assert g(fake, fake, fake, fake, fake, fake, 16, 128, 256, ctypes.c_void_p((1 << 20) + 2), 128, None, None) == -3
     assert g(fake, fake, fake, fake, fake, fake, 0, 128, 256, fake, 128, None, None) == 0     # empty
+
+
+def test_colwise_rht_validation(lib):
+    fake = ctypes.c_void_p(1 << 20)
+    ws = ctypes.c_void_p(1 << 21)
+    c = lib.mixfp4_quantize_colwise_rht
+    assert c(fake, 0, 64, 32, 32, None, fake, fake, fake, ws, 0, 0, None) == -2      # R % 128
+    assert c(fake, 0, 128, 24, 24, None, fake, fake, fake, ws, 0, 0, None) == -2     # C % 16
+    assert c(fake, 0, 128, 32, 32, None, fake, fake, fake, None, 0, 0, None) == -1   # workspace
+    assert c(fake, 0, 0, 32, 32, None, None, None, fake, ws, 0, 1, None) == 0        # empty

@@ -144,3 +144,47 @@ def test_full_size_orientations(oracle):
     for col in sorted(set(rng.integers(0, 4096, 24).tolist()) | {0, 4095}):
         c, s, _ = oracle.quantize(np.ascontiguousarray(xb[:, col][None, :]), s32=s32x)
         assert np.array_equal(qc.codes[col].cpu().numpy(), c[0]) and np.array_equal(qc.scales[col].cpu().numpy(), s[0])
+
+
+@pytest.mark.parametrize("shape", [(128, 16), (256, 80), (384, 272)])
+@pytest.mark.parametrize("mode", [0, 1])
+@pytest.mark.parametrize("with_signs", [False, True])
+def test_colwise_rht_bit_exact(oracle, shape, mode, with_signs):
+    """Rotation of every 128-row chunk of each column, then column-wise
+    Algorithm 1: the rotated X^T quantized bit for bit as the oracle's
+    quantize_f32(rht(X^T)); one and several 64-column tiles, ragged columns."""
+    R, C = shape
+    x = synth.activations(R, C, 9800 + R + C, 9801)
+    signs = None
+    if with_signs:
+        signs = np.random.default_rng(R + C).integers(0, 256, 16).astype(np.uint8)
+    sg = None if signs is None else torch.from_numpy(signs).to(DEV)
+    q = ops().mixfp4_quantize_colwise_rht(x.to(DEV), sg, mode)
+    same(q, oracle.quantize_colwise_rht(synth.bf16_bits(x), signs, mode))
+
+
+def test_colwise_rht_given_scale_and_row_wise_agreement(oracle):
+    """With a given s32, and equal to the row-wise rotated quantizer applied to
+    an explicitly transposed copy of X on the GPU."""
+    x = synth.activations(256, 48, 9802, 9803)
+    s32 = 0.021
+    q = ops().mixfp4_quantize_colwise_rht(x.to(DEV), tensor_scale=torch.tensor([s32], device=DEV))
+    same(q, oracle.quantize_colwise_rht(synth.bf16_bits(x), None, 0, s32=float(np.float32(s32))))
+    qt = ops().mixfp4_quantize_rht(x.t().contiguous().to(DEV))
+    qc = ops().mixfp4_quantize_colwise_rht(x.to(DEV))
+    torch.cuda.synchronize()
+    assert torch.equal(qt.codes, qc.codes) and torch.equal(qt.scales, qc.scales)
+    assert qt.tensor_scale.item() == qc.tensor_scale.item()
+
+
+@pytest.mark.slow
+def test_colwise_rht_attention_activation(oracle):
+    """The attention activation (2048 tokens x 4096) rotated along tokens,
+    against the row-wise rotated quantizer on its explicit transpose."""
+    x = synth.workloads()["attn"].linears[0].make_x().to(DEV)
+    signs = torch.from_numpy(np.random.default_rng(7).integers(0, 256, 16).astype(np.uint8)).to(DEV)
+    qc = ops().mixfp4_quantize_colwise_rht(x, signs)
+    qt = ops().mixfp4_quantize_rht(x.t().contiguous(), signs)
+    torch.cuda.synchronize()
+    assert torch.equal(qt.codes, qc.codes) and torch.equal(qt.scales, qc.scales)
+    assert qt.tensor_scale.item() == qc.tensor_scale.item()
