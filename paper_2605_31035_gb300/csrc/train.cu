@@ -40,12 +40,14 @@ constexpr int kColThreads = 256;        // columns per tile
 constexpr int kColRows = 64;            // rows per tile (four 16-row blocks)
 
 template <int kMode, bool kSR>
-__global__ void __launch_bounds__(kColThreads, 4)
+__global__ void __launch_bounds__(kColThreads, kSR ? 3 : 4)
 quantize_colwise_kernel(const uint16_t* __restrict__ x, int64_t R, int64_t C, int64_t ldx,
                         uint8_t* __restrict__ codes, uint8_t* __restrict__ scales, float* tensor_scale,
                         const uint32_t* amax_word, int scale_given, uint64_t seed, uint64_t offset) {
   __shared__ float4 tab[128];
-  __shared__ __align__(16) uint16_t tile[kColRows][kColThreads];
+  // Row pairs interleaved: pairs[p][c] = x[2p][c] | x[2p + 1][c] << 16, the
+  // bf16 pair of column c that quantize_block takes as one word.
+  __shared__ __align__(16) uint32_t pairs[kColRows / 2][kColThreads];
   griddep_wait();
   griddep_launch_dependents();
   fill_scale_table(tab);
@@ -54,27 +56,43 @@ quantize_colwise_kernel(const uint16_t* __restrict__ x, int64_t R, int64_t C, in
   const int tid = threadIdx.x;
   const int64_t ct_n = (C + kColThreads - 1) / kColThreads, rt_n = (R + kColRows - 1) / kColRows;
   const int64_t nblk_t = R / 16;  // blocks per output row
+  // One 32-byte code store and one 4-byte scale store per full tile column
+  // when every output row starts aligned for them (R a multiple of 64).
+  const bool vec = (R % kColRows) == 0 && (reinterpret_cast<uintptr_t>(codes) & 31) == 0 &&
+                   (reinterpret_cast<uintptr_t>(scales) & 3) == 0;
   for (int64_t t = blockIdx.x; t < ct_n * rt_n; t += gridDim.x) {
     const int64_t r0 = (t / ct_n) * kColRows, c0 = (t % ct_n) * kColThreads;
-    // Stage the tile: 64 rows x 32 chunks of 8 columns (16 bytes).
+    // Stage the tile: 32 row pairs x 32 chunks of 8 columns; a thread loads
+    // the chunk from both rows of a pair (two 16-byte loads) and stores the
+    // eight interleaved words (two 16-byte stores).
 #pragma unroll
-    for (int k = 0; k < kColRows * (kColThreads / 8) / kColThreads; ++k) {
+    for (int k = 0; k < (kColRows / 2) * (kColThreads / 8) / kColThreads; ++k) {
       const int q = tid + k * kColThreads;
-      const int row = q / (kColThreads / 8), ch = q % (kColThreads / 8);
-      uint4 v = make_uint4(0u, 0u, 0u, 0u);
-      if (r0 + row < R && c0 + ch * 8 < C)
-        v = __ldg(reinterpret_cast<const uint4*>(x + (r0 + row) * ldx + c0 + ch * 8));
-      *reinterpret_cast<uint4*>(&tile[row][ch * 8]) = v;
+      const int pr = q / (kColThreads / 8), ch = q % (kColThreads / 8);
+      uint4 a = make_uint4(0u, 0u, 0u, 0u), b = a;
+      if (r0 + 2 * pr < R && c0 + ch * 8 < C) {
+        a = __ldg(reinterpret_cast<const uint4*>(x + (r0 + 2 * pr) * ldx + c0 + ch * 8));
+        b = __ldg(reinterpret_cast<const uint4*>(x + (r0 + 2 * pr + 1) * ldx + c0 + ch * 8));
+      }
+      uint4* dst = reinterpret_cast<uint4*>(&pairs[pr][ch * 8]);
+      dst[0] = make_uint4(prmt(a.x, b.x, 0x5410u), prmt(a.x, b.x, 0x7632u), prmt(a.y, b.y, 0x5410u),
+                          prmt(a.y, b.y, 0x7632u));
+      dst[1] = make_uint4(prmt(a.z, b.z, 0x5410u), prmt(a.z, b.z, 0x7632u), prmt(a.w, b.w, 0x5410u),
+                          prmt(a.w, b.w, 0x7632u));
     }
     __syncthreads();
     const int64_t c = c0 + tid;
     if (c < C) {
-#pragma unroll 1
-      for (int rb = 0; rb < kColRows / 16 && r0 + rb * 16 < R; ++rb) {
+      // The four row blocks of column c are 32 contiguous code bytes (and 4
+      // scale bytes) of output row c: gathered here, stored once.
+      uint32_t out[8] = {0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u}, sc4 = 0u;
+      const int nrb = (int)((R - r0) / 16 < kColRows / 16 ? (R - r0) / 16 : kColRows / 16);
+#pragma unroll
+      for (int rb = 0; rb < kColRows / 16; ++rb) {
+        if (rb >= nrb) break;
         uint32_t w[8];
 #pragma unroll
-        for (int j = 0; j < 8; ++j)
-          w[j] = (uint32_t)tile[rb * 16 + 2 * j][tid] | ((uint32_t)tile[rb * 16 + 2 * j + 1][tid] << 16);
+        for (int j = 0; j < 8; ++j) w[j] = pairs[rb * 8 + j][tid];
         uint32_t lo, hi, sb;
         const int64_t ob = r0 / 16 + rb;  // block index along R
         if (kSR) {
@@ -87,8 +105,23 @@ quantize_colwise_kernel(const uint16_t* __restrict__ x, int64_t R, int64_t C, in
           else if (markstein) quantize_block<kMode, false, true>(w, tc, tab, lo, hi, sb);
           else quantize_block<kMode, false, false>(w, tc, tab, lo, hi, sb);
         }
-        stg64(codes + c * (R / 2) + ob * 8, lo, hi);
-        scales[c * nblk_t + ob] = (uint8_t)sb;
+        out[2 * rb] = lo;
+        out[2 * rb + 1] = hi;
+        sc4 |= sb << (8 * rb);
+      }
+      uint8_t* cdst = codes + c * (R / 2) + (r0 / 16) * 8;
+      uint8_t* sdst = scales + c * nblk_t + r0 / 16;
+      if (vec && nrb == kColRows / 16) {
+        stg256(cdst, out);
+        *reinterpret_cast<uint32_t*>(sdst) = sc4;
+      } else {
+#pragma unroll
+        for (int rb = 0; rb < kColRows / 16; ++rb) {
+          if (rb < nrb) {
+            stg64(cdst + rb * 8, out[2 * rb], out[2 * rb + 1]);
+            sdst[rb] = (uint8_t)(sc4 >> (8 * rb));
+          }
+        }
       }
     }
     __syncthreads();  // the tile is restaged next
