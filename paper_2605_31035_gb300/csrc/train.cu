@@ -22,8 +22,8 @@
 //   quantize_colwise_rht_kernel  the column-wise quantizer with the 128-point
 //       rotation applied along the rows first (the WGRAD inputs).
 //   transpose_2d_kernel  codes and tile scales of the transpose of a
-//       2D-quantized tensor (the DGRAD operand of the weights): 64 x 64
-//       element tiles through shared memory, one 8-byte store per thread.
+//       2D-quantized tensor (the DGRAD operand of the weights): each lane
+//       transposes a 16 x 16 nibble tile in registers.
 // Every kernel shares quantize.cu's per-block arithmetic (quant_core.cuh), so
 // its codes are those of Algorithm 1 on the same values bit for bit.
 #include <cuda_runtime.h>
@@ -283,45 +283,96 @@ quantize_colwise_rht_kernel(const uint16_t* __restrict__ x, int64_t R, int64_t C
   }
 }
 
-constexpr int kTrTile = 64;  // elements per side of a transpose tile
+// Transpose of a 16 x 16 nibble tile held in registers: row i of the tile is
+// lo[i] (elements 0..7, element e at bits 4e) and hi[i] (elements 8..15); on
+// return lo[c] / hi[c] hold column c (tile rows 0..7 / 8..15), packed the same
+// way.  Block-recursive: swap the off-diagonal 8 x 8 blocks (register
+// renaming), then within every 8 x 8 block the 4 x 4 blocks (16-bit fields),
+// the 2 x 2 blocks (bytes) and the single nibbles.
+__device__ __forceinline__ void transpose_nibbles16(uint32_t lo[16], uint32_t hi[16]) {
+#pragma unroll
+  for (int r = 0; r < 8; ++r) {
+    const uint32_t t = lo[r + 8];
+    lo[r + 8] = hi[r];
+    hi[r] = t;
+  }
+#pragma unroll
+  for (int h = 0; h < 2; ++h) {
+    uint32_t* w = h ? hi : lo;
+#pragma unroll
+    for (int r = 0; r < 16; ++r)
+      if ((r & 7) < 4) {
+        const uint32_t x = w[r], y = w[r + 4];
+        w[r] = prmt(x, y, 0x5410u);
+        w[r + 4] = prmt(x, y, 0x7632u);
+      }
+#pragma unroll
+    for (int r = 0; r < 16; ++r)
+      if ((r & 3) < 2) {
+        const uint32_t x = w[r], y = w[r + 2];
+        w[r] = prmt(x, y, 0x6240u);
+        w[r + 2] = prmt(x, y, 0x7351u);
+      }
+#pragma unroll
+    for (int r = 0; r < 16; r += 2) {
+      const uint32_t x = w[r], y = w[r + 1];
+      w[r] = (x & 0x0F0F0F0Fu) | ((y << 4) & 0xF0F0F0F0u);
+      w[r + 1] = ((x >> 4) & 0x0F0F0F0Fu) | (y & 0xF0F0F0F0u);
+    }
+  }
+}
+
+// A warp moves 64 rows x 128 elements per unit; lane (rb = lane & 3,
+// kc = lane >> 2) owns the 16 x 16 tile at rows 16 rb.., elements 16 kc..:
+// sixteen 8-byte loads (8 lanes cover 64 contiguous bytes of a row), the
+// register transpose, sixteen 8-byte stores (the 4 lanes of a kc write 32
+// contiguous bytes of an output row).  No shared memory, no barriers.
+constexpr int kTrUnitRows = 64, kTrUnitCols = 128;
 
 __global__ void __launch_bounds__(256)
 transpose_2d_kernel(const uint8_t* __restrict__ codes, const uint8_t* __restrict__ scales, int64_t rows, int64_t K,
                     uint8_t* __restrict__ codes_t, uint8_t* __restrict__ scales_t) {
-  __shared__ uint8_t in[kTrTile][kTrTile / 2 + 4];  // padded rows: fewer bank conflicts on the column reads
-  const int tid = threadIdx.x;
-  const int64_t ct_n = (K + kTrTile - 1) / kTrTile, rt_n = (rows + kTrTile - 1) / kTrTile;
-  for (int64_t t = blockIdx.x; t < ct_n * rt_n; t += gridDim.x) {
-    const int64_t r0 = (t / ct_n) * kTrTile, k0 = (t % ct_n) * kTrTile;
-    // 64 rows x 32 code bytes: one 8-byte load per thread.
-    {
-      const int row = tid >> 2, q = tid & 3;
-      uint2 v = make_uint2(0u, 0u);
-      if (r0 + row < rows && k0 + q * 16 < K)
-        v = *reinterpret_cast<const uint2*>(codes + (r0 + row) * (K / 2) + k0 / 2 + q * 8);
-      *reinterpret_cast<uint32_t*>(&in[row][q * 8]) = v.x;
-      *reinterpret_cast<uint32_t*>(&in[row][q * 8 + 4]) = v.y;
-    }
-    __syncthreads();
-    // Output row k0 + kk (input column), bytes 8 q .. 8 q + 7 = input rows 16 q .. 16 q + 15.
-    {
-      const int kk = tid >> 2, q = tid & 3;
-      const int64_t k = k0 + kk;
-      if (k < K && r0 + q * 16 < rows) {
-        const int sh = 4 * (kk & 1);
-        uint32_t o[2] = {0u, 0u};
+  const int lane = threadIdx.x & 31, rb = lane & 3, kc = lane >> 2;
+  const int64_t kt_n = (K + kTrUnitCols - 1) / kTrUnitCols, rt_n = (rows + kTrUnitRows - 1) / kTrUnitRows;
+  const int64_t nbt = rows / 16, nb = K / 16;
+  // The four row blocks of a unit write one 4-byte word of each transposed
+  // scale row when those words are aligned (rows a multiple of 64).
+  const bool vec = (rows % kTrUnitRows) == 0 && (reinterpret_cast<uintptr_t>(scales_t) & 3) == 0;
+  const int64_t nwarps = (int64_t)gridDim.x * (blockDim.x / 32);
+  for (int64_t u = (int64_t)blockIdx.x * (blockDim.x / 32) + (threadIdx.x >> 5); u < kt_n * rt_n; u += nwarps) {
+    const int64_t r0 = (u / kt_n) * kTrUnitRows + rb * 16, k0 = (u % kt_n) * kTrUnitCols + kc * 16;
+    const bool live = r0 < rows && k0 < K;
+    uint32_t lo[16], hi[16], s = 0u;
+    if (live) {
 #pragma unroll
-        for (int j = 0; j < 8; ++j) {
-          const uint32_t lo = (in[q * 16 + 2 * j][kk >> 1] >> sh) & 0xFu;
-          const uint32_t hi = (in[q * 16 + 2 * j + 1][kk >> 1] >> sh) & 0xFu;
-          o[j >> 2] |= (lo | (hi << 4)) << (8 * (j & 3));
-        }
-        stg64(codes_t + k * (rows / 2) + r0 / 2 + q * 8, o[0], o[1]);
-        // The tile (r0/16 + q, k/16) scale, shared by the tile's rows.
-        scales_t[k * (rows / 16) + r0 / 16 + q] = scales[(r0 + q * 16) * (K / 16) + k / 16];
+      for (int i = 0; i < 16; ++i) {
+        const uint2 v = __ldg(reinterpret_cast<const uint2*>(codes + (r0 + i) * (K / 2) + k0 / 2));
+        lo[i] = v.x;
+        hi[i] = v.y;
+      }
+      s = scales[r0 * nb + k0 / 16];  // tile (r0 / 16, k0 / 16): the same byte in all its 16 rows
+    } else {
+#pragma unroll
+      for (int i = 0; i < 16; ++i) lo[i] = hi[i] = 0u;
+    }
+    transpose_nibbles16(lo, hi);
+    // Scales of row blocks rb = 0..3 of this kc, byte rb of s4.
+    const int base = lane & ~3;
+    const uint32_t s4 = __shfl_sync(0xffffffffu, s, base) | (__shfl_sync(0xffffffffu, s, base + 1) << 8) |
+                        (__shfl_sync(0xffffffffu, s, base + 2) << 16) | (__shfl_sync(0xffffffffu, s, base + 3) << 24);
+    if (live) {
+#pragma unroll
+      for (int c = 0; c < 16; ++c) stg64(codes_t + (k0 + c) * (rows / 2) + r0 / 2, lo[c], hi[c]);
+      if (vec) {
+        // Lane rb writes output rows k0 + 4 rb .. k0 + 4 rb + 3, row blocks r0 / 16 - rb .. + 3.
+#pragma unroll
+        for (int j = 0; j < 4; ++j)
+          *reinterpret_cast<uint32_t*>(scales_t + (k0 + 4 * rb + j) * nbt + r0 / 16 - rb) = s4;
+      } else {
+#pragma unroll
+        for (int c = 0; c < 16; ++c) scales_t[(k0 + c) * nbt + r0 / 16] = (uint8_t)s;
       }
     }
-    __syncthreads();
   }
 }
 
@@ -424,9 +475,10 @@ int launch_quantize_colwise_rht(const uint16_t* x, int64_t R, int64_t C, int64_t
 
 int launch_transpose_2d(const uint8_t* codes, const uint8_t* scales, int64_t rows, int64_t K, uint8_t* codes_t,
                         uint8_t* scales_t, cudaStream_t stream) {
-  const int64_t tiles = ((K + kTrTile - 1) / kTrTile) * ((rows + kTrTile - 1) / kTrTile);
-  if (tiles == 0) return 0;
-  const int64_t grid = tiles < 152 * 8 ? tiles : 152 * 8;
+  const int64_t units = ((K + kTrUnitCols - 1) / kTrUnitCols) * ((rows + kTrUnitRows - 1) / kTrUnitRows);
+  if (units == 0) return 0;
+  const int64_t blocks = (units + 7) / 8;  // 8 warps per CTA, one unit each per pass
+  const int64_t grid = blocks < 152 * 8 ? blocks : 152 * 8;
   transpose_2d_kernel<<<(unsigned)grid, 256, 0, stream>>>(codes, scales, rows, K, codes_t, scales_t);
   return cudaGetLastError() == cudaSuccess ? 0 : -1;
 }

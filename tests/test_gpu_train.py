@@ -77,7 +77,7 @@ def test_2d_strided_given_scale_and_activations(oracle):
     same(q, oracle.quantize_2d(synth.bf16_bits(x), s32=float(np.float32(s32))))
 
 
-@pytest.mark.parametrize("shape", [(16, 16), (48, 80), (128, 256), (272, 1040)])
+@pytest.mark.parametrize("shape", [(16, 16), (48, 80), (64, 144), (128, 256), (272, 1040), (320, 1040)])
 def test_transpose_2d_bit_exact(oracle, shape):
     rows, K = shape
     w = synth.weights(rows, K, 9300 + rows, 0.02, 0.5)
