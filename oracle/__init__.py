@@ -40,6 +40,8 @@ _SRC = os.path.join(_HERE, "mixfp4_oracle.c")
 _LIB = os.path.join(_HERE, "liboracle.so")
 
 MODE_MIX, MODE_E2M1_ONLY, MODE_E1M2_ONLY = 0, 1, 2
+# Candidates of the ablation quantizer (reading R14), bit c of a candidate mask.
+CAND_E2M1_6, CAND_E1M2, CAND_E2M1_4, CAND_E3M0 = 1, 2, 4, 8
 
 
 def build(force: bool = False) -> str:
@@ -101,6 +103,18 @@ def _L():
         lib.oracle_quantize_sr.restype = ctypes.c_int
         lib.oracle_quantize_sr.argtypes = [P, I64, I64, I64, ctypes.c_int, ctypes.c_int, P, ctypes.c_uint64,
                                            ctypes.c_uint64, P, P]
+        lib.oracle_cand_value.restype = ctypes.c_double
+        lib.oracle_cand_value.argtypes = [ctypes.c_int, ctypes.c_int]
+        lib.oracle_cand_divisor.restype = ctypes.c_float
+        lib.oracle_cand_divisor.argtypes = [ctypes.c_int]
+        lib.oracle_cand_rne.restype = ctypes.c_int
+        lib.oracle_cand_rne.argtypes = [ctypes.c_int, ctypes.c_float]
+        lib.oracle_fake_quantize.restype = ctypes.c_int
+        lib.oracle_fake_quantize.argtypes = [P, I64, I64, I64, ctypes.c_int, ctypes.c_int, ctypes.c_int, P, P, P]
+        lib.oracle_f32_to_bf16.restype = ctypes.c_uint16
+        lib.oracle_f32_to_bf16.argtypes = [ctypes.c_float]
+        lib.oracle_f32_to_bf16_array.restype = None
+        lib.oracle_f32_to_bf16_array.argtypes = [P, I64, P]
         lib.oracle_transpose_2d.restype = ctypes.c_int
         lib.oracle_transpose_2d.argtypes = [P, P, I64, I64, P, P]
         _lib = lib
@@ -348,3 +362,47 @@ def quantize_colwise_rht(x_bf16_bits: np.ndarray, signs: np.ndarray | None = Non
     quantize_f32(rht(X^T))."""
     xt = np.ascontiguousarray(np.asarray(x_bf16_bits, np.uint16).T)
     return quantize_f32(rht(xt, signs), mode, s32)
+
+
+def cand_value(c: int, p: int) -> float:
+    """Magnitude of payload p under candidate c (reading R14)."""
+    return _L().oracle_cand_value(int(c), int(p))
+
+
+def cand_divisor(c: int) -> float:
+    return _L().oracle_cand_divisor(int(c))
+
+
+def cand_rne(c: int, y: float) -> int:
+    return _L().oracle_cand_rne(int(c), float(y))
+
+
+def fake_quantize(x_bf16_bits: np.ndarray, candidates: int, block: int = 16, s32: float | None = None,
+                  out_bf16: bool = False):
+    """Quantize-dequantize of a [rows, K] bf16 tensor under a candidate set
+    (mask of CAND_*) and block size g (reading R14): (out, choice, s32), out
+    fp32 [rows, K] (bf16 bits when out_bf16), choice uint8 [rows, K/g]."""
+    x = np.ascontiguousarray(x_bf16_bits, dtype=np.uint16)
+    rows, K = x.shape
+    out = np.zeros((rows, K), np.float32)
+    choice = np.zeros((rows, K // block if block else 0), np.uint8)
+    s = np.array([0.0 if s32 is None else s32], np.float32)
+    rc = _L().oracle_fake_quantize(_p(x), rows, K, K, int(candidates), int(block), 0 if s32 is None else 1,
+                                   _p(s), _p(out), _p(choice))
+    if rc != 0:
+        raise ValueError("oracle_fake_quantize rejected the arguments or the input")
+    if out_bf16:
+        out = f32_to_bf16_array(out)
+    return out, choice, float(s[0])
+
+
+def f32_to_bf16_array(f: np.ndarray) -> np.ndarray:
+    """bf16 bits (round to nearest even) of a float32 array."""
+    f = np.ascontiguousarray(f, dtype=np.float32)
+    out = np.zeros(f.shape, np.uint16)
+    _L().oracle_f32_to_bf16_array(_p(f), f.size, _p(out))
+    return out
+
+
+def f32_to_bf16(v: float) -> int:
+    return _L().oracle_f32_to_bf16(float(v))

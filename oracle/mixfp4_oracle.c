@@ -41,6 +41,14 @@
  *   oracle_quantize_sr Algorithm 1 with stochastic rounding of the codes
  *                      (App. "Ablation Study of Stochastic Rounding", Sec. 4
  *                      pre-training recipe: SR on gradients); reading R13
+ *   oracle_fake_quantize  Algorithm 1 with the per-block MSE choice taken over
+ *                      a chosen candidate set and block size, returning the
+ *                      quantized-then-dequantized tensor and each block's
+ *                      choice: the candidate-set ablation (Sec. 2.3 "Format
+ *                      Proliferation Has Diminishing Returns", E2M1(4) and
+ *                      E3M0) and the block-size ablation (Sec. 5, Table 5);
+ *                      reading R14
+ *   oracle_f32_to_bf16 binary32 -> bfloat16, round to nearest even
  *
  * Readings where the paper is silent (the same list is kept in the design doc):
  *   R1 X_FP8 = fl32(X / s32) is an fp32 value (no FP8 cast).
@@ -83,6 +91,22 @@
  *      with key (seed low, seed high) and counter (e / 4 low, e / 4 high,
  *      offset low, offset high), word e % 4, e = the element's row-major index
  *      (r * K + k).  The sign bit stays signbit(x).
+ *   R14 candidate sets and block sizes (the ablations; the stored format
+ *      holds one type bit, so these exist only as quantize-dequantize):
+ *      candidate c = 0 E2M1 with largest value 6 (Algorithm 1's E2M1),
+ *      1 E1M2 in x2 units (R3), 2 E2M1 with largest value 4 (block scale
+ *      from B / 4, the same E2M1 codebook and rounding, saturating at 6),
+ *      3 E3M0 (Eq. 1-2 with W_E = 3, W_M = 0, bias 3: {0, 1/4, 1/2, 1, 2, 4,
+ *      8, 16}, block scale from B / 16).  Each candidate follows Algorithm 1
+ *      (R1, R2, R4, R7) with its own divisor; the tensor scale stays
+ *      max|X| / 2688.  A block is g consecutive elements of a row, g in
+ *      {8, 16, 32, 64}; its error sum is R5 on each 16-element chunk (for
+ *      g = 8: the even and the odd elements of the 8), combined for g > 16
+ *      by the pairwise tree (S_0 + S_1) + (S_2 + S_3).  Candidates are taken
+ *      in index order and a later one wins a tie (S <= best), which for
+ *      {E2M1(6), E1M2} is R6.  The output element is
+ *      sign(x) fl32(v s8 s32) (v s8 is exact), the value the dequantizer
+ *      returns; a bf16 output is that fp32 rounded to nearest even.
  */
 #include <math.h>
 #include <stdint.h>
@@ -619,4 +643,124 @@ int oracle_quantize_sr(const uint16_t* x, int64_t rows, int64_t K, int64_t ldx, 
       }
     }
   return 0;
+}
+
+/* ---------------------------------------------------------------------------
+ * R14: candidate-set and block-size ablation (Sec. 2.3, Sec. 5 Table 5).
+ * ------------------------------------------------------------------------- */
+
+/* Magnitude of payload p (0..7) under candidate c (R14). */
+double oracle_cand_value(int c, int p) {
+  if (c == 0 || c == 2) return oracle_fp4_value(0, p);
+  if (c == 1) return oracle_fp4_value(1, p);
+  return fp_code_value(p, 0, 0, 3);                 /* E3M0: W_E=3, W_M=0, bias 3 */
+}
+
+/* Block-max divisor of candidate c: the value the block max is mapped to. */
+float oracle_cand_divisor(int c) {
+  return c == 0 ? 6.0f : c == 1 ? 7.0f : c == 2 ? 4.0f : 16.0f;
+}
+
+/* R4 on candidate c's codebook: the nearest magnitude, ties to the even
+ * payload, saturating at the largest. */
+int oracle_cand_rne(int c, float y) {
+  if ((double)y >= oracle_cand_value(c, 7)) return 7;
+  int best = 0;
+  double bestd = INFINITY;
+  for (int p = 0; p < 8; ++p) {
+    double d = fabs((double)y - oracle_cand_value(c, p));
+    if (d < bestd || (d == bestd && (p & 1) == 0 && (best & 1) == 1)) {
+      best = p;
+      bestd = d;
+    }
+  }
+  return best;
+}
+
+/* Error sum of one block of g element errors (R5 per 16-element chunk, even
+ * and odd chains; pairwise tree over the chunks for g > 16). */
+static float block_error_sum(const float* d, int g) {
+  if (g <= 16) {
+    float se = 0.0f, so = 0.0f;
+    for (int i = 0; i < g; i += 2) se = fmaf(d[i], d[i], se);
+    for (int i = 1; i < g; i += 2) so = fmaf(d[i], d[i], so);
+    return se + so;
+  }
+  float s[4];
+  int n = g / 16;
+  for (int j = 0; j < n; ++j) s[j] = block_error_sum(d + 16 * j, 16);
+  for (; n > 1; n /= 2)
+    for (int j = 0; j < n / 2; ++j) s[j] = s[2 * j] + s[2 * j + 1];
+  return s[0];
+}
+
+/* Quantize-dequantize of a [rows][K] bf16 tensor (row stride ldx elements)
+ * under the candidate set cand_mask (bit c = candidate c of R14) and block
+ * size g.  scale_given / s32 as in oracle_quantize.  out: fp32 [rows][K];
+ * choice: [rows][K/g] candidate index, or NULL.  Returns 0, or -1 on a bad
+ * argument or a non-finite input. */
+int oracle_fake_quantize(const uint16_t* x, int64_t rows, int64_t K, int64_t ldx, int cand_mask, int g,
+                         int scale_given, float* s32, float* out, uint8_t* choice) {
+  if (g != 8 && g != 16 && g != 32 && g != 64) return -1;
+  if (K % 16 != 0 || K % g != 0 || (cand_mask & 15) == 0 || (cand_mask & ~15) != 0) return -1;
+  float amax = 0.0f;
+  for (int64_t r = 0; r < rows; ++r)
+    for (int64_t k = 0; k < K; ++k) {
+      float v = bf16_to_float(x[r * ldx + k]);
+      if (!isfinite(v)) return -1;
+      if (fabsf(v) > amax) amax = fabsf(v);
+    }
+  float s = scale_given ? *s32 : amax / 2688.0f;
+  if (!scale_given) *s32 = s;
+  int64_t nb = K / g;
+  for (int64_t r = 0; r < rows; ++r)
+    for (int64_t b = 0; b < nb; ++b) {
+      float a[64], B = 0.0f;
+      int neg[64];
+      for (int i = 0; i < g; ++i) {
+        float v = bf16_to_float(x[r * ldx + b * g + i]);
+        neg[i] = signbit(v) ? 1 : 0;
+        a[i] = (s > 0.0f) ? fabsf(v) / s : 0.0f;     /* R1, R7 */
+        if (a[i] > B) B = a[i];
+      }
+      int best = -1;
+      float best_S = 0.0f, best_s8 = 0.0f, best_q[64];
+      for (int c = 0; c < 4; ++c) {
+        if (!((cand_mask >> c) & 1)) continue;
+        float s8 = (float)oracle_e4m3_value(oracle_e4m3_rne(B / oracle_cand_divisor(c)));  /* R2 */
+        float q[64], d[64];
+        for (int i = 0; i < g; ++i) {
+          float y = (s8 > 0.0f) ? a[i] / s8 : 0.0f;
+          q[i] = (float)oracle_cand_value(c, oracle_cand_rne(c, y));
+          d[i] = q[i] * s8 - a[i];                    /* the product is exact */
+        }
+        float S = block_error_sum(d, g);
+        if (best < 0 || S <= best_S) {                /* a later candidate wins a tie */
+          best = c;
+          best_S = S;
+          best_s8 = s8;
+          memcpy(best_q, q, sizeof(float) * (size_t)g);
+        }
+      }
+      for (int i = 0; i < g; ++i) {
+        float o = (float)((double)best_q[i] * (double)best_s8 * (double)s);
+        out[r * K + b * g + i] = neg[i] ? -o : o;
+      }
+      if (choice) choice[r * nb + b] = (uint8_t)best;
+    }
+  return 0;
+}
+
+/* binary32 -> bfloat16 bits, round to nearest, ties to even (finite input). */
+uint16_t oracle_f32_to_bf16(float f) {
+  uint32_t u;
+  memcpy(&u, &f, 4);
+  uint32_t keep = u >> 16, rest = u & 0xFFFFu;
+  if (rest > 0x8000u || (rest == 0x8000u && (keep & 1u))) keep += 1u;
+  return (uint16_t)keep;
+}
+
+/* oracle_f32_to_bf16 over an array of n values. */
+void oracle_f32_to_bf16_array(const float* f, int64_t n, uint16_t* out) {
+  for (int64_t i = 0; i < n; ++i) out[i] = oracle_f32_to_bf16(f[i]);
 }

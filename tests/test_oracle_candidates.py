@@ -1,0 +1,233 @@
+"""Pins of the candidate-set / block-size ablation oracle (reading R14:
+Sec. 2.3 candidate sets with E2M1(4) and E3M0, Sec. 5 Table 5 block sizes).
+
+What fixes it from outside itself:
+* Eq. 1-2 give the E3M0 codebook (W_E = 3, W_M = 0, bias 3); E2M1(4) reuses
+  Table 1's E2M1 codebook with the block max mapped to 4.
+* For {E2M1(6), E1M2}, {E2M1(6)} and {E1M2} at g = 16 the ablation is
+  Algorithm 1 followed by the dequantizer, both already pinned: bit-exact
+  equality, and the choice equals the stored type bit.
+* A single candidate at any g is rebuilt from library routines (torch's
+  float8_e4m3fn cast for the block scale, numpy rint / frexp for the codes).
+* Exact grids: a block on one candidate's grid, with its max on that
+  candidate's largest value, comes back unchanged and chooses that candidate.
+* The choice minimises the block's squared error (checked in float64).
+* Ties (an all-zero block) go to the last candidate of the set; scaling by
+  2^k and negation are invariants; a g > 16 block whose other chunks are zero
+  equals the g = 16 block.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2605_31035_gb300 import synth
+
+E2M1 = [0.0, 0.5, 1.0, 1.5, 2.0, 3.0, 4.0, 6.0]
+ALL = oracle.CAND_E2M1_6 | oracle.CAND_E1M2 | oracle.CAND_E2M1_4 | oracle.CAND_E3M0
+
+
+def bits(vals):
+    return synth.bf16_bits(torch.as_tensor(np.asarray(vals, np.float32)).to(torch.bfloat16))
+
+
+def test_codebooks_and_divisors():
+    # Eq. 1-2 with W_E = 3, W_M = 0: bias 2^2 - 1 = 3, E = 0 -> 0, E >= 1 -> 2^(E - 3).
+    e3m0 = [0.0] + [2.0 ** (e - 3) for e in range(1, 8)]
+    assert [oracle.cand_value(3, p) for p in range(8)] == e3m0
+    assert [oracle.cand_value(0, p) for p in range(8)] == E2M1
+    assert [oracle.cand_value(2, p) for p in range(8)] == E2M1
+    assert [oracle.cand_value(1, p) for p in range(8)] == [float(p) for p in range(8)]
+    assert [oracle.cand_divisor(c) for c in range(4)] == [6.0, 7.0, 4.0, 16.0]
+
+
+def _nearest_even(vals, y):
+    d = np.abs(np.asarray(vals, np.float64) - y)
+    near = np.flatnonzero(d == d.min())
+    even = [p for p in near if p % 2 == 0]
+    return int(even[0] if even else near[0])
+
+
+@pytest.mark.parametrize("c", range(4))
+def test_rounding_brute_force(c):
+    vals = [oracle.cand_value(c, p) for p in range(8)]
+    ys = set()
+    for v in vals + [(vals[i] + vals[i + 1]) / 2 for i in range(7)]:
+        f = np.float32(v)
+        ys.update([float(f), float(np.nextafter(f, np.float32(0))), float(np.nextafter(f, np.float32(100)))])
+    ys.update(np.random.default_rng(5).uniform(0, 20, 400).astype(np.float32).tolist())
+    for y in sorted(ys):
+        if y < 0:
+            continue
+        want = 7 if y >= vals[7] else _nearest_even(vals, y)
+        assert oracle.cand_rne(c, y) == want, (c, y)
+    # the E3M0 ties written out: 1/8 -> 0, 3/8 -> 1/2, 12 -> 8; E2M1(4): 5 -> 4
+    assert [oracle.cand_rne(3, y) for y in (0.125, 0.375, 12.0, 12.001, 99.0)] == [0, 2, 6, 7, 7]
+    assert oracle.cand_rne(2, 5.0) == 6
+
+
+@pytest.mark.parametrize("mode,mask", [(oracle.MODE_MIX, oracle.CAND_E2M1_6 | oracle.CAND_E1M2),
+                                       (oracle.MODE_E2M1_ONLY, oracle.CAND_E2M1_6),
+                                       (oracle.MODE_E1M2_ONLY, oracle.CAND_E1M2)])
+@pytest.mark.parametrize("given", [None, 0.0123])
+def test_reduces_to_algorithm1(mode, mask, given):
+    x = synth.bf16_bits(synth.activations(24, 256, 811, 812))
+    s32 = None if given is None else float(np.float32(given))
+    codes, scales, s = oracle.quantize(x, mode, s32)
+    ref = oracle.dequantize(codes, scales, s)
+    out, choice, s2 = oracle.fake_quantize(x, mask, 16, s32)
+    assert np.float32(s2).view(np.uint32) == np.float32(s).view(np.uint32)
+    assert np.array_equal(out.view(np.uint32), ref.view(np.uint32))
+    t = scales >> 7   # type bit: 1 = E1M2 = candidate 1
+    assert np.array_equal(choice, np.where(t == 1, 1, 0).astype(np.uint8))
+
+
+def _library_single(x_bits, c, g):
+    """One candidate rebuilt from library routines: numpy float32 division,
+    torch's E4M3 cast (saturated at 448 first), numpy rint / frexp."""
+    x = (x_bits.astype(np.uint32) << 16).view(np.float32)
+    rows, K = x.shape
+    s32 = np.float32(np.abs(x).max()) / np.float32(2688.0)
+    a = (np.abs(x) / s32).astype(np.float32) if s32 > 0 else np.zeros_like(x)
+    B = a.reshape(rows, K // g, g).max(axis=2)
+    r = (B / np.float32(oracle.cand_divisor(c))).astype(np.float32)
+    s8 = torch.as_tensor(np.minimum(r, np.float32(448.0))).to(torch.float8_e4m3fn).to(torch.float32).numpy()
+    s8e = np.repeat(s8, g, axis=1)
+    with np.errstate(divide="ignore", invalid="ignore"):
+        y = np.where(s8e > 0, a / s8e, np.float32(0)).astype(np.float32)
+    if c == 1:
+        q = np.minimum(np.rint(y), 7.0)
+    elif c == 3:
+        m, e = np.frexp(y.astype(np.float64))          # y = m 2^e, m in [0.5, 1)
+        lo, hi = np.ldexp(1.0, e - 1), np.ldexp(1.0, e)
+        lo_even = ((e - 1 + 3) % 2) == 0                # payload of 2^(e-1) is e + 2
+        q = np.where(m > 0.75, hi, np.where(m < 0.75, lo, np.where(lo_even, lo, hi)))
+        q = np.where(y < 0.25, np.where(y > 0.125, 0.25, 0.0), q)
+        q = np.where(y >= 16.0, 16.0, q)
+    else:
+        V = np.asarray(E2M1)
+        d = np.abs(y[..., None].astype(np.float64) - V)
+        dmin = d.min(axis=-1, keepdims=True)
+        cand = (d == dmin)
+        idx = np.where(cand[..., ::2].any(axis=-1), np.argmax(cand & (np.arange(8) % 2 == 0), axis=-1),
+                       np.argmax(cand, axis=-1))
+        q = np.where(y >= 6.0, 6.0, V[idx])
+    o = (q * s8e.astype(np.float64) * np.float64(s32)).astype(np.float32)
+    return np.where(np.signbit(x), -o, o).astype(np.float32)
+
+
+@pytest.mark.parametrize("c", range(4))
+@pytest.mark.parametrize("g", [8, 16, 32, 64])
+def test_single_candidate_from_library_routines(c, g):
+    x = synth.bf16_bits(synth.activations(16, 256, 820 + g, 821))
+    out, choice, _ = oracle.fake_quantize(x, 1 << c, g)
+    ref = _library_single(x, c, g)
+    assert np.array_equal(out.view(np.uint32), ref.view(np.uint32))
+    assert np.all(choice == c)
+
+
+GRIDS = {0: [6.0, 0.5, 1.5, 3.0], 1: [7.0, 1.0, 5.0, 3.0], 2: [4.0, 0.5, 3.0, 1.5], 3: [16.0, 0.25, 2.0, 1.0]}
+
+
+@pytest.mark.parametrize("g", [8, 16, 32, 64])
+def test_exact_grid_round_trip(g):
+    rng = np.random.default_rng(830 + g)
+    s32, s8 = 2.0 ** -4, 2.0 ** -3
+    rows = []
+    anchor = np.array([6.0, 3.0, 0.5] + [0.0] * (g - 3)) * 448.0 * s32     # tensor max 2688 s32
+    rows.append(anchor)
+    for c in range(4):
+        grid = [v for v in (oracle.cand_value(c, p) for p in range(8)) if v <= GRIDS[c][0]]
+        blk = np.array(GRIDS[c] + list(rng.choice(grid, g - 4))) * s8
+        blk *= rng.choice([-1.0, 1.0], g)
+        rows.append(blk * s32)
+    if g == 8:
+        rows.append(np.zeros(g))   # K a multiple of 16; a zero block ties to E3M0
+    x = np.concatenate(rows)[None, :]
+    xb = bits(x)
+    assert np.array_equal((xb.astype(np.uint32) << 16).view(np.float32), x.astype(np.float32))
+    out, choice, s = oracle.fake_quantize(xb, ALL, g)
+    assert s == s32
+    assert np.array_equal(out, x.astype(np.float32))
+    # The anchor's E2M1(4) scale B / 4 = 672 saturates to 448, the E2M1(6)
+    # scale: both are exact and the tie goes to the later candidate.
+    assert list(choice[0][:5]) == [2, 0, 1, 2, 3]
+
+
+@pytest.mark.parametrize("g", [8, 16, 32, 64])
+@pytest.mark.parametrize("mask", [ALL, oracle.CAND_E2M1_6 | oracle.CAND_E2M1_4,
+                                  oracle.CAND_E2M1_6 | oracle.CAND_E1M2 | oracle.CAND_E3M0])
+def test_choice_minimises_block_error(g, mask):
+    x = synth.bf16_bits(synth.activations(32, 512, 840 + g, 841))
+    xf = (x.astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+    out, choice, s32 = oracle.fake_quantize(x, mask, g)
+    errs = {}
+    for c in range(4):
+        if mask >> c & 1:
+            o, _, _ = oracle.fake_quantize(x, 1 << c, g)
+            errs[c] = ((o.astype(np.float64) - xf) ** 2).reshape(32, -1, g).sum(axis=2)
+    best = np.min(np.stack(list(errs.values())), axis=0)
+    chosen = np.choose(np.searchsorted(sorted(errs), choice), [errs[c] for c in sorted(errs)])
+    # S is a binary32 sum in a fixed order: the chosen error is the minimum up to its rounding.
+    assert np.all(chosen <= best * (1 + 1e-5) + 1e-30)
+    got = ((out.astype(np.float64) - xf) ** 2).reshape(32, -1, g).sum(axis=2)
+    assert np.allclose(got, chosen, rtol=0, atol=0)
+
+
+def test_zero_blocks_tie_to_the_last_candidate():
+    x = np.zeros((2, 64), np.float32)
+    x[1, :] = -0.0
+    x[0, 40] = 3.0
+    xb = bits(x)
+    for mask, last in [(ALL, 3), (oracle.CAND_E2M1_6 | oracle.CAND_E2M1_4, 2), (oracle.CAND_E2M1_6, 0)]:
+        out, choice, _ = oracle.fake_quantize(xb, mask, 16)
+        assert list(choice[1]) == [last] * 4 and list(choice[0][:2]) == [last] * 2
+        assert np.all(out[1] == 0) and np.all(np.signbit(out[1]))
+
+
+@pytest.mark.parametrize("g", [8, 32, 64])
+def test_invariants(g):
+    x = synth.activations(8, 256, 850 + g, 851)
+    xb = synth.bf16_bits(x)
+    out, choice, s = oracle.fake_quantize(xb, ALL, g)
+    out2, choice2, s2 = oracle.fake_quantize(synth.bf16_bits(x * 8), ALL, g)
+    assert s2 == s * 8 and np.array_equal(choice2, choice) and np.array_equal(out2, out * 8)
+    out3, choice3, _ = oracle.fake_quantize(synth.bf16_bits(-x), ALL, g)
+    assert np.array_equal(choice3, choice) and np.array_equal(out3.view(np.uint32), (-out).view(np.uint32))
+
+
+@pytest.mark.parametrize("g", [8, 32, 64])
+def test_block_with_zero_chunks_equals_smaller_block(g):
+    """g = 32, 64: a block whose chunks past the first 16 elements are zero
+    gives that chunk's g = 16 result; g = 8: the first 8-block of a 16-block
+    whose second half is zero gives the g = 16 result (same block max, and
+    zero errors add nothing to the sums)."""
+    x = synth.activations(8, 256, 860 + g, 861).float().numpy()
+    period = max(g, 16)
+    keep = (np.arange(256) % period) < min(g, 16)
+    x = np.where(keep, x, 0.0).astype(np.float32)
+    xb = bits(x)
+    s = float(np.float32(np.abs(x).max()) / np.float32(2688.0))
+    out_g, ch_g, _ = oracle.fake_quantize(xb, ALL, g, s)
+    out_16, ch_16, _ = oracle.fake_quantize(xb, ALL, 16, s)
+    assert np.array_equal(out_g[:, keep].view(np.uint32), out_16[:, keep].view(np.uint32))
+    if g == 8:
+        assert np.array_equal(ch_g[:, ::2], ch_16)
+    else:
+        assert np.array_equal(ch_g, ch_16[:, ::g // 16])
+
+
+def test_bf16_rounding_matches_torch():
+    rng = np.random.default_rng(870)
+    f = np.concatenate([rng.standard_normal(20000).astype(np.float32) * 10.0 ** rng.integers(-30, 30, 20000),
+                        np.array([1.0 + 2.0 ** -8, 1.0 + 3 * 2.0 ** -8, 1.0 + 2.0 ** -9, -2.0 ** -130, 0.0, -0.0],
+                                 np.float32)]).astype(np.float32)
+    want = synth.bf16_bits(torch.from_numpy(f).to(torch.bfloat16))
+    assert np.array_equal(oracle.f32_to_bf16_array(f), want)
+
+
+def test_rejects_bad_arguments():
+    x = bits(np.ones((1, 48), np.float32))
+    for mask, g in [(0, 16), (16, 16), (1, 12), (1, 32)]:
+        with pytest.raises(ValueError):
+            oracle.fake_quantize(x, mask, g)
