@@ -278,6 +278,19 @@ def run_ours(args):
     qc = ops.empty_qtensor(xs.shape[1], xs.shape[0], dev)
     crht_ms = time_quant(lambda: ops.mixfp4_quantize_colwise_rht(xs, out=qc, tensor_scale=given_rht_col))
     del qc
+    # Candidate-set / block-size ablation (quantize-dequantize, bf16 out, the
+    # per-block choice written), tensor scale given.
+    fq_out = torch.empty(xs.shape, dtype=torch.bfloat16, device=dev)
+    fq_ch = torch.empty(xs.shape[0], xs.shape[1] // 8, dtype=torch.uint8, device=dev)
+    ablation = {}
+    for name, mask, g in FQ_SETS:
+        chv = fq_ch[:, : xs.shape[1] // g]
+        ms_ = time_quant(lambda: ops.mixfp4_fake_quantize(xs, mask, g, torch.bfloat16, tensor_scale=given,
+                                                          out=fq_out, choice=chv))
+        gbs = xs.numel() * (4.0 + 1.0 / g) / (ms_ * 1e-3) / 1e9
+        ablation[f"{name}_g{g}"] = {"ms": round(ms_, 4), "alg_gbs": round(gbs, 1),
+                                    "frac_of_hbm": round(gbs / pk["hbm_gbs"], 4)}
+    del fq_out, fq_ch
 
     given_gbs = xs.numel() * QUANT_BYTES_PER_ELEM / (given_ms * 1e-3) / 1e9
     sweep_alg_gbs = xs.numel() * QUANT_BYTES_PER_ELEM / (sweep_ms * 1e-3) / 1e9
@@ -387,6 +400,10 @@ def run_ours(args):
                     "ms": round(sr_ms, 4), "alg_gbs": round(xs_numel * QUANT_BYTES_PER_ELEM / (sr_ms * 1e-3) / 1e9, 1)},
                 "transpose_2d": {"ms": round(transpose_ms, 4),
                                  "alg_gbs": round(xs_numel * 2 * (0.5 + 1.0 / 16) / (transpose_ms * 1e-3) / 1e9, 1)}},
+            "candidate_ablation_2^28": {
+                **ablation,
+                "alg_bytes_per_element": "2 (bf16 in) + 2 (bf16 out) + 1/g (choice)",
+                "note": "quantize-dequantize under a candidate set (E2M1(6), E1M2, E2M1(4), E3M0) and block size g"},
             "rht_quantizer_2^28": {
                 "fused_rotation_quantize_given_scale": {
                     "ms": round(rht_given_ms, 4),
@@ -579,6 +596,11 @@ def run_reference(args):
     print(json.dumps(out), flush=True)
 
 
+# (name, candidate mask, block size) of the ablation lines.
+FQ_SETS = [("mixfp4", 1 | 2, 16), ("four_over_six", 1 | 4, 16), ("e2_e1_e3", 1 | 2 | 8, 16),
+           ("all_four", 15, 16), ("e2_e1_e3", 1 | 2 | 8, 64), ("all_four", 15, 8)]
+
+
 def run_kernel_only(args):
     """One kernel on one workload, for profilers: `--warmup` untimed launches,
     then `--steps` launches, then exit.  Prints the CUDA-event time per launch."""
@@ -628,6 +650,10 @@ def run_kernel_only(args):
         q2 = ops.mixfp4_quantize_2d(x, workspace=ws)
         fn = lambda: ops.mixfp4_transpose_2d(q2)
         work = x.numel() * 2 * (0.5 + 1.0 / 16)
+    elif args.kernel == "fake_quantize":
+        fo = torch.empty(x.shape, dtype=torch.bfloat16, device=dev)
+        fn = lambda: ops.mixfp4_fake_quantize(x, 15, 16, torch.bfloat16, out=fo, workspace=ws)
+        work = x.numel() * (4.0 + 1.0 / 16)
     elif args.kernel == "quantize_rht":
         fn = lambda: ops.mixfp4_quantize_rht(x, out=qx, workspace=ws)
         work = x.numel() * QUANT_BYTES_PER_ELEM
@@ -662,7 +688,7 @@ def main(argv=None):
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-configs", action="store_true", help="skip the other configs' GEMM lines")
     ap.add_argument("--kernel", choices=["gemm", "gemm_native", "gemm_native_fewrows", "split_native", "quantize", "quantize_rht", "quantize_colwise",
-                             "quantize_2d", "transpose_2d", "dequantize"], default=None,
+                             "quantize_2d", "transpose_2d", "fake_quantize", "dequantize"], default=None,
                     help="profiling mode: launch only this kernel")
     ap.add_argument("--workload", default=WORKLOAD,
                     help="tiny|attn|mlp|decode|hadamard|sweepNN (kernel-only mode)")

@@ -53,7 +53,13 @@ enum { MIXFP4_MODE_MIX = 0,        /* Alg. 1: per-block E2M1/E1M2 by lower MSE *
 enum { MIXFP4_SCALE_COMPUTE = 0,   /* compute s32 = fl32(max|x| / 2688), write *tensor_scale */
        MIXFP4_SCALE_GIVEN = 1      /* read s32 from *tensor_scale */ };
 
-enum { MIXFP4_DTYPE_BF16 = 0 };
+enum { MIXFP4_DTYPE_BF16 = 0, MIXFP4_DTYPE_F32 = 1 /* output of mixfp4_fake_quantize only */ };
+
+/* Candidate formats of mixfp4_fake_quantize (bit c of `candidates`). */
+enum { MIXFP4_CAND_E2M1_6 = 1,   /* E2M1, block max mapped to 6 (Algorithm 1's E2M1) */
+       MIXFP4_CAND_E1M2 = 2,     /* E1M2 in x2 units {0..7}, block max mapped to 7 */
+       MIXFP4_CAND_E2M1_4 = 4,   /* E2M1, block max mapped to 4 (the "4/6" candidate) */
+       MIXFP4_CAND_E3M0 = 8      /* E3M0 {0, 1/4, ..., 16}, block max mapped to 16 */ };
 
 /*
  * mixfp4_quantize -- Algorithm 1 (Sec. 3.2) with type-in-scale packing (App. B.3).
@@ -174,6 +180,41 @@ int mixfp4_quantize_sr(const void* x, int dtype, int64_t rows, int64_t K, int64_
 int mixfp4_quantize_colwise_sr(const void* x, int dtype, int64_t R, int64_t C, int64_t ldx, uint8_t* codes,
                                uint8_t* scales, float* tensor_scale, uint32_t* workspace, int mode, int scale_flag,
                                uint64_t seed, uint64_t offset, void* stream);
+
+/*
+ * mixfp4_fake_quantize -- quantize-dequantize under a chosen candidate set
+ * and block size: the paper's candidate-set ablation (Sec. 2.3, candidate
+ * sets {E2M1(6), E2M1(4)} and {E2M1(6), E1M2, E3M0}) and block-size ablation
+ * (Sec. 5, Table 5, g = 8..64).  A block is g consecutive elements of a row.
+ * Every candidate c in `candidates` follows Algorithm 1 with its own divisor
+ * d_c (6, 7, 4, 16): s8 = E4M3_RNE(fl32(B / d_c)) from the block max B of
+ * |x / s32|, codes by round-to-nearest-even of fl32(|x / s32| / s8) onto its
+ * codebook (saturating), error sum S in the order of mixfp4_quantize on each
+ * 16-element chunk (for g = 8: the even and the odd elements of the 8) and,
+ * for g > 16, the pairwise tree (S_0 + S_1) + (S_2 + S_3) of the chunks.
+ * Candidates are visited in bit order and a later one wins a tie (S <= best),
+ * so {E2M1_6, E1M2} at g = 16 is Algorithm 1.  s32 = fl32(max|X| / 2688).
+ * The output is sign(x) fl32(v s8 s32) of the chosen candidate (v its code's
+ * magnitude): for {E2M1_6, E1M2} at g = 16, bit for bit mixfp4_dequantize of
+ * mixfp4_quantize.  Three or more formats, or other block sizes, cannot be
+ * stored in the one type bit, so this entry point returns values, not codes.
+ *
+ * x            device, bf16 [rows][ldx]; 32-byte aligned; ldx % 16 == 0, ldx >= K.
+ * rows, K      K % 16 == 0 and K % block == 0 (else MIXFP4_ERR_SHAPE); 0 is a
+ *              no-op (with SCALE_COMPUTE *tensor_scale is set to 0).
+ * candidates   nonzero mask of MIXFP4_CAND_* (else MIXFP4_ERR_ARG).
+ * block        8, 16, 32 or 64 (else MIXFP4_ERR_ARG).
+ * tensor_scale, workspace, scale_flag, stream: as mixfp4_quantize.
+ * out          device, [rows][ldo] of out_dtype (MIXFP4_DTYPE_F32, or
+ *              MIXFP4_DTYPE_BF16 = that fp32 value rounded to nearest even);
+ *              32-byte aligned, ldo % 16 == 0, ldo >= K.             (output)
+ * choice       device, uint8 [rows][K / block]: index (bit position) of each
+ *              block's chosen candidate; 2-byte aligned; NULL to skip. (output)
+ * Errors: as mixfp4_quantize; MIXFP4_ERR_DTYPE for another out_dtype.
+ */
+int mixfp4_fake_quantize(const void* x, int dtype, int64_t rows, int64_t K, int64_t ldx, int candidates, int block,
+                         float* tensor_scale, uint32_t* workspace, int scale_flag, void* out, int out_dtype,
+                         int64_t ldo, uint8_t* choice, void* stream);
 
 /*
  * mixfp4_quantize_2d -- Algorithm 1 with 16 x 16 blocks, the weight

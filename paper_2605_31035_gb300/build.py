@@ -19,7 +19,7 @@ BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libmixfp4.so")
 INCLUDE = os.path.join(os.path.dirname(HERE), "include")
 
-SOURCES = ["api.cu", "quantize.cu", "train.cu", "gemm.cu", "native.cu", "noalloc.cu", "selftest.cu"]
+SOURCES = ["api.cu", "quantize.cu", "train.cu", "gemm.cu", "native.cu", "candidates.cu", "noalloc.cu", "selftest.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xptxas", "-v",
               "--ftz=false", "--prec-div=true", "--prec-sqrt=true", "--fmad=false",

@@ -236,6 +236,40 @@ int mixfp4_quantize_2d(const void* x, int dtype, int64_t rows, int64_t K, int64_
   return launch_status();
 }
 
+int mixfp4_fake_quantize(const void* x, int dtype, int64_t rows, int64_t K, int64_t ldx, int candidates, int block,
+                         float* tensor_scale, uint32_t* workspace, int scale_flag, void* out, int out_dtype,
+                         int64_t ldo, uint8_t* choice, void* stream) {
+  if (dtype != MIXFP4_DTYPE_BF16) return MIXFP4_ERR_DTYPE;
+  if (out_dtype != MIXFP4_DTYPE_BF16 && out_dtype != MIXFP4_DTYPE_F32) return MIXFP4_ERR_DTYPE;
+  if (candidates <= 0 || candidates > 15) return MIXFP4_ERR_ARG;
+  if (block != 8 && block != 16 && block != 32 && block != 64) return MIXFP4_ERR_ARG;
+  if (scale_flag != MIXFP4_SCALE_COMPUTE && scale_flag != MIXFP4_SCALE_GIVEN) return MIXFP4_ERR_ARG;
+  if (rows < 0 || K < 0 || K % 16 != 0 || K % block != 0 || ldx < K || ldo < K) return MIXFP4_ERR_SHAPE;
+  if (!tensor_scale) return MIXFP4_ERR_NULL;
+  if (scale_flag == MIXFP4_SCALE_COMPUTE && !workspace) return MIXFP4_ERR_NULL;
+  const bool empty = (rows == 0 || K == 0);
+  if (!empty && (!x || !out)) return MIXFP4_ERR_NULL;
+  if (!empty && (!aligned(x, 32) || ldx % 16 != 0 || !aligned(out, 32) || ldo % 16 != 0)) return MIXFP4_ERR_ALIGN;
+  if (choice && !aligned(choice, 2)) return MIXFP4_ERR_ALIGN;
+  if (!aligned(tensor_scale, 4) || (workspace && !aligned(workspace, 4))) return MIXFP4_ERR_ALIGN;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const int given = scale_flag == MIXFP4_SCALE_GIVEN;
+  if (empty) {
+    if (!given && cudaMemsetAsync(tensor_scale, 0, sizeof(float), s) != cudaSuccess) return MIXFP4_ERR_CUDA;
+    return MIXFP4_OK;
+  }
+  const uint16_t* xb = static_cast<const uint16_t*>(x);
+  if (!given) {
+    if (cudaMemsetAsync(workspace, 0, sizeof(uint32_t), s) != cudaSuccess) return MIXFP4_ERR_CUDA;
+    mixfp4::launch_amax(xb, rows, K, ldx, workspace, s);
+    if (int st = launch_status()) return st;
+  }
+  if (mixfp4::launch_fake_quantize(xb, rows, K, ldx, candidates, block, tensor_scale, workspace, given, out,
+                                   out_dtype == MIXFP4_DTYPE_BF16, ldo, choice, s) != 0)
+    return MIXFP4_ERR_CUDA;
+  return launch_status();
+}
+
 int mixfp4_transpose_2d(const uint8_t* codes, const uint8_t* scales, int64_t rows, int64_t K, uint8_t* codes_t,
                         uint8_t* scales_t, void* stream) {
   if (rows < 0 || K < 0 || rows % 16 != 0 || K % 16 != 0) return MIXFP4_ERR_SHAPE;

@@ -32,6 +32,9 @@ int launch_quantize_2d(const uint16_t* x, int64_t rows, int64_t K, int64_t ldx, 
                        cudaStream_t stream);
 int launch_transpose_2d(const uint8_t* codes, const uint8_t* scales, int64_t rows, int64_t K, uint8_t* codes_t,
                         uint8_t* scales_t, cudaStream_t stream);
+int launch_fake_quantize(const uint16_t* x, int64_t rows, int64_t K, int64_t ldx, int candidates, int block,
+                         float* tensor_scale, const uint32_t* amax_word, int scale_given, void* out, int out_bf16,
+                         int64_t ldo, uint8_t* choice, cudaStream_t stream);
 int launch_bounded_wait_selftest(uint32_t* status, uint64_t limit_ns, cudaStream_t stream);
 int launch_dequantize(const uint8_t* codes, const uint8_t* scales, const float* tensor_scale,
                       int64_t rows, int64_t K, float* out, cudaStream_t stream);

@@ -14,7 +14,9 @@ import torch
 
 MODE_MIX, MODE_E2M1_ONLY, MODE_E1M2_ONLY = 0, 1, 2
 SCALE_COMPUTE, SCALE_GIVEN = 0, 1
-DTYPE_BF16 = 0
+DTYPE_BF16, DTYPE_F32 = 0, 1
+# Candidates of mixfp4_fake_quantize, bit c of the mask.
+CAND_E2M1_6, CAND_E1M2, CAND_E2M1_4, CAND_E3M0 = 1, 2, 4, 8
 
 STATUS = {0: "ok", -1: "null pointer", -2: "invalid shape", -3: "misaligned", -4: "unsupported dtype",
           -5: "CUDA error", -6: "device-side wait timed out", -7: "argument out of range"}
@@ -65,6 +67,8 @@ def lib() -> ctypes.CDLL:
         L.mixfp4_gemm_native.argtypes = [P, P, P, P, P, P, P, P, I64, I64, I64, P, I64, P, P]
         L.mixfp4_gemm_native_fewrows.restype = I
         L.mixfp4_gemm_native_fewrows.argtypes = [P, P, P, P, P, P, I64, I64, I64, P, I64, P, P]
+        L.mixfp4_fake_quantize.restype = I
+        L.mixfp4_fake_quantize.argtypes = [P, I, I64, I64, I64, I, I, P, P, I, P, I, I64, P, P]
         L.mixfp4_selftest_bounded_wait.restype = I
         L.mixfp4_selftest_bounded_wait.argtypes = [P, ctypes.c_uint64, P]
         L.mixfp4_status_string.restype = ctypes.c_char_p
@@ -255,6 +259,38 @@ def mixfp4_transpose_2d(q: QTensor, out: QTensor | None = None, stream=None) -> 
                                    _stream(stream))
     _check("mixfp4_transpose_2d", st)
     return t
+
+
+def mixfp4_fake_quantize(x: torch.Tensor, candidates: int, block: int = 16, out_dtype=torch.float32,
+                         tensor_scale: torch.Tensor | None = None, want_choice: bool = True,
+                         out: torch.Tensor | None = None, choice: torch.Tensor | None = None,
+                         workspace: torch.Tensor | None = None, stream=None):
+    """Quantize-dequantize of a bf16 [rows, K] CUDA tensor under a candidate
+    set (mask of CAND_*) and block size (8, 16, 32, 64): returns (out
+    [rows, K] of out_dtype (float32 or bfloat16), choice uint8 [rows, K/block]
+    or None, tensor_scale)."""
+    assert x.dtype == torch.bfloat16 and x.dim() == 2 and x.stride(1) == 1
+    assert out_dtype in (torch.float32, torch.bfloat16)
+    rows, K = x.shape
+    o = out if out is not None else torch.empty(rows, K, dtype=out_dtype, device=x.device)
+    assert o.dtype == out_dtype and o.stride(1) == 1
+    ch = None
+    if want_choice:
+        ch = choice if choice is not None else torch.empty(rows, K // block if block else 0, dtype=torch.uint8,
+                                                           device=x.device)
+    ts = torch.empty(1, dtype=torch.float32, device=x.device)
+    given = tensor_scale is not None
+    if given:
+        ts.copy_(tensor_scale.reshape(1))
+    ws = None
+    if not given:
+        ws = workspace if workspace is not None else torch.empty(1, dtype=torch.int32, device=x.device)
+    st = lib().mixfp4_fake_quantize(_ptr(x), DTYPE_BF16, rows, K, x.stride(0), int(candidates), int(block),
+                                    _ptr(ts), _ptr(ws), SCALE_GIVEN if given else SCALE_COMPUTE, _ptr(o),
+                                    DTYPE_F32 if out_dtype == torch.float32 else DTYPE_BF16, o.stride(0),
+                                    _ptr(ch), _stream(stream))
+    _check("mixfp4_fake_quantize", st)
+    return o, ch, ts
 
 
 def mixfp4_dequantize(q: QTensor, out: torch.Tensor | None = None, stream=None) -> torch.Tensor:

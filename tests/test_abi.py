@@ -172,3 +172,27 @@ def test_colwise_rht_validation(lib):
     assert c(fake, 0, 128, 24, 24, None, fake, fake, fake, ws, 0, 0, None) == -2     # C % 16
     assert c(fake, 0, 128, 32, 32, None, fake, fake, fake, None, 0, 0, None) == -1   # workspace
     assert c(fake, 0, 0, 32, 32, None, None, None, fake, ws, 0, 1, None) == 0        # empty
+
+
+def test_fake_quantize_validation(lib):
+    fake = ctypes.c_void_p(1 << 20)
+    ws = ctypes.c_void_p(1 << 21)
+    f = lib.mixfp4_fake_quantize
+    #        x     dt rows K   ldx cand g   ts    ws  flag out  odt ldo ch    stream
+    assert f(fake, 7, 4, 64, 64, 15, 16, fake, ws, 0, fake, 1, 64, fake, None) == -4    # input dtype
+    assert f(fake, 0, 4, 64, 64, 15, 16, fake, ws, 0, fake, 5, 64, fake, None) == -4    # output dtype
+    assert f(fake, 0, 4, 64, 64, 0, 16, fake, ws, 0, fake, 1, 64, fake, None) == -7     # empty set
+    assert f(fake, 0, 4, 64, 64, 16, 16, fake, ws, 0, fake, 1, 64, fake, None) == -7    # unknown candidate
+    assert f(fake, 0, 4, 64, 64, 15, 12, fake, ws, 0, fake, 1, 64, fake, None) == -7    # block size
+    assert f(fake, 0, 4, 64, 64, 15, 16, fake, ws, 2, fake, 1, 64, fake, None) == -7    # scale flag
+    assert f(fake, 0, 4, 48, 48, 15, 32, fake, ws, 0, fake, 1, 48, fake, None) == -2    # K % g
+    assert f(fake, 0, 4, 24, 24, 15, 8, fake, ws, 0, fake, 1, 24, fake, None) == -2     # K % 16
+    assert f(fake, 0, 4, 64, 64, 15, 16, fake, ws, 0, fake, 1, 48, fake, None) == -2    # ldo < K
+    assert f(fake, 0, 4, 64, 64, 15, 16, None, ws, 0, fake, 1, 64, fake, None) == -1    # tensor scale
+    assert f(fake, 0, 4, 64, 64, 15, 16, fake, None, 0, fake, 1, 64, fake, None) == -1  # workspace
+    assert f(fake, 0, 4, 64, 64, 15, 16, fake, ws, 0, None, 1, 64, fake, None) == -1    # out
+    assert f(fake, 0, 4, 64, 64, 15, 16, fake, ws, 0, ctypes.c_void_p((1 << 20) + 16), 1, 64, fake,
+             None) == -3                                                                  # out alignment
+    assert f(fake, 0, 4, 64, 64, 15, 16, fake, ws, 0, fake, 1, 72, fake, None) == -3    # ldo % 16
+    assert f(fake, 0, 4, 64, 64, 15, 16, fake, ws, 0, fake, 1, 64, ctypes.c_void_p((1 << 20) + 1),
+             None) == -3                                                                  # choice alignment
