@@ -12,54 +12,115 @@
 // g = 8 thread carries two blocks; a g = 32 / 64 block spans 2 / 4 adjacent
 // lanes, which combine the block max and each candidate's error sum with xor
 // shuffles (lane i with i ^ 1, then i ^ 2: the pairwise tree of the 16-element
-// sums, the same on every lane because fp32 addition is commutative).  Every
-// division is the correctly rounded one (__fdiv_rn); the E4M3 scale and the
-// E2M1 codes come from the hardware conversions (round to nearest even,
-// saturating), E1M2 from rint, E3M0 from the exponent and mantissa bits.
+// sums, the same on every lane because fp32 addition is commutative).  The
+// divisions are the quantizer's (quant_core.cuh): x / s32, B / 6, B / 7 and
+// |a| / s8 in the checked two-instruction form on packed pairs (x / s32 with
+// Markstein's correction where the run-time check asks for it); B / 4 and
+// B / 16 are exact scalings.  The E4M3 scale and the E2M1 codes come from the
+// hardware conversions (round to nearest even, saturating), E1M2 from rint,
+// E3M0 from the exponent and mantissa bits.
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <cstdint>
 
 #include "kernels.cuh"
 #include "ptx.cuh"
+#include "quant_core.cuh"
 
 namespace mixfp4 {
 namespace {
 
 constexpr int kFqThreads = 256;
 
-// E4M3 value nearest to v >= 0 (ties to even, saturating at 448, subnormals).
-__device__ __forceinline__ float e4m3_round(float v) {
-  const uint32_t h2 = cvt_f16x2_from_e4m3x2(cvt_e4m3x2(0.0f, v));
-  float lo, hi;
-  f16x2_to_f32(h2, lo, hi);
-  return lo;
-}
-
-// E2M1 magnitude nearest to y >= 0 (ties to the even payload, saturating at 6).
-__device__ __forceinline__ float e2m1_round(float y) {
-  float lo, hi;
-  f16x2_to_f32(cvt_f16x2_from_e2m1x2(cvt_e2m1x2(0.0f, y)), lo, hi);
-  return lo;
-}
-
 // E3M0 magnitude nearest to y >= 0: 0 or 2^e, e = -2..4, ties to the even
-// payload (payload of 2^e is e + 3, so of the two neighbours the one whose
-// biased fp32 exponent is even).
+// payload.  The payload of 2^e is e + 3, so between 2^e and 2^(e+1) a tie
+// (mantissa exactly 1.5) goes up iff the biased fp32 exponent of 2^e is odd:
+// round up iff mantissa + (exponent bit 0) > 2^22.  Then 16 caps the top;
+// below 1/4 the neighbours are 0 and 1/4, with the tie 1/8 going to 0.
 __device__ __forceinline__ float e3m0_round(float y) {
-  if (y >= 16.0f) return 16.0f;
-  if (y < 0.25f) return y > 0.125f ? 0.25f : 0.0f;  // 1/8 is a tie between payloads 0 and 1
   const uint32_t u = __float_as_uint(y);
-  const uint32_t ebits = u & 0x7F800000u, m = u & 0x007FFFFFu;
-  const float lo = __uint_as_float(ebits);
-  const bool up = m > 0x00400000u || (m == 0x00400000u && ((ebits >> 23) & 1u));
-  return up ? 2.0f * lo : lo;
+  const bool up = (u & 0x007FFFFFu) + ((u >> 23) & 1u) > 0x00400000u;
+  const float p2 = fminf(__uint_as_float((u & 0x7F800000u) + (up ? 0x00800000u : 0u)), 16.0f);
+  return y > 0.125f ? fmaxf(p2, 0.25f) : 0.0f;
 }
 
-__device__ __forceinline__ float cand_round(int c, float y) {
-  if (c == 1) return fminf(rintf(y), 7.0f);
-  if (c == 3) return e3m0_round(y);
-  return e2m1_round(y);  // c = 0, 2
+// One candidate of a block part: s8 from the block max, codes of the pairs
+// a[j0 .. j0 + kPairs - 1], their values q (packed, in candidate units) and
+// the error sum (even elements in the low lane chain, odd in the high).
+template <int kPairs>
+__device__ __forceinline__ void candidate_part(int c, const u64* a, float B, const TensorConsts& tc,
+                                               const float4* __restrict__ tab, u64* q, float& s8, float& se,
+                                               float& so) {
+  float bd;  // fl32(B / divisor): 6 and 7 by the checked two-instruction form, 4 and 16 exactly
+  if (c == 0) bd = __fmaf_rn(B, tc.kd6.x, __fmul_rn(B, tc.kd6.y));
+  else if (c == 1) bd = __fmaf_rn(B, tc.kd7.x, __fmul_rn(B, tc.kd7.y));
+  else if (c == 2) bd = __fmul_rn(B, 0.25f);
+  else bd = __fmul_rn(B, 0.0625f);
+  const float4 t = tab[cvt_e4m3x2(0.0f, bd) & 0x7Fu];  // R2: E4M3 RNE, saturating
+  s8 = t.x;
+  const u64 zh8 = pack2(t.y, t.y), zl8 = pack2(t.z, t.z), ns8 = pack2(-t.x, -t.x);
+  u64 acc = 0;
+#pragma unroll
+  for (int j = 0; j < kPairs; ++j) {
+    float ylo, yhi, qlo, qhi;
+    unpack2(div_kd2(a[j], zh8, zl8), ylo, yhi);  // fl32(|a| / s8); s8 = 0 gives 0
+    if (c == 1) {
+      qlo = fminf(rintf(ylo), 7.0f);
+      qhi = fminf(rintf(yhi), 7.0f);
+    } else if (c == 3) {
+      qlo = e3m0_round(ylo);
+      qhi = e3m0_round(yhi);
+    } else {
+      f16x2_to_f32(cvt_f16x2_from_e2m1x2(cvt_e2m1x2(yhi, ylo)), qlo, qhi);
+    }
+    q[j] = pack2(qlo, qhi);
+    const u64 d = fma2(q[j], ns8, a[j]);  // |a| - q s8, the product exact
+    acc = fma2(d, d, acc);
+  }
+  unpack2(acc, se, so);
+}
+
+template <int kG>
+__device__ __forceinline__ void fake_quantize_unit(const u64 a[8], const TensorConsts& tc, float s32,
+                                                   const float4* __restrict__ tab, int mask, float o[16],
+                                                   int best_c[2]) {
+  constexpr int kParts = kG == 8 ? 2 : 1;  // blocks per thread
+  constexpr int kPairs = 8 / kParts;      // element pairs of a block held by one thread
+#pragma unroll
+  for (int p = 0; p < kParts; ++p) {
+    float v[2 * kPairs];
+#pragma unroll
+    for (int j = 0; j < kPairs; ++j) unpack2(a[p * kPairs + j], v[2 * j], v[2 * j + 1]);
+    float B = 0.0f;
+#pragma unroll
+    for (int i = 0; i < 2 * kPairs; ++i) B = fmaxf(B, v[i]);
+    if (kG >= 32) B = fmaxf(B, __shfl_xor_sync(0xffffffffu, B, 1));
+    if (kG == 64) B = fmaxf(B, __shfl_xor_sync(0xffffffffu, B, 2));
+    float best_S = 0.0f, best_s8 = 0.0f;
+    u64 qb[kPairs];
+    best_c[p] = -1;
+#pragma unroll
+    for (int c = 0; c < 4; ++c) {
+      if (!((mask >> c) & 1)) continue;  // uniform over the launch
+      u64 q[kPairs];
+      float s8, se, so;
+      candidate_part<kPairs>(c, a + p * kPairs, B, tc, tab, q, s8, se, so);
+      float S = __fadd_rn(se, so);
+      if (kG >= 32) S = __fadd_rn(S, __shfl_xor_sync(0xffffffffu, S, 1));
+      if (kG == 64) S = __fadd_rn(S, __shfl_xor_sync(0xffffffffu, S, 2));
+      if (best_c[p] < 0 || S <= best_S) {  // a later candidate wins a tie
+        best_c[p] = c;
+        best_S = S;
+        best_s8 = s8;
+#pragma unroll
+        for (int j = 0; j < kPairs; ++j) qb[j] = q[j];
+      }
+    }
+    const u64 s8s = pack2(best_s8, best_s8), s32s = pack2(s32, s32);
+#pragma unroll
+    for (int j = 0; j < kPairs; ++j) unpack2(mul2(mul2(qb[j], s8s), s32s), o[2 * (p * kPairs + j)],
+                                             o[2 * (p * kPairs + j) + 1]);
+  }
 }
 
 template <int kG>
@@ -67,17 +128,13 @@ __global__ void __launch_bounds__(kFqThreads)
 fake_quantize_kernel(const uint16_t* __restrict__ x, int64_t rows, int64_t K, int64_t ldx, int mask,
                      float* tensor_scale, const uint32_t* amax_word, int scale_given, void* __restrict__ out,
                      int out_bf16, int64_t ldo, uint8_t* __restrict__ choice) {
-  constexpr int kParts = kG == 8 ? 2 : 1;  // blocks per thread
-  constexpr int kLen = 16 / kParts;       // elements of a block held by one thread
+  __shared__ float4 tab[128];  // E4M3 code -> {s8, zh, zl, 0}
   griddep_wait();
   griddep_launch_dependents();
-  float s32;
-  if (scale_given) {
-    s32 = *tensor_scale;
-  } else {
-    s32 = __fdiv_rn(__uint_as_float(*amax_word), 2688.0f);  // 6 * 448
-    if (blockIdx.x == 0 && threadIdx.x == 0) *tensor_scale = s32;
-  }
+  fill_scale_table(tab);
+  const TensorConsts tc = tensor_consts(tensor_scale, amax_word, scale_given);
+  const bool markstein = markstein_needed(tc);  // ends with a CTA barrier (tab is ready)
+  const float s32 = tc.scaled ? scalbnf(tc.s32, -tc.k) : tc.s32;  // the tensor's own s32 (exact)
   const int lane = threadIdx.x & 31;
   const int64_t kb = K / 16, nsub = rows * kb;
   const int64_t warp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
@@ -94,93 +151,36 @@ fake_quantize_kernel(const uint16_t* __restrict__ x, int64_t rows, int64_t K, in
 #pragma unroll
       for (int i = 0; i < 8; ++i) w[i] = 0u;
     }
-    float a[16];
-    uint32_t neg = 0u;
-#pragma unroll
-    for (int i = 0; i < 8; ++i) {
-      const float lo = __uint_as_float(w[i] << 16), hi = __uint_as_float(w[i] & 0xFFFF0000u);
-      neg |= ((w[i] >> 15) & 1u) << (2 * i);
-      neg |= (w[i] >> 31) << (2 * i + 1);
-      a[2 * i] = s32 > 0.0f ? __fdiv_rn(fabsf(lo), s32) : 0.0f;      // R1, R7
-      a[2 * i + 1] = s32 > 0.0f ? __fdiv_rn(fabsf(hi), s32) : 0.0f;
-    }
-    float B[kParts];
-#pragma unroll
-    for (int p = 0; p < kParts; ++p) {
-      B[p] = 0.0f;
-#pragma unroll
-      for (int i = 0; i < kLen; ++i) B[p] = fmaxf(B[p], a[p * kLen + i]);
-      if (kG >= 32) B[p] = fmaxf(B[p], __shfl_xor_sync(0xffffffffu, B[p], 1));
-      if (kG == 64) B[p] = fmaxf(B[p], __shfl_xor_sync(0xffffffffu, B[p], 2));
-    }
-    float best_S[kParts], best_s8[kParts], q_best[16];
-    int best_c[kParts];
-#pragma unroll
-    for (int p = 0; p < kParts; ++p) {
-      best_S[p] = 0.0f;
-      best_s8[p] = 0.0f;
-      best_c[p] = -1;
-    }
-#pragma unroll
-    for (int i = 0; i < 16; ++i) q_best[i] = 0.0f;
-#pragma unroll
-    for (int c = 0; c < 4; ++c) {
-      if (!((mask >> c) & 1)) continue;  // uniform over the launch
-      const float div = c == 0 ? 6.0f : c == 1 ? 7.0f : c == 2 ? 4.0f : 16.0f;
-#pragma unroll
-      for (int p = 0; p < kParts; ++p) {
-        const float s8 = e4m3_round(__fdiv_rn(B[p], div));  // R2
-        float q[kLen], se = 0.0f, so = 0.0f;
-#pragma unroll
-        for (int i = 0; i < kLen; ++i) {
-          const float y = s8 > 0.0f ? __fdiv_rn(a[p * kLen + i], s8) : 0.0f;
-          q[i] = cand_round(c, y);
-          const float d = __fmaf_rn(q[i], s8, -a[p * kLen + i]);  // q s8 is exact
-          if (i & 1) so = __fmaf_rn(d, d, so);
-          else se = __fmaf_rn(d, d, se);
-        }
-        float S = __fadd_rn(se, so);
-        if (kG >= 32) S = __fadd_rn(S, __shfl_xor_sync(0xffffffffu, S, 1));
-        if (kG == 64) S = __fadd_rn(S, __shfl_xor_sync(0xffffffffu, S, 2));
-        if (best_c[p] < 0 || S <= best_S[p]) {  // a later candidate wins a tie
-          best_c[p] = c;
-          best_S[p] = S;
-          best_s8[p] = s8;
-#pragma unroll
-          for (int i = 0; i < kLen; ++i) q_best[p * kLen + i] = q[i];
-        }
-      }
-    }
+    float o[16];
+    int best_c[2] = {0, 0};
+    u64 a[8];  // |X_FP8| pairs (R1, R7)
+    if (tc.scaled) x_fp8_magnitudes<true, true>(w, tc, a);
+    else if (markstein) x_fp8_magnitudes<false, true>(w, tc, a);
+    else x_fp8_magnitudes<false, false>(w, tc, a);
+    fake_quantize_unit<kG>(a, tc, s32, tab, mask, o, best_c);
     if (live) {
-      float o[16];
+      uint32_t ow[16];
 #pragma unroll
-      for (int i = 0; i < 16; ++i) {
-        const float v = __fmul_rn(__fmul_rn(q_best[i], best_s8[i / kLen]), s32);
-        o[i] = ((neg >> i) & 1u) ? -v : v;
+      for (int i = 0; i < 8; ++i) {  // sign(x) on the magnitudes
+        ow[2 * i] = __float_as_uint(o[2 * i]) | ((w[i] & 0x8000u) << 16);
+        ow[2 * i + 1] = __float_as_uint(o[2 * i + 1]) | (w[i] & 0x80000000u);
       }
       if (out_bf16) {
-        uint32_t ow[8];
+        uint32_t hw[8];
 #pragma unroll
         for (int i = 0; i < 8; ++i) {
-          const uint32_t lo = __bfloat16_as_ushort(__float2bfloat16_rn(o[2 * i]));
-          const uint32_t hi = __bfloat16_as_ushort(__float2bfloat16_rn(o[2 * i + 1]));
-          ow[i] = lo | (hi << 16);
+          const __nv_bfloat162 h = __floats2bfloat162_rn(__uint_as_float(ow[2 * i]), __uint_as_float(ow[2 * i + 1]));
+          hw[i] = *reinterpret_cast<const uint32_t*>(&h);  // low half: element 2i
         }
-        stg256(static_cast<uint16_t*>(out) + r * ldo + j * 16, ow);
+        stg256(static_cast<uint16_t*>(out) + r * ldo + j * 16, hw);
       } else {
         float* dst = static_cast<float*>(out) + r * ldo + j * 16;
-#pragma unroll
-        for (int h = 0; h < 2; ++h) {
-          uint32_t ow[8];
-#pragma unroll
-          for (int i = 0; i < 8; ++i) ow[i] = __float_as_uint(o[8 * h + i]);
-          stg256(dst + 8 * h, ow);
-        }
+        stg256(dst, ow);
+        stg256(dst + 8, ow + 8);
       }
       if (choice) {
         if (kG == 8) {
-          *reinterpret_cast<uint16_t*>(choice + r * (K / 8) + 2 * j) =
-              (uint16_t)(best_c[0] | (best_c[kParts - 1] << 8));
+          *reinterpret_cast<uint16_t*>(choice + r * (K / 8) + 2 * j) = (uint16_t)(best_c[0] | (best_c[1] << 8));
         } else if (kG == 16) {
           choice[r * kb + j] = (uint8_t)best_c[0];
         } else if ((lane & (kG / 16 - 1)) == 0) {

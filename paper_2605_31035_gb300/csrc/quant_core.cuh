@@ -96,6 +96,25 @@ __device__ __forceinline__ uint32_t sign_bits(uint32_t w0, uint32_t w1, uint32_t
   return (odd & 0x80808080u) | ((even >> 4) & 0x08080808u);
 }
 
+// |X_FP8| = |x| / s32 of 16 bf16 elements held as 8 pairs, as packed fp32
+// pairs (element 2j in the low lane); kScaled / kMarkstein as described at
+// the top of quantize.cu.
+template <bool kScaled, bool kMarkstein>
+__device__ __forceinline__ void x_fp8_magnitudes(const uint32_t w[8], const TensorConsts& tc, u64 a[8]) {
+  const u64 ns32 = pack2(-tc.s32, -tc.s32), r32 = pack2(tc.r32, tc.r32);
+  const u64 zh32 = pack2(tc.kd32.x, tc.kd32.x), zl32 = pack2(tc.kd32.y, tc.kd32.y);
+#pragma unroll
+  for (int j = 0; j < 8; ++j) {
+    const uint32_t u = w[j] & 0x7FFF7FFFu;
+    uint32_t lo = u << 16, hi = u & 0xFFFF0000u;
+    if (kScaled) {
+      lo = __float_as_uint(scalbnf(__uint_as_float(lo), tc.k));
+      hi = __float_as_uint(scalbnf(__uint_as_float(hi), tc.k));
+    }
+    a[j] = kMarkstein ? div_rn2(bits2(lo, hi), ns32, r32) : div_kd2(bits2(lo, hi), zh32, zl32);
+  }
+}
+
 // Algorithm 1 for one 16-element block held as 8 bf16 pairs.
 //
 // Tiny-value note: with s32 in [2^-20, 2^100], an element with |x| < 2^-102
@@ -141,21 +160,8 @@ template <int kMode, bool kScaled, bool kMarkstein, bool kTile = false>
 __device__ __forceinline__ void quantize_block(const uint32_t w[8], const TensorConsts& tc,
                                                const float4* __restrict__ tab, uint32_t& code_lo,
                                                uint32_t& code_hi, uint32_t& scale_byte) {
-  // |x| as packed fp32 pairs (element 2j in the low lane).
   u64 a[8];
-  const u64 ns32 = pack2(-tc.s32, -tc.s32), r32 = pack2(tc.r32, tc.r32);
-  const u64 zh32 = pack2(tc.kd32.x, tc.kd32.x), zl32 = pack2(tc.kd32.y, tc.kd32.y);
-#pragma unroll
-  for (int j = 0; j < 8; ++j) {
-    const uint32_t u = w[j] & 0x7FFF7FFFu;
-    uint32_t lo = u << 16, hi = u & 0xFFFF0000u;
-    if (kScaled) {
-      lo = __float_as_uint(scalbnf(__uint_as_float(lo), tc.k));
-      hi = __float_as_uint(scalbnf(__uint_as_float(hi), tc.k));
-    }
-    // X_FP8 = X / s32 (magnitudes)
-    a[j] = kMarkstein ? div_rn2(bits2(lo, hi), ns32, r32) : div_kd2(bits2(lo, hi), zh32, zl32);
-  }
+  x_fp8_magnitudes<kScaled, kMarkstein>(w, tc, a);
   uint32_t mlo, mhi;
   block_core<kMode, kTile>(a, tc, tab, mlo, mhi, scale_byte);
   code_lo = mlo | sign_bits(w[0], w[1], w[2], w[3]);
