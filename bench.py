@@ -399,7 +399,8 @@ def run_ours(args):
                 "stochastic_rounding_given_scale": {
                     "ms": round(sr_ms, 4), "alg_gbs": round(xs_numel * QUANT_BYTES_PER_ELEM / (sr_ms * 1e-3) / 1e9, 1)},
                 "transpose_2d": {"ms": round(transpose_ms, 4),
-                                 "alg_gbs": round(xs_numel * 2 * (0.5 + 1.0 / 16) / (transpose_ms * 1e-3) / 1e9, 1)}},
+                                 "alg_gbs": round(xs_numel * TRANSPOSE_BYTES_PER_ELEM / (transpose_ms * 1e-3) / 1e9, 1),
+                                 "alg_bytes_per_element": TRANSPOSE_BYTES_PER_ELEM}},
             "candidate_ablation_2^28": {
                 **ablation,
                 "alg_bytes_per_element": "2 (bf16 in) + 2 (bf16 out) + 1/g (choice)",
@@ -596,6 +597,10 @@ def run_reference(args):
     print(json.dumps(out), flush=True)
 
 
+# 2D transpose: codes in and out (0.5 + 0.5), one scale byte read per 16 x 16
+# tile (the tile's rows repeat it) and one written per 16 elements of each
+# output row.
+TRANSPOSE_BYTES_PER_ELEM = 0.5 + 0.5 + 1.0 / 256 + 1.0 / 16
 # (name, candidate mask, block size) of the ablation lines.
 FQ_SETS = [("mixfp4", 1 | 2, 16), ("four_over_six", 1 | 4, 16), ("e2_e1_e3", 1 | 2 | 8, 16),
            ("all_four", 15, 16), ("e2_e1_e3", 1 | 2 | 8, 64), ("all_four", 15, 8)]
@@ -649,7 +654,7 @@ def run_kernel_only(args):
     elif args.kernel == "transpose_2d":
         q2 = ops.mixfp4_quantize_2d(x, workspace=ws)
         fn = lambda: ops.mixfp4_transpose_2d(q2)
-        work = x.numel() * 2 * (0.5 + 1.0 / 16)
+        work = x.numel() * TRANSPOSE_BYTES_PER_ELEM
     elif args.kernel == "fake_quantize":
         fo = torch.empty(x.shape, dtype=torch.bfloat16, device=dev)
         fn = lambda: ops.mixfp4_fake_quantize(x, 15, 16, torch.bfloat16, out=fo, workspace=ws)
