@@ -22,6 +22,7 @@ import argparse
 import hashlib
 import json
 import os
+import platform
 import statistics
 import subprocess
 import sys
@@ -551,6 +552,20 @@ def _calibrated_rows(layer: OracleLayer, n_rows_x: int, budget_s: float, cap: in
     return max(8, min(cap, int(16 * budget_s / (max(secs, 1e-4) * n_rows_x))))
 
 
+def host_cpu() -> dict:
+    """The host the oracle runs on: logical CPUs and the CPU model string."""
+    model = platform.processor() or platform.machine()
+    try:
+        for line in open("/proc/cpuinfo"):
+            key = line.split(":")[0].strip().lower()
+            if key in ("model name", "cpu model", "hardware"):
+                model = line.split(":", 1)[1].strip()
+                break
+    except OSError:
+        pass
+    return {"nproc": os.cpu_count(), "cpu": model, "arch": platform.machine()}
+
+
 def cpu_baseline(lin, x_cpu, budget_s: float = 15.0):
     cap = 2048
     layer = OracleLayer(lin, x_cpu, lin.make_w()[:cap], cap)
@@ -561,7 +576,8 @@ def cpu_baseline(lin, x_cpu, budget_s: float = 15.0):
     secs, flops = layer.run(n_x, n_w)
     return {"value": flops / secs / 1e12, "unit": "TFLOP/s", "cores": 1, "kind": "oracle",
             "sample": f"Algorithm 1 on {n_x} rows of X + float64 GEMM vs {n_w} pre-quantized rows of W "
-                      f"(K={lin.K}), {secs:.1f} s single-threaded"}
+                      f"(K={lin.K}), {secs:.1f} s single-threaded",
+            "host": host_cpu()}
 
 
 def run_reference(args):
@@ -591,7 +607,8 @@ def run_reference(args):
                       "M": lin.M, "N": lin.N, "K": lin.K, "mode": "MixFP4"},
            "cpu_baseline": {"value": value, "unit": "TFLOP/s", "cores": 1, "kind": "oracle",
                             "sample": f"per step: Algorithm 1 on 1 row of X + float64 GEMM vs {n_w} "
-                                      f"pre-quantized rows of W (K={lin.K}), single-threaded"},
+                                      f"pre-quantized rows of W (K={lin.K}), single-threaded",
+                            "host": host_cpu()},
            "gpu_launches": 0,
            "e2e": {"value": value, "unit": "TFLOP/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(out), flush=True)
