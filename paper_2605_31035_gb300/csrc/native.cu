@@ -57,25 +57,27 @@ namespace {
 using namespace sm100;
 
 // ---------------------------------------------------------------- operand split
-// E2M1 codes of the split of an E1M2 payload p (nibble p of each constant).
-constexpr uint32_t kMainOfE1M2 = 0x77665420u;  // e(p): 0,1,2,3,4,4,6,6 -> codes 0,2,4,5,6,6,7,7
-constexpr uint32_t kResOfE1M2 = 0x20200000u;   // r(p): 1 for p = 5, 7 -> code 2
-
-__device__ __forceinline__ void split_word(uint32_t w, bool e1m2, uint32_t& main, uint32_t& res) {
-  if (!e1m2) {
-    main = w;
-    res = 0;
-    return;
-  }
-  main = 0;
-  res = 0;
-#pragma unroll
-  for (int i = 0; i < 8; ++i) {
-    const uint32_t n = (w >> (4 * i)) & 0xFu, p = n & 7u, s = n & 8u;
-    main |= (s | ((kMainOfE1M2 >> (4 * p)) & 0xFu)) << (4 * i);
-    res |= (s | ((kResOfE1M2 >> (4 * p)) & 0xFu)) << (4 * i);
-  }
+// The E2M1 main and residual parts of eight E1M2 nibbles (sign in bit 3 of
+// each, payload p in bits 0-2): main payload bits m0 = p1 (p0 | p2),
+// m1 = p2 | (p0 ~p1), m2 = p2 | p1 (the codes of 0,1,2,3,4,4,6,6), residual
+// payload 2 where p0 p2 (p = 5, 7); both keep the sign bit.  Each line is one
+// three-input logic instruction (lop3; truth-table byte from a = 0xF0,
+// b = 0xCC, c = 0xAA).
+#define MIXFP4_LOP3(d, a, b, c, LUT) asm("lop3.b32 %0, %1, %2, %3, " #LUT ";" : "=r"(d) : "r"(a), "r"(b), "r"(c))
+__device__ __forceinline__ void split_e1m2_word(uint32_t w, uint32_t tmask, uint32_t& main, uint32_t& res) {
+  const uint32_t r1 = w >> 1, r2 = w >> 2, l1 = w << 1;
+  uint32_t m0, m1, t, r;
+  MIXFP4_LOP3(m0, r1, w, r2, 0xE0);                  // p1 & (p0 | p2)          at bit 4i
+  MIXFP4_LOP3(m1, r1, l1, w, 0xF4);                  // p2 | (p0 & ~p1)         at bit 4i+1
+  MIXFP4_LOP3(t, m0, m1, 0x22222222u, 0xD8);         // bit 4i+1 from m1
+  MIXFP4_LOP3(t, t, w | l1, 0x44444444u, 0xD8);      // bit 4i+2: p2 | p1
+  MIXFP4_LOP3(t, t, w, 0x88888888u, 0xD8);           // bit 4i+3: the sign
+  MIXFP4_LOP3(r, l1, r1, 0x22222222u, 0x80);         // p0 & p2                 at bit 4i+1
+  MIXFP4_LOP3(r, r, w, 0x88888888u, 0xF8);           // | the sign
+  MIXFP4_LOP3(main, t, w, tmask, 0xE4);              // tmask ? main : w  (per bit: (a & c) | (b & ~c))
+  res = r & tmask;                                    // E2M1 blocks have no residual
 }
+#undef MIXFP4_LOP3
 
 // Threads [0, n_code) split 32 elements (two blocks, 16 code bytes) each;
 // threads [n_code, n_code + n_sf) write one 16-byte line of the scale tiles
@@ -92,11 +94,12 @@ __global__ void __launch_bounds__(256) split_native_kernel(const uint8_t* __rest
       const int64_t r = i / (K / 32), c = i % (K / 32);  // row, 32-element chunk
       const uint4 w = *reinterpret_cast<const uint4*>(codes + r * (K / 2) + c * 16);
       const uint8_t s0 = scales[r * nb + 2 * c], s1 = scales[r * nb + 2 * c + 1];
+      const uint32_t k0 = (s0 & 0x80u) ? 0xFFFFFFFFu : 0u, k1 = (s1 & 0x80u) ? 0xFFFFFFFFu : 0u;
       uint4 m, q;
-      split_word(w.x, s0 >> 7, m.x, q.x);
-      split_word(w.y, s0 >> 7, m.y, q.y);
-      split_word(w.z, s1 >> 7, m.z, q.z);
-      split_word(w.w, s1 >> 7, m.w, q.w);
+      split_e1m2_word(w.x, k0, m.x, q.x);
+      split_e1m2_word(w.y, k0, m.y, q.y);
+      split_e1m2_word(w.z, k1, m.z, q.z);
+      split_e1m2_word(w.w, k1, m.w, q.w);
       *reinterpret_cast<uint4*>(main_codes + r * (K / 2) + c * 16) = m;
       *reinterpret_cast<uint4*>(res_codes + r * (K / 2) + c * 16) = q;
     } else {
@@ -534,27 +537,6 @@ struct Bars {
 };
 static_assert(sizeof(Bars) <= 256, "barrier block");
 
-// The E2M1 main and residual parts of eight E1M2 nibbles (sign in bit 3 of
-// each, payload p in bits 0-2): main payload bits m0 = p1 (p0 | p2),
-// m1 = p2 | (p0 ~p1), m2 = p2 | p1 (the codes of 0,1,2,3,4,4,6,6), residual
-// payload 2 where p0 p2 (p = 5, 7); both keep the sign bit.  Each line is one
-// three-input logic instruction (lop3; truth-table byte from a = 0xF0,
-// b = 0xCC, c = 0xAA).
-#define MIXFP4_LOP3(d, a, b, c, LUT) asm("lop3.b32 %0, %1, %2, %3, " #LUT ";" : "=r"(d) : "r"(a), "r"(b), "r"(c))
-__device__ __forceinline__ void split_e1m2_word(uint32_t w, uint32_t tmask, uint32_t& main, uint32_t& res) {
-  const uint32_t r1 = w >> 1, r2 = w >> 2, l1 = w << 1;
-  uint32_t m0, m1, t, r;
-  MIXFP4_LOP3(m0, r1, w, r2, 0xE0);                  // p1 & (p0 | p2)          at bit 4i
-  MIXFP4_LOP3(m1, r1, l1, w, 0xF4);                  // p2 | (p0 & ~p1)         at bit 4i+1
-  MIXFP4_LOP3(t, m0, m1, 0x22222222u, 0xD8);         // bit 4i+1 from m1
-  MIXFP4_LOP3(t, t, w | l1, 0x44444444u, 0xD8);      // bit 4i+2: p2 | p1
-  MIXFP4_LOP3(t, t, w, 0x88888888u, 0xD8);           // bit 4i+3: the sign
-  MIXFP4_LOP3(r, l1, r1, 0x22222222u, 0x80);         // p0 & p2                 at bit 4i+1
-  MIXFP4_LOP3(r, r, w, 0x88888888u, 0xF8);           // | the sign
-  MIXFP4_LOP3(main, t, w, tmask, 0xE4);              // tmask ? main : w  (per bit: (a & c) | (b & ~c))
-  res = r & tmask;                                    // E2M1 blocks have no residual
-}
-#undef MIXFP4_LOP3
 
 // Split one 16-byte chunk (two blocks) given the blocks' type bits.
 __device__ __forceinline__ void split_chunk(uint4 c, bool t0, bool t1, uint4& m, uint4& r) {
