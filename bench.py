@@ -150,6 +150,12 @@ def reduce_max(value: float, device) -> float:
     return float(t.item())
 
 
+def job_rate(work_per_rank: float, world: int, max_ms: float) -> float:
+    """Whole-job rate of N independent replicas: the work every rank did,
+    divided by the slowest rank's time (ms), per second."""
+    return world * work_per_rank / (max_ms * 1e-3)
+
+
 def barrier():
     import torch.distributed as dist
     if dist.is_available() and dist.is_initialized():
@@ -206,7 +212,7 @@ def run_ours(args):
     gemm_ms = [e[1].elapsed_time(e[2]) for e in ev]
     total_ms = reduce_max(sum(step_ms), dev)
     ms_per_step = total_ms / args.steps
-    value = world * args.steps * flops / (total_ms * 1e-3) / 1e12
+    value = job_rate(args.steps * flops, world, total_ms) / 1e12
     gemm_avg = statistics.mean(gemm_ms)
     gemm_tflops = flops / (gemm_avg * 1e-3) / 1e12
     quant_avg = statistics.mean(quant_ms)
@@ -348,7 +354,7 @@ def run_ours(args):
     e1.record(s_in)
     torch.cuda.synchronize(dev)
     e2e_ms = reduce_max(e0.elapsed_time(e1), dev)
-    e2e_value = world * e2e_steps * flops / (e2e_ms * 1e-3) / 1e12
+    e2e_value = job_rate(e2e_steps * flops, world, e2e_ms) / 1e12
 
     configs = None if args.no_configs else config_gemms(dev, flush, stream, pk["bf16_tflops"])
 
