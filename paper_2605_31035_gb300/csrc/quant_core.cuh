@@ -287,21 +287,22 @@ __device__ __forceinline__ uint4 philox4x32_10(uint4 c, uint32_t k0, uint32_t k1
 
 // Stochastic payloads of a magnitude m = |a| / s8 (exact fp32 arithmetic
 // throughout): with l <= m < u the codebook neighbours, u iff eps < (m - l) /
-// (u - l); m at or above the largest value saturates.
+// (u - l); m at or above the largest value saturates.  Branch-free (lanes of
+// a warp hold blocks of either type and any magnitude): every gap u - l is a
+// power of two (E2M1: 1/2 below 2, 1 below 4, 2 below 6; E1M2: 1), so
+// v = m / (u - l) is an exact scaling, l's position is floor(v), and
+// (m - l) / (u - l) = v - floor(v) exactly.
 __device__ __forceinline__ uint32_t sr_payload_e1m2(float m, float eps) {
-  if (!(m < 7.0f)) return 7u;
   const float l = floorf(m);
-  return (uint32_t)l + (eps < m - l ? 1u : 0u);
+  const uint32_t p = (uint32_t)l + (eps < m - l ? 1u : 0u);
+  return m < 7.0f ? p : 7u;
 }
 __device__ __forceinline__ uint32_t sr_payload_e2m1(float m, float eps) {
-  if (!(m < 6.0f)) return 7u;                                   // 6
-  if (m >= 4.0f) return 6u + (eps < (m - 4.0f) * 0.5f ? 1u : 0u);  // 4 or 6
-  if (m >= 2.0f) {
-    const float l = floorf(m);                                  // 2 or 3: payloads 4, 5
-    return (uint32_t)l + 2u + (eps < m - l ? 1u : 0u);
-  }
-  const float u = m * 2.0f, l = floorf(u);                      // 0, .5, 1, 1.5: payloads 0..3
-  return (uint32_t)l + (eps < u - l ? 1u : 0u);
+  const float v = m * (m < 2.0f ? 2.0f : (m < 4.0f ? 1.0f : 0.5f));
+  const float fl = floorf(v);
+  // payload of l: 2 v below 2 (0..3), v + 2 below 4 (4, 5), 6 below 6 (v = 2)
+  const uint32_t p = (uint32_t)fl + (m >= 2.0f ? 2u : 0u) + (m >= 4.0f ? 2u : 0u) + (eps < v - fl ? 1u : 0u);
+  return m < 6.0f ? p : 7u;
 }
 
 // Algorithm 1 for one block (format and scale exactly as quantize_block
@@ -347,8 +348,9 @@ __device__ __forceinline__ void quantize_block_sr(const uint32_t w[8], const Ten
       unpack2(div_kd2(a[j], zh8, zl8), mlo, mhi);  // fl32(|a| / s8), as Algorithm 1's quotient
       const float elo = __uint2float_rn(rw[2 * h] >> 8) * 0x1p-24f;
       const float ehi = __uint2float_rn(rw[2 * h + 1] >> 8) * 0x1p-24f;
-      const uint32_t plo = e1m2 ? sr_payload_e1m2(mlo, elo) : sr_payload_e2m1(mlo, elo);
-      const uint32_t phi = e1m2 ? sr_payload_e1m2(mhi, ehi) : sr_payload_e2m1(mhi, ehi);
+      const uint32_t p1lo = sr_payload_e1m2(mlo, elo), p2lo = sr_payload_e2m1(mlo, elo);  // both, then
+      const uint32_t p1hi = sr_payload_e1m2(mhi, ehi), p2hi = sr_payload_e2m1(mhi, ehi);  // a select
+      const uint32_t plo = e1m2 ? p1lo : p2lo, phi = e1m2 ? p1hi : p2hi;
       bytes[j] = plo | (phi << 4);
     }
   }
