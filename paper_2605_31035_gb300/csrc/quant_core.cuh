@@ -292,17 +292,15 @@ __device__ __forceinline__ uint4 philox4x32_10(uint4 c, uint32_t k0, uint32_t k1
 // power of two (E2M1: 1/2 below 2, 1 below 4, 2 below 6; E1M2: 1), so
 // v = m / (u - l) is an exact scaling, l's position is floor(v), and
 // (m - l) / (u - l) = v - floor(v) exactly.
-__device__ __forceinline__ uint32_t sr_payload_e1m2(float m, float eps) {
-  const float l = floorf(m);
-  const uint32_t p = (uint32_t)l + (eps < m - l ? 1u : 0u);
-  return m < 7.0f ? p : 7u;
-}
-__device__ __forceinline__ uint32_t sr_payload_e2m1(float m, float eps) {
-  const float v = m * (m < 2.0f ? 2.0f : (m < 4.0f ? 1.0f : 0.5f));
-  const float fl = floorf(v);
-  // payload of l: 2 v below 2 (0..3), v + 2 below 4 (4, 5), 6 below 6 (v = 2)
-  const uint32_t p = (uint32_t)fl + (m >= 2.0f ? 2u : 0u) + (m >= 4.0f ? 2u : 0u) + (eps < v - fl ? 1u : 0u);
-  return m < 6.0f ? p : 7u;
+// One routine for both formats, its constants chosen per lane: E1M2 has gap
+// 1 everywhere and saturates at 7; E2M1 as described, saturating at 6.
+__device__ __forceinline__ uint32_t sr_payload(bool e1m2, float m, float eps) {
+  const float sc = e1m2 ? 1.0f : (m < 2.0f ? 2.0f : (m < 4.0f ? 1.0f : 0.5f));
+  // payload of l: E1M2 floor(m); E2M1 2 m below 2 (0..3), m + 2 below 4 (4, 5), 6 below 6
+  const uint32_t add = e1m2 ? 0u : (m >= 2.0f ? 2u : 0u) + (m >= 4.0f ? 2u : 0u);
+  const float v = m * sc, fl = floorf(v);
+  const uint32_t p = (uint32_t)fl + add + (eps < v - fl ? 1u : 0u);
+  return m < (e1m2 ? 7.0f : 6.0f) ? p : 7u;
 }
 
 // Algorithm 1 for one block (format and scale exactly as quantize_block
@@ -348,9 +346,7 @@ __device__ __forceinline__ void quantize_block_sr(const uint32_t w[8], const Ten
       unpack2(div_kd2(a[j], zh8, zl8), mlo, mhi);  // fl32(|a| / s8), as Algorithm 1's quotient
       const float elo = __uint2float_rn(rw[2 * h] >> 8) * 0x1p-24f;
       const float ehi = __uint2float_rn(rw[2 * h + 1] >> 8) * 0x1p-24f;
-      const uint32_t p1lo = sr_payload_e1m2(mlo, elo), p2lo = sr_payload_e2m1(mlo, elo);  // both, then
-      const uint32_t p1hi = sr_payload_e1m2(mhi, ehi), p2hi = sr_payload_e2m1(mhi, ehi);  // a select
-      const uint32_t plo = e1m2 ? p1lo : p2lo, phi = e1m2 ? p1hi : p2hi;
+      const uint32_t plo = sr_payload(e1m2, mlo, elo), phi = sr_payload(e1m2, mhi, ehi);
       bytes[j] = plo | (phi << 4);
     }
   }
