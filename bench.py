@@ -678,6 +678,14 @@ def run_kernel_only(args):
         q2 = ops.mixfp4_quantize_2d(x, workspace=ws)
         fn = lambda: ops.mixfp4_transpose_2d(q2)
         work = x.numel() * TRANSPOSE_BYTES_PER_ELEM
+    elif args.kernel == "quantize_colwise_rht":
+        qc = ops.mixfp4_quantize_colwise_rht(x, workspace=ws)   # its s32, then the quantize pass alone
+        ts = qc.tensor_scale.clone()
+        fn = lambda: ops.mixfp4_quantize_colwise_rht(x, out=qc, tensor_scale=ts)
+        work = x.numel() * QUANT_BYTES_PER_ELEM
+    elif args.kernel == "quantize_sr":
+        fn = lambda: ops.mixfp4_quantize_sr(x, 1234, 0, out=qx, workspace=ws)
+        work = x.numel() * QUANT_BYTES_PER_ELEM
     elif args.kernel == "fake_quantize":
         fo = torch.empty(x.shape, dtype=torch.bfloat16, device=dev)
         fn = lambda: ops.mixfp4_fake_quantize(x, 15, 16, torch.bfloat16, out=fo, workspace=ws)
@@ -716,7 +724,8 @@ def main(argv=None):
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-configs", action="store_true", help="skip the other configs' GEMM lines")
     ap.add_argument("--kernel", choices=["gemm", "gemm_native", "gemm_native_fewrows", "split_native", "quantize", "quantize_rht", "quantize_colwise",
-                             "quantize_2d", "transpose_2d", "fake_quantize", "dequantize"], default=None,
+                             "quantize_2d", "transpose_2d", "fake_quantize", "quantize_colwise_rht", "quantize_sr",
+                             "dequantize"], default=None,
                     help="profiling mode: launch only this kernel")
     ap.add_argument("--workload", default=WORKLOAD,
                     help="tiny|attn|mlp|decode|hadamard|sweepNN (kernel-only mode)")
