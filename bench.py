@@ -291,7 +291,7 @@ def run_ours(args):
     fq_ch = torch.empty(xs.shape[0], xs.shape[1] // 8, dtype=torch.uint8, device=dev)
     ablation = {}
     for name, mask, g in FQ_SETS:
-        chv = fq_ch[:, : xs.shape[1] // g]
+        chv = fq_ch.view(-1)[: xs.shape[0] * (xs.shape[1] // g)].view(xs.shape[0], xs.shape[1] // g)
         ms_ = time_quant(lambda: ops.mixfp4_fake_quantize(xs, mask, g, torch.bfloat16, tensor_scale=given,
                                                           out=fq_out, choice=chv))
         gbs = xs.numel() * (4.0 + 1.0 / g) / (ms_ * 1e-3) / 1e9

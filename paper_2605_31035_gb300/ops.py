@@ -278,6 +278,8 @@ def mixfp4_fake_quantize(x: torch.Tensor, candidates: int, block: int = 16, out_
     if want_choice:
         ch = choice if choice is not None else torch.empty(rows, K // block if block else 0, dtype=torch.uint8,
                                                            device=x.device)
+        assert ch.dtype == torch.uint8 and ch.is_contiguous() and ch.numel() == rows * (K // block), \
+            "choice must be a dense uint8 [rows, K / block] tensor"
     ts = torch.empty(1, dtype=torch.float32, device=x.device)
     given = tensor_scale is not None
     if given:
