@@ -50,7 +50,7 @@
  *                      reading R14
  *   oracle_f32_to_bf16 binary32 -> bfloat16, round to nearest even
  *
- * Readings where the paper is silent (the same list is kept in the design doc):
+ * Readings where the paper is silent (binding on the CUDA path as well):
  *   R1 X_FP8 = fl32(X / s32) is an fp32 value (no FP8 cast).
  *   R2 s8 = E4M3_RNE(fl32(blockmax / c)), c = 6 (E2M1) or 7 (E1M2): two
  *      roundings, E4M3 with subnormals, saturating at 448.
