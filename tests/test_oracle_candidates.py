@@ -231,3 +231,26 @@ def test_rejects_bad_arguments():
     for mask, g in [(0, 16), (16, 16), (1, 12), (1, 32)]:
         with pytest.raises(ValueError):
             oracle.fake_quantize(x, mask, g)
+
+
+def test_block_size_trends_of_sec5():
+    """Sec. 5 (Table 5 and its discussion): with coarser blocks the E1M2
+    candidate helps less, and E3M0 becomes the more useful extra format.  A
+    statistical trend on the synthetic stand-ins (not parity): the MSE ratio
+    of {E2M1, E1M2} to NVFP4 rises with g for activations and weights, and on
+    the outlier-heavy activations {E2M1, E3M0} gains on {E2M1, E1M2} from
+    g = 8 to g = 64."""
+    tensors = {"act": synth.activations(128, 4096, 5, 6), "w": synth.weights(128, 4096, 7, 0.02, 0.5)}
+    ratio = {}
+    for name, x in tensors.items():
+        xb, xf = synth.bf16_bits(x), x.float().numpy().astype(np.float64)
+        for g in (8, 16, 32, 64):
+            mse = {}
+            for mask in (1, 1 | 2, 1 | 8):
+                o, _, _ = oracle.fake_quantize(xb, mask, g)
+                mse[mask] = np.mean((o.astype(np.float64) - xf) ** 2)
+            ratio[name, g] = (mse[1 | 2] / mse[1], mse[1 | 8] / mse[1 | 2])
+    for name in tensors:
+        e1 = [ratio[name, g][0] for g in (8, 16, 32, 64)]
+        assert all(a < b for a, b in zip(e1, e1[1:])) and e1[-1] < 1.0, (name, e1)
+    assert ratio["act", 64][1] < ratio["act", 8][1] < 1.0
