@@ -558,17 +558,22 @@ def _calibrated_rows(layer: OracleLayer, n_rows_x: int, budget_s: float, cap: in
     return max(8, min(cap, int(16 * budget_s / (max(secs, 1e-4) * n_rows_x))))
 
 
-def host_cpu() -> dict:
-    """The host the oracle runs on: logical CPUs and the CPU model string."""
+def host_cpu(cpuinfo: str = "/proc/cpuinfo") -> dict:
+    """The host the oracle runs on: logical CPUs and the CPU model (the model
+    name where the kernel reports one, else the Arm implementer / part codes)."""
     model = platform.processor() or platform.machine()
+    fields = {}
     try:
-        for line in open("/proc/cpuinfo"):
-            key = line.split(":")[0].strip().lower()
-            if key in ("model name", "cpu model", "hardware"):
-                model = line.split(":", 1)[1].strip()
-                break
+        for line in open(cpuinfo):
+            if ":" in line:
+                key, val = line.split(":", 1)
+                fields.setdefault(key.strip().lower(), val.strip())
     except OSError:
         pass
+    if fields.get("model name"):
+        model = fields["model name"]
+    elif fields.get("cpu part"):
+        model = f"implementer {fields.get('cpu implementer', '?')} part {fields['cpu part']}"
     return {"nproc": os.cpu_count(), "cpu": model, "arch": platform.machine()}
 
 
