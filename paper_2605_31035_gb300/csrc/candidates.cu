@@ -179,12 +179,11 @@ fake_quantize_kernel(const uint16_t* __restrict__ x, int64_t rows, int64_t K, in
         stg256(dst + 8, ow + 8);
       }
       if (choice) {
-        if (kG == 8) {
+        constexpr int kLanes = kG >= 16 ? kG / 16 : 1;  // lanes sharing one block
+        if constexpr (kG == 8) {
           *reinterpret_cast<uint16_t*>(choice + r * (K / 8) + 2 * j) = (uint16_t)(best_c[0] | (best_c[1] << 8));
-        } else if (kG == 16) {
-          choice[r * kb + j] = (uint8_t)best_c[0];
-        } else if ((lane & (kG / 16 - 1)) == 0) {
-          choice[r * (K / kG) + j / (kG / 16)] = (uint8_t)best_c[0];
+        } else if ((lane & (kLanes - 1)) == 0) {
+          choice[r * (K / kG) + j / kLanes] = (uint8_t)best_c[0];
         }
       }
     }

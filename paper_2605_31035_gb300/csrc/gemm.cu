@@ -824,13 +824,9 @@ int launch_pair(const uint8_t* a_codes, const uint8_t* a_scales, const float* a_
       !make_map(&tas, a_scales, (uint64_t)K / 16, (uint64_t)M, BKC / 16, BM, CU_TENSOR_MAP_SWIZZLE_NONE) ||
       !make_map(&tbs, b_scales, (uint64_t)K / 16, (uint64_t)N, BKC / 16, kTileN / 2, CU_TENSOR_MAP_SWIZZLE_NONE))
     return MIXFP4_ERR_CUDA;
-  static bool attr_set = false;
-  if (!attr_set) {
-    if (cudaFuncSetAttribute(mixfp4_gemm_kernel<kTileN>, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_ALLOC) !=
-        cudaSuccess)
-      return MIXFP4_ERR_CUDA;
-    attr_set = true;
-  }
+  static std::atomic<uint64_t> smem_set{0};
+  if (!set_dynamic_smem_once(reinterpret_cast<const void*>(mixfp4_gemm_kernel<kTileN>), SMEM_ALLOC, smem_set))
+    return MIXFP4_ERR_CUDA;
   const int64_t ntiles_n = (N + kTileN - 1) / kTileN;
   if (dp_tiles < tiles) {
     // Zero C from the first stream-K tile's row band down (tile t: mt = t / ntiles_n,
@@ -869,13 +865,10 @@ int launch_gemm(const uint8_t* a_codes, const uint8_t* a_scales, const float* a_
         !make_map(&tws, b_scales, (uint64_t)K / 16, (uint64_t)N, BKC / 16, skinny::BN, CU_TENSOR_MAP_SWIZZLE_NONE) ||
         !make_map(&txs, a_scales, (uint64_t)K / 16, (uint64_t)M, BKC / 16, nx, CU_TENSOR_MAP_SWIZZLE_NONE))
       return MIXFP4_ERR_CUDA;
-    static bool skinny_attr = false;
-    if (!skinny_attr) {
-      if (cudaFuncSetAttribute(skinny::mixfp4_gemm_skinny_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                               skinny::SMEM_ALLOC) != cudaSuccess)
-        return MIXFP4_ERR_CUDA;
-      skinny_attr = true;
-    }
+    static std::atomic<uint64_t> skinny_smem_set{0};
+    if (!set_dynamic_smem_once(reinterpret_cast<const void*>(skinny::mixfp4_gemm_skinny_kernel), skinny::SMEM_ALLOC,
+                               skinny_smem_set))
+      return MIXFP4_ERR_CUDA;
     if (cudaMemset2DAsync(C, (size_t)ldc * sizeof(float), 0, (size_t)N * sizeof(float), (size_t)M, stream) !=
         cudaSuccess)
       return MIXFP4_ERR_CUDA;

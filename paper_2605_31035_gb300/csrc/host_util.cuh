@@ -1,9 +1,11 @@
 // Host helpers shared by the GEMM launchers: the driver's tensor-map encoder
-// (resolved once through the runtime) and the device's SM count.
+// (resolved once through the runtime), the current device's SM count, and the
+// once-per-device setting of a kernel's dynamic shared memory limit.
 #pragma once
 #include <cuda.h>
 #include <cudaTypedefs.h>
 #include <cuda_runtime.h>
+#include <atomic>
 #include <cstdint>
 
 namespace mixfp4 {
@@ -35,15 +37,35 @@ inline bool make_map(CUtensorMap* m, const void* base, uint64_t row_bytes, uint6
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+constexpr int kMaxDevices = 64;  // devices tracked by the per-device caches below
+
+inline int current_device() {
+  int d = 0;
+  if (cudaGetDevice(&d) != cudaSuccess || d < 0 || d >= kMaxDevices) d = 0;
+  return d;
+}
+
+// SM count of the current device (cached per device).
 inline int num_sms() {
-  static int n = 0;
-  if (!n) {
-    int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess ||
-        cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0)
-      n = 148;
+  static std::atomic<int> n[kMaxDevices];
+  const int d = current_device();
+  int v = n[d].load(std::memory_order_relaxed);
+  if (v <= 0) {
+    if (cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, d) != cudaSuccess || v <= 0) v = 148;
+    n[d].store(v, std::memory_order_relaxed);
   }
-  return n;
+  return v;
+}
+
+// Raise `kernel`'s dynamic shared memory limit to `bytes` on the current
+// device, once per device: `done` is the call site's bit mask of devices
+// already set (function attributes belong to a device's context).
+inline bool set_dynamic_smem_once(const void* kernel, int bytes, std::atomic<uint64_t>& done) {
+  const uint64_t bit = 1ull << current_device();
+  if (done.load(std::memory_order_acquire) & bit) return true;
+  if (cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes) != cudaSuccess) return false;
+  done.fetch_or(bit, std::memory_order_release);
+  return true;
 }
 
 }  // namespace mixfp4

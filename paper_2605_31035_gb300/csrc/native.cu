@@ -426,13 +426,9 @@ int launch(const uint8_t* a_main, const uint8_t* a_res, const uint8_t* a_sf, con
       !make_map(&tar, kARes ? a_res : a_main, (uint64_t)K / 2, (uint64_t)M, ROW_BYTES, BM, swz) ||
       !make_map(&tbr, kBRes ? b_res : b_main, (uint64_t)K / 2, (uint64_t)N, ROW_BYTES, BM, swz))
     return MIXFP4_ERR_CUDA;
-  static bool attr_set = false;
-  if (!attr_set) {
-    if (cudaFuncSetAttribute(nvf4_gemm_kernel<kARes, kBRes>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             L::SMEM_ALLOC) != cudaSuccess)
-      return MIXFP4_ERR_CUDA;
-    attr_set = true;
-  }
+  static std::atomic<uint64_t> smem_set{0};
+  if (!set_dynamic_smem_once(reinterpret_cast<const void*>(nvf4_gemm_kernel<kARes, kBRes>), L::SMEM_ALLOC, smem_set))
+    return MIXFP4_ERR_CUDA;
   const int64_t mtiles = (M + TILE_M - 1) / TILE_M, ntiles_n = (N + TILE_N - 1) / TILE_N;
   const int64_t tiles = mtiles * ntiles_n, num_kc = K / BKC;
   int64_t clusters = num_sms() / 2;
@@ -845,13 +841,9 @@ int launch(const uint8_t* a_codes, const uint8_t* a_scales, const float* a_ts, c
       !make_map(&txs, a_scales, (uint64_t)K / 16, (uint64_t)M, 16, (uint32_t)nx, CU_TENSOR_MAP_SWIZZLE_NONE))
     return MIXFP4_ERR_CUDA;
   const int smem = OFF_RINGS + code_stages(nx) * code_stage_bytes(nx) + kSplitStages * SPLIT_STAGE + 1024;
-  static bool attr_set = false;
-  if (!attr_set) {
-    if (cudaFuncSetAttribute(nvf4_fewrows_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, 232448) !=
-        cudaSuccess)
-      return MIXFP4_ERR_CUDA;
-    attr_set = true;
-  }
+  static std::atomic<uint64_t> smem_set{0};
+  if (!set_dynamic_smem_once(reinterpret_cast<const void*>(nvf4_fewrows_kernel), 232448, smem_set))
+    return MIXFP4_ERR_CUDA;
   cudaError_t e;
   if (ldc == N)
     e = cudaMemsetAsync(C, 0, (size_t)M * (size_t)N * sizeof(float), stream);
