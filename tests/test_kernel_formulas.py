@@ -9,6 +9,7 @@ pin the derivations the kernels rely on.
 * branch-free E3M0 rounding (candidate-set ablation, reading R14)
 * the stochastic-rounding payload shared by both formats (reading R13)
 * the 16 x 16 nibble transpose in registers (2D transpose)
+* the decode of a code word to f16 operands in the GEMM (reading R8)
 """
 import numpy as np
 import pytest
@@ -148,3 +149,40 @@ def test_register_nibble_transpose_is_the_transpose():
             for r in range(16):
                 w = L[c] if r < 8 else H[c]
                 assert (w >> (4 * (r % 8))) & 0xF == M[r, c]
+
+
+# gemm.cu decode8: f16 high bytes of u = 2 v by payload, E2M1 and E1M2.
+LUT = {0: (0x42403C00, 0x4A484644), 1: (0x46444000, 0x4B4A4948)}
+
+
+def decode8_kernel(w: int, t: int):
+    """gemm.cu decode8 before the scale multiply: the eight f16 bit patterns
+    of a code word, element 2j from the low nibble of byte j."""
+    lo, hi = LUT[t]
+    wp = w & 0x77777777
+    ws = (w * 16) & M32
+    u0 = prmt(lo, hi, wp & 0xFFFF)
+    u1 = prmt(lo, hi, (wp >> 16) & 0xFFFF)          # __umulhi(wp, 0x10000)
+    g0 = prmt(w, ws, 0x1504)
+    g1 = prmt(w, ws, 0x3726)
+    v0 = u0 | (g0 & 0x80808080)
+    v1 = u1 | (g1 & 0x80808080)
+    words = [prmt(v0, 0, 0x1404), prmt(v0, 0, 0x3424), prmt(v1, 0, 0x1404), prmt(v1, 0, 0x3424)]
+    return [(x >> (16 * h)) & 0xFFFF for x in words for h in (0, 1)]
+
+
+@pytest.mark.parametrize("t", [0, 1])
+def test_gemm_decode_gives_the_exact_f16_of_twice_each_value(oracle, t):
+    """Every nibble in every position decodes to the f16 of 2 v with the
+    nibble's sign (negative zero for 0x8), v the oracle's magnitude of the
+    payload (the E2M1 value, or the E1M2 payload in x2 units, R3); the GEMM
+    epilogue removes the factor 4 that the two doubled operands carry."""
+    for pos in range(8):
+        for nib in range(16):
+            w = (nib << (4 * pos)) | (((nib * 7 + 3) & 15) << (4 * ((pos + 5) % 8)))
+            got = decode8_kernel(w, t)
+            for e in range(8):
+                n = (w >> (4 * e)) & 0xF
+                v = 2.0 * oracle.fp4_value(t, n & 7)
+                want = np.float16(-v if n & 8 else v)
+                assert got[e] == int(want.view(np.uint16)), (hex(w), t, e)
