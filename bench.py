@@ -240,6 +240,7 @@ def run_ours(args):
         return statistics.median(a.elapsed_time(b) for a, b in evs)
 
     given_ms = time_quant(lambda: ops.mixfp4_quantize(xs, out=qs, tensor_scale=given))
+    four_six_ms = time_quant(lambda: ops.mixfp4_quantize(xs, ops.MODE_FOUR_SIX, out=qs, tensor_scale=given))
     sweep_ms = time_quant(lambda: ops.mixfp4_quantize(xs, out=qs, workspace=ws))
     ops.mixfp4_quantize_rht(xs, out=qs, workspace=ws)
     given_rht = qs.tensor_scale.clone()
@@ -388,6 +389,9 @@ def run_ours(args):
                 "with_amax_pass": {"ms": round(sweep_ms, 4), "alg_gbs": round(sweep_alg_gbs, 1),
                                    "alg_frac_of_hbm": round(sweep_alg_gbs / pk["hbm_gbs"], 4),
                                    "bytes_incl_amax_read_gbs": round(sweep_read_gbs, 1)},
+                "four_over_six_mode_given_scale": {
+                    "ms": round(four_six_ms, 4),
+                    "alg_gbs": round(xs_numel * QUANT_BYTES_PER_ELEM / (four_six_ms * 1e-3) / 1e9, 1)},
                 "alg_bytes_per_element": QUANT_BYTES_PER_ELEM, "hbm_peak_gbs": pk["hbm_gbs"]},
             "native_fp4_variant": {
                 "gemm_native_ms": round(native_gemm_ms, 5),

@@ -48,7 +48,11 @@ typedef enum {
 
 enum { MIXFP4_MODE_MIX = 0,        /* Alg. 1: per-block E2M1/E1M2 by lower MSE */
        MIXFP4_MODE_E2M1_ONLY = 1,  /* every block E2M1, T = 0 (plain NVFP4 bits) */
-       MIXFP4_MODE_E1M2_ONLY = 2   /* every block E1M2, T = 1 (NVINT4 lattice) */ };
+       MIXFP4_MODE_E1M2_ONLY = 2,  /* every block E1M2, T = 1 (NVINT4 lattice) */
+       MIXFP4_MODE_FOUR_SIX = 3    /* the {E2M1(6), E2M1(4)} candidate set of Sec. 2.3 ("4/6"):
+                                      per block the lower-MSE of s8 from B/6 or B/4 (B/4 on a
+                                      tie), E2M1 codes, T = 0 (plain NVFP4 bits, so both GEMMs
+                                      take it); mixfp4_quantize and mixfp4_quantize_noalloc only */ };
 
 enum { MIXFP4_SCALE_COMPUTE = 0,   /* compute s32 = fl32(max|x| / 2688), write *tensor_scale */
        MIXFP4_SCALE_GIVEN = 1      /* read s32 from *tensor_scale */ };

@@ -37,7 +37,7 @@ int mixfp4_quantize(const void* x, int dtype, int64_t rows, int64_t K, int64_t l
                     uint8_t* codes, uint8_t* scales, float* tensor_scale, uint32_t* workspace,
                     int mode, int scale_flag, void* stream) {
   if (dtype != MIXFP4_DTYPE_BF16) return MIXFP4_ERR_DTYPE;
-  if (mode < MIXFP4_MODE_MIX || mode > MIXFP4_MODE_E1M2_ONLY) return MIXFP4_ERR_ARG;
+  if (mode < MIXFP4_MODE_MIX || mode > MIXFP4_MODE_FOUR_SIX) return MIXFP4_ERR_ARG;
   if (scale_flag != MIXFP4_SCALE_COMPUTE && scale_flag != MIXFP4_SCALE_GIVEN) return MIXFP4_ERR_ARG;
   if (rows < 0 || K < 0 || K % 16 != 0 || ldx < K) return MIXFP4_ERR_SHAPE;
   if (!tensor_scale) return MIXFP4_ERR_NULL;

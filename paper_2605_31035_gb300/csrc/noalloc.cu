@@ -64,7 +64,7 @@ extern "C" int mixfp4_quantize_noalloc(const void* x, int dtype, int64_t rows, i
                                        int64_t ldx, uint8_t* codes, uint8_t* scales,
                                        float* tensor_scale, int mode, void* stream) {
   if (dtype != MIXFP4_DTYPE_BF16) return MIXFP4_ERR_DTYPE;
-  if (mode < MIXFP4_MODE_MIX || mode > MIXFP4_MODE_E1M2_ONLY) return MIXFP4_ERR_ARG;
+  if (mode < MIXFP4_MODE_MIX || mode > MIXFP4_MODE_FOUR_SIX) return MIXFP4_ERR_ARG;
   if (rows < 0 || K < 0 || K % 16 != 0 || ldx < K) return MIXFP4_ERR_SHAPE;
   if (kAmaxWords > kNoAllocScratchWords) return MIXFP4_ERR_SHAPE;
   if (!tensor_scale) return MIXFP4_ERR_NULL;

@@ -168,6 +168,45 @@ __device__ __forceinline__ void quantize_block(const uint32_t w[8], const Tensor
   code_hi = mhi | sign_bits(w[4], w[5], w[6], w[7]);
 }
 
+// One E2M1 candidate of a block with scale table entry t = {s8, zh, zl}:
+// the payload bytes (element 2j low) packed into two words and, with kErr,
+// the R5 error sum (even / odd chains in the two lanes of a packed pair).
+template <bool kErr, bool kTile>
+__device__ __forceinline__ void e2m1_candidate(const u64 a[8], const float4 t, uint32_t& p_lo, uint32_t& p_hi,
+                                               float& S) {
+  const u64 zh8 = pack2(t.y, t.y), zl8 = pack2(t.z, t.z);
+  const uint16_t ns8h = __half_as_ushort(__float2half_rn(-t.x));  // exact: E4M3 values are f16 values
+  u64 acc = 0;  // (+0, +0): even / odd chains
+  uint32_t e[8];
+#pragma unroll
+  for (int j = 0; j < 8; ++j) {
+    const u64 y = div_kd2(a[j], zh8, zl8);
+    float ylo, yhi;
+    unpack2(y, ylo, yhi);
+    uint32_t h2;
+    e[j] = e2m1_pair(ylo, yhi, h2);
+    if (kErr) {
+      float alo, ahi, dlo, dhi;
+      unpack2(a[j], alo, ahi);
+      // d = |a| - q s8 (exact), with q taken straight from its f16 decode
+      asm("{ .reg .f16 ql, qh; mov.b32 {ql, qh}, %2;\n"
+          " fma.rn.f32.f16 %0, ql, %3, %4;\n fma.rn.f32.f16 %1, qh, %3, %5; }"
+          : "=f"(dlo), "=f"(dhi) : "r"(h2), "h"(ns8h), "f"(alo), "f"(ahi));
+      const u64 d = pack2(dlo, dhi);
+      acc = fma2(d, d, acc);
+    }
+  }
+  p_lo = pack_low_bytes(e[0], e[1], e[2], e[3]);
+  p_hi = pack_low_bytes(e[4], e[5], e[6], e[7]);
+  S = 0.0f;
+  if (kErr) {
+    float se, so;
+    unpack2(acc, se, so);
+    S = se + so;
+    if (kTile) S = tile_tree16(S);
+  }
+}
+
 template <int kMode, bool kTile>
 __device__ __forceinline__ void block_core(const u64 a[8], const TensorConsts& tc, const float4* __restrict__ tab,
                                            uint32_t& mag_lo, uint32_t& mag_hi, uint32_t& scale_byte) {
@@ -183,45 +222,31 @@ __device__ __forceinline__ void block_core(const u64 a[8], const TensorConsts& t
   const u64 bq = div_kd2(pack2(B, B), pack2(tc.kd6.x, tc.kd7.x), pack2(tc.kd6.y, tc.kd7.y));
   float b6, b7;
   unpack2(bq, b6, b7);
+
+  if (kMode == MIXFP4_MODE_FOUR_SIX) {
+    // {E2M1(6), E2M1(4)} (Sec. 2.3, reading R14): the second scale from
+    // fl32(B/4) = B/4 exactly; both candidates are E2M1 (T = 0) and the later
+    // one, E2M1(4), wins a tie.
+    const uint32_t sc = cvt_e4m3x2(__fmul_rn(B, 0.25f), b6);  // low byte: B/6 code, high: B/4
+    const uint32_t c6 = sc & 0x7Fu, c4 = (sc >> 8) & 0x7Fu;
+    uint32_t p6lo, p6hi, p4lo, p4hi;
+    float S6, S4;
+    e2m1_candidate<true, kTile>(a, tab[c6], p6lo, p6hi, S6);
+    e2m1_candidate<true, kTile>(a, tab[c4], p4lo, p4hi, S4);
+    const bool four = S4 <= S6;
+    mag_lo = four ? p4lo : p6lo;
+    mag_hi = four ? p4hi : p6hi;
+    scale_byte = four ? c4 : c6;
+    return;
+  }
+
   const uint32_t sc = cvt_e4m3x2(b7, b6);  // low byte: E2M1 scale code, high: E1M2
   const uint32_t c2 = sc & 0x7Fu, c1 = (sc >> 8) & 0x7Fu;
 
   float S2 = 0.0f, S1 = 0.0f;
   uint32_t p2lo = 0, p2hi = 0, p1lo = 0, p1hi = 0;
-  if (kMode != MIXFP4_MODE_E1M2_ONLY) {
-    // E2M1 candidate.
-    const float4 t = tab[c2];
-    const u64 zh8 = pack2(t.y, t.y), zl8 = pack2(t.z, t.z);
-    const uint16_t ns8h = __half_as_ushort(__float2half_rn(-t.x));  // exact: E4M3 values are f16 values
-    u64 acc = 0;  // (+0, +0): even / odd chains
-    uint32_t e[8];
-#pragma unroll
-    for (int j = 0; j < 8; ++j) {
-      const u64 y = div_kd2(a[j], zh8, zl8);
-      float ylo, yhi;
-      unpack2(y, ylo, yhi);
-      uint32_t h2;
-      e[j] = e2m1_pair(ylo, yhi, h2);
-      if (kMode == MIXFP4_MODE_MIX) {
-        float alo, ahi, dlo, dhi;
-        unpack2(a[j], alo, ahi);
-        // d = |a| - q s8 (exact), with q taken straight from its f16 decode
-        asm("{ .reg .f16 ql, qh; mov.b32 {ql, qh}, %2;\n"
-            " fma.rn.f32.f16 %0, ql, %3, %4;\n fma.rn.f32.f16 %1, qh, %3, %5; }"
-            : "=f"(dlo), "=f"(dhi) : "r"(h2), "h"(ns8h), "f"(alo), "f"(ahi));
-        const u64 d = pack2(dlo, dhi);
-        acc = fma2(d, d, acc);
-      }
-    }
-    p2lo = pack_low_bytes(e[0], e[1], e[2], e[3]);
-    p2hi = pack_low_bytes(e[4], e[5], e[6], e[7]);
-    if (kMode == MIXFP4_MODE_MIX) {
-      float se, so;
-      unpack2(acc, se, so);
-      S2 = se + so;
-      if (kTile) S2 = tile_tree16(S2);
-    }
-  }
+  if (kMode != MIXFP4_MODE_E1M2_ONLY)
+    e2m1_candidate<kMode == MIXFP4_MODE_MIX, kTile>(a, tab[c2], p2lo, p2hi, S2);
   if (kMode != MIXFP4_MODE_E2M1_ONLY) {
     // E1M2 candidate (x2 units: integers 0..7).
     const float4 t = tab[c1];

@@ -265,6 +265,7 @@ int launch_quantize(const uint16_t* x, int64_t rows, int64_t K, int64_t ldx, uin
   switch (mode) {
     case MIXFP4_MODE_MIX: MIXFP4_LAUNCH_Q(MIXFP4_MODE_MIX); break;
     case MIXFP4_MODE_E2M1_ONLY: MIXFP4_LAUNCH_Q(MIXFP4_MODE_E2M1_ONLY); break;
+    case MIXFP4_MODE_FOUR_SIX: MIXFP4_LAUNCH_Q(MIXFP4_MODE_FOUR_SIX); break;
     default: MIXFP4_LAUNCH_Q(MIXFP4_MODE_E1M2_ONLY); break;
   }
 #undef MIXFP4_LAUNCH_Q

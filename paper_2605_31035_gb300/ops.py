@@ -12,7 +12,7 @@ from dataclasses import dataclass
 
 import torch
 
-MODE_MIX, MODE_E2M1_ONLY, MODE_E1M2_ONLY = 0, 1, 2
+MODE_MIX, MODE_E2M1_ONLY, MODE_E1M2_ONLY, MODE_FOUR_SIX = 0, 1, 2, 3
 SCALE_COMPUTE, SCALE_GIVEN = 0, 1
 DTYPE_BF16, DTYPE_F32 = 0, 1
 # Candidates of mixfp4_fake_quantize, bit c of the mask.

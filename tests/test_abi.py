@@ -45,7 +45,7 @@ def test_quantize_validation(lib):
     assert q(fake, 0, 4, 24, 24, fake, fake, fake, ws, 0, 0, None) == -2        # K % 16
     assert q(fake, 0, 4, 32, 16, fake, fake, fake, ws, 0, 0, None) == -2        # ldx < K
     assert q(fake, 0, -1, 32, 32, fake, fake, fake, ws, 0, 0, None) == -2       # rows < 0
-    assert q(fake, 0, 4, 32, 32, fake, fake, fake, ws, 3, 0, None) == -7        # mode
+    assert q(fake, 0, 4, 32, 32, fake, fake, fake, ws, 4, 0, None) == -7        # mode
     assert q(fake, 0, 4, 32, 32, fake, fake, fake, ws, 0, 2, None) == -7        # scale flag
     assert q(None, 0, 4, 32, 32, fake, fake, fake, ws, 0, 0, None) == -1        # x null
     assert q(fake, 0, 4, 32, 32, fake, fake, fake, None, 0, 0, None) == -1      # workspace
@@ -196,3 +196,12 @@ def test_fake_quantize_validation(lib):
     assert f(fake, 0, 4, 64, 64, 15, 16, fake, ws, 0, fake, 1, 72, fake, None) == -3    # ldo % 16
     assert f(fake, 0, 4, 64, 64, 15, 16, fake, ws, 0, fake, 1, 64, ctypes.c_void_p((1 << 20) + 1),
              None) == -3                                                                  # choice alignment
+
+
+def test_four_six_mode_only_where_declared(lib):
+    fake = ctypes.c_void_p(1 << 20)
+    ws = ctypes.c_void_p(1 << 21)
+    assert lib.mixfp4_quantize(fake, 0, 4, 32, 32, fake, fake, fake, ws, 4, 0, None) == -7   # past FOUR_SIX
+    assert lib.mixfp4_quantize_colwise(fake, 0, 32, 32, 32, fake, fake, fake, ws, 3, 0, None) == -7
+    assert lib.mixfp4_quantize_2d(fake, 0, 32, 32, 32, fake, fake, fake, ws, 3, 0, None) == -7
+    assert lib.mixfp4_quantize_noalloc(fake, 0, 4, 32, 32, fake, fake, fake, 4, None) == -7

@@ -117,3 +117,50 @@ def test_full_size_sampled_rows(oracle):
         ref, rch, _ = oracle.fake_quantize(synth.bf16_bits(x[rows]), ALL, g, s32)
         assert np.array_equal(y[rows].cpu().numpy().view(np.uint32), ref.view(np.uint32))
         assert np.array_equal(ch[rows].cpu().numpy(), rch)
+
+
+@pytest.mark.parametrize("shape", [(1, 16), (40, 512), (37, 272)])
+@pytest.mark.parametrize("given", [False, True])
+def test_four_six_mode_packs_the_46_candidate_set(oracle, shape, given):
+    """MIXFP4_MODE_FOUR_SIX: the codes the GPU stores decode (oracle
+    dequantizer) to exactly the oracle's {E2M1(6), E2M1(4)} quantize-dequantize
+    at g = 16, every type bit is 0, and each scale byte is E4M3 of B/6 or B/4
+    as the oracle chose."""
+    o = ops()
+    rows, K = shape
+    x = synth.activations(rows, K, 7500 + rows + K, 7501)
+    bits = synth.bf16_bits(x)
+    s32 = float(np.float32(0.0173)) if given else None
+    ts = None if s32 is None else torch.tensor([s32], device=DEV)
+    q = o.mixfp4_quantize(x.to(DEV), o.MODE_FOUR_SIX, tensor_scale=ts)
+    torch.cuda.synchronize()
+    codes, scales, t = q.codes.cpu().numpy(), q.scales.cpu().numpy(), float(q.tensor_scale.item())
+    ref, choice, rs = oracle.fake_quantize(bits, 1 | 4, 16, s32)
+    assert np.float32(t).view(np.uint32) == np.float32(rs).view(np.uint32)
+    assert not np.any(scales & 0x80)
+    deq = oracle.dequantize(codes, scales, t)
+    assert np.array_equal(deq.view(np.uint32), ref.view(np.uint32))
+    xf = (bits.astype(np.uint32) << 16).view(np.float32)
+    a = (np.abs(xf) / np.float32(rs)).astype(np.float32) if rs > 0 else np.zeros_like(xf)
+    B = a.reshape(rows, K // 16, 16).max(axis=2)
+    div = np.where(choice == 2, np.float32(4.0), np.float32(6.0))
+    want = np.vectorize(lambda v: oracle.e4m3_rne(float(v)))((B / div).astype(np.float32))
+    assert np.array_equal(scales, want.astype(np.uint8))
+
+
+def test_four_six_operands_in_both_gemms(oracle):
+    """4/6 operands are plain NVFP4 bits: the decode-path GEMM and the native
+    variant (one E2M1 product) take them, within the 1e-5 bound."""
+    o = ops()
+    X = synth.activations(256, 512, 7600, 7601)
+    W = synth.weights(384, 512, 7602, 0.02, 0.5)
+    qx, qw = o.mixfp4_quantize(X.to(DEV), o.MODE_FOUR_SIX), o.mixfp4_quantize(W.to(DEV), o.MODE_FOUR_SIX)
+    C1 = o.mixfp4_gemm(qx, qw)
+    C2 = o.mixfp4_gemm_native(o.mixfp4_split_native(qx), o.mixfp4_split_native(qw))
+    torch.cuda.synchronize()
+    ra = (qx.codes.cpu().numpy(), qx.scales.cpu().numpy(), float(qx.tensor_scale.item()))
+    rb = (qw.codes.cpu().numpy(), qw.scales.cpu().numpy(), float(qw.tensor_scale.item()))
+    Cref = oracle.gemm_f64(ra, rb)
+    D = np.abs(oracle.dequant_rows_f64(*ra, range(256))) @ np.abs(oracle.dequant_rows_f64(*rb, range(384))).T
+    for C in (C1, C2):
+        assert np.all(np.abs(C.cpu().numpy().astype(np.float64) - Cref) <= 1e-5 * D)
