@@ -39,7 +39,7 @@ _HERE = os.path.dirname(os.path.abspath(__file__))
 _SRC = os.path.join(_HERE, "mixfp4_oracle.c")
 _LIB = os.path.join(_HERE, "liboracle.so")
 
-MODE_MIX, MODE_E2M1_ONLY, MODE_E1M2_ONLY = 0, 1, 2
+MODE_MIX, MODE_E2M1_ONLY, MODE_E1M2_ONLY, MODE_FOUR_SIX = 0, 1, 2, 3
 # Candidates of the ablation quantizer (reading R14), bit c of a candidate mask.
 CAND_E2M1_6, CAND_E1M2, CAND_E2M1_4, CAND_E3M0 = 1, 2, 4, 8
 

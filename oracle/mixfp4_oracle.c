@@ -187,9 +187,8 @@ static float bf16_to_float(uint16_t h) {
 
 /* One candidate of Algorithm 1 for one 16-element block: scale, quantize,
  * dequantize, error.  a[] holds X_FP8 for the block, B its block max. */
-static void candidate(int type, const float a[16], float B, int* s8code,
-                      int payload[16], float* S) {
-  float cmax = (type == 0) ? 6.0f : 7.0f;          /* largest magnitude */
+static void candidate_div(int type, float cmax, const float a[16], float B, int* s8code,
+                          int payload[16], float* S) {
   float ratio = B / cmax;                           /* fl32(B / c) */
   int code = oracle_e4m3_rne(ratio);                /* E4M3 RNE, R2 */
   float s8 = (float)oracle_e4m3_value(code);        /* exact in fp32 */
@@ -209,8 +208,16 @@ static void candidate(int type, const float a[16], float B, int* s8code,
   *s8code = code;
 }
 
+/* Algorithm 1's candidates: E2M1 with the block max mapped to 6, E1M2 to 7. */
+static void candidate(int type, const float a[16], float B, int* s8code,
+                      int payload[16], float* S) {
+  candidate_div(type, (type == 0) ? 6.0f : 7.0f, a, B, s8code, payload, S);
+}
+
 /* Algorithm 1 over a [rows][K] fp32 tensor (row stride ldx elements).
- *   mode 0 = MixFP4, 1 = E2M1 only (NVFP4), 2 = E1M2 only (NVINT4)
+ *   mode 0 = MixFP4, 1 = E2M1 only (NVFP4), 2 = E1M2 only (NVINT4),
+ *   3 = the {E2M1(6), E2M1(4)} set of R14 packed as E2M1 codes with T = 0
+ *       (the error arrays then hold S of E2M1(6) and of E2M1(4))
  *   scale_given 0: s32 = fl32(max|X| / 2688) is computed and written to *s32;
  *   scale_given 1: *s32 is read.
  * Optional err_e2m1 / err_e1m2 ([rows][K/16]) receive each block's S.
@@ -242,14 +249,29 @@ int oracle_quantize_f32(const float* x, int64_t rows, int64_t K, int64_t ldx,
       }
       int c2 = 0, c1 = 0, p2[16], p1[16];
       float S2 = 0.0f, S1 = 0.0f;
-      if (mode != 2) candidate(0, a, B, &c2, p2, &S2);
-      if (mode != 1) candidate(1, a, B, &c1, p1, &S1);
       int T;
-      if (mode == 1) T = 0;
-      else if (mode == 2) T = 1;
-      else T = (S2 < S1) ? 0 : 1;                   /* R6: strict < */
-      const int* p = T ? p1 : p2;
-      int code = T ? c1 : c2;
+      const int* p;
+      int code;
+      if (mode == 3) {
+        /* {E2M1(6), E2M1(4)} (R14): both E2M1, T = 0; E2M1(4) wins a tie */
+        int c4 = 0, p4[16];
+        float S4 = 0.0f;
+        candidate(0, a, B, &c2, p2, &S2);
+        candidate_div(0, 4.0f, a, B, &c4, p4, &S4);
+        T = 0;
+        p = (S4 <= S2) ? p4 : p2;
+        code = (S4 <= S2) ? c4 : c2;
+        if (err_e2m1) err_e2m1[r * nb + b] = S2;
+        if (err_e1m2) err_e1m2[r * nb + b] = S4;
+      } else {
+        if (mode != 2) candidate(0, a, B, &c2, p2, &S2);
+        if (mode != 1) candidate(1, a, B, &c1, p1, &S1);
+        if (mode == 1) T = 0;
+        else if (mode == 2) T = 1;
+        else T = (S2 < S1) ? 0 : 1;                 /* R6: strict < */
+        p = T ? p1 : p2;
+        code = T ? c1 : c2;
+      }
       uint8_t* crow = codes + r * (K / 2) + b * 8;
       for (int j = 0; j < 8; ++j) {
         int lo = (sign[2 * j] << 3) | p[2 * j];
@@ -257,8 +279,10 @@ int oracle_quantize_f32(const float* x, int64_t rows, int64_t K, int64_t ldx,
         crow[j] = (uint8_t)(lo | (hi << 4));        /* R9 */
       }
       scales[r * nb + b] = (uint8_t)((T << 7) | code);  /* App. B.3 */
-      if (err_e2m1) err_e2m1[r * nb + b] = S2;
-      if (err_e1m2) err_e1m2[r * nb + b] = S1;
+      if (mode != 3) {
+        if (err_e2m1) err_e2m1[r * nb + b] = S2;
+        if (err_e1m2) err_e1m2[r * nb + b] = S1;
+      }
     }
   }
   return 0;

@@ -254,3 +254,26 @@ def test_block_size_trends_of_sec5():
         e1 = [ratio[name, g][0] for g in (8, 16, 32, 64)]
         assert all(a < b for a, b in zip(e1, e1[1:])) and e1[-1] < 1.0, (name, e1)
     assert ratio["act", 64][1] < ratio["act", 8][1] < 1.0
+
+
+@pytest.mark.parametrize("given", [None, 0.0173])
+def test_packed_four_six_mode_is_the_46_candidate_set(given):
+    """Mode 3 of the packed quantizer: E2M1 codes with T = 0 whose decode is
+    the {E2M1(6), E2M1(4)} quantize-dequantize bit for bit; each scale byte is
+    E4M3 of B/6 or B/4 as that set chose; blocks that kept B/6 carry the
+    E2M1-only (NVFP4) mode's bytes."""
+    x = synth.bf16_bits(synth.activations(48, 512, 880, 881))
+    s32 = None if given is None else float(np.float32(given))
+    codes, scales, s = oracle.quantize(x, oracle.MODE_FOUR_SIX, s32)
+    ref, choice, s2 = oracle.fake_quantize(x, oracle.CAND_E2M1_6 | oracle.CAND_E2M1_4, 16, s32)
+    assert s == s2 and not np.any(scales & 0x80)
+    assert np.array_equal(oracle.dequantize(codes, scales, s).view(np.uint32), ref.view(np.uint32))
+    xf = (x.astype(np.uint32) << 16).view(np.float32)
+    B = (np.abs(xf) / np.float32(s)).astype(np.float32).reshape(48, 32, 16).max(axis=2)
+    div = np.where(choice == 2, np.float32(4.0), np.float32(6.0))
+    want = np.vectorize(lambda v: oracle.e4m3_rne(float(v)))((B / div).astype(np.float32))
+    assert np.array_equal(scales, want.astype(np.uint8))
+    c1, s1, _ = oracle.quantize(x, oracle.MODE_E2M1_ONLY, s32)
+    keep6 = np.repeat(choice == 0, 8, axis=1)
+    assert np.array_equal(codes[keep6], c1[keep6]) and np.array_equal(scales[choice == 0], s1[choice == 0])
+    assert 0 < np.mean(choice == 2) < 1                 # both candidates occur on these tensors
