@@ -79,6 +79,22 @@ def lib() -> ctypes.CDLL:
     return _lib
 
 
+def _require(cond: bool, msg: str):
+    """Argument check that stays on under python -O (raises ValueError)."""
+    if not cond:
+        raise ValueError(msg)
+
+
+def _check_x(x: torch.Tensor):
+    _require(isinstance(x, torch.Tensor) and x.is_cuda and x.dtype == torch.bfloat16 and x.dim() == 2
+             and x.stride(1) == 1, "x must be a 2-D bf16 CUDA tensor with unit column stride")
+
+
+def _check_signs(signs):
+    _require(signs is None or (signs.dtype == torch.uint8 and signs.numel() == 16 and signs.is_contiguous()
+                               and signs.is_cuda), "signs must be 16 contiguous uint8 bytes on the GPU")
+
+
 def _ptr(t):
     return None if t is None else ctypes.c_void_p(t.data_ptr())
 
@@ -123,7 +139,7 @@ def mixfp4_quantize(x: torch.Tensor, mode: int = MODE_MIX, tensor_scale: torch.T
     With tensor_scale=None the per-tensor scale is computed (max|x| / 2688);
     otherwise the given 1-element fp32 tensor is used as s32.
     """
-    assert x.dtype == torch.bfloat16 and x.dim() == 2 and x.stride(1) == 1
+    _check_x(x)
     rows, K = x.shape
     q = out if out is not None else empty_qtensor(rows, K, x.device)
     given = tensor_scale is not None
@@ -145,8 +161,8 @@ def mixfp4_quantize_rht(x: torch.Tensor, signs: torch.Tensor | None = None, mode
     """Rotate every 128-element chunk of each row of a bf16 [rows, K] CUDA tensor
     (sign flips from the 16-byte `signs`, then the normalised Walsh-Hadamard
     transform) and quantize the result; K % 128 == 0."""
-    assert x.dtype == torch.bfloat16 and x.dim() == 2 and x.stride(1) == 1
-    assert signs is None or (signs.dtype == torch.uint8 and signs.numel() == 16 and signs.is_contiguous())
+    _check_x(x)
+    _check_signs(signs)
     rows, K = x.shape
     q = out if out is not None else empty_qtensor(rows, K, x.device)
     given = tensor_scale is not None
@@ -168,7 +184,7 @@ def mixfp4_quantize_colwise(x: torch.Tensor, mode: int = MODE_MIX, tensor_scale:
     """Quantize a bf16 [R, C] CUDA tensor with 16-row blocks down each column
     (the orientation of a GEMM reducing over R): returns the MixFP4 tensor of
     X^T, codes [C, R/2], scales [C, R/16]."""
-    assert x.dtype == torch.bfloat16 and x.dim() == 2 and x.stride(1) == 1
+    _check_x(x)
     R, C = x.shape
     q = out if out is not None else empty_qtensor(C, R, x.device)
     given = tensor_scale is not None
@@ -189,8 +205,8 @@ def mixfp4_quantize_colwise_rht(x: torch.Tensor, signs: torch.Tensor | None = No
                                 workspace: torch.Tensor | None = None, stream=None) -> QTensor:
     """Rotate every 128-row chunk of each column of a bf16 [R, C] CUDA tensor and
     quantize down the columns: the MixFP4 tensor of the rotated X^T."""
-    assert x.dtype == torch.bfloat16 and x.dim() == 2 and x.stride(1) == 1
-    assert signs is None or (signs.dtype == torch.uint8 and signs.numel() == 16 and signs.is_contiguous())
+    _check_x(x)
+    _check_signs(signs)
     R, C = x.shape
     q = out if out is not None else empty_qtensor(C, R, x.device)
     given = tensor_scale is not None
@@ -211,7 +227,7 @@ def mixfp4_quantize_sr(x: torch.Tensor, seed: int, offset: int = 0, mode: int = 
                        workspace: torch.Tensor | None = None, colwise: bool = False, stream=None) -> QTensor:
     """mixfp4_quantize (or, with colwise=True, mixfp4_quantize_colwise) with
     stochastic rounding of the codes drawn from (seed, offset)."""
-    assert x.dtype == torch.bfloat16 and x.dim() == 2 and x.stride(1) == 1
+    _check_x(x)
     rows, K = x.shape
     q = out if out is not None else (empty_qtensor(K, rows, x.device) if colwise else empty_qtensor(rows, K, x.device))
     given = tensor_scale is not None
@@ -233,7 +249,7 @@ def mixfp4_quantize_2d(x: torch.Tensor, mode: int = MODE_MIX, tensor_scale: torc
                        stream=None) -> QTensor:
     """Quantize a bf16 [rows, K] CUDA tensor with 16 x 16 blocks (one scale
     and format per tile, repeated on the tile's rows)."""
-    assert x.dtype == torch.bfloat16 and x.dim() == 2 and x.stride(1) == 1
+    _check_x(x)
     rows, K = x.shape
     q = out if out is not None else empty_qtensor(rows, K, x.device)
     given = tensor_scale is not None
@@ -269,17 +285,19 @@ def mixfp4_fake_quantize(x: torch.Tensor, candidates: int, block: int = 16, out_
     set (mask of CAND_*) and block size (8, 16, 32, 64): returns (out
     [rows, K] of out_dtype (float32 or bfloat16), choice uint8 [rows, K/block]
     or None, tensor_scale)."""
-    assert x.dtype == torch.bfloat16 and x.dim() == 2 and x.stride(1) == 1
-    assert out_dtype in (torch.float32, torch.bfloat16)
+    _check_x(x)
+    _require(out_dtype in (torch.float32, torch.bfloat16), "out_dtype must be torch.float32 or torch.bfloat16")
+    _require(block in (8, 16, 32, 64), "block must be 8, 16, 32 or 64")
     rows, K = x.shape
     o = out if out is not None else torch.empty(rows, K, dtype=out_dtype, device=x.device)
-    assert o.dtype == out_dtype and o.stride(1) == 1
+    _require(o.dtype == out_dtype and o.dim() == 2 and o.shape == x.shape and o.stride(1) == 1,
+             "out must be a [rows, K] tensor of out_dtype with unit column stride")
     ch = None
     if want_choice:
-        ch = choice if choice is not None else torch.empty(rows, K // block if block else 0, dtype=torch.uint8,
+        ch = choice if choice is not None else torch.empty(rows, K // block, dtype=torch.uint8,
                                                            device=x.device)
-        assert ch.dtype == torch.uint8 and ch.is_contiguous() and ch.numel() == rows * (K // block), \
-            "choice must be a dense uint8 [rows, K / block] tensor"
+        _require(ch.dtype == torch.uint8 and ch.is_contiguous() and ch.numel() == rows * (K // block),
+                 "choice must be a dense uint8 [rows, K / block] tensor")
     ts = torch.empty(1, dtype=torch.float32, device=x.device)
     given = tensor_scale is not None
     if given:
@@ -306,7 +324,7 @@ def mixfp4_dequantize(q: QTensor, out: torch.Tensor | None = None, stream=None) 
 def mixfp4_gemm(a: QTensor, b: QTensor, out: torch.Tensor | None = None,
                 status_word: torch.Tensor | None = None, stream=None) -> torch.Tensor:
     """C = A_deq . B_deq^T in fp32; a is M x K, b is N x K."""
-    assert a.K == b.K
+    _require(a.K == b.K, "operands must share K")
     M, N, K = a.rows, b.rows, a.K
     C = out if out is not None else torch.empty(M, N, dtype=torch.float32, device=a.codes.device)
     st = lib().mixfp4_gemm(_ptr(a.codes), _ptr(a.scales), _ptr(a.tensor_scale),
@@ -346,7 +364,7 @@ def mixfp4_split_native(q: QTensor, keep_residual: bool = True, out: NativeTenso
     (MODE_E2M1_ONLY).  `out` (with a residual buffer) is reused when given."""
     dev = q.codes.device
     if out is not None:
-        assert out.res is not None and out.main.shape == q.codes.shape
+        _require(out.res is not None and out.main.shape == q.codes.shape, "out must match the operand's shape")
         main, res, sf = out.main, out.res, out.sf
     else:
         main = torch.empty_like(q.codes)
@@ -361,7 +379,7 @@ def mixfp4_split_native(q: QTensor, keep_residual: bool = True, out: NativeTenso
 def mixfp4_gemm_native(a: NativeTensor, b: NativeTensor, out: torch.Tensor | None = None,
                        status_word: torch.Tensor | None = None, stream=None) -> torch.Tensor:
     """C = A . B^T on the block-scaled FP4 tensor path; a is M x K, b is N x K."""
-    assert a.K == b.K
+    _require(a.K == b.K, "operands must share K")
     M, N, K = a.rows, b.rows, a.K
     C = out if out is not None else torch.empty(M, N, dtype=torch.float32, device=a.main.device)
     st = lib().mixfp4_gemm_native(_ptr(a.main), _ptr(a.res), _ptr(a.sf), _ptr(a.tensor_scale),
@@ -375,7 +393,7 @@ def mixfp4_gemm_native_fewrows(a: QTensor, b: QTensor, out: torch.Tensor | None 
                                status_word: torch.Tensor | None = None, stream=None) -> torch.Tensor:
     """C = A_deq . B_deq^T for a with at most 64 rows, on the block-scaled FP4
     tensor path with the operands split on the fly."""
-    assert a.K == b.K and a.rows <= 64
+    _require(a.K == b.K and a.rows <= 64, "operands must share K, and A have at most 64 rows")
     M, N, K = a.rows, b.rows, a.K
     C = out if out is not None else torch.empty(M, N, dtype=torch.float32, device=a.codes.device)
     st = lib().mixfp4_gemm_native_fewrows(_ptr(a.codes), _ptr(a.scales), _ptr(a.tensor_scale),

@@ -92,3 +92,24 @@ def test_stale_traffic_figure_is_dropped(tmp_path, monkeypatch):
     (fake_root / "paper_2605_31035_gb300" / "csrc" / "gemm.cu").write_text("// another kernel\n")
     monkeypatch.setattr(bench, "ROOT", str(fake_root))
     assert bench.ncu_traffic("gemm_attn", "gemm.cu") is None
+
+
+def test_binding_rejects_bad_arguments_before_the_library(monkeypatch):
+    """The binding's checks raise ValueError (they stay on under python -O)
+    and run before any library call: a CPU tensor, a wrong dtype, a bad block
+    size or output dtype never reaches the C ABI."""
+    import torch
+    from paper_2605_31035_gb300 import ops
+
+    def no_lib():
+        raise AssertionError("the library must not be reached")
+    monkeypatch.setattr(ops, "lib", no_lib)
+    x_cpu = torch.zeros(4, 64, dtype=torch.bfloat16)
+    with pytest.raises(ValueError, match="CUDA"):
+        ops.mixfp4_quantize(x_cpu)
+    with pytest.raises(ValueError, match="CUDA"):
+        ops.mixfp4_quantize_2d(x_cpu.float())
+    with pytest.raises(ValueError):
+        ops.mixfp4_fake_quantize(x_cpu, 15, 16)
+    with pytest.raises(ValueError):
+        ops.mixfp4_quantize_rht(x_cpu, signs=torch.zeros(8, dtype=torch.uint8))
