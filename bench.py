@@ -249,6 +249,12 @@ def run_ours(args):
     # Native block-scaled FP4 variant on the same workload: the weights are
     # split once (like their quantization), the activations every call.
     nw = ops.mixfp4_split_native(w_q)
+    # Share of blocks that chose E1M2 (type bit set) in the quantized X and W.
+    try:
+        e1m2_share = {"x": round(float((q_x.scales >> 7).float().mean().item()), 4),
+                      "w": round(float((w_q.scales >> 7).float().mean().item()), 4)}
+    except Exception:  # a reporting extra; never costs the bench line
+        e1m2_share = None
     nx = ops.mixfp4_split_native(q_x)
     Cn = torch.empty_like(C)
 
@@ -381,11 +387,13 @@ def run_ours(args):
                      "traffic": traffic},
         "kernels": {
             "gemm_ms": round(gemm_avg, 5), "gemm_tflops": round(gemm_tflops, 2),
+            "e1m2_block_share": e1m2_share,
             "quantize_with_amax_ms": round(quant_avg, 5),
             "quantize_with_amax_gbs_alg": round(M * K * QUANT_BYTES_PER_ELEM / (quant_avg * 1e-3) / 1e9, 1),
             "quantizer_2^28": {
                 "quantize_kernel_given_scale": {"ms": round(given_ms, 4), "alg_gbs": round(given_gbs, 1),
-                                                "frac_of_hbm": round(given_gbs / pk["hbm_gbs"], 4)},
+                                                "frac_of_hbm": round(given_gbs / pk["hbm_gbs"], 4),
+                                                "frac_of_hbm_spec_7900": round(given_gbs / 7900.0, 4)},
                 "with_amax_pass": {"ms": round(sweep_ms, 4), "alg_gbs": round(sweep_alg_gbs, 1),
                                    "alg_frac_of_hbm": round(sweep_alg_gbs / pk["hbm_gbs"], 4),
                                    "bytes_incl_amax_read_gbs": round(sweep_read_gbs, 1)},
