@@ -49,7 +49,7 @@ typedef enum {
 enum { MIXFP4_MODE_MIX = 0,        /* Alg. 1: per-block E2M1/E1M2 by lower MSE */
        MIXFP4_MODE_E2M1_ONLY = 1,  /* every block E2M1, T = 0 (plain NVFP4 bits) */
        MIXFP4_MODE_E1M2_ONLY = 2,  /* every block E1M2, T = 1 (NVINT4 lattice) */
-       MIXFP4_MODE_FOUR_SIX = 3    /* the {E2M1(6), E2M1(4)} candidate set of Sec. 2.3 ("4/6"):
+       MIXFP4_MODE_FOUR_SIX = 3    /* the {E2M1(6), E2M1(4)} candidate set of Sec. 2.4 ("4/6"):
                                       per block the lower-MSE of s8 from B/6 or B/4 (B/4 on a
                                       tie), E2M1 codes, T = 0 (plain NVFP4 bits, so both GEMMs
                                       take it); mixfp4_quantize and mixfp4_quantize_noalloc only */ };
@@ -96,8 +96,8 @@ int mixfp4_quantize(const void* x, int dtype, int64_t rows, int64_t K, int64_t l
 
 /*
  * mixfp4_quantize_rht -- the 128-point Walsh-Hadamard rotation applied before
- * quantization (the random Hadamard transform of Sec. 4 "+RHT" and the
- * Sec. 3.4 training flow), fused with Algorithm 1 (as mixfp4_quantize).
+ * quantization (the random Hadamard transform of Sec. 4.1 "+RHT" and the
+ * Sec. 3.2 training flow), fused with Algorithm 1 (as mixfp4_quantize).
  *
  *   every 128-element chunk of a row along K, on its own:
  *     v_i = -x_i if bit i of `signs` is set, else x_i        (i = 0..127)
@@ -122,7 +122,7 @@ int mixfp4_quantize_rht(const void* x, int dtype, int64_t rows, int64_t K, int64
 /*
  * mixfp4_quantize_colwise -- Algorithm 1 with every 16-element block running
  * down a column: the operand orientation of a GEMM that reduces over the rows
- * of X, as in the weight-gradient GEMM of the training flow (Sec. 3.4, WGRAD
+ * of X, as in the weight-gradient GEMM of the training flow (Sec. 3.2, WGRAD
  * reduces over tokens; DGRAD over the weights' output dimension).  The
  * result is bit for bit mixfp4_quantize of the transpose X^T:
  *   codes  [C][R/2]   element r of column c in nibble r % 2 of byte r / 2
@@ -143,7 +143,7 @@ int mixfp4_quantize_colwise(const void* x, int dtype, int64_t R, int64_t C, int6
 /*
  * mixfp4_quantize_colwise_rht -- mixfp4_quantize_colwise with the 128-point
  * Walsh-Hadamard rotation of mixfp4_quantize_rht applied along the rows first:
- * the weight-gradient inputs of the training recipe (Sec. 3.4, Sec. 4: the
+ * the weight-gradient inputs of the training recipe (Sec. 3.2, Sec. 4.2: the
  * RHT is applied to both WGRAD operands, whose reduction runs over R).  Every
  * 128-row chunk of each column is rotated (signs, butterfly order and scaling
  * as mixfp4_quantize_rht) and the rotated column is quantized down its rows:
@@ -159,7 +159,7 @@ int mixfp4_quantize_colwise_rht(const void* x, int dtype, int64_t R, int64_t C, 
 /*
  * mixfp4_quantize_sr, mixfp4_quantize_colwise_sr -- mixfp4_quantize and
  * mixfp4_quantize_colwise with stochastic rounding of the codes, the
- * gradient quantization of the training flow (Sec. 4 pre-training recipe;
+ * gradient quantization of the training flow (Sec. 4.2 pre-training recipe;
  * the paper's stochastic-rounding ablation).  Format and block scale are
  * chosen exactly as Algorithm 1 chooses them (round-to-nearest candidates, so
  * scale bytes and s32 equal those of the rounding-to-nearest entry point);
@@ -187,9 +187,9 @@ int mixfp4_quantize_colwise_sr(const void* x, int dtype, int64_t R, int64_t C, i
 
 /*
  * mixfp4_fake_quantize -- quantize-dequantize under a chosen candidate set
- * and block size: the paper's candidate-set ablation (Sec. 2.3, candidate
+ * and block size: the paper's candidate-set ablation (Sec. 2.4, candidate
  * sets {E2M1(6), E2M1(4)} and {E2M1(6), E1M2, E3M0}) and block-size ablation
- * (Sec. 5, Table 5, g = 8..64).  A block is g consecutive elements of a row.
+ * (Sec. 4.3, Table 5, g = 8..64).  A block is g consecutive elements of a row.
  * Every candidate c in `candidates` follows Algorithm 1 with its own divisor
  * d_c (6, 7, 4, 16): s8 = E4M3_RNE(fl32(B / d_c)) from the block max B of
  * |x / s32|, codes by round-to-nearest-even of fl32(|x / s32| / s8) onto its
@@ -222,7 +222,7 @@ int mixfp4_fake_quantize(const void* x, int dtype, int64_t rows, int64_t K, int6
 
 /*
  * mixfp4_quantize_2d -- Algorithm 1 with 16 x 16 blocks, the weight
- * quantization of the training flow (Sec. 3.4: weights in 2D blocks).  The
+ * quantization of the training flow (Sec. 3.2: weights in 2D blocks).  The
  * tile of rows 16t..16t+15 and columns 16b..16b+15 has one block max (the
  * tile's), one E4M3 scale per candidate and one type bit; each candidate's
  * error is the per-row sum of mixfp4_quantize, combined over the tile's 16
@@ -368,7 +368,8 @@ int mixfp4_gemm_native_fewrows(const uint8_t* a_codes, const uint8_t* a_scales, 
  * tensor_scale (device, one float) receives s32.
  *
  * The first call on a device looks up the array's device address for that
- * device (make it before any stream capture).  Every call shares the array,
+ * device (make it before any stream capture); a call that finds a different
+ * context current on the device (after cudaDeviceReset) looks it up again.  Every call shares the array,
  * and the array keeps the last call's contents (it is cleared before each
  * use); calls that overlap on the GPU race on it and must be ordered.  Any
  * shape needs one 32-bit word of the 64 the array holds; a larger need would

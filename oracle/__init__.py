@@ -18,9 +18,9 @@ Function map (paper passages are cited in ``mixfp4_oracle.c``):
                             layout (the native FP4 GEMM variant)
   quantize_colwise          Algorithm 1 along the other dimension (blocks of 16
                             rows in one column): quantize of the transpose, the
-                            WGRAD / DGRAD operand orientation (Sec. 3.4)
+                            WGRAD / DGRAD operand orientation (Sec. 3.2)
   quantize_2d               Algorithm 1 with 16 x 16 tiles (2D weight blocks of
-                            the training flow, Sec. 3.4), reading R12
+                            the training flow, Sec. 3.2), reading R12
   transpose_2d              the transposed operand of a 2D-quantized tensor
   philox4x32_10             Salmon et al.'s counter-based generator (SC'11)
   quantize_sr               Algorithm 1 with stochastic rounding of the chosen

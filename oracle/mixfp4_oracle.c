@@ -19,7 +19,7 @@
  *                      App. B.3 (type-in-scale packing); oracle_quantize_f32
  *                      is the same steps on an fp32 tensor
  *   oracle_rht         the random Hadamard transform applied before
- *                      quantization (Sec. 4 "+RHT", Sec. 3.4 training flow):
+ *                      quantization (Sec. 4.1 "+RHT", Sec. 3.2 training flow):
  *                      128-point Sylvester Walsh-Hadamard per chunk (reading
  *                      R11)
  *   oracle_dequantize  App. B.2/B.3 decode (scale_ue4m3 = scale with bit 7
@@ -31,7 +31,7 @@
  *                      sharing its scales (Table 1 codebooks; 5 = 4 + 1,
  *                      7 = 6 + 1), scales in the tensor core's tiled layout
  *   oracle_quantize_2d Algorithm 1 with 2D 16 x 16 blocks, the weight
- *                      quantization of the training flow (Sec. 3.4, Sec. 4
+ *                      quantization of the training flow (Sec. 3.2, Sec. 4.2
  *                      pre-training recipe); reading R12
  *   oracle_transpose_2d  the transposed operand (DGRAD orientation) of a
  *                      2D-quantized tensor: codes and tile scales transposed
@@ -39,14 +39,14 @@
  *                      "Parallel random numbers: as easy as 1, 2, 3" (SC'11),
  *                      source of the stochastic-rounding uniforms
  *   oracle_quantize_sr Algorithm 1 with stochastic rounding of the codes
- *                      (App. "Ablation Study of Stochastic Rounding", Sec. 4
+ *                      (App. D "Ablation Study of Stochastic Rounding", Sec. 4.2
  *                      pre-training recipe: SR on gradients); reading R13
  *   oracle_fake_quantize  Algorithm 1 with the per-block MSE choice taken over
  *                      a chosen candidate set and block size, returning the
  *                      quantized-then-dequantized tensor and each block's
- *                      choice: the candidate-set ablation (Sec. 2.3 "Format
+ *                      choice: the candidate-set ablation (Sec. 2.4 "Format
  *                      Proliferation Has Diminishing Returns", E2M1(4) and
- *                      E3M0) and the block-size ablation (Sec. 5, Table 5);
+ *                      E3M0) and the block-size ablation (Sec. 4.3, Table 5);
  *                      reading R14
  *   oracle_f32_to_bf16 binary32 -> bfloat16, round to nearest even
  *
@@ -493,8 +493,8 @@ int oracle_split_native(const uint8_t* codes, const uint8_t* scales, int64_t row
 }
 
 /* ---------------------------------------------------------------------------
- * 2D block quantization (Sec. 3.4: weights are quantized in 2D blocks in the
- * training flow; Sec. 4 pre-training recipe), reading R12: Algorithm 1 with
+ * 2D block quantization (Sec. 3.2: weights are quantized in 2D blocks in the
+ * training flow; Sec. 4.2 pre-training recipe), reading R12: Algorithm 1 with
  * the block taken as a 16 x 16 tile.
  * ------------------------------------------------------------------------- */
 static float tree16(const float s[16]) {
@@ -670,7 +670,7 @@ int oracle_quantize_sr(const uint16_t* x, int64_t rows, int64_t K, int64_t ldx, 
 }
 
 /* ---------------------------------------------------------------------------
- * R14: candidate-set and block-size ablation (Sec. 2.3, Sec. 5 Table 5).
+ * R14: candidate-set and block-size ablation (Sec. 2.4, Sec. 4.3 Table 5).
  * ------------------------------------------------------------------------- */
 
 /* Magnitude of payload p (0..7) under candidate c (R14). */

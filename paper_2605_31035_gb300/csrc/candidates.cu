@@ -3,7 +3,7 @@
 // -- E2M1 with largest value 6 (Algorithm 1's E2M1), E1M2 in x2 units, E2M1
 // with the block max mapped to 4, and E3M0 (Eq. 1-2 with W_E = 3, W_M = 0:
 // {0, 1/4, ..., 16}) -- and blocks of g = 8, 16, 32 or 64 elements.  These are
-// the paper's ablations (Sec. 2.3 candidate sets, Sec. 5 Table 5 block
+// the paper's ablations (Sec. 2.4 candidate sets, Sec. 4.3 Table 5 block
 // sizes).  The stored MixFP4 format holds one type bit, so the kernel returns
 // what the ablations measure: the dequantized tensor (fp32 or bf16) and each
 // block's chosen candidate.
@@ -23,6 +23,7 @@
 #include <cuda_runtime.h>
 #include <cstdint>
 
+#include "host_util.cuh"
 #include "kernels.cuh"
 #include "ptx.cuh"
 #include "quant_core.cuh"
@@ -198,7 +199,7 @@ int launch_fake_quantize(const uint16_t* x, int64_t rows, int64_t K, int64_t ldx
   const int64_t nsub = rows * (K / 16);
   if (nsub == 0) return 0;
   int64_t grid = (nsub + kFqThreads - 1) / kFqThreads;
-  if (grid > 152 * 8) grid = 152 * 8;
+  if (grid > num_sms() * 8) grid = num_sms() * 8;
   cudaError_t e;
 #define MIXFP4_LAUNCH_FQ(G)                                                                                  \
   e = launch_pdl(fake_quantize_kernel<G>, (unsigned)grid, kFqThreads, 0, stream, x, rows, K, ldx, candidates, \

@@ -19,12 +19,17 @@
 //   * In host code the array's name is only a host-side stand-in; the device
 //     address is obtained with cudaGetSymbolAddress once per device, with that
 //     device current, on the first call made on it.  Make that first call
-//     before any stream capture begins.
+//     before any stream capture begins.  The address is cached together with
+//     the unique id of the context it was looked up in: after a
+//     cudaDeviceReset the library's module is loaded again in a new context,
+//     possibly at another address, so a call that finds a different current
+//     context looks the address up again (as a first call does).
 //   * All calls share the one array and it keeps the last call's contents; the
 //     word is cleared on the stream before each use.  Calls that overlap on the
 //     GPU (different streams without ordering, or several host threads) race
 //     on it and may produce a wrong scale: order them.
 //   * No cudaMalloc, cudaFree or other allocating routine is called.
+#include <cuda.h>
 #include <cuda_runtime.h>
 #include <cstdint>
 #include <mutex>
@@ -41,17 +46,49 @@ static __device__ __align__(256) uint32_t g_noalloc_scratch[kNoAllocScratchWords
 
 std::mutex g_setup_mutex;
 uint32_t* g_scratch_ptr[kMaxDevices] = {};
+unsigned long long g_scratch_ctx[kMaxDevices] = {};  // context id the address belongs to (0: none)
 
-// Device address of the scratch array on the current device (set up once per
-// device); nullptr on failure.
+using CtxGetCurrentFn = CUresult (*)(CUcontext*);
+using CtxGetIdFn = CUresult (*)(CUcontext, unsigned long long*);
+
+// Unique id of the current context (ids are never reused within a process);
+// 0 when there is no current context or the driver does not report ids.
+unsigned long long current_context_id() {
+  static CtxGetCurrentFn get_current = nullptr;
+  static CtxGetIdFn get_id = nullptr;
+  static bool resolved = false;
+  if (!resolved) {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      get_current = reinterpret_cast<CtxGetCurrentFn>(p);
+    p = nullptr;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetId", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      get_id = reinterpret_cast<CtxGetIdFn>(p);
+    resolved = true;
+  }
+  CUcontext ctx = nullptr;
+  unsigned long long id = 0;
+  if (!get_current || !get_id || get_current(&ctx) != CUDA_SUCCESS || !ctx || get_id(ctx, &id) != CUDA_SUCCESS)
+    return 0;
+  return id;
+}
+
+// Device address of the scratch array on the current device, looked up on
+// the first call on each device (and again when the device's context has
+// changed since, e.g. after cudaDeviceReset); nullptr on failure.
 uint32_t* scratch_for_current_device() {
   int dev = -1;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return nullptr;
   std::lock_guard<std::mutex> lock(g_setup_mutex);
-  if (!g_scratch_ptr[dev]) {
+  const unsigned long long ctx = current_context_id();
+  if (!g_scratch_ptr[dev] || ctx == 0 || ctx != g_scratch_ctx[dev]) {
     void* p = nullptr;
     if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || !p) return nullptr;
     g_scratch_ptr[dev] = static_cast<uint32_t*>(p);
+    g_scratch_ctx[dev] = current_context_id();  // the lookup above made the context current if it was not
   }
   return g_scratch_ptr[dev];
 }

@@ -224,7 +224,7 @@ __device__ __forceinline__ void block_core(const u64 a[8], const TensorConsts& t
   unpack2(bq, b6, b7);
 
   if (kMode == MIXFP4_MODE_FOUR_SIX) {
-    // {E2M1(6), E2M1(4)} (Sec. 2.3, reading R14): the second scale from
+    // {E2M1(6), E2M1(4)} (Sec. 2.4, reading R14): the second scale from
     // fl32(B/4) = B/4 exactly; both candidates are E2M1 (T = 0) and the later
     // one, E2M1(4), wins a tie.
     const uint32_t sc = cvt_e4m3x2(__fmul_rn(B, 0.25f), b6);  // low byte: B/6 code, high: B/4
@@ -417,7 +417,7 @@ __device__ __forceinline__ const uint16_t* block_src(const uint16_t* x, int64_t 
 }
 
 // ---- 128-point Walsh-Hadamard rotation before quantization ----------------
-// Reading R11 of the random Hadamard transform (Sec. 4 "+RHT", Sec. 3.4): each
+// Reading R11 of the random Hadamard transform (Sec. 4.1 "+RHT", Sec. 3.2): each
 // 128-element chunk of a row along K is rotated on its own: elements whose bit
 // in the caller's 128-bit sign vector is set are negated, the Sylvester
 // product H_128 v is formed by the radix-2 butterfly in fp32 with strides

@@ -31,6 +31,7 @@
 #include <cuda_runtime.h>
 #include <cstdint>
 
+#include "host_util.cuh"
 #include "kernels.cuh"
 #include "ptx.cuh"
 #include "quant_core.cuh"
@@ -235,7 +236,7 @@ int launch_amax(const uint16_t* x, int64_t rows, int64_t K, int64_t ldx, uint32_
   const int64_t kblocks = K / 16, nblocks = rows * kblocks;
   if (nblocks == 0) return 0;
   int64_t grid = (nblocks + 256 * kAmaxUnroll - 1) / (256 * kAmaxUnroll);
-  if (grid > 152 * 8) grid = 152 * 8;
+  if (grid > num_sms() * 8) grid = num_sms() * 8;
   if (ldx == K) amax_kernel<true><<<(unsigned)grid, 256, 0, stream>>>(x, nblocks, kblocks, ldx, amax_word);
   else amax_kernel<false><<<(unsigned)grid, 256, 0, stream>>>(x, nblocks, kblocks, ldx, amax_word);
   return 0;
@@ -245,10 +246,10 @@ int launch_quantize(const uint16_t* x, int64_t rows, int64_t K, int64_t ldx, uin
                     uint8_t* scales, float* tensor_scale, const uint32_t* amax_word, int mode,
                     int scale_given, cudaStream_t stream) {
   const int64_t kblocks = K / 16, nblocks = rows * kblocks;
-  // Persistent grid: 4 CTAs per SM of a 152-SM GB300, fewer for small tensors
+  // Persistent grid: 4 CTAs per SM of the device, fewer for small tensors
   // (each thread takes at least two blocks).
   int64_t grid = (nblocks + 2 * kQuantThreads - 1) / (2 * kQuantThreads);
-  if (grid > 152 * 4) grid = 152 * 4;
+  if (grid > num_sms() * 4) grid = num_sms() * 4;
   if (grid == 0) return 0;
   // Launched as a programmatic dependent: it overlaps its launch with the tail
   // of the kernel before it (see the waits at the top of quantize_kernel).
@@ -277,7 +278,7 @@ int launch_rht_amax(const uint16_t* x, int64_t rows, int64_t K, int64_t ldx, con
   const int64_t kblocks = K / 16, nblocks = rows * kblocks;
   if (nblocks == 0) return 0;
   int64_t grid = (nblocks + 255) / 256;
-  if (grid > 152 * 8) grid = 152 * 8;
+  if (grid > num_sms() * 8) grid = num_sms() * 8;
   if (ldx == K) rht_amax_kernel<true><<<(unsigned)grid, 256, 0, stream>>>(x, nblocks, kblocks, ldx, signs, amax_word);
   else rht_amax_kernel<false><<<(unsigned)grid, 256, 0, stream>>>(x, nblocks, kblocks, ldx, signs, amax_word);
   return 0;
@@ -288,7 +289,7 @@ int launch_rht_quantize(const uint16_t* x, int64_t rows, int64_t K, int64_t ldx,
                         int scale_given, cudaStream_t stream) {
   const int64_t kblocks = K / 16, nblocks = rows * kblocks;
   int64_t grid = (nblocks + kQuantThreads - 1) / kQuantThreads;
-  if (grid > 152 * 3) grid = 152 * 3;
+  if (grid > num_sms() * 3) grid = num_sms() * 3;
   if (grid == 0) return 0;
   const int after_amax = !scale_given;
 #define MIXFP4_LAUNCH_R(MODE)                                                                            \

@@ -1,4 +1,4 @@
-// Quantizer orientations of the MixFP4 training flow (Sec. 3.4: FPROP, DGRAD
+// Quantizer orientations of the MixFP4 training flow (Sec. 3.2: FPROP, DGRAD
 // and WGRAD all run on MixFP4 operands; weights use 2D blocks) for sm_103a.
 //
 //   quantize_colwise_kernel  Algorithm 1 with each 16-element block running
@@ -29,6 +29,7 @@
 #include <cuda_runtime.h>
 #include <cstdint>
 
+#include "host_util.cuh"
 #include "kernels.cuh"
 #include "ptx.cuh"
 #include "quant_core.cuh"
@@ -196,7 +197,7 @@ quantize_2d_kernel(const uint16_t* __restrict__ x, int64_t rows, int64_t K, int6
 }
 
 // Column-wise quantization with the 128-point rotation along the rows (the
-// weight-gradient inputs of the training recipe, Sec. 3.4 / Sec. 4: the RHT
+// weight-gradient inputs of the training recipe, Sec. 3.2 / Sec. 4.2: the RHT
 // is applied to both WGRAD operands, whose reduction runs over tokens): every
 // 128-row chunk of each column is rotated (reading R11: the caller's sign
 // vector, the same butterfly order) and the rotated column is quantized down
@@ -383,7 +384,7 @@ int launch_quantize_colwise(const uint16_t* x, int64_t R, int64_t C, int64_t ldx
                             uint64_t seed, uint64_t offset, cudaStream_t stream) {
   const int64_t tiles = ((C + kColThreads - 1) / kColThreads) * ((R + kColRows - 1) / kColRows);
   if (tiles == 0) return 0;
-  int64_t grid = tiles < 152 * 4 ? tiles : 152 * 4;
+  int64_t grid = tiles < num_sms() * 4 ? tiles : num_sms() * 4;
   cudaError_t e;
 #define MIXFP4_LAUNCH_C(MODE, SR)                                                                            \
   e = launch_pdl(quantize_colwise_kernel<MODE, SR>, (unsigned)grid, kColThreads, 0, stream, x, R, C, ldx, codes, \
@@ -409,7 +410,7 @@ int launch_quantize_sr(const uint16_t* x, int64_t rows, int64_t K, int64_t ldx, 
   const int64_t kblocks = K / 16, nblocks = rows * kblocks;
   if (nblocks == 0) return 0;
   int64_t grid = (nblocks + 255) / 256;
-  if (grid > 152 * 3) grid = 152 * 3;
+  if (grid > num_sms() * 3) grid = num_sms() * 3;
   cudaError_t e;
 #define MIXFP4_LAUNCH_S(MODE)                                                                               \
   e = (ldx == K) ? launch_pdl(quantize_sr_kernel<MODE, true>, (unsigned)grid, 256, 0, stream, x, nblocks, kblocks, \
@@ -431,7 +432,7 @@ int launch_quantize_2d(const uint16_t* x, int64_t rows, int64_t K, int64_t ldx, 
   const int64_t units = ((rows + 15) / 16) * ((K / 16 + 1) / 2);
   if (units == 0) return 0;
   int64_t grid = (units + k2dThreads / 32 - 1) / (k2dThreads / 32);
-  if (grid > 152 * 4) grid = 152 * 4;
+  if (grid > num_sms() * 4) grid = num_sms() * 4;
   cudaError_t e;
   switch (mode) {
     case MIXFP4_MODE_MIX:
@@ -455,7 +456,7 @@ int launch_quantize_colwise_rht(const uint16_t* x, int64_t R, int64_t C, int64_t
                                 int scale_given, int amax_pass, cudaStream_t stream) {
   const int64_t tiles = ((C + kCrCols - 1) / kCrCols) * (R / kCrRows);
   if (tiles == 0) return 0;
-  const int64_t grid = tiles < 152 * 3 ? tiles : 152 * 3;
+  const int64_t grid = tiles < num_sms() * 3 ? tiles : num_sms() * 3;
   cudaError_t e;
 #define MIXFP4_LAUNCH_CR(MODE, AMAX)                                                                           \
   e = launch_pdl(quantize_colwise_rht_kernel<MODE, AMAX>, (unsigned)grid, 256, 0, stream, x, R, C, ldx, signs, codes, \
@@ -478,7 +479,7 @@ int launch_transpose_2d(const uint8_t* codes, const uint8_t* scales, int64_t row
   const int64_t units = ((K + kTrUnitCols - 1) / kTrUnitCols) * ((rows + kTrUnitRows - 1) / kTrUnitRows);
   if (units == 0) return 0;
   const int64_t blocks = (units + 7) / 8;  // 8 warps per CTA, one unit each per pass
-  const int64_t grid = blocks < 152 * 8 ? blocks : 152 * 8;
+  const int64_t grid = blocks < num_sms() * 8 ? blocks : num_sms() * 8;
   transpose_2d_kernel<<<(unsigned)grid, 256, 0, stream>>>(codes, scales, rows, K, codes_t, scales_t);
   return cudaGetLastError() == cudaSuccess ? 0 : -1;
 }

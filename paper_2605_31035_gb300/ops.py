@@ -95,6 +95,65 @@ def _check_signs(signs):
                                and signs.is_cuda), "signs must be 16 contiguous uint8 bytes on the GPU")
 
 
+def _check_dev(t, device, what: str):
+    """t must be a CUDA tensor on `device` (the device of the call's main input)."""
+    _require(isinstance(t, torch.Tensor) and t.is_cuda and t.device == device,
+             f"{what} must be a CUDA tensor on {device}")
+
+
+def _check_u8(t, shape, device, what: str):
+    _check_dev(t, device, what)
+    _require(t.dtype == torch.uint8 and tuple(t.shape) == tuple(shape) and t.is_contiguous(),
+             f"{what} must be a dense uint8 tensor of shape {tuple(shape)}")
+
+
+def _check_scalar_f32(t, device, what: str):
+    _check_dev(t, device, what)
+    _require(t.dtype == torch.float32 and t.numel() >= 1, f"{what} must hold at least one float32")
+
+
+def _check_qtensor(q, rows: int, K: int, device, what: str):
+    """A MixFP4 operand: codes uint8 [rows, K/2], scales uint8 [rows, K/16], s32 float32, all on `device`."""
+    _require(isinstance(q, QTensor), f"{what} must be a QTensor")
+    _check_u8(q.codes, (rows, K // 2), device, f"{what}.codes")
+    _check_u8(q.scales, (rows, K // 16), device, f"{what}.scales")
+    _check_scalar_f32(q.tensor_scale, device, f"{what}.tensor_scale")
+
+
+def _check_operand(q, what: str):
+    """A GEMM operand: a QTensor on a CUDA device, consistent with its own codes shape."""
+    _require(isinstance(q, QTensor) and isinstance(q.codes, torch.Tensor) and q.codes.dim() == 2,
+             f"{what} must be a QTensor with 2-D codes")
+    _check_qtensor(q, q.rows, q.K, q.codes.device, what)
+
+
+def _check_c(C, M: int, N: int, device):
+    """GEMM output: float32 [M, N] on `device`, unit column stride (row stride >= N)."""
+    _check_dev(C, device, "out")
+    _require(C.dtype == torch.float32 and C.dim() == 2 and tuple(C.shape) == (M, N)
+             and (C.stride(1) == 1 or N <= 1) and C.stride(0) >= max(N, 1),
+             f"out must be a float32 [{M}, {N}] tensor with unit column stride")
+
+
+def _check_workspace(ws, device):
+    if ws is not None:
+        _check_dev(ws, device, "workspace")
+        _require(ws.numel() * ws.element_size() >= 4 and ws.is_contiguous(),
+                 "workspace must be a dense CUDA tensor of at least 4 bytes")
+
+
+def _check_status(sw, device):
+    if sw is not None:
+        _check_dev(sw, device, "status_word")
+        _require(sw.numel() >= 1 and sw.element_size() == 4 and not sw.dtype.is_floating_point,
+                 "status_word must be a CUDA tensor of 32-bit integers with at least one element")
+
+
+def _check_given_scale(ts):
+    if ts is not None:
+        _require(isinstance(ts, torch.Tensor) and ts.numel() == 1, "tensor_scale must be a 1-element tensor")
+
+
 def _ptr(t):
     return None if t is None else ctypes.c_void_p(t.data_ptr())
 
@@ -142,12 +201,15 @@ def mixfp4_quantize(x: torch.Tensor, mode: int = MODE_MIX, tensor_scale: torch.T
     _check_x(x)
     rows, K = x.shape
     q = out if out is not None else empty_qtensor(rows, K, x.device)
+    _check_qtensor(q, rows, K, x.device, "out")
+    _check_given_scale(tensor_scale)
     given = tensor_scale is not None
     if given:
         q.tensor_scale.copy_(tensor_scale.reshape(1))
     ws = None
     if not given:
         ws = workspace if workspace is not None else torch.empty(1, dtype=torch.int32, device=x.device)
+        _check_workspace(ws, x.device)
     st = lib().mixfp4_quantize(_ptr(x), DTYPE_BF16, rows, K, x.stride(0), _ptr(q.codes), _ptr(q.scales),
                                _ptr(q.tensor_scale), _ptr(ws), int(mode),
                                SCALE_GIVEN if given else SCALE_COMPUTE, _stream(stream))
@@ -165,12 +227,15 @@ def mixfp4_quantize_rht(x: torch.Tensor, signs: torch.Tensor | None = None, mode
     _check_signs(signs)
     rows, K = x.shape
     q = out if out is not None else empty_qtensor(rows, K, x.device)
+    _check_qtensor(q, rows, K, x.device, "out")
+    _check_given_scale(tensor_scale)
     given = tensor_scale is not None
     if given:
         q.tensor_scale.copy_(tensor_scale.reshape(1))
     ws = None
     if not given:
         ws = workspace if workspace is not None else torch.empty(1, dtype=torch.int32, device=x.device)
+        _check_workspace(ws, x.device)
     st = lib().mixfp4_quantize_rht(_ptr(x), DTYPE_BF16, rows, K, x.stride(0), _ptr(signs), _ptr(q.codes),
                                    _ptr(q.scales), _ptr(q.tensor_scale), _ptr(ws), int(mode),
                                    SCALE_GIVEN if given else SCALE_COMPUTE, _stream(stream))
@@ -187,12 +252,15 @@ def mixfp4_quantize_colwise(x: torch.Tensor, mode: int = MODE_MIX, tensor_scale:
     _check_x(x)
     R, C = x.shape
     q = out if out is not None else empty_qtensor(C, R, x.device)
+    _check_qtensor(q, C, R, x.device, "out")
+    _check_given_scale(tensor_scale)
     given = tensor_scale is not None
     if given:
         q.tensor_scale.copy_(tensor_scale.reshape(1))
     ws = None
     if not given:
         ws = workspace if workspace is not None else torch.empty(1, dtype=torch.int32, device=x.device)
+        _check_workspace(ws, x.device)
     st = lib().mixfp4_quantize_colwise(_ptr(x), DTYPE_BF16, R, C, x.stride(0), _ptr(q.codes), _ptr(q.scales),
                                        _ptr(q.tensor_scale), _ptr(ws), int(mode),
                                        SCALE_GIVEN if given else SCALE_COMPUTE, _stream(stream))
@@ -209,12 +277,15 @@ def mixfp4_quantize_colwise_rht(x: torch.Tensor, signs: torch.Tensor | None = No
     _check_signs(signs)
     R, C = x.shape
     q = out if out is not None else empty_qtensor(C, R, x.device)
+    _check_qtensor(q, C, R, x.device, "out")
+    _check_given_scale(tensor_scale)
     given = tensor_scale is not None
     if given:
         q.tensor_scale.copy_(tensor_scale.reshape(1))
     ws = None
     if not given:
         ws = workspace if workspace is not None else torch.empty(1, dtype=torch.int32, device=x.device)
+        _check_workspace(ws, x.device)
     st = lib().mixfp4_quantize_colwise_rht(_ptr(x), DTYPE_BF16, R, C, x.stride(0), _ptr(signs), _ptr(q.codes),
                                            _ptr(q.scales), _ptr(q.tensor_scale), _ptr(ws), int(mode),
                                            SCALE_GIVEN if given else SCALE_COMPUTE, _stream(stream))
@@ -230,12 +301,15 @@ def mixfp4_quantize_sr(x: torch.Tensor, seed: int, offset: int = 0, mode: int = 
     _check_x(x)
     rows, K = x.shape
     q = out if out is not None else (empty_qtensor(K, rows, x.device) if colwise else empty_qtensor(rows, K, x.device))
+    _check_qtensor(q, K if colwise else rows, rows if colwise else K, x.device, "out")
+    _check_given_scale(tensor_scale)
     given = tensor_scale is not None
     if given:
         q.tensor_scale.copy_(tensor_scale.reshape(1))
     ws = None
     if not given:
         ws = workspace if workspace is not None else torch.empty(1, dtype=torch.int32, device=x.device)
+        _check_workspace(ws, x.device)
     fn = lib().mixfp4_quantize_colwise_sr if colwise else lib().mixfp4_quantize_sr
     st = fn(_ptr(x), DTYPE_BF16, rows, K, x.stride(0), _ptr(q.codes), _ptr(q.scales), _ptr(q.tensor_scale),
             _ptr(ws), int(mode), SCALE_GIVEN if given else SCALE_COMPUTE, int(seed) & (2 ** 64 - 1),
@@ -252,12 +326,15 @@ def mixfp4_quantize_2d(x: torch.Tensor, mode: int = MODE_MIX, tensor_scale: torc
     _check_x(x)
     rows, K = x.shape
     q = out if out is not None else empty_qtensor(rows, K, x.device)
+    _check_qtensor(q, rows, K, x.device, "out")
+    _check_given_scale(tensor_scale)
     given = tensor_scale is not None
     if given:
         q.tensor_scale.copy_(tensor_scale.reshape(1))
     ws = None
     if not given:
         ws = workspace if workspace is not None else torch.empty(1, dtype=torch.int32, device=x.device)
+        _check_workspace(ws, x.device)
     st = lib().mixfp4_quantize_2d(_ptr(x), DTYPE_BF16, rows, K, x.stride(0), _ptr(q.codes), _ptr(q.scales),
                                   _ptr(q.tensor_scale), _ptr(ws), int(mode),
                                   SCALE_GIVEN if given else SCALE_COMPUTE, _stream(stream))
@@ -268,9 +345,12 @@ def mixfp4_quantize_2d(x: torch.Tensor, mode: int = MODE_MIX, tensor_scale: torc
 def mixfp4_transpose_2d(q: QTensor, out: QTensor | None = None, stream=None) -> QTensor:
     """The transpose of a 2D-quantized tensor (rows and K multiples of 16);
     the tensor scale is shared with the input."""
+    _check_operand(q, "q")
     t = out if out is not None else QTensor(
         torch.empty(q.K, q.rows // 2, dtype=torch.uint8, device=q.codes.device),
         torch.empty(q.K, q.rows // 16, dtype=torch.uint8, device=q.codes.device), q.tensor_scale)
+    _check_u8(t.codes, (q.K, q.rows // 2), q.codes.device, "out.codes")
+    _check_u8(t.scales, (q.K, q.rows // 16), q.codes.device, "out.scales")
     st = lib().mixfp4_transpose_2d(_ptr(q.codes), _ptr(q.scales), q.rows, q.K, _ptr(t.codes), _ptr(t.scales),
                                    _stream(stream))
     _check("mixfp4_transpose_2d", st)
@@ -290,14 +370,17 @@ def mixfp4_fake_quantize(x: torch.Tensor, candidates: int, block: int = 16, out_
     _require(block in (8, 16, 32, 64), "block must be 8, 16, 32 or 64")
     rows, K = x.shape
     o = out if out is not None else torch.empty(rows, K, dtype=out_dtype, device=x.device)
+    _check_dev(o, x.device, "out")
     _require(o.dtype == out_dtype and o.dim() == 2 and o.shape == x.shape and o.stride(1) == 1,
              "out must be a [rows, K] tensor of out_dtype with unit column stride")
     ch = None
     if want_choice:
         ch = choice if choice is not None else torch.empty(rows, K // block, dtype=torch.uint8,
                                                            device=x.device)
+        _check_dev(ch, x.device, "choice")
         _require(ch.dtype == torch.uint8 and ch.is_contiguous() and ch.numel() == rows * (K // block),
                  "choice must be a dense uint8 [rows, K / block] tensor")
+    _check_given_scale(tensor_scale)
     ts = torch.empty(1, dtype=torch.float32, device=x.device)
     given = tensor_scale is not None
     if given:
@@ -305,6 +388,7 @@ def mixfp4_fake_quantize(x: torch.Tensor, candidates: int, block: int = 16, out_
     ws = None
     if not given:
         ws = workspace if workspace is not None else torch.empty(1, dtype=torch.int32, device=x.device)
+        _check_workspace(ws, x.device)
     st = lib().mixfp4_fake_quantize(_ptr(x), DTYPE_BF16, rows, K, x.stride(0), int(candidates), int(block),
                                     _ptr(ts), _ptr(ws), SCALE_GIVEN if given else SCALE_COMPUTE, _ptr(o),
                                     DTYPE_F32 if out_dtype == torch.float32 else DTYPE_BF16, o.stride(0),
@@ -314,7 +398,11 @@ def mixfp4_fake_quantize(x: torch.Tensor, candidates: int, block: int = 16, out_
 
 
 def mixfp4_dequantize(q: QTensor, out: torch.Tensor | None = None, stream=None) -> torch.Tensor:
+    _check_operand(q, "q")
     o = out if out is not None else torch.empty(q.rows, q.K, dtype=torch.float32, device=q.codes.device)
+    _check_dev(o, q.codes.device, "out")
+    _require(o.dtype == torch.float32 and tuple(o.shape) == (q.rows, q.K) and o.is_contiguous(),
+             "out must be a dense float32 [rows, K] tensor")
     st = lib().mixfp4_dequantize(_ptr(q.codes), _ptr(q.scales), _ptr(q.tensor_scale), q.rows, q.K,
                                  _ptr(o), _stream(stream))
     _check("mixfp4_dequantize", st)
@@ -324,9 +412,13 @@ def mixfp4_dequantize(q: QTensor, out: torch.Tensor | None = None, stream=None) 
 def mixfp4_gemm(a: QTensor, b: QTensor, out: torch.Tensor | None = None,
                 status_word: torch.Tensor | None = None, stream=None) -> torch.Tensor:
     """C = A_deq . B_deq^T in fp32; a is M x K, b is N x K."""
-    _require(a.K == b.K, "operands must share K")
+    _check_operand(a, "a")
+    _check_operand(b, "b")
+    _require(a.K == b.K and a.codes.device == b.codes.device, "operands must share K and device")
     M, N, K = a.rows, b.rows, a.K
     C = out if out is not None else torch.empty(M, N, dtype=torch.float32, device=a.codes.device)
+    _check_c(C, M, N, a.codes.device)
+    _check_status(status_word, a.codes.device)
     st = lib().mixfp4_gemm(_ptr(a.codes), _ptr(a.scales), _ptr(a.tensor_scale),
                            _ptr(b.codes), _ptr(b.scales), _ptr(b.tensor_scale),
                            M, N, K, _ptr(C), C.stride(0), _ptr(status_word), _stream(stream))
@@ -357,14 +449,27 @@ def sf_tiled_bytes(rows: int, K: int) -> int:
     return ((rows + 255) // 256) * 256 * (K // 16)
 
 
+def _check_native(t, rows: int, K: int, device, what: str):
+    """Native operand: main (and residual, if any) uint8 [rows, K/2], tiled scales, s32, all on `device`."""
+    _check_u8(t.main, (rows, K // 2), device, f"{what}.main")
+    if t.res is not None:
+        _check_u8(t.res, (rows, K // 2), device, f"{what}.res")
+    _check_dev(t.sf, device, f"{what}.sf")
+    _require(t.sf.dtype == torch.uint8 and t.sf.is_contiguous() and t.sf.numel() >= sf_tiled_bytes(rows, K),
+             f"{what}.sf must be a dense uint8 buffer of at least {sf_tiled_bytes(rows, K)} bytes")
+    _check_scalar_f32(t.tensor_scale, device, f"{what}.tensor_scale")
+
+
 def mixfp4_split_native(q: QTensor, keep_residual: bool = True, out: NativeTensor | None = None,
                         stream=None) -> NativeTensor:
     """Split a MixFP4 tensor into native E2M1 operands.  keep_residual=False
     drops the residual, which is exact only for tensors without E1M2 blocks
     (MODE_E2M1_ONLY).  `out` (with a residual buffer) is reused when given."""
+    _check_operand(q, "q")
     dev = q.codes.device
     if out is not None:
-        _require(out.res is not None and out.main.shape == q.codes.shape, "out must match the operand's shape")
+        _require(out.res is not None, "out must carry a residual buffer")
+        _check_native(out, q.rows, q.K, dev, "out")
         main, res, sf = out.main, out.res, out.sf
     else:
         main = torch.empty_like(q.codes)
@@ -379,9 +484,16 @@ def mixfp4_split_native(q: QTensor, keep_residual: bool = True, out: NativeTenso
 def mixfp4_gemm_native(a: NativeTensor, b: NativeTensor, out: torch.Tensor | None = None,
                        status_word: torch.Tensor | None = None, stream=None) -> torch.Tensor:
     """C = A . B^T on the block-scaled FP4 tensor path; a is M x K, b is N x K."""
+    _require(isinstance(a, NativeTensor) and isinstance(b, NativeTensor) and a.main.dim() == 2
+             and b.main.dim() == 2, "operands must be NativeTensors")
+    dev = a.main.device
+    _check_native(a, a.rows, a.K, dev, "a")
+    _check_native(b, b.rows, b.K, dev, "b")
     _require(a.K == b.K, "operands must share K")
     M, N, K = a.rows, b.rows, a.K
     C = out if out is not None else torch.empty(M, N, dtype=torch.float32, device=a.main.device)
+    _check_c(C, M, N, dev)
+    _check_status(status_word, dev)
     st = lib().mixfp4_gemm_native(_ptr(a.main), _ptr(a.res), _ptr(a.sf), _ptr(a.tensor_scale),
                                   _ptr(b.main), _ptr(b.res), _ptr(b.sf), _ptr(b.tensor_scale),
                                   M, N, K, _ptr(C), C.stride(0), _ptr(status_word), _stream(stream))
@@ -393,9 +505,14 @@ def mixfp4_gemm_native_fewrows(a: QTensor, b: QTensor, out: torch.Tensor | None 
                                status_word: torch.Tensor | None = None, stream=None) -> torch.Tensor:
     """C = A_deq . B_deq^T for a with at most 64 rows, on the block-scaled FP4
     tensor path with the operands split on the fly."""
-    _require(a.K == b.K and a.rows <= 64, "operands must share K, and A have at most 64 rows")
+    _check_operand(a, "a")
+    _check_operand(b, "b")
+    _require(a.K == b.K and a.rows <= 64 and a.codes.device == b.codes.device,
+             "operands must share K and device, and A have at most 64 rows")
     M, N, K = a.rows, b.rows, a.K
     C = out if out is not None else torch.empty(M, N, dtype=torch.float32, device=a.codes.device)
+    _check_c(C, M, N, a.codes.device)
+    _check_status(status_word, a.codes.device)
     st = lib().mixfp4_gemm_native_fewrows(_ptr(a.codes), _ptr(a.scales), _ptr(a.tensor_scale),
                                           _ptr(b.codes), _ptr(b.scales), _ptr(b.tensor_scale),
                                           M, N, K, _ptr(C), C.stride(0), _ptr(status_word), _stream(stream))

@@ -113,3 +113,68 @@ def test_binding_rejects_bad_arguments_before_the_library(monkeypatch):
         ops.mixfp4_fake_quantize(x_cpu, 15, 16)
     with pytest.raises(ValueError):
         ops.mixfp4_quantize_rht(x_cpu, signs=torch.zeros(8, dtype=torch.uint8))
+
+
+def test_binding_rejects_bad_operands_and_outputs(monkeypatch):
+    """GEMM, dequantize, split and quantizer outputs: a CPU operand, a
+    wrong-shape or wrong-dtype C, a short workspace or a mismatched QTensor
+    raise ValueError before any library call (a bad pointer never reaches a
+    kernel).  Device placement is checked first; to reach the shape and dtype
+    checks on this CPU-only host, the device check is relaxed to "all on the
+    same device" for the second half."""
+    import torch
+    from paper_2605_31035_gb300 import ops
+
+    def no_lib():
+        raise AssertionError("the library must not be reached")
+    monkeypatch.setattr(ops, "lib", no_lib)
+
+    def qt(rows, K, dtype=torch.uint8):
+        return ops.QTensor(torch.zeros(rows, K // 2, dtype=dtype), torch.zeros(rows, K // 16, dtype=dtype),
+                           torch.ones(1))
+    a, b = qt(8, 256), qt(16, 256)
+    with pytest.raises(ValueError, match="CUDA"):
+        ops.mixfp4_gemm(a, b)
+    with pytest.raises(ValueError, match="CUDA"):
+        ops.mixfp4_dequantize(a)
+    with pytest.raises(ValueError, match="CUDA"):
+        ops.mixfp4_split_native(a)
+    with pytest.raises(ValueError, match="CUDA"):
+        ops.mixfp4_gemm_native_fewrows(a, b)
+
+    def same_device(t, device, what):
+        ops._require(isinstance(t, torch.Tensor) and t.device == device, f"{what} must be on {device}")
+    monkeypatch.setattr(ops, "_check_dev", same_device)
+    with pytest.raises(ValueError, match="out must be a float32"):
+        ops.mixfp4_gemm(a, b, out=torch.zeros(8, 15))
+    with pytest.raises(ValueError, match="out must be a float32"):
+        ops.mixfp4_gemm(a, b, out=torch.zeros(8, 16, dtype=torch.float64))
+    with pytest.raises(ValueError, match="out must be a float32"):
+        ops.mixfp4_gemm(a, b, out=torch.zeros(16, 8).t())
+    with pytest.raises(ValueError, match="share K"):
+        ops.mixfp4_gemm(a, qt(16, 512))
+    with pytest.raises(ValueError, match="status_word"):
+        ops.mixfp4_gemm(a, b, status_word=torch.zeros(1, dtype=torch.float32))
+    bad = ops.QTensor(a.codes, torch.zeros(8, 8, dtype=torch.uint8), a.tensor_scale)
+    with pytest.raises(ValueError, match="scales"):
+        ops.mixfp4_gemm(bad, b)
+    with pytest.raises(ValueError, match="codes"):
+        ops.mixfp4_gemm(qt(8, 256, torch.int8), b)
+    with pytest.raises(ValueError, match="tensor_scale"):
+        ops.mixfp4_gemm(ops.QTensor(a.codes, a.scales, torch.ones(1, dtype=torch.float64)), b)
+    with pytest.raises(ValueError, match="at most 64 rows"):
+        ops.mixfp4_gemm_native_fewrows(qt(65, 256), b)
+    with pytest.raises(ValueError, match="dense float32"):
+        ops.mixfp4_dequantize(a, out=torch.zeros(8, 128))
+    x = torch.zeros(8, 256, dtype=torch.bfloat16)
+    monkeypatch.setattr(ops, "_check_x", lambda t: None)
+    with pytest.raises(ValueError, match="out.codes"):
+        ops.mixfp4_quantize(x, out=qt(8, 128))
+    with pytest.raises(ValueError, match="workspace"):
+        ops.mixfp4_quantize(x, out=qt(8, 256), workspace=torch.zeros(1, dtype=torch.uint8))
+    with pytest.raises(ValueError, match="tensor_scale"):
+        ops.mixfp4_quantize(x, out=qt(8, 256), tensor_scale=torch.ones(2))
+    with pytest.raises(ValueError, match="out.codes"):
+        ops.mixfp4_quantize_colwise(x, out=qt(8, 256))
+    with pytest.raises(ValueError, match="choice"):
+        ops.mixfp4_fake_quantize(x, 3, 16, choice=torch.zeros(8, 8, dtype=torch.int32))

@@ -1,5 +1,5 @@
 """GPU parity of the candidate-set / block-size quantize-dequantize (reading
-R14; Sec. 2.3 candidate sets, Sec. 5 Table 5 block sizes): outputs (fp32 and
+R14; Sec. 2.4 candidate sets, Sec. 4.3 Table 5 block sizes): outputs (fp32 and
 bf16), per-block choices and the tensor scale bit-exact against the CPU
 oracle, through the C ABI."""
 import numpy as np

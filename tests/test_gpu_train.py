@@ -1,4 +1,4 @@
-"""GPU parity of the training-flow quantizer orientations (Sec. 3.4):
+"""GPU parity of the training-flow quantizer orientations (Sec. 3.2):
 column-wise blocks (WGRAD / DGRAD operands), 2D 16 x 16 weight blocks
 (reading R12) and the transpose of a 2D-quantized tensor, each bit-exact
 against the CPU oracle, plus the GEMMs they feed within the 1e-5 bound.

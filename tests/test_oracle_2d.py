@@ -1,6 +1,6 @@
 """Pins of the training-side quantizer orientations in the oracle.
 
-* quantize_2d (Algorithm 1 with 16 x 16 weight blocks, Sec. 3.4; reading R12)
+* quantize_2d (Algorithm 1 with 16 x 16 weight blocks, Sec. 3.2; reading R12)
   is pinned against the 1D oracle on tiles that reduce to one row (identical
   rows, a single nonzero row), against exact rational arithmetic on small
   dyadic tiles, and by the sign and power-of-two invariances.

@@ -1,5 +1,5 @@
 """Pins of the candidate-set / block-size ablation oracle (reading R14:
-Sec. 2.3 candidate sets with E2M1(4) and E3M0, Sec. 5 Table 5 block sizes).
+Sec. 2.4 candidate sets with E2M1(4) and E3M0, Sec. 4.3 Table 5 block sizes).
 
 What fixes it from outside itself:
 * Eq. 1-2 give the E3M0 codebook (W_E = 3, W_M = 0, bias 3); E2M1(4) reuses
@@ -234,7 +234,7 @@ def test_rejects_bad_arguments():
 
 
 def test_block_size_trends_of_sec5():
-    """Sec. 5 (Table 5 and its discussion): with coarser blocks the E1M2
+    """Sec. 4.3 (Table 5 and its discussion): with coarser blocks the E1M2
     candidate helps less, and E3M0 becomes the more useful extra format.  A
     statistical trend on the synthetic stand-ins (not parity): the MSE ratio
     of {E2M1, E1M2} to NVFP4 rises with g for activations and weights, and on

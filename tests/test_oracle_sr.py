@@ -1,5 +1,5 @@
 """Pins of stochastic rounding in the oracle (reading R13; the paper's SR
-ablation appendix and Sec. 4 pre-training recipe).
+ablation appendix and Sec. 4.2 pre-training recipe).
 
 * The generator: Philox4x32-10 against its published known-answer vectors
   (tests/golden/philox_kat.txt).

@@ -35,7 +35,7 @@ def _ptr(t):
     return ctypes.c_void_p(t.data_ptr())
 
 
-@pytest.mark.parametrize("mode", [0, 1, 2])
+@pytest.mark.parametrize("mode", [0, 1, 2, 3])
 def test_noalloc_matches_workspace_entry_point(mode):
     L = _lib()
     dev = torch.device("cuda:0")
