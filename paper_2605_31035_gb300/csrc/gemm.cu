@@ -7,12 +7,21 @@
 // tensor cores contract f16 x f16 with fp32 accumulation (tcgen05.mma
 // kind::f16, K = 16 per instruction) and the epilogue applies s32A * s32B / 4.
 //
+// Accumulation length.  The tensor cores add each K step's products into the
+// fp32 accumulator with an error that grows with the number of steps added
+// into one accumulator (relative to |A|.|B|, about 1e-6 per 1024 of K on
+// outlier-heavy operands whose outlier channels coincide).  So the work
+// schedule cuts every tile's K into chunks of at most 16 K slices (4096 K):
+// each chunk is accumulated from zero, and the epilogue stores the first
+// chunk of a tile into C and adds the later ones with red.global.add, so the
+// bound no longer depends on K.
+//
 // Work decomposition: persistent CTA pairs (clusters of 2, cta_group::2).  A
 // pair owns 256 x 256 output tiles; each CTA holds 128 rows of A and 128 rows
-// (half) of B.  Tiles of the full waves are dealt whole; when the tile count
-// leaves a partial last wave, that wave's (tile, K slice) units are split
-// evenly over all pairs (stream-K) and their partial sums are added into C
-// with red.global.add after the host zeroed those tiles.  Tiles are numbered
+// (half) of B.  Tiles of the full waves are dealt whole (chunk by chunk);
+// when the tile count leaves a partial last wave, that wave's (tile, K slice)
+// units are split evenly over all pairs (stream-K) and their partial sums are
+// added into C with red.global.add after the host zeroed those tiles.  Tiles are numbered
 // row band by row band (t = mt * ntiles_n + nt).  Decoded A never touches
 // shared memory: it is written to tensor memory (tcgen05.st) and the MMA reads
 // it from there; decoded B goes through shared memory.  Per CTA:
@@ -179,7 +188,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
 mixfp4_gemm_kernel(const __grid_constant__ CUtensorMap tm_ac, const __grid_constant__ CUtensorMap tm_bc,
                    const __grid_constant__ CUtensorMap tm_as, const __grid_constant__ CUtensorMap tm_bs,
                    const float* __restrict__ a_ts, const float* __restrict__ b_ts,
-                   int M, int N, int K, float* __restrict__ C, long long ldc, int dp_tiles,
+                   int M, int N, int K, float* __restrict__ C, long long ldc, int dp_tiles, int chunk_kc,
                    uint32_t* status_word) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -241,7 +250,7 @@ mixfp4_gemm_kernel(const __grid_constant__ CUtensorMap tm_ac, const __grid_const
       int last_it = -1;  // last code-stage use issued (its copies may be in flight)
       int it = 0;
       bool ok = true;
-      Sched sched(cluster_id, nclusters, dp_tiles, ntiles, num_kc);
+      Sched sched(cluster_id, nclusters, dp_tiles, ntiles, num_kc, chunk_kc);
       int t, k0, k1;
       while (ok && sched.next(t, k0, k1)) {
         const int mt = t / ntiles_n, nt = t % ntiles_n;
@@ -279,7 +288,7 @@ mixfp4_gemm_kernel(const __grid_constant__ CUtensorMap tm_ac, const __grid_const
       int d = 0;
       uint32_t dph = 0;
       bool ok = true;
-      Sched sched(cluster_id, nclusters, dp_tiles, ntiles, num_kc);
+      Sched sched(cluster_id, nclusters, dp_tiles, ntiles, num_kc, chunk_kc);
       int t, k0, k1;
       for (int i = 0; ok && sched.next(t, k0, k1); ++i) {
         if (!mbar_wait_cluster(smem_u32(&bars->acc_empty), (i & 1) ^ 1, abort_flag, kWaitLimitNs)) {
@@ -318,7 +327,7 @@ mixfp4_gemm_kernel(const __grid_constant__ CUtensorMap tm_ac, const __grid_const
       int d = 0;
       uint32_t dph = 0;
       bool ok = true;
-      Sched sched(cluster_id, nclusters, dp_tiles, ntiles, num_kc);
+      Sched sched(cluster_id, nclusters, dp_tiles, ntiles, num_kc, chunk_kc);
       int t, k0, k1;
       while (ok && sched.next(t, k0, k1)) {
         for (int st = 0; st < (k1 - k0) * kSub; ++st) {
@@ -348,7 +357,7 @@ mixfp4_gemm_kernel(const __grid_constant__ CUtensorMap tm_ac, const __grid_const
     uint32_t dph = 0;
     int it = 0;
     bool ok = true;
-    Sched sched(cluster_id, nclusters, dp_tiles, ntiles, num_kc);
+    Sched sched(cluster_id, nclusters, dp_tiles, ntiles, num_kc, chunk_kc);
     int t, k0, k1;
     while (ok && sched.next(t, k0, k1)) {
       for (int kc = k0; kc < k1 && ok; ++kc, ++it) {
@@ -430,10 +439,12 @@ mixfp4_gemm_kernel(const __grid_constant__ CUtensorMap tm_ac, const __grid_const
     const uint32_t acc_empty_leader = mapa_shared(smem_u32(&bars->acc_empty), 0);
     const uint32_t stage = sbase + OFF_EPI + (uint32_t)(warp - kFirstEpi) * EPI_BYTES;
     const uint32_t wr_row = stage + (uint32_t)lane * 64u, wr_swz = (uint32_t)(lane >> 1) & 3u;
-    Sched sched(cluster_id, nclusters, dp_tiles, ntiles, num_kc);
+    Sched sched(cluster_id, nclusters, dp_tiles, ntiles, num_kc, chunk_kc);
     int t, k0, k1;
     for (int i = 0; sched.next(t, k0, k1); ++i) {
-      const bool whole = k0 == 0 && k1 == num_kc;  // else: add into C (zeroed by the host)
+      // The first chunk of a whole tile is stored; every other segment is
+      // added into C (after that chunk, or into rows the host zeroed).
+      const bool whole = sched.store;
       const bool acc_ok = mbar_wait_cluster(smem_u32(&bars->acc_full), i & 1, abort_flag, kWaitLimitNs);
       tc_fence_after();
       // tcgen05.ld is warp-collective: decide for the whole warp.
@@ -510,7 +521,10 @@ mixfp4_gemm_kernel(const __grid_constant__ CUtensorMap tm_ac, const __grid_const
 // Work = (weight tile of 256 rows, 256-wide K slice) units split evenly over
 // all CTAs (stream-K); each CTA adds its partial tiles into C (zeroed first)
 // with red.global.add, so bits depend on the summation order but every result
-// is within the fp32-accumulation bound.
+// is within the fp32-accumulation bound.  A CTA's run of consecutive K slices
+// of one weight tile is cut every `chunk_units` slices (2048 K), so no TMEM
+// accumulation is longer than that (see the accumulation-length note at the
+// top of this file).
 // Per CTA: warp 0 TMA, warp 1 TMEM allocator + MMA thread, warps 2-17 weight
 // decoders (two threads per weight row, one 32-code chunk each per stage),
 // warps 18-21 X decoders (warp % 4 = TMEM lane quarter = 32 X rows), warps
@@ -561,7 +575,8 @@ __global__ void __launch_bounds__(kThreads, 1)
 mixfp4_gemm_skinny_kernel(const __grid_constant__ CUtensorMap tm_wc, const __grid_constant__ CUtensorMap tm_xc,
                           const __grid_constant__ CUtensorMap tm_ws, const __grid_constant__ CUtensorMap tm_xs,
                           const float* __restrict__ a_ts, const float* __restrict__ b_ts, int Mx, int N, int K,
-                          float* __restrict__ C, long long ldc, uint32_t idesc, uint32_t* status_word) {
+                          float* __restrict__ C, long long ldc, uint32_t idesc, int chunk_units,
+                          uint32_t* status_word) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   Bars* bars = reinterpret_cast<Bars*>(smem + OFF_BAR);
@@ -573,6 +588,14 @@ mixfp4_gemm_skinny_kernel(const __grid_constant__ CUtensorMap tm_wc, const __gri
   const long long units = (long long)((N + BN - 1) / BN) * num_kc;
   const long long u_begin = units * blockIdx.x / gridDim.x, u_end = units * (blockIdx.x + 1) / gridDim.x;
   const uint32_t stage_bytes = W_CODE + W_SCALE + (uint32_t)nx * (BKC / 2 + BKC / 16);
+  // End of the accumulation run that starts at unit u: the end of its weight
+  // tile, of this CTA's units, or of its accumulation chunk, whichever is first.
+  auto run_end_of = [&](long long u) {
+    long long e = (u / num_kc + 1) * num_kc;
+    if (e > u_end) e = u_end;
+    if (e > u + chunk_units) e = u + chunk_units;
+    return e;
+  };
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kCodeStages; ++s) {
@@ -648,8 +671,7 @@ mixfp4_gemm_skinny_kernel(const __grid_constant__ CUtensorMap tm_wc, const __gri
       // carry: shared addresses stay below 256 KiB).
       const uint64_t bdesc0 = smem_desc_noswizzle(sbase + OFF_DEC, kLBO, kSBO);
       for (long long u = u_begin; u < u_end && ok;) {
-        const int wt = (int)(u / num_kc);
-        const long long run_end = (long long)(wt + 1) * num_kc < u_end ? (long long)(wt + 1) * num_kc : u_end;
+        const long long run_end = run_end_of(u);
         if (!mbar_wait(smem_u32(&bars->acc_empty), (ntile & 1) ^ 1, abort_flag, kWaitLimitNs)) {
           fail(2u);
           break;
@@ -759,7 +781,7 @@ mixfp4_gemm_skinny_kernel(const __grid_constant__ CUtensorMap tm_wc, const __gri
     int ntile = 0;
     for (long long u = u_begin; u < u_end; ++ntile) {
       const int wt = (int)(u / num_kc);
-      u = (long long)(wt + 1) * num_kc < u_end ? (long long)(wt + 1) * num_kc : u_end;
+      u = run_end_of(u);
       const bool acc_ok = mbar_wait(smem_u32(&bars->acc_full), ntile & 1, abort_flag, kWaitLimitNs);
       tc_fence_after();
       const bool go = __all_sync(0xffffffffu, acc_ok && !*abort_flag);
@@ -810,6 +832,7 @@ mixfp4_gemm_skinny_kernel(const __grid_constant__ CUtensorMap tm_wc, const __gri
 
 }  // namespace skinny
 
+
 }  // namespace
 
 // Launch the pair kernel with tile width kTileN over `tiles` tiles, the first
@@ -845,8 +868,8 @@ int launch_pair(const uint8_t* a_codes, const uint8_t* a_scales, const float* a_
   // tail of the kernel before it; the TMA producer and the epilogue wait for
   // that kernel before they read the operands or the tensor scales.
   if (launch_pdl(mixfp4_gemm_kernel<kTileN>, (unsigned)(2 * clusters), kThreads, SMEM_ALLOC, stream, tac, tbc, tas,
-                 tbs, a_ts, b_ts, (int)M, (int)N, (int)K, C, (long long)ldc, (int)dp_tiles, status_word) !=
-      cudaSuccess)
+                 tbs, a_ts, b_ts, (int)M, (int)N, (int)K, C, (long long)ldc, (int)dp_tiles, kAccumChunkK / BKC,
+                 status_word) != cudaSuccess)
     return MIXFP4_ERR_CUDA;
   return MIXFP4_OK;
 }
@@ -877,7 +900,7 @@ int launch_gemm(const uint8_t* a_codes, const uint8_t* a_scales, const float* a_
     if (grid > units) grid = units;
     skinny::mixfp4_gemm_skinny_kernel<<<(unsigned)grid, skinny::kThreads, skinny::SMEM_ALLOC, stream>>>(
         twc, txc, tws, txs, a_ts, b_ts, (int)M, (int)N, (int)K, C, (long long)ldc,
-        idesc_f16_f32(128, skinny::BN), status_word);
+        idesc_f16_f32(128, skinny::BN), kAccumChunkK / skinny::BKC, status_word);
     return MIXFP4_OK;
   }
   // Tile width: the pair tiles are 256 rows of A by kTileN rows of B.  With

@@ -20,7 +20,8 @@
 // multiple of 256 with zero bytes.
 //
 // nvf4_gemm_kernel: persistent CTA pairs (cta_group::2), 256 x 256 output
-// tiles, the stream-K split of the last wave as in the decoding kernel.  Per
+// tiles, the stream-K split of the last wave and the accumulation chunks of
+// at most 4096 K (later chunks added into C) as in the decoding kernel.  Per
 // CTA:
 //   warp 0      TMA producer: the main (and residual) code tiles of its 128
 //               rows of A and 128 rows of B for a 256-wide K slice (128-byte
@@ -179,7 +180,7 @@ nvf4_gemm_kernel(const __grid_constant__ CUtensorMap tm_am, const __grid_constan
                  const __grid_constant__ CUtensorMap tm_bm, const __grid_constant__ CUtensorMap tm_br,
                  const uint8_t* __restrict__ a_sf, const uint8_t* __restrict__ b_sf, const float* __restrict__ a_ts,
                  const float* __restrict__ b_ts, int M, int N, int K, float* __restrict__ C, long long ldc,
-                 int dp_tiles, uint32_t* status_word) {
+                 int dp_tiles, int chunk_kc, uint32_t* status_word) {
   using L = Layout<kARes, kBRes>;
   constexpr int S = L::kStages;
   extern __shared__ uint8_t smem_raw[];
@@ -233,7 +234,7 @@ nvf4_gemm_kernel(const __grid_constant__ CUtensorMap tm_am, const __grid_constan
       griddep_wait();
       int last_it = -1, it = 0;
       bool ok = true;
-      Sched sched(cluster_id, nclusters, dp_tiles, ntiles, num_kc);
+      Sched sched(cluster_id, nclusters, dp_tiles, ntiles, num_kc, chunk_kc);
       int t, k0, k1;
       while (ok && sched.next(t, k0, k1)) {
         const int mt = t / ntiles_n, nt = t % ntiles_n;
@@ -276,7 +277,7 @@ nvf4_gemm_kernel(const __grid_constant__ CUtensorMap tm_am, const __grid_constan
       constexpr uint32_t kIdesc = idesc_nvf4_f32(TILE_M, TILE_N);
       int it = 0;
       bool ok = true;
-      Sched sched(cluster_id, nclusters, dp_tiles, ntiles, num_kc);
+      Sched sched(cluster_id, nclusters, dp_tiles, ntiles, num_kc, chunk_kc);
       int t, k0, k1;
       for (int i = 0; ok && sched.next(t, k0, k1); ++i) {
         if (!mbar_wait_cluster(smem_u32(&bars->acc_empty), (i & 1) ^ 1, abort_flag, kWaitLimitNs)) {
@@ -332,7 +333,7 @@ nvf4_gemm_kernel(const __grid_constant__ CUtensorMap tm_am, const __grid_constan
       const uint32_t ready_leader0 = mapa_shared(smem_u32(&bars->ready[0]), 0);
       int it = 0;
       bool ok = true;
-      Sched sched(cluster_id, nclusters, dp_tiles, ntiles, num_kc);
+      Sched sched(cluster_id, nclusters, dp_tiles, ntiles, num_kc, chunk_kc);
       int t, k0, k1;
       while (ok && sched.next(t, k0, k1)) {
         for (int kc = k0; kc < k1; ++kc, ++it) {
@@ -355,10 +356,12 @@ nvf4_gemm_kernel(const __grid_constant__ CUtensorMap tm_am, const __grid_constan
     const bool vec_ok = ((ldc & 3) == 0) && ((reinterpret_cast<uintptr_t>(C) & 15) == 0);
     const uint32_t acc_empty_leader = mapa_shared(smem_u32(&bars->acc_empty), 0);
     const uint32_t tbase = tmem_base + (uint32_t)(cg * kEpiCols) + ((uint32_t)(q * 32) << 16);
-    Sched sched(cluster_id, nclusters, dp_tiles, ntiles, num_kc);
+    Sched sched(cluster_id, nclusters, dp_tiles, ntiles, num_kc, chunk_kc);
     int t, k0, k1;
     for (int i = 0; sched.next(t, k0, k1); ++i) {
-      const bool whole = k0 == 0 && k1 == num_kc;
+      // The first chunk of a whole tile is stored; every other segment is
+      // added into C (after that chunk, or into rows the host zeroed).
+      const bool whole = sched.store;
       const bool acc_ok = mbar_wait_cluster(smem_u32(&bars->acc_full), i & 1, abort_flag, kWaitLimitNs);
       tc_fence_after();
       const bool go = __all_sync(0xffffffffu, acc_ok && !*abort_flag);
@@ -449,7 +452,7 @@ int launch(const uint8_t* a_main, const uint8_t* a_res, const uint8_t* a_sf, con
   }
   if (launch_pdl(nvf4_gemm_kernel<kARes, kBRes>, (unsigned)(2 * clusters), kThreads, L::SMEM_ALLOC, stream, tam,
                  tar, tbm, tbr, a_sf, b_sf, a_ts, b_ts, (int)M, (int)N, (int)K, C, (long long)ldc, (int)dp_tiles,
-                 status_word) != cudaSuccess)
+                 kAccumChunkK / BKC, status_word) != cudaSuccess)
     return MIXFP4_ERR_CUDA;
   return MIXFP4_OK;
 }
@@ -550,7 +553,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 nvf4_fewrows_kernel(const __grid_constant__ CUtensorMap tm_wc, const __grid_constant__ CUtensorMap tm_ws,
                     const __grid_constant__ CUtensorMap tm_xc, const __grid_constant__ CUtensorMap tm_xs,
                     const float* __restrict__ a_ts, const float* __restrict__ b_ts, int Mx, int nx, int N, int K,
-                    float* __restrict__ C, long long ldc, uint32_t* status_word) {
+                    float* __restrict__ C, long long ldc, int chunk_units, uint32_t* status_word) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   Bars* bars = reinterpret_cast<Bars*>(smem);
@@ -559,6 +562,15 @@ nvf4_fewrows_kernel(const __grid_constant__ CUtensorMap tm_wc, const __grid_cons
   const int num_kc = K / BKC;
   const long long units = (long long)((N + WR - 1) / WR) * num_kc;
   const long long u_begin = units * blockIdx.x / gridDim.x, u_end = units * (blockIdx.x + 1) / gridDim.x;
+  // End of the accumulation run that starts at unit u: the end of its weight
+  // tile, of this CTA's units, or of its accumulation chunk (chunk_units K
+  // slices), whichever is first.
+  auto run_end_of = [&](long long u) {
+    long long e = (u / num_kc + 1) * num_kc;
+    if (e > u_end) e = u_end;
+    if (e > u + chunk_units) e = u + chunk_units;
+    return e;
+  };
   const uint32_t stage_bytes = WR * ROWB + WR * 16 + (uint32_t)nx * (ROWB + 16);
   const int CS = code_stage_bytes(nx), NCS = code_stages(nx);
   const uint32_t OFF_XS = (uint32_t)(OFF_XC + nx * ROWB);
@@ -641,8 +653,7 @@ nvf4_fewrows_kernel(const __grid_constant__ CUtensorMap tm_wc, const __grid_cons
       int it = 0, run = 0;
       bool ok = true;
       for (long long u = u_begin; u < u_end && ok; ++run) {
-        const int g = (int)(u / num_kc);
-        const long long run_end = (long long)(g + 1) * num_kc < u_end ? (long long)(g + 1) * num_kc : u_end;
+        const long long run_end = run_end_of(u);
         if (!mbar_wait(smem_u32(&bars->acc_empty), (run & 1) ^ 1, abort_flag, kWaitLimitNs)) {
           fail(2u);
           break;
@@ -781,7 +792,7 @@ nvf4_fewrows_kernel(const __grid_constant__ CUtensorMap tm_wc, const __grid_cons
     int run = 0;
     for (long long u = u_begin; u < u_end; ++run) {
       const int g = (int)(u / num_kc);
-      u = (long long)(g + 1) * num_kc < u_end ? (long long)(g + 1) * num_kc : u_end;
+      u = run_end_of(u);
       const bool acc_ok = mbar_wait(smem_u32(&bars->acc_full), run & 1, abort_flag, kWaitLimitNs);
       tc_fence_after();
       const bool go = __all_sync(0xffffffffu, acc_ok && !*abort_flag);
@@ -854,7 +865,7 @@ int launch(const uint8_t* a_codes, const uint8_t* a_scales, const float* a_ts, c
   int64_t grid = num_sms();
   if (grid > units) grid = units;
   if (launch_pdl(nvf4_fewrows_kernel, (unsigned)grid, kThreads, smem, stream, twc, tws, txc, txs, a_ts, b_ts,
-                 (int)M, nx, (int)N, (int)K, C, (long long)ldc, status_word) != cudaSuccess)
+                 (int)M, nx, (int)N, (int)K, C, (long long)ldc, kAccumChunkK / BKC, status_word) != cudaSuccess)
     return MIXFP4_ERR_CUDA;
   return MIXFP4_OK;
 }

@@ -85,7 +85,8 @@ def test_stale_traffic_figure_is_dropped(tmp_path, monkeypatch):
     sys.path.insert(0, ROOT)
     bench = importlib.import_module("bench")
     entry = json.load(open(os.path.join(ROOT, "profiles", "ncu_traffic.json")))["gemm_attn"]
-    assert bench.ncu_traffic("gemm_attn", "gemm.cu") == entry["dram_bytes_per_launch"]
+    current = entry["source_sha"] == bench.kernel_hash("gemm.cu")
+    assert bench.ncu_traffic("gemm_attn", "gemm.cu") == (entry["dram_bytes_per_launch"] if current else None)
     fake_root = tmp_path / "r"
     shutil.copytree(os.path.join(ROOT, "profiles"), fake_root / "profiles")
     os.makedirs(fake_root / "paper_2605_31035_gb300" / "csrc")

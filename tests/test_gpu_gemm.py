@@ -110,32 +110,118 @@ def test_strided_output(oracle):
     assert_close(big[:, :200].cpu().numpy(), Cref, A, B)
 
 
-def sampled_check(oracle, qa, qb, nsample=400, seed=0):
-    """Large shapes: compare sampled C entries with float64 dots of the
-    oracle's dequantized rows."""
+def rows_cols_check(oracle, qa, qb, C, rows, cols, block=2048):
+    """Whole rows of C against every column and whole columns against every
+    row: float64 dots of the oracle's dequantized operands, the full operand
+    dequantized block by block to bound host memory."""
     ac, as_, at = qa.codes.cpu().numpy(), qa.scales.cpu().numpy(), qa.tensor_scale.item()
     bc, bs, bt = qb.codes.cpu().numpy(), qb.scales.cpu().numpy(), qb.tensor_scale.item()
-    C = ops().mixfp4_gemm(qa, qb)
-    torch.cuda.synchronize()
-    rng = np.random.default_rng(seed)
     M, N = C.shape
-    ms = np.unique(np.concatenate([[0, M - 1], rng.integers(0, M, 24)]))
-    ns = np.unique(np.concatenate([[0, N - 1], rng.integers(0, N, nsample // 24)]))
-    A = oracle.dequant_rows_f64(ac, as_, at, ms)
-    B = oracle.dequant_rows_f64(bc, bs, bt, ns)
-    Cg = C[torch.from_numpy(ms).to(DEV)][:, torch.from_numpy(ns).to(DEV)].cpu().numpy()
-    return assert_close(Cg, A @ B.T, A, B)
+    rows = np.unique(np.asarray(rows, dtype=np.int64).clip(0, M - 1))
+    cols = np.unique(np.asarray(cols, dtype=np.int64).clip(0, N - 1))
+    C_rows = C[torch.from_numpy(rows).to(C.device)].cpu().numpy()
+    C_cols = C[:, torch.from_numpy(cols).to(C.device)].cpu().numpy()
+    A_r = oracle.dequant_rows_f64(ac, as_, at, rows)
+    B_c = oracle.dequant_rows_f64(bc, bs, bt, cols)
+    worst = 0.0
+    for n0 in range(0, N, block):
+        B_blk = oracle.dequant_rows_f64(bc, bs, bt, range(n0, min(N, n0 + block)))
+        worst = max(worst, assert_close(C_rows[:, n0:n0 + block], A_r @ B_blk.T, A_r, B_blk))
+    for m0 in range(0, M, block):
+        A_blk = oracle.dequant_rows_f64(ac, as_, at, range(m0, min(M, m0 + block)))
+        worst = max(worst, assert_close(C_cols[m0:m0 + block], A_blk @ B_c.T, A_blk, B_c))
+    return worst
+
+
+def boundary_indices(n, tile_widths=(224, 192, 256), extra=16, seed=0):
+    """First and last index, both sides of every candidate tile edge near the
+    start and the end, plus random indices."""
+    rng = np.random.default_rng(seed)
+    idx = [0, n - 1]
+    for w in tile_widths:
+        for e in (w, 2 * w, (n // w) * w):
+            idx += [e - 1, e]
+    return np.concatenate([np.array(idx), rng.integers(0, n, extra)])
 
 
 @pytest.mark.slow
 @pytest.mark.parametrize("name", ["attn", "mlp", "decode", "hadamard"])
 def test_full_size_workloads(oracle, name):
+    """Every linear of the workload at full size, in the launch configuration
+    the bench times: whole rows of C (every column) and whole columns (every
+    row) against float64 from the oracle's dequantized operands."""
     wl = synth.workloads()[name]
     o = ops()
     for lin in wl.linears:
         qa = o.mixfp4_quantize(lin.make_x().to(DEV))
         qb = o.mixfp4_quantize(lin.make_w().to(DEV))
-        sampled_check(oracle, qa, qb, seed=sum(map(ord, lin.name)))
+        status = torch.zeros(1, dtype=torch.int32, device=DEV)
+        C = o.mixfp4_gemm(qa, qb, status_word=status)
+        torch.cuda.synchronize()
+        assert status.item() == 0
+        seed = sum(map(ord, lin.name))
+        rows_cols_check(oracle, qa, qb, C, boundary_indices(lin.M, seed=seed), boundary_indices(lin.N, seed=seed + 1))
+
+
+def coinciding_outliers(M, N, K, seed):
+    """Activations and weights whose x50 outlier channels are the same 1 % of
+    K (weights without row scales): the products of two outliers dominate
+    every dot product, so the accumulator runs far from the typical partial
+    sum -- the case in which a long fp32 accumulation on the tensor cores
+    drifts furthest (relative to |A|.|B|) from the exact result."""
+    x = synth.activations(M, K, seed, 3000 + K)
+    w = synth.weights(N, K, seed + 100, 0.02, None, 3000 + K)
+    return x, w
+
+
+@pytest.mark.parametrize("K", [14336, 28672])
+@pytest.mark.parametrize("M", [256, 16, 600])
+def test_long_k_accumulation_bound(oracle, M, K):
+    """Long reductions on outlier-heavy operands stay within 1e-5 of |A|.|B|:
+    the GEMMs cut every TMEM accumulation into chunks of at most 4096 K and
+    add the chunks into C in fp32.  M = 256 and 600 take the CTA-pair kernel
+    (600: ragged, several tiles), M = 16 the few-row kernel; the native FP4
+    GEMM (and, for M = 16, its few-row form) on the same operands; every
+    element of C is checked."""
+    N = 512
+    x, w = coinciding_outliers(M, N, K, 9500 + K + M)
+    o = ops()
+    qa, qb = o.mixfp4_quantize(x.to(DEV)), o.mixfp4_quantize(w.to(DEV))
+    status = torch.zeros(1, dtype=torch.int32, device=DEV)
+    C = o.mixfp4_gemm(qa, qb, status_word=status)
+    torch.cuda.synchronize()
+    assert status.item() == 0
+    A = oracle.dequant_rows_f64(qa.codes.cpu().numpy(), qa.scales.cpu().numpy(), qa.tensor_scale.item(), range(M))
+    B = oracle.dequant_rows_f64(qb.codes.cpu().numpy(), qb.scales.cpu().numpy(), qb.tensor_scale.item(), range(N))
+    Cref = A @ B.T
+    assert_close(C.cpu().numpy(), Cref, A, B)
+    # The native block-scaled FP4 path accumulates on the same tensor cores.
+    Cn = o.mixfp4_gemm_native(o.mixfp4_split_native(qa), o.mixfp4_split_native(qb), status_word=status)
+    torch.cuda.synchronize()
+    assert status.item() == 0
+    assert_close(Cn.cpu().numpy(), Cref, A, B)
+    if M <= 64:
+        Cf = o.mixfp4_gemm_native_fewrows(qa, qb, status_word=status)
+        torch.cuda.synchronize()
+        assert status.item() == 0
+        assert_close(Cf.cpu().numpy(), Cref, A, B)
+
+
+@pytest.mark.slow
+def test_long_k_full_size_down_projection(oracle):
+    """The MLP down projection shape (4096 x 4096, K = 14336) with coinciding
+    outlier channels: whole rows and columns of C, including the stream-K
+    tail and the four accumulation chunks of every whole tile."""
+    M = N = 4096
+    K = 14336
+    x, w = coinciding_outliers(M, N, K, 9700)
+    o = ops()
+    qa, qb = o.mixfp4_quantize(x.to(DEV)), o.mixfp4_quantize(w.to(DEV))
+    status = torch.zeros(1, dtype=torch.int32, device=DEV)
+    C = o.mixfp4_gemm(qa, qb, status_word=status)
+    torch.cuda.synchronize()
+    assert status.item() == 0
+    rows_cols_check(oracle, qa, qb, C, boundary_indices(M, seed=3), boundary_indices(N, seed=4))
 
 
 def test_stream_k_tail(oracle):
@@ -183,3 +269,21 @@ def test_narrow_tile_widths(oracle, M, N, K):
     A = oracle.dequant_rows_f64(qa.codes.cpu().numpy(), qa.scales.cpu().numpy(), qa.tensor_scale.item(), range(M))
     B = oracle.dequant_rows_f64(qb.codes.cpu().numpy(), qb.scales.cpu().numpy(), qb.tensor_scale.item(), range(N))
     assert_close(C.cpu().numpy(), A @ B.T, A, B)
+
+
+@pytest.mark.slow
+def test_stream_k_chunked_segments(oracle):
+    """126 tiles of 256 x 256 with K = 14336 (56 K slices): on 76 CTA pairs
+    the 50 tiles past the first wave are shared out as about 37 K slices per
+    pair, so stream-K shares cross accumulation-chunk edges (every 16 K
+    slices) and are cut there; whole tiles run as four chunks.  Whole rows
+    and columns are checked."""
+    M, N, K = 768, 10528, 14336
+    x, w = coinciding_outliers(M, N, K, 9800)
+    o = ops()
+    qa, qb = o.mixfp4_quantize(x.to(DEV)), o.mixfp4_quantize(w.to(DEV))
+    status = torch.zeros(1, dtype=torch.int32, device=DEV)
+    C = o.mixfp4_gemm(qa, qb, status_word=status)
+    torch.cuda.synchronize()
+    assert status.item() == 0
+    rows_cols_check(oracle, qa, qb, C, boundary_indices(M, seed=5), boundary_indices(N, seed=6))
