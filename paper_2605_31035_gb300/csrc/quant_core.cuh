@@ -34,6 +34,25 @@ __device__ __forceinline__ float2 kd_consts(float b) {
   return make_float2(zh, __fdiv_rn(__fmaf_rn(-b, zh, 1.0f), b));
 }
 
+// The same pair for a divisor whose (zh, zl) is checked before use (the
+// tensor scale, see markstein_needed): zl by Markstein's correction with the
+// reciprocal zh instead of a correctly rounded division (cheaper on the
+// critical path of every CTA; a zl that were off would only send the tensor
+// to the Markstein path).
+__device__ __forceinline__ float2 kd_consts_checked(float b) {
+  if (!(b > 0.0f)) return make_float2(0.0f, 0.0f);
+  const float zh = __frcp_rn(b);
+  const float r = __fmaf_rn(-b, zh, 1.0f);
+  const float q0 = __fmul_rn(r, zh);
+  return make_float2(zh, __fmaf_rn(__fmaf_rn(-q0, b, r), zh, q0));
+}
+
+// (zh, zl) of the block-scale divisors 6 and 7 (kd_consts(6), kd_consts(7),
+// fixed bit patterns: 6 * RN(1/6) = 1 + 2^-25, so zl = RN(-2^-25 / 6); the
+// pairs are recomputed from their definition by a CPU test).
+constexpr uint32_t kZh6Bits = 0x3e2aaaabu, kZl6Bits = 0xb1aaaaabu;
+constexpr uint32_t kZh7Bits = 0x3e124925u, kZl7Bits = 0xb1db6db7u;
+
 __device__ __forceinline__ uint32_t lo32(u64 v) { return (uint32_t)v; }
 __device__ __forceinline__ uint32_t hi32(u64 v) { return (uint32_t)(v >> 32); }
 
@@ -66,9 +85,9 @@ __device__ __forceinline__ TensorConsts tensor_consts(float* tensor_scale, const
   }
   c.s32 = s32;
   c.r32 = (s32 > 0.0f) ? __frcp_rn(s32) : 0.0f;
-  c.kd32 = kd_consts(s32);
-  c.kd6 = kd_consts(6.0f);
-  c.kd7 = kd_consts(7.0f);
+  c.kd32 = kd_consts_checked(s32);
+  c.kd6 = make_float2(__uint_as_float(kZh6Bits), __uint_as_float(kZl6Bits));
+  c.kd7 = make_float2(__uint_as_float(kZh7Bits), __uint_as_float(kZl7Bits));
   return c;
 }
 
@@ -394,17 +413,21 @@ __device__ __forceinline__ void fill_scale_table(float4* tab) {
 // quotient for all 128 bf16 significands (the quotient scales exactly with
 // x's exponent) and its correction term a*zl stays normal for every quotient
 // that can matter (|a| >= 2^-82; see the tiny-value note): the remainder
-// 1 - s32*zh is 0 or at least 2^-44 in magnitude.  Threads 0..127 check one
-// significand each; every thread of the CTA must call this (it ends with a
-// CTA barrier) and all get the same answer: true = use Markstein's form.
+// 1 - s32*zh is 0 or at least 2^-44 in magnitude.  The reference quotient is
+// Markstein's form, which equals the IEEE quotient for every bf16 numerator
+// significand and every fp32 divisor significand (checked exhaustively on the
+// host).  Threads 0..127 check one significand each; every thread of the CTA
+// must call this (it ends with a CTA barrier) and all get the same answer:
+// true = use Markstein's form.
 __device__ __forceinline__ bool markstein_needed(const TensorConsts& tc) {
   bool kd_ok = true;
   if (threadIdx.x < 128 && !tc.scaled) {
     const float xs = __uint_as_float(0x3F800000u | (threadIdx.x << 16));
-    const u64 q = div_kd2(pack2(xs, xs), pack2(tc.kd32.x, tc.kd32.x), pack2(tc.kd32.y, tc.kd32.y));
+    const u64 x2 = pack2(xs, xs);
+    const u64 q = div_kd2(x2, pack2(tc.kd32.x, tc.kd32.x), pack2(tc.kd32.y, tc.kd32.y));
+    const u64 ref = div_rn2(x2, pack2(-tc.s32, -tc.s32), pack2(tc.r32, tc.r32));
     const float rem = __fmaf_rn(-tc.s32, tc.kd32.x, 1.0f);
-    kd_ok = tc.s32 > 0.0f && lo32(q) == __float_as_uint(__fdiv_rn(xs, tc.s32)) &&
-            (rem == 0.0f || fabsf(rem) >= 0x1p-44f);
+    kd_ok = tc.s32 > 0.0f && lo32(q) == lo32(ref) && (rem == 0.0f || fabsf(rem) >= 0x1p-44f);
   }
   return !__syncthreads_and(kd_ok);
 }

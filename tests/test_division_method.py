@@ -14,9 +14,11 @@ import os
 import shutil
 import subprocess
 
+import numpy as np
 import pytest
 
 HERE = os.path.dirname(os.path.abspath(__file__))
+ROOT = os.path.dirname(HERE)
 
 
 @pytest.mark.skipif(shutil.which("gcc") is None, reason="needs gcc")
@@ -47,3 +49,32 @@ def test_known_divisor_division_matches_ieee(tmp_path):
     assert len(lines) == 3 and all(l.endswith("mismatches=0") for l in lines), res.stdout
     rejected = int(res.stdout.split("rejected=")[1].split()[0])
     assert 0 < rejected < 1000, res.stdout  # a handful of s32 significands fall back to Markstein
+
+
+def _rn32_bits(x):
+    """Binary32 nearest to the rational x (ties to even), as bits."""
+    from fractions import Fraction
+    import struct
+    f = np.float32(float(x))
+    cands = [np.nextafter(f, np.float32(-np.inf)), f, np.nextafter(f, np.float32(np.inf))]
+    bits = [struct.unpack("<I", struct.pack("<f", c))[0] for c in cands]
+    best = min(range(3), key=lambda i: (abs(Fraction(float(cands[i])) - x), bits[i] & 1))
+    return bits[best]
+
+
+def test_block_scale_divisor_constants():
+    """The fixed (zh, zl) pairs of the divisors 6 and 7 in quant_core.cuh are
+    RN(1/b) and RN(RN(1 - b zh) / b), recomputed here in exact rational
+    arithmetic."""
+    import re
+    import struct
+    from fractions import Fraction
+    src = open(os.path.join(ROOT, "paper_2605_31035_gb300", "csrc", "quant_core.cuh")).read()
+    for b in (6, 7):
+        zh_bits = int(re.search(rf"kZh{b}Bits = (0x[0-9a-f]+)u", src).group(1), 16)
+        zl_bits = int(re.search(rf"kZl{b}Bits = (0x[0-9a-f]+)u", src).group(1), 16)
+        assert zh_bits == _rn32_bits(Fraction(1, b))
+        zh = Fraction(struct.unpack("<f", struct.pack("<I", zh_bits))[0])
+        r_bits = _rn32_bits(1 - b * zh)
+        r = Fraction(struct.unpack("<f", struct.pack("<I", r_bits))[0])
+        assert zl_bits == _rn32_bits(r / b)
