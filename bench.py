@@ -364,6 +364,7 @@ def run_ours(args):
     e2e_value = job_rate(e2e_steps * flops, world, e2e_ms) / 1e12
 
     configs = None if args.no_configs else config_gemms(dev, flush, stream, pk["bf16_tflops"])
+    sweep = None if args.no_sweep else quantizer_sweep(dev, flush, stream, pk["hbm_gbs"])
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -432,6 +433,7 @@ def run_ours(args):
                     "ms": round(rht_ms, 4),
                     "alg_gbs": round(xs_numel * QUANT_BYTES_PER_ELEM / (rht_ms * 1e-3) / 1e9, 1)}}},
         "configs_gemm": configs,
+        "quantizer_sweep": sweep,
         "clocks": clocks,
         "e2e": {"value": round(e2e_value, 2), "unit": "TFLOP/s",
                 "h2d_bytes_per_step": x_host.numel() * 2, "d2h_bytes_per_step": c_host[0].numel() * 4,
@@ -441,6 +443,78 @@ def run_ours(args):
     }
     if rank == 0:
         print(json.dumps(out), flush=True)
+
+
+# --------------------------------------------------------------- quantizer sweep
+def gpu_t3(dev, rows: int, K: int, seed: int, outliers: bool = True):
+    """Student-t(3) x 0.5 activations with floor(0.01 K) x50 outlier channels,
+    drawn on the GPU from a seeded generator (the synth.py distribution)."""
+    import math
+    import torch
+    g = torch.Generator(device=dev)
+    g.manual_seed(seed)
+    out = torch.empty(rows, K, dtype=torch.bfloat16, device=dev)
+    step = max(1, (1 << 25) // K)
+    gc = torch.Generator(device="cpu")
+    gc.manual_seed(seed + 1)
+    ch = torch.randperm(K, generator=gc)[:int(math.floor(0.01 * K))].to(dev)
+    for r0 in range(0, rows, step):
+        r1 = min(rows, r0 + step)
+        z = torch.randn(4, r1 - r0, K, device=dev, generator=g)
+        v = z[0] / torch.sqrt((z[1] * z[1] + z[2] * z[2] + z[3] * z[3]) / 3.0) * 0.5
+        if outliers:
+            v[:, ch] *= 50.0
+        out[r0:r1] = v.to(torch.bfloat16)
+    return out
+
+
+def quant_rates(x, flush, stream, hbm_gbs, reps=10):
+    """Quantizer rates on x: MixFP4 and E2M1-only (NVFP4) modes, the quantize
+    kernel alone (tensor scale given) and with the amax pass; L2 flushed
+    before every launch.  GB/s counts the algorithmic 2.5625 B/element."""
+    import torch
+    from paper_2605_31035_gb300 import ops
+    dev = x.device
+    q = ops.empty_qtensor(x.shape[0], x.shape[1], dev)
+    ws = torch.empty(1, dtype=torch.int32, device=dev)
+    ops.mixfp4_quantize(x, out=q, workspace=ws)
+    given = q.tensor_scale.clone()
+
+    def timed(fn):
+        for _ in range(3):
+            fn()
+        evs = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(reps)]
+        for e in evs:
+            flush()
+            e[0].record(stream)
+            fn()
+            e[1].record(stream)
+        torch.cuda.synchronize(dev)
+        return statistics.median(a.elapsed_time(b) for a, b in evs)
+
+    n = x.numel()
+    rec = {"elements": n}
+    for mname, mode in (("mixfp4", ops.MODE_MIX), ("e2m1_only", ops.MODE_E2M1_ONLY)):
+        for sname, fn in (("given_scale", lambda: ops.mixfp4_quantize(x, mode, out=q, tensor_scale=given)),
+                          ("with_amax", lambda: ops.mixfp4_quantize(x, mode, out=q, workspace=ws))):
+            ms = timed(fn)
+            gbs = n * QUANT_BYTES_PER_ELEM / (ms * 1e-3) / 1e9
+            rec[f"{mname}_{sname}"] = {"us": round(ms * 1e3, 2), "alg_gbs": round(gbs, 1),
+                                       "frac_of_hbm": round(gbs / hbm_gbs, 4)}
+    return rec
+
+
+def quantizer_sweep(dev, flush, stream, hbm_gbs, k_min=20, k_max=30):
+    """The quantizer-only sweep: the attention activation distribution as
+    [2^k / 4096, 4096] for k = k_min..k_max."""
+    import torch
+    out = {}
+    for k in range(k_min, k_max + 1):
+        x = gpu_t3(dev, (1 << k) // 4096, 4096, 5000 + k)
+        out[f"2^{k}"] = quant_rates(x, flush, stream, hbm_gbs, reps=10 if k >= 26 else 20)
+        del x
+        torch.cuda.empty_cache()
+    return out
 
 
 # ------------------------------------------------------ the other configs' GEMMs
@@ -511,8 +585,16 @@ def config_gemms(dev, flush, stream, peak_t):
              ("hadamard_8192", 8192, 8192, 8192, lambda: hadamard(t3(8192, 8192, 17)),
               lambda: hadamard(normal(8192, 8192, 18, 0.02, None, outliers=True)))]
     out = {}
+    hbm = peaks()["hbm_gbs"]
     for name, M, N, K, mx, mw in cases:
-        qx, qw = ops.mixfp4_quantize(mx()), ops.mixfp4_quantize(mw())
+        xin, win = mx(), mw()
+        quant = None
+        if name == "mlp_down":        # the MLP's X' (4096 x 14336), quantized online every call
+            quant = {"x": quant_rates(xin, flush, stream, hbm)}
+        elif name == "hadamard_8192":  # the rotated 8192 x 8192 X and W
+            quant = {"x": quant_rates(xin, flush, stream, hbm), "w": quant_rates(win, flush, stream, hbm)}
+        qx, qw = ops.mixfp4_quantize(xin), ops.mixfp4_quantize(win)
+        del xin, win
         C = torch.empty(M, N, dtype=torch.float32, device=dev)
         fl = 2.0 * M * N * K
         ms = timed(lambda: ops.mixfp4_gemm(qx, qw, out=C))
@@ -532,6 +614,8 @@ def config_gemms(dev, flush, stream, peak_t):
             rec["native_ms"] = round(ms_n, 4)
             rec["native_tflops"] = round(fl / (ms_n * 1e-3) / 1e12, 1)
             del nx, nw
+        if quant is not None:
+            rec["quantizer"] = quant
         out[name] = rec
         del qx, qw, C
         torch.cuda.empty_cache()
@@ -589,7 +673,35 @@ def host_cpu(cpuinfo: str = "/proc/cpuinfo") -> dict:
     return {"nproc": os.cpu_count(), "cpu": model, "arch": platform.machine()}
 
 
+def _oracle_job(job):
+    """One oracle task in a worker process (spawned: it shares nothing with
+    the CUDA context of the bench process).  Returns its seconds."""
+    kind, x_bits, s32, wq = job
+    import oracle
+    t0 = time.perf_counter()
+    xq = oracle.quantize(x_bits, s32=s32)
+    if kind == "layer":
+        oracle.gemm_f64(xq, wq)
+    return time.perf_counter() - t0
+
+
+def oracle_all_cores(kind: str, x_bits, s32: float, wq, nproc: int):
+    """Rows of x_bits split over nproc spawned processes (the oracle itself
+    is serial C); returns (wall seconds, processes)."""
+    import multiprocessing as mp
+    import numpy as np
+    parts = [p for p in np.array_split(x_bits, nproc) if len(p)]
+    with mp.get_context("spawn").Pool(len(parts)) as pool:
+        pool.map(_oracle_job, [("quantize", parts[0][:1], s32, None)] * len(parts))  # workers up and warm
+        t0 = time.perf_counter()
+        pool.map(_oracle_job, [(kind, p, s32, wq) for p in parts])
+        return time.perf_counter() - t0, len(parts)
+
+
 def cpu_baseline(lin, x_cpu, budget_s: float = 15.0):
+    """The oracle on the host cores: the layer (Algorithm 1 on rows of X + the
+    float64 GEMM against pre-quantized rows of W) single-threaded and on all
+    cores (rows split over processes), and Algorithm 1 alone (elements/s)."""
     cap = 2048
     layer = OracleLayer(lin, x_cpu, lin.make_w()[:cap], cap)
     secs, _ = layer.run(1, 64)
@@ -597,10 +709,33 @@ def cpu_baseline(lin, x_cpu, budget_s: float = 15.0):
     n_w = cap
     n_x = max(4, min(512, int(budget_s / max(per_row * n_w, 1e-9))))
     secs, flops = layer.run(n_x, n_w)
-    return {"value": flops / secs / 1e12, "unit": "TFLOP/s", "cores": 1, "kind": "oracle",
-            "sample": f"Algorithm 1 on {n_x} rows of X + float64 GEMM vs {n_w} pre-quantized rows of W "
-                      f"(K={lin.K}), {secs:.1f} s single-threaded",
-            "host": host_cpu()}
+    nproc = os.cpu_count() or 1
+    out = {"value": flops / secs / 1e12, "unit": "TFLOP/s", "cores": 1, "kind": "oracle",
+           "sample": f"Algorithm 1 on {n_x} rows of X + float64 GEMM vs {n_w} pre-quantized rows of W "
+                     f"(K={lin.K}), {secs:.1f} s single-threaded",
+           "host": host_cpu()}
+    wq = (layer.wq[0][:n_w], layer.wq[1][:n_w], layer.wq[2])
+    try:
+        n_all = max(nproc, min(lin.M, n_x * nproc))
+        wall, used = oracle_all_cores("layer", layer.x_bits[:n_all], layer.s32, wq, nproc)
+        out["all_cores"] = {"value": 2.0 * n_all * n_w * lin.K / wall / 1e12, "unit": "TFLOP/s", "cores": used,
+                            "sample": f"{n_all} rows of X vs {n_w} rows of W split over {used} processes, "
+                                      f"{wall:.1f} s"}
+        rows_q = min(lin.M, 256)
+        t0 = time.perf_counter()
+        import oracle
+        oracle.quantize(layer.x_bits[:rows_q], s32=layer.s32)
+        tq = time.perf_counter() - t0
+        n_q = rows_q * lin.K
+        wall_q, used_q = oracle_all_cores("quantize", layer.x_bits, layer.s32, None, nproc)
+        out["quantizer"] = {
+            "unit": "elements/s", "one_core": n_q / tq,
+            "all_cores": lin.M * lin.K / wall_q, "cores": used_q,
+            "sample": f"Algorithm 1 on {rows_q} rows (one core, {tq:.1f} s) and on all {lin.M} rows of X split "
+                      f"over {used_q} processes ({wall_q:.1f} s)"}
+    except Exception as e:  # a reporting extra; never costs the bench line
+        out["all_cores_error"] = repr(e)
+    return out
 
 
 def run_reference(args):
@@ -740,6 +875,7 @@ def main(argv=None):
     ap.add_argument("--cpu-budget", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-configs", action="store_true", help="skip the other configs' GEMM lines")
+    ap.add_argument("--no-sweep", action="store_true", help="skip the quantizer sweep over 2^20..2^30 elements")
     ap.add_argument("--kernel", choices=["gemm", "gemm_native", "gemm_native_fewrows", "split_native", "quantize", "quantize_rht", "quantize_colwise",
                              "quantize_2d", "transpose_2d", "fake_quantize", "quantize_colwise_rht", "quantize_sr",
                              "dequantize"], default=None,

@@ -400,6 +400,27 @@ int mixfp4_version(void);
  */
 int mixfp4_selftest_bounded_wait(uint32_t* status_word, uint64_t limit_ns, void* stream);
 
+/*
+ * mixfp4_selftest_gemm_missed_stage -- check of the failure path of the
+ * CTA-pair GEMM kernel itself (no counterpart in the paper): mixfp4_gemm's
+ * pair kernel (256-wide tiles, any M) runs with every pipeline wait limited
+ * to limit_ns and with the first code stage of every CTA never issued (no
+ * copy, no arrival).  The waits on that stage run out, each role that gives
+ * up ORs its bit into *status_word (1 producer, 2 / 4 MMA thread, 8 drain,
+ * 16 / 32 decoders, 64 epilogue, 128 peer forwarder), raises its CTA's abort
+ * flag, lets the copies and MMAs it issued complete, frees its tensor memory
+ * and exits; C is not written.  Nothing faults or hangs, and the device stays
+ * usable: a later mixfp4_gemm on it runs normally.
+ *
+ * Operands, M, N, K, C, ldc: as mixfp4_gemm (M, N >= 1, K >= 256).
+ * status_word  device, one uint32, 4-byte aligned, required (zeroed first).
+ * limit_ns     1 .. 2e9 (else MIXFP4_ERR_ARG); the call takes a few limit_ns.
+ */
+int mixfp4_selftest_gemm_missed_stage(const uint8_t* a_codes, const uint8_t* a_scales, const float* a_ts,
+                                      const uint8_t* b_codes, const uint8_t* b_scales, const float* b_ts, int64_t M,
+                                      int64_t N, int64_t K, float* C, int64_t ldc, uint32_t* status_word,
+                                      uint64_t limit_ns, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -390,6 +390,25 @@ int mixfp4_gemm_native(const uint8_t* a_main, const uint8_t* a_res, const uint8_
 
 }  // extern "C"
 
+int mixfp4_selftest_gemm_missed_stage(const uint8_t* a_codes, const uint8_t* a_scales, const float* a_ts,
+                                      const uint8_t* b_codes, const uint8_t* b_scales, const float* b_ts, int64_t M,
+                                      int64_t N, int64_t K, float* C, int64_t ldc, uint32_t* status_word,
+                                      uint64_t limit_ns, void* stream) {
+  if (M < 1 || N < 1 || K < 256 || K % 256 != 0 || ldc < N) return MIXFP4_ERR_SHAPE;
+  if (M > (1 << 30) || N > (1 << 30) || K > (1 << 30)) return MIXFP4_ERR_SHAPE;
+  if (limit_ns == 0 || limit_ns > 2000000000ull) return MIXFP4_ERR_ARG;
+  if (!a_codes || !a_scales || !a_ts || !b_codes || !b_scales || !b_ts || !C || !status_word) return MIXFP4_ERR_NULL;
+  if (!aligned(a_codes, 16) || !aligned(a_scales, 16) || !aligned(b_codes, 16) || !aligned(b_scales, 16) ||
+      !aligned(a_ts, 4) || !aligned(b_ts, 4) || !aligned(C, 4) || !aligned(status_word, 4))
+    return MIXFP4_ERR_ALIGN;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (cudaMemsetAsync(status_word, 0, sizeof(uint32_t), s) != cudaSuccess) return MIXFP4_ERR_CUDA;
+  int st = mixfp4::launch_gemm_missed_stage_selftest(a_codes, a_scales, a_ts, b_codes, b_scales, b_ts, M, N, K, C,
+                                                     ldc, status_word, limit_ns, s);
+  if (st) return st;
+  return launch_status();
+}
+
 int mixfp4_selftest_bounded_wait(uint32_t* status_word, uint64_t limit_ns, void* stream) {
   if (!status_word) return MIXFP4_ERR_NULL;
   if (!aligned(status_word, 4)) return MIXFP4_ERR_ALIGN;

@@ -40,8 +40,12 @@
 // TMEM per CTA (512 columns): fp32 accumulator 128 lanes x 256 columns, then
 // kDecStages A stages of 64 columns (128 K of f16 pairs).  The leader's MMA
 // waits for both CTAs' decoders (remote mbarrier arrivals).
-// All pipeline waits are bounded; a wait that gives up records a nonzero
-// status word and the CTA drains and exits without touching C.
+// All pipeline waits are bounded (1 s each, or the self-test's limit); a
+// wait that gives up ORs its role's bit into the status word (1 producer,
+// 2 MMA thread waiting for the accumulator, 4 MMA thread waiting for a
+// decoded stage, 8 final drain, 16 / 32 decoders, 64 epilogue, 128 peer
+// forwarder), raises the CTA's abort flag, and the CTA lets its issued copies
+// and MMAs land, frees TMEM and exits without touching C.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 #include <cuda_runtime.h>
@@ -189,7 +193,7 @@ mixfp4_gemm_kernel(const __grid_constant__ CUtensorMap tm_ac, const __grid_const
                    const __grid_constant__ CUtensorMap tm_as, const __grid_constant__ CUtensorMap tm_bs,
                    const float* __restrict__ a_ts, const float* __restrict__ b_ts,
                    int M, int N, int K, float* __restrict__ C, long long ldc, int dp_tiles, int chunk_kc,
-                   uint32_t* status_word) {
+                   uint32_t* status_word, uint64_t wait_ns, int skip_first_stage) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   Bars* bars = reinterpret_cast<Bars*>(smem + OFF_BAR);
@@ -256,9 +260,12 @@ mixfp4_gemm_kernel(const __grid_constant__ CUtensorMap tm_ac, const __grid_const
         const int mt = t / ntiles_n, nt = t % ntiles_n;
         const int ma = mt * TILE_M + (int)rank * BM, nb = nt * kTileN + (int)rank * kBRows;
         for (int kc = k0; kc < k1; ++kc, ++it) {
+          // Self-test of the failure path: the first code stage is never
+          // issued (no copy, no arrival), so the waits on it run out.
+          if (skip_first_stage && it == 0) continue;
           const int s = it % kCodeStages;
           const uint32_t ph = (it / kCodeStages) & 1;
-          if (!mbar_wait(smem_u32(&bars->code_empty[s]), ph ^ 1, abort_flag, kWaitLimitNs)) {
+          if (!mbar_wait(smem_u32(&bars->code_empty[s]), ph ^ 1, abort_flag, wait_ns)) {
             fail(1u);
             ok = false;
             break;
@@ -277,9 +284,9 @@ mixfp4_gemm_kernel(const __grid_constant__ CUtensorMap tm_ac, const __grid_const
       if (*abort_flag) {
         // Let the copies this thread started land before the CTA may exit.
         for (int u = last_it - kCodeStages + 1; u <= last_it; ++u)
-          if (u >= 0)
+          if (u >= 0 && !(skip_first_stage && u == 0))
             mbar_wait(smem_u32(&bars->code_full[u % kCodeStages]), (uint32_t)((u / kCodeStages) & 1), nullptr,
-                      kWaitLimitNs);
+                      wait_ns);
       }
     }
   } else if (warp == 1) {
@@ -291,14 +298,14 @@ mixfp4_gemm_kernel(const __grid_constant__ CUtensorMap tm_ac, const __grid_const
       Sched sched(cluster_id, nclusters, dp_tiles, ntiles, num_kc, chunk_kc);
       int t, k0, k1;
       for (int i = 0; ok && sched.next(t, k0, k1); ++i) {
-        if (!mbar_wait_cluster(smem_u32(&bars->acc_empty), (i & 1) ^ 1, abort_flag, kWaitLimitNs)) {
+        if (!mbar_wait_cluster(smem_u32(&bars->acc_empty), (i & 1) ^ 1, abort_flag, wait_ns)) {
           fail(2u);
           break;
         }
         tc_fence_after();
         for (int kc = k0; kc < k1 && ok; ++kc) {
           for (int sub = 0; sub < kSub; ++sub) {
-            if (!mbar_wait_cluster(smem_u32(&bars->dec_full[d]), dph, abort_flag, kWaitLimitNs)) {
+            if (!mbar_wait_cluster(smem_u32(&bars->dec_full[d]), dph, abort_flag, wait_ns)) {
               fail(4u);
               ok = false;
               break;
@@ -320,7 +327,7 @@ mixfp4_gemm_kernel(const __grid_constant__ CUtensorMap tm_ac, const __grid_const
       // Every MMA issued above completes before the drain barrier fires; wait
       // for it (ignoring the abort flag) so TMEM is never freed under an MMA.
       mma_commit_pair(smem_u32(&bars->drain), 1);
-      if (!mbar_wait_cluster(smem_u32(&bars->drain), 0, nullptr, kWaitLimitNs)) fail(8u);
+      if (!mbar_wait_cluster(smem_u32(&bars->drain), 0, nullptr, wait_ns)) fail(8u);
     } else if (!leader && lane == 0) {
       // ---------------- forwarder (peer CTA) ----------------
       const uint32_t dec_full_leader0 = mapa_shared(smem_u32(&bars->dec_full[0]), 0);
@@ -331,7 +338,7 @@ mixfp4_gemm_kernel(const __grid_constant__ CUtensorMap tm_ac, const __grid_const
       int t, k0, k1;
       while (ok && sched.next(t, k0, k1)) {
         for (int st = 0; st < (k1 - k0) * kSub; ++st) {
-          if (!mbar_wait(smem_u32(&bars->peer_ready[d]), dph, abort_flag, kWaitLimitNs)) {
+          if (!mbar_wait(smem_u32(&bars->peer_ready[d]), dph, abort_flag, wait_ns)) {
             fail(128u);
             ok = false;
             break;
@@ -363,7 +370,7 @@ mixfp4_gemm_kernel(const __grid_constant__ CUtensorMap tm_ac, const __grid_const
       for (int kc = k0; kc < k1 && ok; ++kc, ++it) {
         const int s = it % kCodeStages;
         const uint32_t ph = (it / kCodeStages) & 1;
-        if (!mbar_wait(smem_u32(&bars->code_full[s]), ph, abort_flag, kWaitLimitNs)) {
+        if (!mbar_wait(smem_u32(&bars->code_full[s]), ph, abort_flag, wait_ns)) {
           fail(16u);
           ok = false;
           break;
@@ -378,7 +385,7 @@ mixfp4_gemm_kernel(const __grid_constant__ CUtensorMap tm_ac, const __grid_const
             const int chunk = sub * kChunksPerSub + part * kChunksPerThread + j;
             c[j] = lds128(st + code_off + (((uint32_t)chunk ^ swz) << 4));
           }
-          if (!mbar_wait_cluster(smem_u32(&bars->dec_empty[d]), dph ^ 1, abort_flag, kWaitLimitNs)) {
+          if (!mbar_wait_cluster(smem_u32(&bars->dec_empty[d]), dph ^ 1, abort_flag, wait_ns)) {
             fail(32u);
             ok = false;
             break;
@@ -445,7 +452,7 @@ mixfp4_gemm_kernel(const __grid_constant__ CUtensorMap tm_ac, const __grid_const
       // The first chunk of a whole tile is stored; every other segment is
       // added into C (after that chunk, or into rows the host zeroed).
       const bool whole = sched.store;
-      const bool acc_ok = mbar_wait_cluster(smem_u32(&bars->acc_full), i & 1, abort_flag, kWaitLimitNs);
+      const bool acc_ok = mbar_wait_cluster(smem_u32(&bars->acc_full), i & 1, abort_flag, wait_ns);
       tc_fence_after();
       // tcgen05.ld is warp-collective: decide for the whole warp.
       const bool go = __all_sync(0xffffffffu, acc_ok && !*abort_flag);
@@ -840,7 +847,8 @@ mixfp4_gemm_skinny_kernel(const __grid_constant__ CUtensorMap tm_wc, const __gri
 template <int kTileN>
 int launch_pair(const uint8_t* a_codes, const uint8_t* a_scales, const float* a_ts, const uint8_t* b_codes,
                 const uint8_t* b_scales, const float* b_ts, int64_t M, int64_t N, int64_t K, float* C, int64_t ldc,
-                uint32_t* status_word, int64_t clusters, int64_t tiles, int64_t dp_tiles, cudaStream_t stream) {
+                uint32_t* status_word, int64_t clusters, int64_t tiles, int64_t dp_tiles, cudaStream_t stream,
+                uint64_t wait_ns = kWaitLimitNs, int skip_first_stage = 0) {
   CUtensorMap tac, tbc, tas, tbs;
   if (!make_map(&tac, a_codes, (uint64_t)K / 2, (uint64_t)M, BKC / 2, BM, CU_TENSOR_MAP_SWIZZLE_128B) ||
       !make_map(&tbc, b_codes, (uint64_t)K / 2, (uint64_t)N, BKC / 2, kTileN / 2, CU_TENSOR_MAP_SWIZZLE_128B) ||
@@ -869,9 +877,24 @@ int launch_pair(const uint8_t* a_codes, const uint8_t* a_scales, const float* a_
   // that kernel before they read the operands or the tensor scales.
   if (launch_pdl(mixfp4_gemm_kernel<kTileN>, (unsigned)(2 * clusters), kThreads, SMEM_ALLOC, stream, tac, tbc, tas,
                  tbs, a_ts, b_ts, (int)M, (int)N, (int)K, C, (long long)ldc, (int)dp_tiles, kAccumChunkK / BKC,
-                 status_word) != cudaSuccess)
+                 status_word, wait_ns, skip_first_stage) != cudaSuccess)
     return MIXFP4_ERR_CUDA;
   return MIXFP4_OK;
+}
+
+// The pair kernel on 256-wide tiles with every pipeline wait limited to
+// wait_ns and the first code stage of every CTA never issued: each CTA's
+// waits on that stage run out, its status bits are set and it exits (the
+// self-test of the failure path; C is not written).
+int launch_gemm_missed_stage_selftest(const uint8_t* a_codes, const uint8_t* a_scales, const float* a_ts,
+                                      const uint8_t* b_codes, const uint8_t* b_scales, const float* b_ts, int64_t M,
+                                      int64_t N, int64_t K, float* C, int64_t ldc, uint32_t* status_word,
+                                      uint64_t wait_ns, cudaStream_t stream) {
+  const int64_t tiles = ((M + TILE_M - 1) / TILE_M) * ((N + 255) / 256);
+  int64_t clusters = num_sms() / 2;
+  if (clusters > tiles) clusters = tiles;
+  return launch_pair<256>(a_codes, a_scales, a_ts, b_codes, b_scales, b_ts, M, N, K, C, ldc, status_word, clusters,
+                          tiles, tiles, stream, wait_ns, 1);
 }
 
 int launch_gemm(const uint8_t* a_codes, const uint8_t* a_scales, const float* a_ts,

@@ -36,6 +36,10 @@ int launch_fake_quantize(const uint16_t* x, int64_t rows, int64_t K, int64_t ldx
                          float* tensor_scale, const uint32_t* amax_word, int scale_given, void* out, int out_bf16,
                          int64_t ldo, uint8_t* choice, cudaStream_t stream);
 int launch_bounded_wait_selftest(uint32_t* status, uint64_t limit_ns, cudaStream_t stream);
+int launch_gemm_missed_stage_selftest(const uint8_t* a_codes, const uint8_t* a_scales, const float* a_ts,
+                                      const uint8_t* b_codes, const uint8_t* b_scales, const float* b_ts, int64_t M,
+                                      int64_t N, int64_t K, float* C, int64_t ldc, uint32_t* status_word,
+                                      uint64_t wait_ns, cudaStream_t stream);
 int launch_dequantize(const uint8_t* codes, const uint8_t* scales, const float* tensor_scale,
                       int64_t rows, int64_t K, float* out, cudaStream_t stream);
 int launch_gemm(const uint8_t* a_codes, const uint8_t* a_scales, const float* a_ts,

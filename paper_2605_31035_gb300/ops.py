@@ -69,6 +69,9 @@ def lib() -> ctypes.CDLL:
         L.mixfp4_gemm_native_fewrows.argtypes = [P, P, P, P, P, P, I64, I64, I64, P, I64, P, P]
         L.mixfp4_fake_quantize.restype = I
         L.mixfp4_fake_quantize.argtypes = [P, I, I64, I64, I64, I, I, P, P, I, P, I, I64, P, P]
+        L.mixfp4_selftest_gemm_missed_stage.restype = I
+        L.mixfp4_selftest_gemm_missed_stage.argtypes = [P, P, P, P, P, P, I64, I64, I64, P, I64, P,
+                                                         ctypes.c_uint64, P]
         L.mixfp4_selftest_bounded_wait.restype = I
         L.mixfp4_selftest_bounded_wait.argtypes = [P, ctypes.c_uint64, P]
         L.mixfp4_status_string.restype = ctypes.c_char_p
@@ -526,6 +529,25 @@ def selftest_bounded_wait(limit_ns: int = 20_000_000, stream=None) -> int:
     _check("mixfp4_selftest_bounded_wait",
            lib().mixfp4_selftest_bounded_wait(_ptr(status), int(limit_ns), _stream(stream)))
     torch.cuda.synchronize()
+    return int(status.item())
+
+
+def selftest_gemm_missed_stage(a: QTensor, b: QTensor, out: torch.Tensor, limit_ns: int = 5_000_000,
+                               stream=None) -> int:
+    """Run the pair GEMM kernel with its first code stage withheld and short
+    wait limits; returns the status bits it reported (nonzero when the
+    failure path worked).  `out` is not written."""
+    _check_operand(a, "a")
+    _check_operand(b, "b")
+    _require(a.K == b.K and a.codes.device == b.codes.device, "operands must share K and device")
+    _check_c(out, a.rows, b.rows, a.codes.device)
+    status = torch.zeros(1, dtype=torch.int32, device=a.codes.device)
+    _check("mixfp4_selftest_gemm_missed_stage",
+           lib().mixfp4_selftest_gemm_missed_stage(_ptr(a.codes), _ptr(a.scales), _ptr(a.tensor_scale),
+                                                   _ptr(b.codes), _ptr(b.scales), _ptr(b.tensor_scale), a.rows,
+                                                   b.rows, a.K, _ptr(out), out.stride(0), _ptr(status),
+                                                   int(limit_ns), _stream(stream)))
+    torch.cuda.synchronize(a.codes.device)
     return int(status.item())
 
 
