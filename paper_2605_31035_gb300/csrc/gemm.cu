@@ -31,12 +31,19 @@
 //                 MMA-issuing thread; in the peer CTA one thread that forwards
 //                 "stage decoded" to the leader as a single remote arrival (16
 //                 remote arrivals on one barrier word serialise across SMs);
-//   warps 2-9     A decoders, two threads per A row (lane quarter = warp % 4),
-//                 64 K of the row per stage -> f16 pairs in TMEM columns;
-//   warps 10-17   B decoders, two threads per B row, 64 K of the row per stage
-//                 -> f16 in the canonical K-major no-swizzle UMMA layout;
-//   warps 18-25   epilogue: tcgen05.ld -> x s32A s32B / 4 -> a per-warp shared
+//   warps 2-9     A decoders, two groups of four (lane quarter = warp % 4): the
+//                 first group decodes the first 128-K stage of every code
+//                 stage, the second group the second, one thread per A row,
+//                 128 K of the row -> f16 pairs in TMEM columns;
+//   next 6-8      B decoders in the same two groups, one thread per B row of
+//                 the tile (kTileN / 2 rows; a 224-wide tile puts the last 16
+//                 rows of both groups in one shared warp), 128 K of the row ->
+//                 f16 in the canonical K-major no-swizzle UMMA layout;
+//   last 8 warps  epilogue: tcgen05.ld -> x s32A s32B / 4 -> a per-warp shared
 //                 staging tile -> coalesced fp32 stores (or red.add) to C.
+// Each decoder warp synchronises once per code stage instead of once per
+// decoded stage, so the decoders spend a smaller share of their time in
+// barrier waits (their ALU work bounds the main loop).
 // TMEM per CTA (512 columns): fp32 accumulator 128 lanes x 256 columns, then
 // kDecStages A stages of 64 columns (128 K of f16 pairs).  The leader's MMA
 // waits for both CTAs' decoders (remote mbarrier arrivals).
@@ -70,19 +77,30 @@ constexpr int BKD = 128;                      // K per decoded stage
 constexpr int kSub = BKC / BKD;
 constexpr int kCodeStages = 2;
 constexpr int kDecStages = 4;
-constexpr int kTPR = 2;                       // decode threads per operand row
 constexpr int kChunksPerSub = BKD / 32;       // 16-byte code chunks (32 codes) per row per stage
-constexpr int kChunksPerThread = kChunksPerSub / kTPR;
-static_assert(kChunksPerThread % 2 == 0, "A decoders store two chunks (32 TMEM columns) at a time");
-constexpr int kDecodeWarpsA = kTPR * BM / 32;   // 8
-constexpr int kDecodeWarpsB = kTPR * BNH / 32;  // 8
+static_assert(kSub == 2 && kChunksPerSub == 4, "two decoder groups, one per 128-K stage of a code stage");
+constexpr int kDecodeWarpsA = kSub * BM / 32;   // 8: one thread per A row in each group
 constexpr int kEpiWarps = 8;
 constexpr int kFirstDecA = 2;
 constexpr int kFirstDecB = kFirstDecA + kDecodeWarpsA;   // 10
-constexpr int kFirstEpi = kFirstDecB + kDecodeWarpsB;    // 18
-constexpr int kThreads = 32 * (kFirstEpi + kEpiWarps);   // 832
-constexpr int kDecodeWarps = kDecodeWarpsA + kDecodeWarpsB;
 static_assert(kFirstDecA % 4 == 2 && kDecodeWarpsA % 4 == 0, "A decoders cover every TMEM lane quarter");
+
+// Warp roles that depend on the tile width: one B decoder thread per B row of
+// the CTA in each group; with kTileN / 2 = 32 f + 16 rows the last 16 rows of
+// both groups share one warp (lanes 0-15 first group, 16-31 second).
+template <int kTileN>
+struct PairRoles {
+  static constexpr int kBRows = kTileN / 2;
+  static constexpr int kBFull = kBRows / 32;                  // B warps per group with 32 rows
+  static constexpr int kBMixed = (kBRows % 32) ? 1 : 0;       // the shared warp
+  static_assert(kBRows % 32 == 0 || kBRows % 32 == 16, "B rows per CTA: a multiple of 16");
+  static constexpr int kBWarps = kSub * kBFull + kBMixed;
+  static constexpr int kFirstEpi = kFirstDecB + kBWarps;
+  static constexpr int kThreads = 32 * (kFirstEpi + kEpiWarps);
+  static constexpr int kDecodeWarps = kDecodeWarpsA + kBWarps;  // arrivals per code stage
+  // Arrivals on a decoded stage: its A group, its full B warps, the shared warp.
+  static constexpr int kStageArrivals = kDecodeWarpsA / kSub + kBFull + kBMixed;
+};
 
 constexpr uint32_t kAccCols = TILE_N;                 // fp32 accumulator columns
 constexpr uint32_t kAStageCols = BKD / 2;             // f16 pairs per A row per stage
@@ -117,8 +135,8 @@ constexpr int kMinStreamKGainSlices = 8;           // stream-K must save this ma
 struct Bars {
   uint64_t code_full[kCodeStages];
   uint64_t code_empty[kCodeStages];
-  uint64_t dec_full[kDecStages];    // leader: its kDecodeWarps + 1 forwarded peer arrival
-  uint64_t peer_ready[kDecStages];  // peer: its kDecodeWarps arrivals, forwarded as one
+  uint64_t dec_full[kDecStages];    // leader: its stage's decoder warps + 1 forwarded peer arrival
+  uint64_t peer_ready[kDecStages];  // peer: its stage's decoder warps, forwarded as one
   uint64_t dec_empty[kDecStages];   // MMA commit (multicast to both CTAs)
   uint64_t acc_full;                // MMA commit (multicast)
   uint64_t acc_empty;               // leader: 2 x kEpiWarps arrivals
@@ -185,10 +203,9 @@ __device__ __forceinline__ uint32_t scale_pair(const uint4& sc, int chunk) {
 
 // kTileN: pair tile width (256, 224 or 192; each CTA holds kTileN / 2 rows of
 // B).  Shared and tensor memory are laid out for 256; narrower tiles leave the
-// tail of the B regions unused (decoders may write those rows; the MMA never
-// reads them).
+// tail of the B regions unused.
 template <int kTileN>
-__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairRoles<kTileN>::kThreads, 1)
 mixfp4_gemm_kernel(const __grid_constant__ CUtensorMap tm_ac, const __grid_constant__ CUtensorMap tm_bc,
                    const __grid_constant__ CUtensorMap tm_as, const __grid_constant__ CUtensorMap tm_bs,
                    const float* __restrict__ a_ts, const float* __restrict__ b_ts,
@@ -204,7 +221,9 @@ mixfp4_gemm_kernel(const __grid_constant__ CUtensorMap tm_ac, const __grid_const
   const bool leader = rank == 0;
   const int num_kc = K / BKC;
   static_assert(kTileN % 32 == 0 && kTileN >= 64 && kTileN <= TILE_N, "tile width");
-  constexpr int kBRows = kTileN / 2;  // B rows per CTA
+  using Roles = PairRoles<kTileN>;
+  constexpr int kBRows = Roles::kBRows;  // B rows per CTA
+  constexpr int kFirstEpi = Roles::kFirstEpi;
   constexpr uint32_t kStageTx = A_CODE_BYTES + A_SCALE_BYTES + kBRows * (BKC / 2 + BKC / 16);
   constexpr uint32_t kIdescT = idesc_f16_f32(TILE_M, kTileN);
   const int mtiles = (M + TILE_M - 1) / TILE_M, ntiles_n = (N + kTileN - 1) / kTileN;
@@ -214,11 +233,11 @@ mixfp4_gemm_kernel(const __grid_constant__ CUtensorMap tm_ac, const __grid_const
   if (threadIdx.x == 0) {
     for (int s = 0; s < kCodeStages; ++s) {
       mbar_init(smem_u32(&bars->code_full[s]), 1);
-      mbar_init(smem_u32(&bars->code_empty[s]), kDecodeWarps);
+      mbar_init(smem_u32(&bars->code_empty[s]), Roles::kDecodeWarps);
     }
     for (int s = 0; s < kDecStages; ++s) {
-      mbar_init(smem_u32(&bars->dec_full[s]), kDecodeWarps + 1);
-      mbar_init(smem_u32(&bars->peer_ready[s]), kDecodeWarps);
+      mbar_init(smem_u32(&bars->dec_full[s]), Roles::kStageArrivals + 1);
+      mbar_init(smem_u32(&bars->peer_ready[s]), Roles::kStageArrivals);
       mbar_init(smem_u32(&bars->dec_empty[s]), 1);
     }
     mbar_init(smem_u32(&bars->acc_full), 1);
@@ -350,18 +369,31 @@ mixfp4_gemm_kernel(const __grid_constant__ CUtensorMap tm_ac, const __grid_const
     }
   } else if (warp < kFirstEpi) {
     // ---------------- decoders ----------------
+    // Group g decodes decoded stage g (K 128 g .. 128 g + 127) of every code
+    // stage: A warps by warp index, B threads by warp and, in the shared
+    // warp, by lane.
     const bool is_a = warp < kFirstDecB;
     const int dw = warp - (is_a ? kFirstDecA : kFirstDecB);
-    const int part = dw >> 2;                      // which half of a stage's chunks
-    // A decoders: rows follow the warp's TMEM lane quarter (warp % 4).
-    const int rl = is_a ? ((warp & 3) * 32 + lane) : (dw & 3) * 32 + lane;
+    int sub, rl;
+    if (is_a) {
+      sub = dw >> 2;
+      rl = (warp & 3) * 32 + lane;  // rows follow the warp's TMEM lane quarter
+    } else if (dw < kSub * Roles::kBFull) {
+      sub = dw / Roles::kBFull;
+      rl = (dw % Roles::kBFull) * 32 + lane;
+    } else {
+      sub = lane >> 4;
+      rl = Roles::kBFull * 32 + (lane & 15);
+    }
+    const bool mixed = Roles::kBMixed && !is_a && dw >= kSub * Roles::kBFull;
     const uint32_t code_off = (is_a ? 0 : A_CODE_BYTES) + rl * (BKC / 2);
-    const uint32_t scale_off = A_CODE_BYTES + B_CODE_BYTES + (is_a ? 0 : A_SCALE_BYTES) + rl * (BKC / 16);
+    const uint32_t scale_off =
+        A_CODE_BYTES + B_CODE_BYTES + (is_a ? 0 : A_SCALE_BYTES) + rl * (BKC / 16) + sub * (BKD / 16);
     const uint32_t b_off = OFF_DEC + (rl >> 3) * kSBO + (rl & 7) * 16;
     const uint32_t a_lane = (uint32_t)((warp & 3) * 32) << 16;
-    const uint32_t swz = rl & 7;
-    int d = 0;
-    uint32_t dph = 0;
+    // 16-byte chunk c of the row sits at chunk c ^ (row % 8) (128-byte swizzle);
+    // this thread's chunks are sub * 4 + j, j = 0..3.
+    const uint32_t cswz = (uint32_t)(sub * kChunksPerSub) ^ (uint32_t)(rl & 7);
     int it = 0;
     bool ok = true;
     Sched sched(cluster_id, nclusters, dp_tiles, ntiles, num_kc, chunk_kc);
@@ -376,59 +408,61 @@ mixfp4_gemm_kernel(const __grid_constant__ CUtensorMap tm_ac, const __grid_const
           break;
         }
         const uint32_t st = sbase + s * CODE_STAGE_BYTES;
-        const uint4 sc = lds128(st + scale_off);  // the row's 16 block scales of this code stage
-#pragma unroll
-        for (int sub = 0; sub < kSub; ++sub) {
-          uint4 c[kChunksPerThread];
-#pragma unroll
-          for (int j = 0; j < kChunksPerThread; ++j) {
-            const int chunk = sub * kChunksPerSub + part * kChunksPerThread + j;
-            c[j] = lds128(st + code_off + (((uint32_t)chunk ^ swz) << 4));
-          }
-          if (!mbar_wait_cluster(smem_u32(&bars->dec_empty[d]), dph ^ 1, abort_flag, wait_ns)) {
-            fail(32u);
-            ok = false;
-            break;
-          }
-          if (is_a) {
-            // The thread's kChunksPerThread * 32 K of the row = 16 f16 pairs per
-            // chunk -> TMEM columns [part * 16 * kChunksPerThread, ...) of stage d,
-            // stored two chunks (32 columns) at a time.
-#pragma unroll
-            for (int j = 0; j < kChunksPerThread; j += 2) {
-              uint32_t o[32];
-              decode_chunk(c[j], scale_pair(sc, sub * kChunksPerSub + part * kChunksPerThread + j), o);
-              decode_chunk(c[j + 1], scale_pair(sc, sub * kChunksPerSub + part * kChunksPerThread + j + 1), o + 16);
-              tmem_st_32x32b_x32(tmem_a0 + a_lane + (uint32_t)d * kAStageCols +
-                                     (uint32_t)(part * 16 * kChunksPerThread + 16 * j), o);
-            }
-            tmem_st_wait();
-            tc_fence_before();
-          } else {
-            const uint32_t dst = sbase + b_off + d * B_DEC_BYTES;
-#pragma unroll
-            for (int j = 0; j < kChunksPerThread; ++j) {
-              const int chunk = sub * kChunksPerSub + part * kChunksPerThread + j;
-              uint32_t o[16];
-              decode_chunk(c[j], scale_pair(sc, chunk), o);
-              const int kchunk0 = (chunk - sub * kChunksPerSub) * 4;  // first 8-element K chunk
-#pragma unroll
-              for (int q = 0; q < 4; ++q)
-                sts128(dst + (kchunk0 + q) * kLBO, o[4 * q], o[4 * q + 1], o[4 * q + 2], o[4 * q + 3]);
-            }
-            fence_proxy_async_smem();
-          }
-          __syncwarp();
-          if (lane == 0) mbar_arrive(smem_u32(leader ? &bars->dec_full[d] : &bars->peer_ready[d]));
-          if (++d == kDecStages) { d = 0; dph ^= 1; }
-          if (sub == kSub - 1) {
-            // Release the code stage only now: every value loaded from it has
-            // been consumed (the decoded stores depend on it), so the TMA
-            // refill cannot overtake a pending shared-memory load.
-            __syncwarp();
-            if (lane == 0) mbar_arrive(smem_u32(&bars->code_empty[s]));
-          }
+        const uint32_t crow = st + code_off;
+        const uint2 sc = lds64(st + scale_off);  // this stage's 8 block scales of the row
+        const int gstage = it * kSub + sub;
+        const int d = gstage % kDecStages;
+        const uint32_t dph = (uint32_t)(gstage / kDecStages) & 1u;
+        uint4 c0 = lds128(crow + ((cswz ^ 0u) << 4)), c1 = lds128(crow + ((cswz ^ 1u) << 4));
+        // The shared warp waits for both stages' slots (its lanes fill both).
+        const int d_first = mixed ? (it * kSub) % kDecStages : d;
+        const int d_last = mixed ? (it * kSub + kSub - 1) % kDecStages : d;
+        const uint32_t ph_first = mixed ? (uint32_t)((it * kSub) / kDecStages) & 1u : dph;
+        const uint32_t ph_last = mixed ? (uint32_t)((it * kSub + kSub - 1) / kDecStages) & 1u : dph;
+        if (!mbar_wait_cluster(smem_u32(&bars->dec_empty[d_first]), ph_first ^ 1, abort_flag, wait_ns) ||
+            (mixed && !mbar_wait_cluster(smem_u32(&bars->dec_empty[d_last]), ph_last ^ 1, abort_flag, wait_ns))) {
+          fail(32u);
+          ok = false;
+          break;
         }
+        if (is_a) {
+          // 128 K of the row = 64 f16 pairs -> TMEM columns of stage d, 16
+          // columns (one chunk) per store.
+#pragma unroll
+          for (int j = 0; j < kChunksPerSub; ++j) {
+            const uint4 cj = j == 0 ? c0 : j == 1 ? c1 : lds128(crow + ((cswz ^ (uint32_t)j) << 4));
+            const uint32_t sw = j < 2 ? sc.x : sc.y;
+            uint32_t o[16];
+            decode_chunk(cj, (j & 1) ? (sw >> 16) : (sw & 0xFFFFu), o);
+            tmem_st_32x32b_x16(tmem_a0 + a_lane + (uint32_t)d * kAStageCols + (uint32_t)(16 * j), o);
+          }
+          tmem_st_wait();
+          tc_fence_before();
+        } else {
+          const uint32_t dst = sbase + b_off + d * B_DEC_BYTES;
+#pragma unroll
+          for (int j = 0; j < kChunksPerSub; ++j) {
+            const uint4 cj = j == 0 ? c0 : j == 1 ? c1 : lds128(crow + ((cswz ^ (uint32_t)j) << 4));
+            const uint32_t sw = j < 2 ? sc.x : sc.y;
+            uint32_t o[16];
+            decode_chunk(cj, (j & 1) ? (sw >> 16) : (sw & 0xFFFFu), o);
+#pragma unroll
+            for (int q = 0; q < 4; ++q)
+              sts128(dst + (j * 4 + q) * kLBO, o[4 * q], o[4 * q + 1], o[4 * q + 2], o[4 * q + 3]);
+          }
+          fence_proxy_async_smem();
+        }
+        __syncwarp();
+        if (lane == 0) {
+          const uint32_t full0 = smem_u32(leader ? &bars->dec_full[0] : &bars->peer_ready[0]);
+          mbar_arrive(full0 + 8u * (uint32_t)d_first);
+          if (mixed) mbar_arrive(full0 + 8u * (uint32_t)d_last);
+        }
+        // Release the code stage only now: every value loaded from it has been
+        // consumed (the decoded stores depend on it), so the TMA refill cannot
+        // overtake a pending shared-memory load.
+        __syncwarp();
+        if (lane == 0) mbar_arrive(smem_u32(&bars->code_empty[s]));
       }
     }
   } else {
@@ -442,6 +476,7 @@ mixfp4_gemm_kernel(const __grid_constant__ CUtensorMap tm_ac, const __grid_const
     const int chalf = (warp - kFirstEpi) >> 2;  // column half
     griddep_wait();
     const float sa = 0.25f * __ldg(a_ts), sb = __ldg(b_ts);
+    const u64 sa2 = pack2(sa, sa), sb2 = pack2(sb, sb);
     const bool vec_ok = ((ldc & 3) == 0) && ((reinterpret_cast<uintptr_t>(C) & 15) == 0);
     const uint32_t acc_empty_leader = mapa_shared(smem_u32(&bars->acc_empty), 0);
     const uint32_t stage = sbase + OFF_EPI + (uint32_t)(warp - kFirstEpi) * EPI_BYTES;
@@ -476,7 +511,11 @@ mixfp4_gemm_kernel(const __grid_constant__ CUtensorMap tm_ac, const __grid_const
           if (lane == 0) mbar_arrive_cluster(acc_empty_leader);
         }
 #pragma unroll
-        for (int k = 0; k < EPI_CHUNK; ++k) o[k] = __float_as_uint(__fmul_rn(__fmul_rn(__uint_as_float(o[k]), sa), sb));
+        for (int k = 0; k < EPI_CHUNK; k += 2) {  // (acc x sa) x sb, two columns per instruction
+          const u64 v = mul2(mul2(bits2(o[k], o[k + 1]), sa2), sb2);
+          o[k] = (uint32_t)v;
+          o[k + 1] = (uint32_t)(v >> 32);
+        }
         const int col = n0 + cc * EPI_CHUNK;
         if (vec_ok && col + EPI_CHUNK <= N) {
 #pragma unroll
@@ -875,7 +914,8 @@ int launch_pair(const uint8_t* a_codes, const uint8_t* a_scales, const float* a_
   // A programmatic dependent: barrier set-up and TMEM allocation overlap the
   // tail of the kernel before it; the TMA producer and the epilogue wait for
   // that kernel before they read the operands or the tensor scales.
-  if (launch_pdl(mixfp4_gemm_kernel<kTileN>, (unsigned)(2 * clusters), kThreads, SMEM_ALLOC, stream, tac, tbc, tas,
+  if (launch_pdl(mixfp4_gemm_kernel<kTileN>, (unsigned)(2 * clusters), PairRoles<kTileN>::kThreads, SMEM_ALLOC, stream,
+                 tac, tbc, tas,
                  tbs, a_ts, b_ts, (int)M, (int)N, (int)K, C, (long long)ldc, (int)dp_tiles, kAccumChunkK / BKC,
                  status_word, wait_ns, skip_first_stage) != cudaSuccess)
     return MIXFP4_ERR_CUDA;
