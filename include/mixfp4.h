@@ -407,7 +407,7 @@ int mixfp4_selftest_bounded_wait(uint32_t* status_word, uint64_t limit_ns, void*
  * to limit_ns and with the first code stage of every CTA never issued (no
  * copy, no arrival).  The waits on that stage run out, each role that gives
  * up ORs its bit into *status_word (1 producer, 2 / 4 MMA thread, 8 drain,
- * 16 / 32 decoders, 64 epilogue, 128 peer forwarder), raises its CTA's abort
+ * 16 / 32 decoders, 64 epilogue), raises its CTA's abort
  * flag, lets the copies and MMAs it issued complete, frees its tensor memory
  * and exits; C is not written.  Nothing faults or hangs, and the device stays
  * usable: a later mixfp4_gemm on it runs normally.

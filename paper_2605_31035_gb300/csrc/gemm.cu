@@ -28,9 +28,7 @@
 //   warp 0        TMA producer: codes [rows][128 B] (128-byte swizzle) and
 //                 scales [rows][16 B] of a 256-wide K slice into a 2-deep ring;
 //   warp 1        TMEM allocator (both CTAs); in the leader CTA also the single
-//                 MMA-issuing thread; in the peer CTA one thread that forwards
-//                 "stage decoded" to the leader as a single remote arrival (16
-//                 remote arrivals on one barrier word serialise across SMs);
+//                 MMA-issuing thread;
 //   warps 2-9     A decoders, two groups of four (lane quarter = warp % 4): the
 //                 first group decodes the first 128-K stage of every code
 //                 stage, the second group the second, one thread per A row,
@@ -46,12 +44,13 @@
 // barrier waits (their ALU work bounds the main loop).
 // TMEM per CTA (512 columns): fp32 accumulator 128 lanes x 256 columns, then
 // kDecStages A stages of 64 columns (128 K of f16 pairs).  The leader's MMA
-// waits for both CTAs' decoders (remote mbarrier arrivals).
+// waits for both CTAs' decoders: every decoder warp of a stage arrives on the
+// leader's barrier, the peer's through a remote arrival.
 // All pipeline waits are bounded (1 s each, or the self-test's limit); a
 // wait that gives up ORs its role's bit into the status word (1 producer,
 // 2 MMA thread waiting for the accumulator, 4 MMA thread waiting for a
-// decoded stage, 8 final drain, 16 / 32 decoders, 64 epilogue, 128 peer
-// forwarder), raises the CTA's abort flag, and the CTA lets its issued copies
+// decoded stage, 8 final drain, 16 / 32 decoders, 64 epilogue), raises the
+// CTA's abort flag, and the CTA lets its issued copies
 // and MMAs land, frees TMEM and exits without touching C.
 #include <cuda.h>
 #include <cudaTypedefs.h>
@@ -135,8 +134,7 @@ constexpr int kMinStreamKGainSlices = 8;           // stream-K must save this ma
 struct Bars {
   uint64_t code_full[kCodeStages];
   uint64_t code_empty[kCodeStages];
-  uint64_t dec_full[kDecStages];    // leader: its stage's decoder warps + 1 forwarded peer arrival
-  uint64_t peer_ready[kDecStages];  // peer: its stage's decoder warps, forwarded as one
+  uint64_t dec_full[kDecStages];    // leader: the stage's decoder warps of both CTAs
   uint64_t dec_empty[kDecStages];   // MMA commit (multicast to both CTAs)
   uint64_t acc_full;                // MMA commit (multicast)
   uint64_t acc_empty;               // leader: 2 x kEpiWarps arrivals
@@ -236,8 +234,7 @@ mixfp4_gemm_kernel(const __grid_constant__ CUtensorMap tm_ac, const __grid_const
       mbar_init(smem_u32(&bars->code_empty[s]), Roles::kDecodeWarps);
     }
     for (int s = 0; s < kDecStages; ++s) {
-      mbar_init(smem_u32(&bars->dec_full[s]), Roles::kStageArrivals + 1);
-      mbar_init(smem_u32(&bars->peer_ready[s]), Roles::kStageArrivals);
+      mbar_init(smem_u32(&bars->dec_full[s]), 2 * Roles::kStageArrivals);
       mbar_init(smem_u32(&bars->dec_empty[s]), 1);
     }
     mbar_init(smem_u32(&bars->acc_full), 1);
@@ -347,25 +344,6 @@ mixfp4_gemm_kernel(const __grid_constant__ CUtensorMap tm_ac, const __grid_const
       // for it (ignoring the abort flag) so TMEM is never freed under an MMA.
       mma_commit_pair(smem_u32(&bars->drain), 1);
       if (!mbar_wait_cluster(smem_u32(&bars->drain), 0, nullptr, wait_ns)) fail(8u);
-    } else if (!leader && lane == 0) {
-      // ---------------- forwarder (peer CTA) ----------------
-      const uint32_t dec_full_leader0 = mapa_shared(smem_u32(&bars->dec_full[0]), 0);
-      int d = 0;
-      uint32_t dph = 0;
-      bool ok = true;
-      Sched sched(cluster_id, nclusters, dp_tiles, ntiles, num_kc, chunk_kc);
-      int t, k0, k1;
-      while (ok && sched.next(t, k0, k1)) {
-        for (int st = 0; st < (k1 - k0) * kSub; ++st) {
-          if (!mbar_wait(smem_u32(&bars->peer_ready[d]), dph, abort_flag, wait_ns)) {
-            fail(128u);
-            ok = false;
-            break;
-          }
-          mbar_arrive_cluster(dec_full_leader0 + d * 8);
-          if (++d == kDecStages) { d = 0; dph ^= 1; }
-        }
-      }
     }
   } else if (warp < kFirstEpi) {
     // ---------------- decoders ----------------
@@ -454,9 +432,10 @@ mixfp4_gemm_kernel(const __grid_constant__ CUtensorMap tm_ac, const __grid_const
         }
         __syncwarp();
         if (lane == 0) {
-          const uint32_t full0 = smem_u32(leader ? &bars->dec_full[0] : &bars->peer_ready[0]);
-          mbar_arrive(full0 + 8u * (uint32_t)d_first);
-          if (mixed) mbar_arrive(full0 + 8u * (uint32_t)d_last);
+          // The leader's barrier, locally or through a remote arrival.
+          const uint32_t full0 = mapa_shared(smem_u32(&bars->dec_full[0]), 0);
+          mbar_arrive_cluster(full0 + 8u * (uint32_t)d_first);
+          if (mixed) mbar_arrive_cluster(full0 + 8u * (uint32_t)d_last);
         }
         // Release the code stage only now: every value loaded from it has been
         // consumed (the decoded stores depend on it), so the TMA refill cannot
