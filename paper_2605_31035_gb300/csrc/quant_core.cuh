@@ -91,13 +91,21 @@ __device__ __forceinline__ TensorConsts tensor_consts(float* tensor_scale, const
   return c;
 }
 
-// E2M1 quantization of a pair (RNE, saturating): returns the byte of the two
-// nibbles (first element low) and the dequantized pair as f16x2.
-__device__ __forceinline__ uint32_t e2m1_pair(float lo, float hi, uint32_t& h2) {
-  uint32_t byte;
-  asm("{ .reg .b8 t; cvt.rn.satfinite.e2m1x2.f32 t, %2, %3; cvt.rn.f16x2.e2m1x2 %1, t; cvt.u32.u8 %0, t; }"
-      : "=r"(byte), "=r"(h2) : "f"(hi), "f"(lo));
-  return byte;
+// E2M1 codes of four pairs packed into one word (pair j in byte j, first
+// element low), and each pair decoded back to f16x2.
+__device__ __forceinline__ uint32_t e2m1_quad(const float (&lo)[4], const float (&hi)[4], uint32_t (&h2)[4]) {
+  uint32_t word;
+  asm("{ .reg .b8 t0, t1, t2, t3;\n"
+      " cvt.rn.satfinite.e2m1x2.f32 t0, %6, %5;\n"
+      " cvt.rn.satfinite.e2m1x2.f32 t1, %8, %7;\n"
+      " cvt.rn.satfinite.e2m1x2.f32 t2, %10, %9;\n"
+      " cvt.rn.satfinite.e2m1x2.f32 t3, %12, %11;\n"
+      " cvt.rn.f16x2.e2m1x2 %1, t0;\n cvt.rn.f16x2.e2m1x2 %2, t1;\n"
+      " cvt.rn.f16x2.e2m1x2 %3, t2;\n cvt.rn.f16x2.e2m1x2 %4, t3;\n"
+      " mov.b32 %0, {t0, t1, t2, t3}; }"
+      : "=r"(word), "=r"(h2[0]), "=r"(h2[1]), "=r"(h2[2]), "=r"(h2[3])
+      : "f"(lo[0]), "f"(hi[0]), "f"(lo[1]), "f"(hi[1]), "f"(lo[2]), "f"(hi[2]), "f"(lo[3]), "f"(hi[3]));
+  return word;
 }
 
 // Four byte values (each in the low byte of a word) packed into one word.
@@ -196,27 +204,30 @@ __device__ __forceinline__ void e2m1_candidate(const u64 a[8], const float4 t, u
   const u64 zh8 = pack2(t.y, t.y), zl8 = pack2(t.z, t.z);
   const uint16_t ns8h = __half_as_ushort(__float2half_rn(-t.x));  // exact: E4M3 values are f16 values
   u64 acc = 0;  // (+0, +0): even / odd chains
-  uint32_t e[8];
+  uint32_t pw[2];
 #pragma unroll
-  for (int j = 0; j < 8; ++j) {
-    const u64 y = div_kd2(a[j], zh8, zl8);
-    float ylo, yhi;
-    unpack2(y, ylo, yhi);
-    uint32_t h2;
-    e[j] = e2m1_pair(ylo, yhi, h2);
-    if (kErr) {
+  for (int g = 0; g < 2; ++g) {
+    float ylo[4], yhi[4];
+    uint32_t hq[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) unpack2(div_kd2(a[4 * g + i], zh8, zl8), ylo[i], yhi[i]);
+    pw[g] = e2m1_quad(ylo, yhi, hq);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      if (!kErr) continue;
+      const int j = 4 * g + i;
       float alo, ahi, dlo, dhi;
       unpack2(a[j], alo, ahi);
       // d = |a| - q s8 (exact), with q taken straight from its f16 decode
       asm("{ .reg .f16 ql, qh; mov.b32 {ql, qh}, %2;\n"
           " fma.rn.f32.f16 %0, ql, %3, %4;\n fma.rn.f32.f16 %1, qh, %3, %5; }"
-          : "=f"(dlo), "=f"(dhi) : "r"(h2), "h"(ns8h), "f"(alo), "f"(ahi));
+          : "=f"(dlo), "=f"(dhi) : "r"(hq[i]), "h"(ns8h), "f"(alo), "f"(ahi));
       const u64 d = pack2(dlo, dhi);
       acc = fma2(d, d, acc);
     }
   }
-  p_lo = pack_low_bytes(e[0], e[1], e[2], e[3]);
-  p_hi = pack_low_bytes(e[4], e[5], e[6], e[7]);
+  p_lo = pw[0];
+  p_hi = pw[1];
   S = 0.0f;
   if (kErr) {
     float se, so;

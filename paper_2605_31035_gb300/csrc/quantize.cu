@@ -2,9 +2,10 @@
 // (App. B.2/B.3) for sm_103a.
 //
 // Design (HBM-bound, 2.5625 algorithmic bytes per element):
-//   * one thread owns one 16-element block: a single 256-bit coalesced load
-//     (a warp reads 1 KiB of contiguous bf16), one 64-bit code store and one
-//     scale-byte store (a warp writes 256 B and 32 B contiguous);
+//   * one thread owns one 16-element block at a time: a single 256-bit
+//     coalesced load (a warp reads 1 KiB of contiguous bf16), one 64-bit code
+//     store and one scale-byte store (a warp writes 256 B and 32 B
+//     contiguous); each thread quantizes two such blocks side by side;
 //   * all per-element fp32 work runs on packed f32x2 instructions;
 //   * every division of Algorithm 1 (x/s32, B/6, B/7, |a|/s8) is evaluated as
 //     IEEE round-to-nearest with a divisor known in advance, in two packed
@@ -40,9 +41,34 @@ namespace mixfp4 {
 
 namespace {
 
-// Persistent grid: each thread walks blocks b, b + nthr, b + 2 nthr, ... and
-// keeps the next block's 32-byte load in flight while it quantizes the
-// current one.  The first loads are issued before any set-up work.
+// Persistent grid: each thread walks blocks b, b + nthr, b + 2 nthr, ... two
+// at a time (a, b): both blocks of a pair are quantized before either is
+// stored, so their independent dependency chains interleave, and the loads of
+// the next pair are in flight meanwhile.  The division method is fixed per
+// launch, so each method gets its own copy of the loop.
+template <int kMode, bool kContig, bool kScaled, bool kMarkstein>
+__device__ __forceinline__ void quantize_pairs(const uint16_t* __restrict__ x, int64_t b, int64_t nthr,
+                                               int64_t nblocks, int64_t kblocks, int64_t ldx,
+                                               uint8_t* __restrict__ codes, uint8_t* __restrict__ scales,
+                                               const TensorConsts& tc, const float4* __restrict__ tab,
+                                               uint32_t (&wa)[8], uint32_t (&wb)[8]) {
+  for (; b < nblocks; b += 2 * nthr) {
+    const int64_t b1 = b + nthr;
+    uint32_t lo0, hi0, sb0, lo1, hi1, sb1;
+    quantize_block<kMode, kScaled, kMarkstein>(wa, tc, tab, lo0, hi0, sb0);
+    quantize_block<kMode, kScaled, kMarkstein>(wb, tc, tab, lo1, hi1, sb1);  // wb past the end: unused
+    stg64(codes + b * 8, lo0, hi0);
+    scales[b] = (uint8_t)sb0;
+    if (b + 2 * nthr < nblocks) ldg256_stream(block_src<kContig>(x, b + 2 * nthr, kblocks, ldx), wa);
+    if (b1 < nblocks) {
+      stg64(codes + b1 * 8, lo1, hi1);
+      scales[b1] = (uint8_t)sb1;
+      if (b1 + 2 * nthr < nblocks) ldg256_stream(block_src<kContig>(x, b1 + 2 * nthr, kblocks, ldx), wb);
+    }
+  }
+}
+
+// The first loads are issued before any set-up work.
 template <int kMode, bool kContig>
 __global__ void __launch_bounds__(kQuantThreads, 4)
 quantize_kernel(const uint16_t* __restrict__ x, int64_t nblocks, int64_t kblocks, int64_t ldx,
@@ -55,32 +81,22 @@ quantize_kernel(const uint16_t* __restrict__ x, int64_t nblocks, int64_t kblocks
   if (!after_amax) griddep_wait();
   griddep_launch_dependents();
   const int64_t nthr = (int64_t)gridDim.x * kQuantThreads;
-  int64_t b = (int64_t)blockIdx.x * kQuantThreads + threadIdx.x;
+  const int64_t b = (int64_t)blockIdx.x * kQuantThreads + threadIdx.x;
   uint32_t wa[8], wb[8];
+#pragma unroll
+  for (int j = 0; j < 8; ++j) wb[j] = 0u;  // defined values for a missing second block
   if (b < nblocks) ldg256_stream(block_src<kContig>(x, b, kblocks, ldx), wa);
   if (b + nthr < nblocks) ldg256_stream(block_src<kContig>(x, b + nthr, kblocks, ldx), wb);
   fill_scale_table(tab);
   if (after_amax) griddep_wait();
   const TensorConsts tc = tensor_consts(tensor_scale, amax_word, scale_given);
   const bool markstein = markstein_needed(tc);
-  for (; b < nblocks; b += 2 * nthr) {
-    uint32_t lo, hi, sb;
-    if (tc.scaled) quantize_block<kMode, true, true>(wa, tc, tab, lo, hi, sb);
-    else if (markstein) quantize_block<kMode, false, true>(wa, tc, tab, lo, hi, sb);
-    else quantize_block<kMode, false, false>(wa, tc, tab, lo, hi, sb);
-    stg64(codes + b * 8, lo, hi);
-    scales[b] = (uint8_t)sb;
-    if (b + 2 * nthr < nblocks) ldg256_stream(block_src<kContig>(x, b + 2 * nthr, kblocks, ldx), wa);
-    const int64_t b1 = b + nthr;
-    if (b1 < nblocks) {
-      if (tc.scaled) quantize_block<kMode, true, true>(wb, tc, tab, lo, hi, sb);
-      else if (markstein) quantize_block<kMode, false, true>(wb, tc, tab, lo, hi, sb);
-      else quantize_block<kMode, false, false>(wb, tc, tab, lo, hi, sb);
-      stg64(codes + b1 * 8, lo, hi);
-      scales[b1] = (uint8_t)sb;
-      if (b1 + 2 * nthr < nblocks) ldg256_stream(block_src<kContig>(x, b1 + 2 * nthr, kblocks, ldx), wb);
-    }
-  }
+  if (tc.scaled)
+    quantize_pairs<kMode, kContig, true, true>(x, b, nthr, nblocks, kblocks, ldx, codes, scales, tc, tab, wa, wb);
+  else if (markstein)
+    quantize_pairs<kMode, kContig, false, true>(x, b, nthr, nblocks, kblocks, ldx, codes, scales, tc, tab, wa, wb);
+  else
+    quantize_pairs<kMode, kContig, false, false>(x, b, nthr, nblocks, kblocks, ldx, codes, scales, tc, tab, wa, wb);
 }
 
 template <int kMode, bool kContig>
