@@ -56,6 +56,7 @@
 #include <cudaTypedefs.h>
 #include <cuda_runtime.h>
 #include <cstdint>
+#include <cstring>
 
 #include "host_util.cuh"
 #include "kernels.cuh"
@@ -206,6 +207,7 @@ template <int kTileN>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairRoles<kTileN>::kThreads, 1)
 mixfp4_gemm_kernel(const __grid_constant__ CUtensorMap tm_ac, const __grid_constant__ CUtensorMap tm_bc,
                    const __grid_constant__ CUtensorMap tm_as, const __grid_constant__ CUtensorMap tm_bs,
+                   const __grid_constant__ CUtensorMap tm_c, int c_tma,
                    const float* __restrict__ a_ts, const float* __restrict__ b_ts,
                    int M, int N, int K, float* __restrict__ C, long long ldc, int dp_tiles, int chunk_kc,
                    uint32_t* status_word, uint64_t wait_ns, int skip_first_stage) {
@@ -446,26 +448,42 @@ mixfp4_gemm_kernel(const __grid_constant__ CUtensorMap tm_ac, const __grid_const
     }
   } else {
     // ---------------- epilogue (two warps per TMEM lane quarter) ----------------
-    // Each warp drains 32 rows x 128 columns in 16-column steps: tcgen05.ld
-    // (lane = row) -> scale -> its shared staging tile (row-major, 16-byte
-    // chunks XOR-swizzled by row so writes and reads are conflict-free) ->
-    // read back four lanes per row, so every global store instruction writes
-    // 64 contiguous bytes in each of 8 rows.
+    // Each warp drains 32 rows x kTileN / 2 columns in 16-column steps:
+    // tcgen05.ld (lane = row) -> scale -> its shared staging tile (row-major,
+    // 64 bytes a row, 16-byte chunks XOR-swizzled by row: the 64-byte swizzle
+    // of the tensor map of C) -> one TMA store (or TMA add) of the 32 x 16
+    // box, which reads the tile and writes C asynchronously: the next step's
+    // tcgen05.ld does not wait for the stores, so the accumulator is released
+    // sooner and the C writes overlap the next tile's main loop.  Parts of a
+    // box outside C are not written.  Without the tensor map (C or ldc not
+    // 16-byte aligned) each lane stores its row's 16 values one by one.
     const int q = warp & 3;                  // TMEM lane quarter of this warp
     const int chalf = (warp - kFirstEpi) >> 2;  // column half
     griddep_wait();
     const float sa = 0.25f * __ldg(a_ts), sb = __ldg(b_ts);
     const u64 sa2 = pack2(sa, sa), sb2 = pack2(sb, sb);
-    const bool vec_ok = ((ldc & 3) == 0) && ((reinterpret_cast<uintptr_t>(C) & 15) == 0);
     const uint32_t acc_empty_leader = mapa_shared(smem_u32(&bars->acc_empty), 0);
-    const uint32_t stage = sbase + OFF_EPI + (uint32_t)(warp - kFirstEpi) * EPI_BYTES;
-    const uint32_t wr_row = stage + (uint32_t)lane * 64u, wr_swz = (uint32_t)(lane >> 1) & 3u;
+    // Staging tiles: the warp's own, and for tiles of at most 224 columns a
+    // second one in the unused B rows 112-127 of a decoded-B stage (never
+    // written by the decoders nor read by the MMA), so consecutive steps
+    // alternate and a step's store need not finish reading before the next.
+    constexpr bool kTwoStages = kBRows <= 112;
+    const int ew = warp - kFirstEpi;
+    const uint32_t stage0 = sbase + OFF_EPI + (uint32_t)ew * EPI_BYTES;
+    const uint32_t stage1 = kTwoStages ? sbase + OFF_DEC + (uint32_t)(ew >> 1) * B_DEC_BYTES + 14u * kSBO +
+                                             (uint32_t)(ew & 1) * EPI_BYTES
+                                       : stage0;
+    const uint32_t wr_off = (uint32_t)lane * 64u, wr_swz = (uint32_t)(lane >> 1) & 3u;
     Sched sched(cluster_id, nclusters, dp_tiles, ntiles, num_kc, chunk_kc);
     int t, k0, k1;
     for (int i = 0; sched.next(t, k0, k1); ++i) {
       // The first chunk of a whole tile is stored; every other segment is
       // added into C (after that chunk, or into rows the host zeroed).
       const bool whole = sched.store;
+      // An add into C must follow the earlier segments' stores into the same
+      // tile: bulk operations of different groups are not ordered, so wait
+      // for their completion (issued a main loop ago, they are done).
+      if (!whole && c_tma && lane == 0) bulk_wait_all();
       const bool acc_ok = mbar_wait_cluster(smem_u32(&bars->acc_full), i & 1, abort_flag, wait_ns);
       tc_fence_after();
       // tcgen05.ld is warp-collective: decide for the whole warp.
@@ -496,26 +514,27 @@ mixfp4_gemm_kernel(const __grid_constant__ CUtensorMap tm_ac, const __grid_const
           o[k + 1] = (uint32_t)(v >> 32);
         }
         const int col = n0 + cc * EPI_CHUNK;
-        if (vec_ok && col + EPI_CHUNK <= N) {
+        if (c_tma) {
+          const uint32_t stage = (kTwoStages && (cc & 1)) ? stage1 : stage0;
+          // The store that last used this staging tile must have read it.
+          if (lane == 0) {
+            if (kTwoStages) bulk_wait_read_one();
+            else bulk_wait_read_all();
+          }
+          __syncwarp();
 #pragma unroll
           for (int j = 0; j < 4; ++j)
-            sts128(wr_row + (((uint32_t)j ^ wr_swz) << 4), o[4 * j], o[4 * j + 1], o[4 * j + 2], o[4 * j + 3]);
+            sts128(stage + wr_off + (((uint32_t)j ^ wr_swz) << 4), o[4 * j], o[4 * j + 1], o[4 * j + 2],
+                   o[4 * j + 3]);
+          fence_proxy_async_smem();
           __syncwarp();
-          const int cq = lane & 3;
-#pragma unroll
-          for (int p = 0; p < 4; ++p) {
-            const int rr = (lane >> 2) + 8 * p;
-            const uint4 val = lds128(stage + (uint32_t)rr * 64u + (((uint32_t)cq ^ ((uint32_t)(rr >> 1) & 3u)) << 4));
-            if (row0 + rr < M) {
-              float* dst = C + (long long)(row0 + rr) * ldc + col + 4 * cq;
-              if (whole)
-                *reinterpret_cast<uint4*>(dst) = val;
-              else
-                red_add_v4(dst, __uint_as_float(val.x), __uint_as_float(val.y), __uint_as_float(val.z),
-                           __uint_as_float(val.w));
+          if (lane == 0) {
+            if (row0 < M && col < N) {  // boxes wholly outside C are skipped
+              if (whole) tma_store_2d(&tm_c, stage, col, row0);
+              else tma_reduce_add_2d(&tm_c, stage, col, row0);
             }
+            bulk_commit_group();  // one group per step, empty or not: the waits count groups
           }
-          __syncwarp();  // the staging tile is rewritten by the next step
         } else if (row0 + lane < M) {
           float* crow = C + (long long)(row0 + lane) * ldc + col;
           for (int k = 0; k < EPI_CHUNK; ++k)
@@ -526,6 +545,8 @@ mixfp4_gemm_kernel(const __grid_constant__ CUtensorMap tm_ac, const __grid_const
         }
       }
     }
+    // The CTA's stores into C complete before it exits.
+    if (c_tma && lane == 0) bulk_wait_all();
   }
 
   tc_fence_before();
@@ -873,6 +894,14 @@ int launch_pair(const uint8_t* a_codes, const uint8_t* a_scales, const float* a_
       !make_map(&tas, a_scales, (uint64_t)K / 16, (uint64_t)M, BKC / 16, BM, CU_TENSOR_MAP_SWIZZLE_NONE) ||
       !make_map(&tbs, b_scales, (uint64_t)K / 16, (uint64_t)N, BKC / 16, kTileN / 2, CU_TENSOR_MAP_SWIZZLE_NONE))
     return MIXFP4_ERR_CUDA;
+  // C by TMA stores: 32 x 16 fp32 boxes, 64-byte swizzle (the staging tiles'
+  // layout), when C and its row stride are 16-byte aligned.
+  CUtensorMap tmc;
+  memset(&tmc, 0, sizeof(tmc));
+  const int c_tma = ((ldc & 3) == 0) && ((reinterpret_cast<uintptr_t>(C) & 15) == 0);
+  if (c_tma && !make_map_f32(&tmc, C, (uint64_t)N, (uint64_t)M, (uint64_t)ldc, EPI_CHUNK, 32,
+                             CU_TENSOR_MAP_SWIZZLE_64B))
+    return MIXFP4_ERR_CUDA;
   static std::atomic<uint64_t> smem_set{0};
   if (!set_dynamic_smem_once(reinterpret_cast<const void*>(mixfp4_gemm_kernel<kTileN>), SMEM_ALLOC, smem_set))
     return MIXFP4_ERR_CUDA;
@@ -894,9 +923,8 @@ int launch_pair(const uint8_t* a_codes, const uint8_t* a_scales, const float* a_
   // tail of the kernel before it; the TMA producer and the epilogue wait for
   // that kernel before they read the operands or the tensor scales.
   if (launch_pdl(mixfp4_gemm_kernel<kTileN>, (unsigned)(2 * clusters), PairRoles<kTileN>::kThreads, SMEM_ALLOC, stream,
-                 tac, tbc, tas,
-                 tbs, a_ts, b_ts, (int)M, (int)N, (int)K, C, (long long)ldc, (int)dp_tiles, kAccumChunkK / BKC,
-                 status_word, wait_ns, skip_first_stage) != cudaSuccess)
+                 tac, tbc, tas, tbs, tmc, c_tma, a_ts, b_ts, (int)M, (int)N, (int)K, C, (long long)ldc,
+                 (int)dp_tiles, kAccumChunkK / BKC, status_word, wait_ns, skip_first_stage) != cudaSuccess)
     return MIXFP4_ERR_CUDA;
   return MIXFP4_OK;
 }

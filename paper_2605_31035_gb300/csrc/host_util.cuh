@@ -23,6 +23,21 @@ inline PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
   return fn;
 }
 
+// 2D fp32 tensor [rows][cols] with row stride ld elements (ld * 4 a multiple
+// of 16 bytes, base 16-byte aligned), box [box_rows][box_cols].
+inline bool make_map_f32(CUtensorMap* m, const float* base, uint64_t cols, uint64_t rows, uint64_t ld,
+                         uint32_t box_cols, uint32_t box_rows, CUtensorMapSwizzle swz) {
+  auto fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[2] = {cols, rows};
+  cuuint64_t strides[1] = {ld * sizeof(float)};
+  cuuint32_t box[2] = {box_cols, box_rows};
+  cuuint32_t estr[2] = {1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, const_cast<float*>(base), dims, strides, box, estr,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, swz, CU_TENSOR_MAP_L2_PROMOTION_NONE,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 // 2D uint8 tensor [rows][row_bytes] (dense), box [box_rows][box_bytes].
 inline bool make_map(CUtensorMap* m, const void* base, uint64_t row_bytes, uint64_t rows, uint32_t box_bytes,
                      uint32_t box_rows, CUtensorMapSwizzle swz) {
