@@ -13,15 +13,16 @@
 // outlier-heavy operands whose outlier channels coincide).  So the work
 // schedule cuts every tile's K into chunks of at most 16 K slices (4096 K):
 // each chunk is accumulated from zero, and the epilogue stores the first
-// chunk of a tile into C and adds the later ones with red.global.add, so the
+// chunk of a tile into C and adds the later ones (TMA add), so the
 // bound no longer depends on K.
 //
 // Work decomposition: persistent CTA pairs (clusters of 2, cta_group::2).  A
-// pair owns 256 x 256 output tiles; each CTA holds 128 rows of A and 128 rows
-// (half) of B.  Tiles of the full waves are dealt whole (chunk by chunk);
+// pair owns 256 x kTileN output tiles (kTileN = 256, 224 or 192); each CTA
+// holds 128 rows of A and kTileN / 2 rows of B.  Tiles of the full waves are
+// dealt whole (chunk by chunk);
 // when the tile count leaves a partial last wave, that wave's (tile, K slice)
 // units are split evenly over all pairs (stream-K) and their partial sums are
-// added into C with red.global.add after the host zeroed those tiles.  Tiles are numbered
+// added into C (TMA add) after the host zeroed those tiles.  Tiles are numbered
 // row band by row band (t = mt * ntiles_n + nt).  Decoded A never touches
 // shared memory: it is written to tensor memory (tcgen05.st) and the MMA reads
 // it from there; decoded B goes through shared memory.  Per CTA:
@@ -38,7 +39,7 @@
 //                 rows of both groups in one shared warp), 128 K of the row ->
 //                 f16 in the canonical K-major no-swizzle UMMA layout;
 //   last 8 warps  epilogue: tcgen05.ld -> x s32A s32B / 4 -> a per-warp shared
-//                 staging tile -> coalesced fp32 stores (or red.add) to C.
+//                 staging tile -> TMA store (or TMA add) of the 32 x 16 box.
 // Each decoder warp synchronises once per code stage instead of once per
 // decoded stage, so the decoders spend a smaller share of their time in
 // barrier waits (their ALU work bounds the main loop).
