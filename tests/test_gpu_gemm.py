@@ -110,6 +110,27 @@ def test_strided_output(oracle):
     assert_close(big[:, :200].cpu().numpy(), Cref, A, B)
 
 
+@pytest.mark.parametrize("K", [512, 8192])
+def test_unaligned_output(oracle, K):
+    """C whose base and row stride are not 16-byte aligned: the epilogue
+    cannot use TMA stores of C and writes element by element (stores for the
+    first accumulation chunk, atomic adds for the second at K = 8192); the
+    columns around the output are untouched."""
+    x = synth.activations(130, K, 31 + K, 32)
+    w = synth.weights(200, K, 33 + K, 0.02)
+    qa, ra = quant_both(oracle, x)
+    qb, rb = quant_both(oracle, w)
+    big = torch.full((130, 203), -1.0, device=DEV)
+    out = big[:, 1:201]  # base 4 bytes past a 16-byte boundary, ldc = 203
+    ops().mixfp4_gemm(qa, qb, out=out)
+    torch.cuda.synchronize()
+    assert torch.all(big[:, 0] == -1.0) and torch.all(big[:, 201:] == -1.0)
+    Cref = oracle.gemm_f64(ra, rb)
+    A = oracle.dequant_rows_f64(ra[0], ra[1], ra[2], range(130))
+    B = oracle.dequant_rows_f64(rb[0], rb[1], rb[2], range(200))
+    assert_close(out.cpu().numpy(), Cref, A, B)
+
+
 def rows_cols_check(oracle, qa, qb, C, rows, cols, block=2048):
     """Whole rows of C against every column and whole columns against every
     row: float64 dots of the oracle's dequantized operands, the full operand
