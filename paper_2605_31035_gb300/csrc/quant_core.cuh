@@ -542,7 +542,7 @@ __device__ __forceinline__ void rht_block(const u64 y[8], const TensorConsts& tc
   code_hi = mhi | f32_sign_bits(y + 4);
 }
 
-// Rotation + Algorithm 1.  One block per thread per iteration; the grid
-// stride is a multiple of 8 blocks, so the 8 lanes of a chunk stay together.
+// Rotation + Algorithm 1 (rht_quantize_kernel): the grid stride is a multiple
+// of 8 blocks, so the 8 lanes of a chunk stay together at every step.
 }  // namespace
 }  // namespace mixfp4

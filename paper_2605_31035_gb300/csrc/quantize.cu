@@ -99,8 +99,10 @@ quantize_kernel(const uint16_t* __restrict__ x, int64_t nblocks, int64_t kblocks
     quantize_pairs<kMode, kContig, false, false>(x, b, nthr, nblocks, kblocks, ldx, codes, scales, tc, tab, wa, wb);
 }
 
+// Rotation + Algorithm 1, two blocks per thread side by side (as in
+// quantize_kernel); the rotated pairs take 2 CTAs per SM of registers.
 template <int kMode, bool kContig>
-__global__ void __launch_bounds__(kQuantThreads, 3)
+__global__ void __launch_bounds__(kQuantThreads, 2)
 rht_quantize_kernel(const uint16_t* __restrict__ x, int64_t nblocks, int64_t kblocks, int64_t ldx,
                     const uint8_t* __restrict__ signs, uint8_t* __restrict__ codes, uint8_t* __restrict__ scales,
                     float* tensor_scale, const uint32_t* amax_word, int scale_given, int after_amax) {
@@ -110,8 +112,11 @@ rht_quantize_kernel(const uint16_t* __restrict__ x, int64_t nblocks, int64_t kbl
   const int lane = threadIdx.x & 31;
   const int64_t nthr = (int64_t)gridDim.x * kQuantThreads;
   int64_t b = (int64_t)blockIdx.x * kQuantThreads + threadIdx.x;
-  uint32_t w[8];
+  uint32_t w[8], w2[8];
+#pragma unroll
+  for (int j = 0; j < 8; ++j) w2[j] = 0u;
   if (b < nblocks) ldg256_stream(block_src<kContig>(x, b, kblocks, ldx), w);
+  if (b + nthr < nblocks) ldg256_stream(block_src<kContig>(x, b + nthr, kblocks, ldx), w2);
   if (threadIdx.x < 128) {
     float s8 = 0.0f, unused;
     if (threadIdx.x < 0x7F) f16x2_to_f32(cvt_f16x2_from_e4m3x2((uint16_t)threadIdx.x), s8, unused);
@@ -123,15 +128,27 @@ rht_quantize_kernel(const uint16_t* __restrict__ x, int64_t nblocks, int64_t kbl
   if (after_amax) griddep_wait();
   const TensorConsts tc = tensor_consts(tensor_scale, amax_word, scale_given);
   __syncthreads();
-  for (; b < nblocks; b += nthr) {
-    u64 y[8];
+  for (; b < nblocks; b += 2 * nthr) {
+    const int64_t b1 = b + nthr;
+    u64 y[8], y2[8];
     rht_rotate(w, sw, lane, y);
-    if (b + nthr < nblocks) ldg256_stream(block_src<kContig>(x, b + nthr, kblocks, ldx), w);
-    uint32_t lo, hi, sb;
-    if (tc.scaled) rht_block<kMode, true>(y, tc, tab, lo, hi, sb);
-    else rht_block<kMode, false>(y, tc, tab, lo, hi, sb);
+    rht_rotate(w2, sw, lane, y2);  // the 8 lanes of a chunk agree on b1 < nblocks
+    if (b + 2 * nthr < nblocks) ldg256_stream(block_src<kContig>(x, b + 2 * nthr, kblocks, ldx), w);
+    if (b1 + 2 * nthr < nblocks) ldg256_stream(block_src<kContig>(x, b1 + 2 * nthr, kblocks, ldx), w2);
+    uint32_t lo, hi, sb, lo2, hi2, sb2;
+    if (tc.scaled) {
+      rht_block<kMode, true>(y, tc, tab, lo, hi, sb);
+      rht_block<kMode, true>(y2, tc, tab, lo2, hi2, sb2);
+    } else {
+      rht_block<kMode, false>(y, tc, tab, lo, hi, sb);
+      rht_block<kMode, false>(y2, tc, tab, lo2, hi2, sb2);
+    }
     stg64(codes + b * 8, lo, hi);
     scales[b] = (uint8_t)sb;
+    if (b1 < nblocks) {
+      stg64(codes + b1 * 8, lo2, hi2);
+      scales[b1] = (uint8_t)sb2;
+    }
   }
 }
 
@@ -305,7 +322,7 @@ int launch_rht_quantize(const uint16_t* x, int64_t rows, int64_t K, int64_t ldx,
                         int scale_given, cudaStream_t stream) {
   const int64_t kblocks = K / 16, nblocks = rows * kblocks;
   int64_t grid = (nblocks + kQuantThreads - 1) / kQuantThreads;
-  if (grid > num_sms() * 3) grid = num_sms() * 3;
+  if (grid > num_sms() * 2) grid = num_sms() * 2;
   if (grid == 0) return 0;
   const int after_amax = !scale_given;
 #define MIXFP4_LAUNCH_R(MODE)                                                                            \
