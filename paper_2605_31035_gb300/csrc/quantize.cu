@@ -162,13 +162,18 @@ rht_amax_kernel(const uint16_t* __restrict__ x, int64_t nblocks, int64_t kblocks
   rht_sign_words(signs, lane, sw);
   uint32_t m = 0;
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
-  for (int64_t b = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; b < nblocks; b += stride) {
-    uint32_t w[8];
-    ldg256_stream(block_src<kContig>(x, b, kblocks, ldx), w);
+  int64_t b = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  uint32_t w[8];
+  if (b < nblocks) ldg256_stream(block_src<kContig>(x, b, kblocks, ldx), w);
+  for (; b < nblocks; b += stride) {
+    uint32_t wn[8];  // the next block's load is in flight during this block's rotation
+    if (b + stride < nblocks) ldg256_stream(block_src<kContig>(x, b + stride, kblocks, ldx), wn);
     u64 y[8];
     rht_rotate(w, sw, lane, y);
 #pragma unroll
     for (int j = 0; j < 8; ++j) m = max(m, max(lo32(y[j]) & 0x7FFFFFFFu, hi32(y[j]) & 0x7FFFFFFFu));
+#pragma unroll
+    for (int j = 0; j < 8; ++j) w[j] = wn[j];
   }
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) m = max(m, __shfl_xor_sync(0xffffffffu, m, o));
