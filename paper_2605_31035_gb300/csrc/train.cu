@@ -129,6 +129,27 @@ quantize_colwise_kernel(const uint16_t* __restrict__ x, int64_t R, int64_t C, in
   }
 }
 
+// Grid-stride loop of the stochastic-rounding quantizer with the division
+// method fixed; the next block's load is in flight while a block is quantized.
+template <int kMode, bool kContig, bool kScaled, bool kMarkstein>
+__device__ __forceinline__ void sr_loop(const uint16_t* __restrict__ x, int64_t b, int64_t nthr, int64_t nblocks,
+                                        int64_t kblocks, int64_t ldx, uint8_t* __restrict__ codes,
+                                        uint8_t* __restrict__ scales, const TensorConsts& tc,
+                                        const float4* __restrict__ tab, uint64_t seed, uint64_t offset) {
+  uint32_t w[8];
+  if (b < nblocks) ldg256_stream(block_src<kContig>(x, b, kblocks, ldx), w);
+  for (; b < nblocks; b += nthr) {
+    uint32_t wn[8];
+    if (b + nthr < nblocks) ldg256_stream(block_src<kContig>(x, b + nthr, kblocks, ldx), wn);
+    uint32_t lo, hi, sb;
+    quantize_block_sr<kMode, kScaled, kMarkstein>(w, tc, tab, seed, offset, (uint64_t)b * 16, lo, hi, sb);
+    stg64(codes + b * 8, lo, hi);
+    scales[b] = (uint8_t)sb;
+#pragma unroll
+    for (int j = 0; j < 8; ++j) w[j] = wn[j];
+  }
+}
+
 // Row-wise quantization with stochastic rounding (R13): one thread per
 // 16-element block, grid-stride; the element index of block b's first element
 // is 16 b (row-major over [rows][K]).
@@ -144,17 +165,10 @@ quantize_sr_kernel(const uint16_t* __restrict__ x, int64_t nblocks, int64_t kblo
   const TensorConsts tc = tensor_consts(tensor_scale, amax_word, scale_given);
   const bool markstein = markstein_needed(tc);
   const int64_t nthr = (int64_t)gridDim.x * blockDim.x;
-  for (int64_t b = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; b < nblocks; b += nthr) {
-    uint32_t w[8];
-    ldg256_stream(block_src<kContig>(x, b, kblocks, ldx), w);
-    uint32_t lo, hi, sb;
-    const uint64_t e0 = (uint64_t)b * 16;
-    if (tc.scaled) quantize_block_sr<kMode, true, true>(w, tc, tab, seed, offset, e0, lo, hi, sb);
-    else if (markstein) quantize_block_sr<kMode, false, true>(w, tc, tab, seed, offset, e0, lo, hi, sb);
-    else quantize_block_sr<kMode, false, false>(w, tc, tab, seed, offset, e0, lo, hi, sb);
-    stg64(codes + b * 8, lo, hi);
-    scales[b] = (uint8_t)sb;
-  }
+  const int64_t b0 = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (tc.scaled) sr_loop<kMode, kContig, true, true>(x, b0, nthr, nblocks, kblocks, ldx, codes, scales, tc, tab, seed, offset);
+  else if (markstein) sr_loop<kMode, kContig, false, true>(x, b0, nthr, nblocks, kblocks, ldx, codes, scales, tc, tab, seed, offset);
+  else sr_loop<kMode, kContig, false, false>(x, b0, nthr, nblocks, kblocks, ldx, codes, scales, tc, tab, seed, offset);
 }
 
 constexpr int k2dThreads = 256;
