@@ -574,8 +574,8 @@ mixfp4_gemm_kernel(const __grid_constant__ CUtensorMap tm_ac, const __grid_const
 // top of this file).
 // Per CTA: warp 0 TMA, warp 1 TMEM allocator + MMA thread, warps 2-17 weight
 // decoders (two threads per weight row, one 32-code chunk each per stage),
-// warps 18-21 X decoders (warp % 4 = TMEM lane quarter = 32 X rows), warps
-// 22-25 epilogue.
+// warps 18-25 X decoders (warp % 4 = TMEM lane quarter = 32 X rows; two warps
+// per quarter, one chunk each per stage), warps 26-29 epilogue.
 // ============================================================================
 namespace skinny {
 
@@ -584,10 +584,10 @@ constexpr int MXMAX = 64;                        // max activation rows (MMA M i
 constexpr int BKC = 256, BKD = 64, kSub = BKC / BKD;
 constexpr int kCodeStages = 2, kDecStages = 4;
 constexpr int kWarpsW = 2 * BN / 32;             // 16
-constexpr int kWarpsX = 4;
-constexpr int kFirstW = 2, kFirstX = kFirstW + kWarpsW, kFirstEpi = kFirstX + kWarpsX;  // 2, 18, 22
+constexpr int kWarpsX = 8;                       // two per TMEM lane quarter: one chunk of a stage each
+constexpr int kFirstW = 2, kFirstX = kFirstW + kWarpsW, kFirstEpi = kFirstX + kWarpsX;  // 2, 18, 26
 constexpr int kEpiWarps = 4;
-constexpr int kThreads = 32 * (kFirstEpi + kEpiWarps);  // 832
+constexpr int kThreads = 32 * (kFirstEpi + kEpiWarps);  // 960
 static_assert(kFirstX % 4 == 2 && kFirstEpi % 4 == 2, "warp w covers TMEM lane quarter w % 4");
 constexpr int W_CODE = BN * BKC / 2, X_CODE = MXMAX * BKC / 2;
 constexpr int W_SCALE = BN * BKC / 16, X_SCALE = MXMAX * BKC / 16;
@@ -753,10 +753,10 @@ mixfp4_gemm_skinny_kernel(const __grid_constant__ CUtensorMap tm_wc, const __gri
     // ---------------- decoders ----------------
     const bool is_w = warp < kFirstX;
     // W: row = (dw % 8) * 32 + lane, chunk part = dw / 8 of each 64-K stage.
-    // X: row = (warp % 4) * 32 + lane = its TMEM lane; both chunks of a stage.
+    // X: row = (warp % 4) * 32 + lane = its TMEM lane, chunk part = (warp - 18) / 4.
     const int dw = warp - kFirstW;
     const int row = is_w ? ((dw & 7) * 32 + lane) : ((warp & 3) * 32 + lane);
-    const int part = is_w ? (dw >> 3) : 0;
+    const int part = is_w ? (dw >> 3) : ((warp - kFirstX) >> 2);
     const bool active = is_w || (warp & 3) * 32 < nx;  // X warps past the fetched rows idle
     const uint32_t code_row = (is_w ? 0u : (uint32_t)OFF_XC) + (uint32_t)row * (BKC / 2);
     const uint32_t scale_row = (is_w ? (uint32_t)OFF_WS : (uint32_t)OFF_XS) + (uint32_t)row * (BKC / 16);
@@ -780,12 +780,7 @@ mixfp4_gemm_skinny_kernel(const __grid_constant__ CUtensorMap tm_wc, const __gri
       for (int sub = 0; sub < kSub; ++sub) {
         uint4 c[2];
         if (active) {
-          if (is_w) {
-            c[0] = lds128(st + code_row + ((((uint32_t)(sub * 2 + part)) ^ swz) << 4));
-          } else {
-            c[0] = lds128(st + code_row + ((((uint32_t)(sub * 2)) ^ swz) << 4));
-            c[1] = lds128(st + code_row + ((((uint32_t)(sub * 2 + 1)) ^ swz) << 4));
-          }
+          c[0] = lds128(st + code_row + ((((uint32_t)(sub * 2 + part)) ^ swz) << 4));
         }
         if (!mbar_wait(smem_u32(&bars->dec_empty[d]), dph ^ 1, abort_flag, kWaitLimitNs)) {
           fail(32u);
@@ -801,10 +796,9 @@ mixfp4_gemm_skinny_kernel(const __grid_constant__ CUtensorMap tm_wc, const __gri
             sts128(dst + (uint32_t)(part * 4 + q) * kLBO, o[4 * q], o[4 * q + 1], o[4 * q + 2], o[4 * q + 3]);
           fence_proxy_async_smem();
         } else if (active) {
-          uint32_t o[32];
-          decode_chunk(c[0], scale_pair(sc, sub * 2), o);
-          decode_chunk(c[1], scale_pair(sc, sub * 2 + 1), o + 16);
-          tmem_st_32x32b_x32(tmem_x0 + x_lane + (uint32_t)d * kXStageCols, o);
+          uint32_t o[16];
+          decode_chunk(c[0], scale_pair(sc, sub * 2 + part), o);
+          tmem_st_32x32b_x16(tmem_x0 + x_lane + (uint32_t)d * kXStageCols + (uint32_t)(16 * part), o);
           tmem_st_wait();
           tc_fence_before();
         }
