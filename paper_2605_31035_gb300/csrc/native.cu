@@ -78,7 +78,6 @@ __device__ __forceinline__ void split_e1m2_word(uint32_t w, uint32_t tmask, uint
   MIXFP4_LOP3(main, t, w, tmask, 0xE4);              // tmask ? main : w  (per bit: (a & c) | (b & ~c))
   res = r & tmask;                                    // E2M1 blocks have no residual
 }
-#undef MIXFP4_LOP3
 
 // Threads [0, n_code) split 32 elements (two blocks, 16 code bytes) each;
 // threads [n_code, n_code + n_sf) write one 16-byte line of the scale tiles
@@ -460,74 +459,90 @@ int launch(const uint8_t* a_main, const uint8_t* a_res, const uint8_t* a_sf, con
 }  // namespace nv
 
 // ============================================================================
-// Few-row native variant (M <= 64 activation rows, the decode shape): the
-// MixFP4 operands are split into E2M1 main + residual parts on the fly, in
-// shared memory, instead of beforehand.  Weight rows go on the MMA N side in
-// units of 128 rows x one 256-wide K slice: the split writes the 128 main rows
-// to rows 0-127 and the 128 residual rows to rows 128-255 of one N = 256
-// operand tile, and the activation rows' main and residual parts to rows
-// 0-63 and 64-127 of the M = 128 operand tile, so ONE kind::mxf4nvf4 MMA per
-// 64-K step forms all four products; the epilogue adds the accumulator's four
-// quadrants: C[m][n] = D[m][n] + D[m][128+n] + D[64+m][n] + D[64+m][128+n].
+// Few-row native variant (M <= 64 activation rows, the decode shape).
+//
+// Decomposition used here (every product exact, same block scales):
+//   main part     = the stored MixFP4 code itself read as an E2M1 code;
+//   residual part = E2M1 code {0,1,2,3,4,4,4,2}[p] of the magnitude p (sign
+//                   kept), scaled by the block's scale for an E1M2 block and
+//                   by 0 for an E2M1 block.
+// For an E2M1 block the main part is the block and the residual has scale 0.
+// For an E1M2 block, E2M1 value e(p) + e(res(p)) = p for every p in 0..7
+// (0, .5+.5, 1+1, 1.5+1.5, 2+2, 3+2, 4+2, 6+1), which is the E1M2 value of p
+// under the same scale.  So the main codes need no rewriting: TMA lands them
+// straight in the MMA operand tiles, and the splitters only write the
+// residual rows (one bit-sliced function of the nibbles, no per-block type
+// select) and the two scale tiles per operand (main: the scale with the type
+// bit cleared; residual: the same where the type bit is set, else 0).
+//
+// Weight rows go on the MMA N side in units of 128 rows x one 256-wide K
+// slice: rows 0-127 of the N = 256 operand tile hold the main codes, rows
+// 128-255 the residual codes; the activation rows' main codes sit in rows
+// 0..XR-1 of the M = 128 tile and their residual codes in rows XR..2XR-1
+// (XR = 16, 32 or 64 by the row count; rows from 2XR on are never written,
+// the MMA reads whatever follows in the stage there and the epilogue never
+// loads those accumulator lanes).  ONE kind::mxf4nvf4 MMA per 64-K step forms
+// all four products; C[m][n] = D[m][n] + D[m][128+n] + D[XR+m][n] +
+// D[XR+m][128+n], the epilogue adding each accumulator lane's two column
+// halves into C row (lane row mod XR).
 // Per CTA (one per SM, units split evenly over all SMs, partial sums added
 // into C which the host zeroed):
-//   warp 0      TMA: 128 x 128-byte weight code tile (128-byte swizzle), its
-//               128 x 16-byte scale tile, the activation rows' code and scale
-//               tiles, into a ring of 2-4 stages (21-27 KB each, by the row
-//               count), ahead of a 3-stage ring of split operand tiles;
-//   warp 1      TMEM allocation; lane 0 issues the MMAs (one per 64-K step);
-//   warps 2-17  split the weight codes (four threads per row, two 16-byte
-//               chunks each: E2M1 blocks copied, E1M2 nibbles p -> main
-//               {0,2,4,5,6,6,7,7}[p] and residual (p in {5,7} ? 2 : 0) by
-//               bit logic on eight nibbles at a time) into the swizzled
-//               operand tile, and the scale bytes into the tensor core's
-//               tiled layout; warps 18-21 the same for the activation rows;
+//   warp 0      TMA: weight codes (128 x 128 bytes, 128-byte swizzle) into
+//               the operand tile, its 128 x 16-byte scale rows, the
+//               activation rows' codes into the A tile and their scale rows,
+//               into a ring of 3-5 stages (by the row count);
+//   warp 1      TMEM allocation; lane 0 issues the MMAs (one per 64-K step)
+//               and frees the stage with their commit;
+//   warps 2-17  weight residual rows (four threads per row, two 16-byte
+//               chunks each) and weight scale tiles; warps 18-21 the same
+//               for the activation rows;
 //   warps 22-25 epilogue, one TMEM lane quarter each;
-//   warps 26-27 copy each split stage's scale tiles into tensor memory
-//               (tcgen05.cp, half of the K steps each) and commit, so that
-//               scale copies and MMAs are issued by three threads in parallel
-//               (each tcgen05 instruction holds its issuing thread ~50 ns).
+//   warps 26-27 copy each stage's scale tiles into tensor memory
+//               (tcgen05.cp, half of the K steps each) and commit.
 // ============================================================================
 namespace nvs {
 
 constexpr int WR = 128;                    // weight rows per unit (MMA N = 2 x 128)
-constexpr int XR = 64;                     // activation rows (MMA M = 2 x 64)
 constexpr int BKC = 256;                   // K per unit
 constexpr int ROWB = BKC / 2;              // 128 code bytes per row per unit
-constexpr int kMaxCodeStages = 4, kSplitStages = 3;
-// Code stage (ring of TMA destinations): weight codes and scales, then the
-// nx activation rows' codes and scales; its size depends on nx (host side).
-constexpr int OFF_WC = 0, OFF_WS = WR * ROWB, OFF_XC = OFF_WS + WR * 16;
-constexpr int S_B = 0, S_A = 2 * WR * ROWB, S_SFA = S_A + 2 * XR * ROWB, S_SFB = S_SFA + 4 * 512;
-constexpr int SPLIT_STAGE = S_SFB + 4 * 512;                     // 52 KB
+constexpr int kMaxStages = 5;
+constexpr int SF_T = 4 * 512;              // tiled scales of 128 rows for the unit's four K steps
+// Stage layout (offsets from the stage base): A tile (2 XR rows), weight main
+// rows, weight residual rows, weight scale rows (TMA), activation scale rows
+// (TMA, at most 64 x 16 bytes), then the tiled scales of the A tile, of the
+// weight main rows and of the weight residual rows.
+__host__ __device__ constexpr int xr_of(int nx) { return nx <= 16 ? 16 : (nx <= 32 ? 32 : 64); }
+__host__ __device__ constexpr int off_b(int xr) { return 2 * xr * ROWB; }
+__host__ __device__ constexpr int off_ws(int xr) { return off_b(xr) + 2 * WR * ROWB; }
+__host__ __device__ constexpr int off_xs(int xr) { return off_ws(xr) + WR * 16; }
+__host__ __device__ constexpr int off_sfa(int xr) { return off_xs(xr) + 64 * 16; }
+__host__ __device__ constexpr int off_sfb(int xr) { return off_sfa(xr) + SF_T; }
+__host__ __device__ constexpr int off_sfr(int xr) { return off_sfb(xr) + SF_T; }
+__host__ __device__ constexpr int stage_bytes_of(int xr) { return ((off_sfr(xr) + SF_T + 1023) / 1024) * 1024; }
 constexpr int OFF_RINGS = 1024;                                  // after the barrier block
 constexpr int kSmemBudget = 232448 - 1024;                       // 1024 for the alignment of the base
-static_assert(OFF_XC % 1024 == 0 && SPLIT_STAGE % 1024 == 0 && S_A % 1024 == 0,
-              "swizzled tiles need 1024-byte alignment");
-__host__ __device__ constexpr int code_stage_bytes(int nx) { return ((OFF_XC + nx * (ROWB + 16) + 1023) / 1024) * 1024; }
-__host__ __device__ constexpr int code_stages(int nx) {
-  return (kSmemBudget - OFF_RINGS - kSplitStages * SPLIT_STAGE) / code_stage_bytes(nx) < kMaxCodeStages
-             ? (kSmemBudget - OFF_RINGS - kSplitStages * SPLIT_STAGE) / code_stage_bytes(nx)
-             : kMaxCodeStages;
+__host__ __device__ constexpr int stages_of(int xr) {
+  return (kSmemBudget - OFF_RINGS) / stage_bytes_of(xr) < kMaxStages ? (kSmemBudget - OFF_RINGS) / stage_bytes_of(xr)
+                                                                     : kMaxStages;
 }
-static_assert(code_stages(XR) >= 2, "shared memory budget");
+static_assert(stages_of(16) == 5 && stages_of(32) == 4 && stages_of(64) == 3, "ring depths");
+static_assert(off_b(16) % 1024 == 0 && stage_bytes_of(16) >= 128 * ROWB, "the M = 128 operand read stays in the stage");
 constexpr int kWSplitWarps = 16, kXSplitWarps = 4;
 constexpr int kFirstW = 2, kFirstX = kFirstW + kWSplitWarps, kFirstEpi = kFirstX + kXSplitWarps;  // 2, 18, 22
 constexpr int kCopyWarp = kFirstEpi + 4, kCopyWarps = 2;                                          // 26, 27
 constexpr int kThreads = 32 * (kCopyWarp + kCopyWarps);                                           // 896
 static_assert(kFirstEpi % 4 == 2, "epilogue warps cover the four TMEM lane quarters");
 constexpr uint32_t kAccCols = 2 * WR;                            // 256 fp32 columns
-constexpr uint32_t kSfCols = 12;                                 // per K step: 4 (A) + 8 (B)
+constexpr uint32_t kSfCols = 12;                                 // per K step: 4 (A) + 8 (B main, residual)
 constexpr uint32_t kTmemCols = 512;
 constexpr uint64_t kWaitLimitNs = 1000000000ull;
-static_assert(kAccCols + kSplitStages * 4 * kSfCols <= kTmemCols, "TMEM budget");
+static_assert(kAccCols + kMaxStages * 4 * kSfCols <= kTmemCols, "TMEM budget");
 
 struct Bars {
-  uint64_t code_full[kMaxCodeStages];
-  uint64_t code_empty[kMaxCodeStages];
-  uint64_t split_full[kSplitStages];
-  uint64_t sf_full[kSplitStages];   // the stage's scales are in tensor memory (commit of the copy warp)
-  uint64_t split_empty[kSplitStages];
+  uint64_t full[kMaxStages];        // TMA landed
+  uint64_t split_full[kMaxStages];  // residual rows and scale tiles written
+  uint64_t sf_full[kMaxStages];     // the stage's scales are in tensor memory (commit of the copy warps)
+  uint64_t empty[kMaxStages];       // the stage's MMAs completed
   uint64_t acc_full;
   uint64_t acc_empty;
   uint64_t drain;
@@ -536,14 +551,26 @@ struct Bars {
 };
 static_assert(sizeof(Bars) <= 256, "barrier block");
 
-
-// Split one 16-byte chunk (two blocks) given the blocks' type bits.
-__device__ __forceinline__ void split_chunk(uint4 c, bool t0, bool t1, uint4& m, uint4& r) {
-  const uint32_t k0 = t0 ? 0xFFFFFFFFu : 0u, k1 = t1 ? 0xFFFFFFFFu : 0u;
-  split_e1m2_word(c.x, k0, m.x, r.x);
-  split_e1m2_word(c.y, k0, m.y, r.y);
-  split_e1m2_word(c.z, k1, m.z, r.z);
-  split_e1m2_word(c.w, k1, m.w, r.w);
+// Residual E2M1 codes of eight nibbles (sign in bit 3, payload p in bits
+// 0-2): payload {0,1,2,3,4,4,4,2}[p] = p & F with F's bit 0 = ~p2, bit 1 =
+// ~p2 | p0, bit 2 = ~(p1 & p0), and the sign kept.  Checked exhaustively on
+// the host against the table.
+__device__ __forceinline__ uint32_t residual_word(uint32_t w) {
+  const uint32_t r1 = w >> 1, r2 = w >> 2, l1 = w << 1, l2 = w << 2;
+  uint32_t a, b, c, d;
+  MIXFP4_LOP3(a, 0x22222222u, r1, l1, 0xBF);        // ~K | ~r1 | l1
+  MIXFP4_LOP3(b, 0x44444444u, l1, l2, 0x7F);        // ~K | ~(l1 & l2)
+  MIXFP4_LOP3(c, w, a, b, 0x80);                    // w & a & b
+  MIXFP4_LOP3(d, c, r2, 0x11111111u, 0x70);         // c & (~r2 | ~K)
+  return d;
+}
+// Scale bytes of a residual row: the scale (type bit cleared) where the type
+// bit is set, else 0 (prmt with the sign-replicate selectors gives 0xFF per
+// byte whose bit 7 is set).
+__device__ __forceinline__ uint32_t residual_scales(uint32_t sw) {
+  uint32_t m;
+  asm("prmt.b32 %0, %1, %2, 0xBA98;" : "=r"(m) : "r"(sw), "r"(0u));
+  return sw & m & 0x7F7F7F7Fu;
 }
 
 // Row r's four ue4m3 scales of K step j in the tiled layout of a 128-row tile.
@@ -571,26 +598,20 @@ nvf4_fewrows_kernel(const __grid_constant__ CUtensorMap tm_wc, const __grid_cons
     if (e > u + chunk_units) e = u + chunk_units;
     return e;
   };
-  const uint32_t stage_bytes = WR * ROWB + WR * 16 + (uint32_t)nx * (ROWB + 16);
-  const int CS = code_stage_bytes(nx), NCS = code_stages(nx);
-  const uint32_t OFF_XS = (uint32_t)(OFF_XC + nx * ROWB);
-  const uint32_t sbase = smem_u32(smem) + OFF_RINGS;          // code ring, then the split ring
-  const uint32_t OFF_SPLIT = (uint32_t)(NCS * CS);
+  const int XR = xr_of(nx);
+  const uint32_t OB = (uint32_t)off_b(XR), OWS = (uint32_t)off_ws(XR), OXS = (uint32_t)off_xs(XR);
+  const uint32_t OSFA = (uint32_t)off_sfa(XR), OSFB = (uint32_t)off_sfb(XR), OSFR = (uint32_t)off_sfr(XR);
+  const uint32_t SB = (uint32_t)stage_bytes_of(XR);
+  const int NST = stages_of(XR);
+  const uint32_t tx_bytes = WR * ROWB + WR * 16 + (uint32_t)nx * (ROWB + 16);
+  const uint32_t sbase = smem_u32(smem) + OFF_RINGS;
 
-  // Split stages start as zeros: activation rows >= nx (and their residual
-  // rows and scales) are never written, so they stay zero.
-  for (uint32_t i = threadIdx.x; i < (uint32_t)(kSplitStages * SPLIT_STAGE / 16); i += blockDim.x)
-    sts128(sbase + OFF_SPLIT + i * 16, 0u, 0u, 0u, 0u);
-  fence_proxy_async_smem();
   if (threadIdx.x == 0) {
-    for (int s = 0; s < NCS; ++s) {
-      mbar_init(smem_u32(&bars->code_full[s]), 1);
-      mbar_init(smem_u32(&bars->code_empty[s]), kWSplitWarps + kXSplitWarps);
-    }
-    for (int s = 0; s < kSplitStages; ++s) {
+    for (int s = 0; s < NST; ++s) {
+      mbar_init(smem_u32(&bars->full[s]), 1);
       mbar_init(smem_u32(&bars->split_full[s]), kWSplitWarps + kXSplitWarps);
       mbar_init(smem_u32(&bars->sf_full[s]), kCopyWarps);
-      mbar_init(smem_u32(&bars->split_empty[s]), 1);
+      mbar_init(smem_u32(&bars->empty[s]), 1);
     }
     mbar_init(smem_u32(&bars->acc_full), 1);
     mbar_init(smem_u32(&bars->acc_empty), 4);
@@ -625,31 +646,30 @@ nvf4_fewrows_kernel(const __grid_constant__ CUtensorMap tm_wc, const __grid_cons
       int it = 0;
       long long last = -1;
       for (long long u = u_begin; u < u_end; ++u, ++it) {
-        const int s = it % NCS;
-        if (!mbar_wait(smem_u32(&bars->code_empty[s]), ((it / NCS) & 1) ^ 1, abort_flag, kWaitLimitNs)) {
+        const int s = it % NST;
+        if (!mbar_wait(smem_u32(&bars->empty[s]), ((it / NST) & 1) ^ 1, abort_flag, kWaitLimitNs)) {
           fail(1u);
           break;
         }
         const int g = (int)(u / num_kc), kc = (int)(u % num_kc);
-        const uint32_t st = sbase + s * CS;
-        const uint32_t fb = smem_u32(&bars->code_full[s]);
-        mbar_arrive_expect_tx(fb, stage_bytes);
-        tma_load_2d(st + OFF_WC, &tm_wc, kc * ROWB, g * WR, fb);
-        tma_load_2d(st + OFF_WS, &tm_ws, kc * 16, g * WR, fb);
-        tma_load_2d(st + OFF_XC, &tm_xc, kc * ROWB, 0, fb);
-        tma_load_2d(st + OFF_XS, &tm_xs, kc * 16, 0, fb);
+        const uint32_t st = sbase + s * SB;
+        const uint32_t fb = smem_u32(&bars->full[s]);
+        mbar_arrive_expect_tx(fb, tx_bytes);
+        tma_load_2d(st + OB, &tm_wc, kc * ROWB, g * WR, fb);
+        tma_load_2d(st + OWS, &tm_ws, kc * 16, g * WR, fb);
+        tma_load_2d(st, &tm_xc, kc * ROWB, 0, fb);
+        tma_load_2d(st + OXS, &tm_xs, kc * 16, 0, fb);
         last = it;
       }
       if (*abort_flag)
-        for (long long v = last - NCS + 1; v <= last; ++v)
+        for (long long v = last - NST + 1; v <= last; ++v)
           if (v >= 0)
-            mbar_wait(smem_u32(&bars->code_full[v % NCS]), (uint32_t)((v / NCS) & 1), nullptr,
-                      kWaitLimitNs);
+            mbar_wait(smem_u32(&bars->full[v % NST]), (uint32_t)((v / NST) & 1), nullptr, kWaitLimitNs);
     }
   } else if (warp == 1) {
     // ---------------- MMA issuer ----------------
     if (lane == 0) {
-      constexpr uint32_t kIdesc = idesc_nvf4_f32(2 * XR, 2 * WR);
+      constexpr uint32_t kIdesc = idesc_nvf4_f32(128, 2 * WR);
       int it = 0, run = 0;
       bool ok = true;
       for (long long u = u_begin; u < u_end && ok; ++run) {
@@ -661,23 +681,22 @@ nvf4_fewrows_kernel(const __grid_constant__ CUtensorMap tm_wc, const __grid_cons
         tc_fence_after();
         bool first = true;
         for (; u < run_end; ++u, ++it) {
-          const int s = it % kSplitStages;
-          if (!mbar_wait(smem_u32(&bars->sf_full[s]), (uint32_t)((it / kSplitStages) & 1), abort_flag,
-                         kWaitLimitNs)) {
+          const int s = it % NST;
+          if (!mbar_wait(smem_u32(&bars->sf_full[s]), (uint32_t)((it / NST) & 1), abort_flag, kWaitLimitNs)) {
             fail(4u);
             ok = false;
             break;
           }
           tc_fence_after();
-          const uint32_t sp = sbase + OFF_SPLIT + s * SPLIT_STAGE;
+          const uint32_t sp = sbase + s * SB;
 #pragma unroll
           for (int j = 0; j < BKC / 64; ++j) {
             const uint32_t sfa = tmem_sf0 + (uint32_t)(s * 4 + j) * kSfCols, sfb = sfa + 4;
-            mma_nvf4(tmem_base, smem_desc_sw128(sp + S_A + j * 32), smem_desc_sw128(sp + S_B + j * 32), kIdesc, sfa,
-                     sfb, first ? 0u : 1u);
+            mma_nvf4(tmem_base, smem_desc_sw128(sp + j * 32), smem_desc_sw128(sp + OB + j * 32), kIdesc, sfa, sfb,
+                     first ? 0u : 1u);
             first = false;
           }
-          mma_commit(smem_u32(&bars->split_empty[s]));
+          mma_commit(smem_u32(&bars->empty[s]));
         }
         if (ok) mma_commit(smem_u32(&bars->acc_full));
       }
@@ -686,39 +705,38 @@ nvf4_fewrows_kernel(const __grid_constant__ CUtensorMap tm_wc, const __grid_cons
     }
   } else if (warp >= kCopyWarp) {
     // ---------------- scale copies ----------------
-    // Once a stage is split, its A and B scale tiles go to tensor memory
-    // (tcgen05.cp, replicated to the four lane quarters; the B tile twice, for
-    // the main and residual halves of N) and the commits tell the MMA thread;
-    // the two copy warps take K steps 0-1 and 2-3.  A stage's columns are
-    // rewritten only after its next split, which waits for the MMAs that
-    // read them.
+    // Once a stage's scale tiles are written, the A tile's scales, the weight
+    // main rows' scales and the weight residual rows' scales go to tensor
+    // memory (tcgen05.cp, replicated to the four lane quarters) and the
+    // commit tells the MMA thread; the two copy warps take K steps 0-1 and
+    // 2-3.  A stage's columns are rewritten only after its next split, which
+    // follows the MMAs that read them.
     const int j0 = 2 * (warp - kCopyWarp);
     if (lane == 0) {
       int it = 0;
       for (long long u = u_begin; u < u_end; ++u, ++it) {
-        const int s = it % kSplitStages;
-        if (!mbar_wait(smem_u32(&bars->split_full[s]), (uint32_t)((it / kSplitStages) & 1), abort_flag,
-                       kWaitLimitNs)) {
+        const int s = it % NST;
+        if (!mbar_wait(smem_u32(&bars->split_full[s]), (uint32_t)((it / NST) & 1), abort_flag, kWaitLimitNs)) {
           fail(128u);
           break;
         }
         tc_fence_after();
-        const uint32_t sp = sbase + OFF_SPLIT + s * SPLIT_STAGE;
+        const uint32_t sp = sbase + s * SB;
 #pragma unroll
         for (int j = j0; j < j0 + 2; ++j) {
           const uint32_t sfa = tmem_sf0 + (uint32_t)(s * 4 + j) * kSfCols, sfb = sfa + 4;
-          tmem_cp_32x128b_x4(sfa, smem_desc_noswizzle(sp + S_SFA + j * 512, 128, 128));
-          tmem_cp_32x128b_x4(sfb, smem_desc_noswizzle(sp + S_SFB + j * 512, 128, 128));
-          tmem_cp_32x128b_x4(sfb + 4, smem_desc_noswizzle(sp + S_SFB + j * 512, 128, 128));
+          tmem_cp_32x128b_x4(sfa, smem_desc_noswizzle(sp + OSFA + j * 512, 128, 128));
+          tmem_cp_32x128b_x4(sfb, smem_desc_noswizzle(sp + OSFB + j * 512, 128, 128));
+          tmem_cp_32x128b_x4(sfb + 4, smem_desc_noswizzle(sp + OSFR + j * 512, 128, 128));
         }
         mma_commit(smem_u32(&bars->sf_full[s]));
       }
     }
   } else if (warp < kFirstEpi) {
-    // ---------------- splitters ----------------
-    // Weights: thread t of 512 splits row t / 4, chunks 2 (t % 4) and +1
-    // (blocks 4 (t % 4) .. +3, scale word t % 4).  Activations: thread t of
-    // 128 splits chunks q = t + 128 i (row q / 8, chunk q % 8) of rows < nx.
+    // ---------------- residual rows and scale tiles ----------------
+    // Weights: thread t of 512 takes row t / 4, chunks 2 (t % 4) and +1 and
+    // scale word t % 4 (K step t % 4).  Activations: thread t of 128 takes
+    // chunks q = t + 128 i (row q / 8, chunk q % 8) of rows < nx.
     const bool is_w = warp < kFirstX;
     const int t = is_w ? (warp - kFirstW) * 32 + lane : (warp - kFirstX) * 32 + lane;
     auto pick = [](const uint4& v, int i) {  // v[i] without dynamic indexing
@@ -726,68 +744,55 @@ nvf4_fewrows_kernel(const __grid_constant__ CUtensorMap tm_wc, const __grid_cons
     };
     int it = 0;
     for (long long u = u_begin; u < u_end; ++u, ++it) {
-      const int s = it % NCS, sps = it % kSplitStages;
-      if (!mbar_wait(smem_u32(&bars->code_full[s]), (uint32_t)((it / NCS) & 1), abort_flag,
-                     kWaitLimitNs)) {
+      const int s = it % NST;
+      if (!mbar_wait(smem_u32(&bars->full[s]), (uint32_t)((it / NST) & 1), abort_flag, kWaitLimitNs)) {
         fail(16u);
         break;
       }
-      if (!mbar_wait(smem_u32(&bars->split_empty[sps]), (uint32_t)(((it / kSplitStages) & 1) ^ 1), abort_flag,
-                     kWaitLimitNs)) {
-        fail(32u);
-        break;
-      }
-      const uint32_t st = sbase + s * CS, sp = sbase + OFF_SPLIT + sps * SPLIT_STAGE;
+      const uint32_t sp = sbase + s * SB;
       if (is_w) {
         const int row = t >> 2, q4 = t & 3;
         const uint32_t swz = (uint32_t)(row & 7);
-        const uint4 sc = lds128(st + OFF_WS + (uint32_t)row * 16);
-        const uint32_t sw = pick(sc, q4);
 #pragma unroll
         for (int k = 0; k < 2; ++k) {
-          const uint32_t pc = ((uint32_t)(2 * q4 + k) ^ swz) << 4;
-          const uint32_t tb = sw >> (16 * k);
-          uint4 m, r;
-          split_chunk(lds128(st + OFF_WC + (uint32_t)row * ROWB + pc), (tb & 0x80u) != 0, (tb & 0x8000u) != 0, m, r);
-          sts128(sp + S_B + (uint32_t)row * ROWB + pc, m.x, m.y, m.z, m.w);
-          sts128(sp + S_B + (uint32_t)(row + WR) * ROWB + pc, r.x, r.y, r.z, r.w);
+          const uint32_t a = sp + OB + (uint32_t)row * ROWB + ((((uint32_t)(2 * q4 + k)) ^ swz) << 4);
+          const uint4 c = lds128(a);
+          sts128(a + WR * ROWB, residual_word(c.x), residual_word(c.y), residual_word(c.z), residual_word(c.w));
         }
-        // Scales of K step q4 into the tiled layout (bit 7, the type, cleared).
-        sts32(sp + S_SFB + q4 * 512 + sf_offset(row), sw & 0x7F7F7F7Fu);
+        const uint32_t sw = lds32(sp + OWS + (uint32_t)row * 16 + (uint32_t)q4 * 4);
+        sts32(sp + OSFB + q4 * 512 + sf_offset(row), sw & 0x7F7F7F7Fu);
+        sts32(sp + OSFR + q4 * 512 + sf_offset(row), residual_scales(sw));
       } else {
 #pragma unroll 1
         for (int q = t; q < nx * 8; q += kXSplitWarps * 32) {
-          const int row = q >> 3, c = q & 7;
-          const uint32_t pc = ((uint32_t)c ^ (uint32_t)(row & 7)) << 4;
-          const uint4 sc = lds128(st + OFF_XS + (uint32_t)row * 16);
-          const uint32_t sw = pick(sc, c >> 1), tb = sw >> (16 * (c & 1));
-          uint4 m, r;
-          split_chunk(lds128(st + OFF_XC + (uint32_t)row * ROWB + pc), (tb & 0x80u) != 0, (tb & 0x8000u) != 0, m, r);
-          sts128(sp + S_A + (uint32_t)row * ROWB + pc, m.x, m.y, m.z, m.w);
-          sts128(sp + S_A + (uint32_t)(row + XR) * ROWB + pc, r.x, r.y, r.z, r.w);
-          if ((c & 1) == 0) {  // scale word c / 2 = K step c / 2, for the main and residual rows
-            sts32(sp + S_SFA + (c >> 1) * 512 + sf_offset(row), sw & 0x7F7F7F7Fu);
-            sts32(sp + S_SFA + (c >> 1) * 512 + sf_offset(row + XR), sw & 0x7F7F7F7Fu);
+          const int row = q >> 3, c8 = q & 7;
+          const uint32_t a = sp + (uint32_t)row * ROWB + ((((uint32_t)c8) ^ (uint32_t)(row & 7)) << 4);
+          const uint4 c = lds128(a);
+          sts128(a + (uint32_t)XR * ROWB, residual_word(c.x), residual_word(c.y), residual_word(c.z),
+                 residual_word(c.w));
+          if (c8 < 4) {  // scale word c8 = K step c8, for the main and residual rows
+            const uint32_t sw = lds32(sp + OXS + (uint32_t)row * 16 + (uint32_t)c8 * 4);
+            sts32(sp + OSFA + c8 * 512 + sf_offset(row), sw & 0x7F7F7F7Fu);
+            sts32(sp + OSFA + c8 * 512 + sf_offset(row + XR), residual_scales(sw));
           }
         }
       }
       fence_proxy_async_smem();
       __syncwarp();
-      if (lane == 0) {
-        mbar_arrive(smem_u32(&bars->split_full[sps]));
-        mbar_arrive(smem_u32(&bars->code_empty[s]));
-      }
+      if (lane == 0) mbar_arrive(smem_u32(&bars->split_full[s]));
     }
   } else {
     // ---------------- epilogue ----------------
-    // Warps for lane quarters 0, 1 hold the activation rows' main products,
-    // quarters 2, 3 their residual products (row m + 64); both add into C.
+    // Accumulator lane d (quarter q = warp % 4, d = 32 q + lane) holds
+    // activation row d mod XR: main products for d < XR, residual products
+    // for XR <= d < 2 XR; both add into C.
     const int q = warp & 3;
-    const int m = (q & 1) * 32 + lane;
+    const int d = q * 32 + lane;
+    const int m = d % XR;
     griddep_wait();
     const float sa = __ldg(a_ts), sb = __ldg(b_ts);
     const bool vec_ok = ((ldc & 3) == 0) && ((reinterpret_cast<uintptr_t>(C) & 15) == 0);
-    const bool mine = (q & 1) * 32 < Mx;
+    const bool mine = q * 32 < 2 * XR && (q * 32) % XR < Mx;
     const uint32_t tb = tmem_base + ((uint32_t)(q * 32) << 16);
     int run = 0;
     for (long long u = u_begin; u < u_end; ++run) {
@@ -815,7 +820,7 @@ nvf4_fewrows_kernel(const __grid_constant__ CUtensorMap tm_wc, const __grid_cons
           if (lane == 0) mbar_arrive(smem_u32(&bars->acc_empty));
         }
         const int n0 = g * WR + cc * 16;
-        if (mine && m < Mx) {
+        if (mine && d < 2 * XR && m < Mx) {
           float* crow = C + (long long)m * ldc + n0;
           float o[16];
 #pragma unroll
@@ -851,7 +856,8 @@ int launch(const uint8_t* a_codes, const uint8_t* a_scales, const float* a_ts, c
       !make_map(&txc, a_codes, (uint64_t)K / 2, (uint64_t)M, ROWB, (uint32_t)nx, CU_TENSOR_MAP_SWIZZLE_128B) ||
       !make_map(&txs, a_scales, (uint64_t)K / 16, (uint64_t)M, 16, (uint32_t)nx, CU_TENSOR_MAP_SWIZZLE_NONE))
     return MIXFP4_ERR_CUDA;
-  const int smem = OFF_RINGS + code_stages(nx) * code_stage_bytes(nx) + kSplitStages * SPLIT_STAGE + 1024;
+  const int xr = xr_of(nx);
+  const int smem = OFF_RINGS + stages_of(xr) * stage_bytes_of(xr) + 1024;
   static std::atomic<uint64_t> smem_set{0};
   if (!set_dynamic_smem_once(reinterpret_cast<const void*>(nvf4_fewrows_kernel), 232448, smem_set))
     return MIXFP4_ERR_CUDA;

@@ -161,11 +161,14 @@ def test_native_full_size_workloads(oracle, name):
         assert_close(Cg, A @ B.T, A, B)
 
 
-@pytest.mark.parametrize("M,N,K", [(1, 128, 256), (16, 300, 768), (33, 1000, 512), (64, 256, 2048), (7, 129, 1280)])
+@pytest.mark.parametrize("M,N,K", [(1, 128, 256), (16, 300, 768), (33, 1000, 512), (64, 256, 2048), (7, 129, 1280),
+                                   (20, 384, 1024), (32, 640, 4352)])
 def test_fewrows_native_gemm(oracle, M, N, K):
     """The few-row native path splits the stored MixFP4 operands on the fly:
     one or several 128-row weight groups, a ragged last group, activation
-    rows from 1 to 64, several K slices per CTA."""
+    rows from 1 to 64 (all three activation tile heights: up to 16, 32 and 64
+    rows), several K slices per CTA, a run crossing a 4096-K accumulation
+    chunk."""
     x = synth.activations(M, K, 8600 + M, 8601)
     w = synth.weights(N, K, 8602 + N, 0.02, 0.5)
     qa, ra = quant_both(oracle, x)

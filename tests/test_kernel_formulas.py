@@ -6,6 +6,8 @@ include every tie.  The GPU parity tests check the kernels themselves; these
 pin the derivations the kernels rely on.
 
 * the E1M2 main / residual split (native FP4 variant): eight `lop3` per word
+* the few-row native kernel's residual of a stored code (four `lop3` per word)
+  and its residual scale bytes (`prmt` sign replication)
 * branch-free E3M0 rounding (candidate-set ablation, reading R14)
 * the stochastic-rounding payload shared by both formats (reading R13)
 * the 16 x 16 nibble transpose in registers (2D transpose)
@@ -65,6 +67,54 @@ def test_lop3_split_matches_oracle_for_every_nibble_and_position(oracle, t):
         m, r = split_e1m2_word(w, M32 if t else 0)
         assert m == int(np.frombuffer(main[i, :4].tobytes(), np.uint32)[0]), (hex(w), t)
         assert r == int(np.frombuffer(res[i, :4].tobytes(), np.uint32)[0]), (hex(w), t)
+
+
+def residual_word(w: int) -> int:
+    """The few-row native kernel's residual codes of eight nibbles,
+    instruction by instruction: payload {0,1,2,3,4,4,4,2}[p], sign kept."""
+    r1, r2, l1, l2 = w >> 1, w >> 2, (w << 1) & M32, (w << 2) & M32
+    a = lop3(0x22222222, r1, l1, 0xBF)
+    b = lop3(0x44444444, l1, l2, 0x7F)
+    c = lop3(w, a, b, 0x80)
+    return lop3(c, r2, 0x11111111, 0x70)
+
+
+def prmt_sign_replicate(a: int) -> int:
+    """prmt.b32 d, a, 0, 0xBA98: selector nibbles 8..B pick bytes 0..3 of a
+    with the sign-replicate bit set, so each byte becomes 0xFF or 0x00 by its
+    bit 7."""
+    return sum((0xFF if (a >> (8 * i)) & 0x80 else 0) << (8 * i) for i in range(4))
+
+
+def residual_scales(sw: int) -> int:
+    return sw & prmt_sign_replicate(sw) & 0x7F7F7F7F
+
+
+@pytest.mark.parametrize("t", [0, 1])
+def test_fewrows_residual_reconstructs_every_value(oracle, t):
+    """The stored code read as E2M1 (scale with the type bit cleared) plus the
+    residual code (scale from residual_scales) equals the MixFP4 value of the
+    stored code, for every nibble in every position and both block types;
+    values from the oracle's dequantizer.  Scale 0x38 (1.0) and 0x01 (the
+    smallest subnormal) both checked."""
+    for scale in (0x38, 0x01):
+        sbyte = scale | (t << 7)
+        rows = []
+        for pos in range(8):
+            for nib in range(16):
+                rows.append((nib << (4 * pos)) | (((nib + 5) & 15) << (4 * ((pos + 3) % 8))))
+        codes = np.zeros((len(rows), 8), np.uint8)       # K = 16: one block per row
+        res = np.zeros_like(codes)
+        for i, w in enumerate(rows):
+            codes[i, :4] = np.frombuffer(np.uint32(w).tobytes(), np.uint8)
+            res[i, :4] = np.frombuffer(np.uint32(residual_word(w)).tobytes(), np.uint8)
+        sw = sbyte * 0x01010101
+        main_scale = np.full((len(rows), 1), (sw & 0x7F7F7F7F) & 0xFF, np.uint8)
+        res_scale = np.full((len(rows), 1), residual_scales(sw) & 0xFF, np.uint8)
+        want = oracle.dequantize(codes, np.full((len(rows), 1), sbyte, np.uint8), 1.0).astype(np.float64)
+        got = (oracle.dequantize(codes, main_scale, 1.0).astype(np.float64)
+               + oracle.dequantize(res, res_scale, 1.0).astype(np.float64))
+        assert np.array_equal(got, want), (t, scale)
 
 
 def f32(v):
