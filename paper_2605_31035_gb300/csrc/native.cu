@@ -493,9 +493,10 @@ int launch(const uint8_t* a_main, const uint8_t* a_res, const uint8_t* a_sf, con
 //               into a ring of 3-5 stages (by the row count);
 //   warp 1      TMEM allocation; lane 0 issues the MMAs (one per 64-K step)
 //               and frees the stage with their commit;
-//   warps 2-17  weight residual rows (four threads per row, two 16-byte
-//               chunks each) and weight scale tiles; warps 18-21 the same
-//               for the activation rows;
+//   warps 2-17  weight scale tiles (announced first, so their copies to
+//               tensor memory overlap the rest), then the weight residual
+//               rows (four threads per row, two 16-byte chunks each); warps
+//               18-21 the same for the activation rows;
 //   warps 22-25 epilogue, one TMEM lane quarter each;
 //   warps 26-27 copy each stage's scale tiles into tensor memory
 //               (tcgen05.cp, half of the K steps each) and commit.
@@ -540,8 +541,9 @@ static_assert(kAccCols + kMaxStages * 4 * kSfCols <= kTmemCols, "TMEM budget");
 
 struct Bars {
   uint64_t full[kMaxStages];        // TMA landed
-  uint64_t split_full[kMaxStages];  // residual rows and scale tiles written
+  uint64_t split_full[kMaxStages];  // residual rows written
   uint64_t sf_full[kMaxStages];     // the stage's scales are in tensor memory (commit of the copy warps)
+  uint64_t sf_ready[kMaxStages];    // the stage's scale tiles are written
   uint64_t empty[kMaxStages];       // the stage's MMAs completed
   uint64_t acc_full;
   uint64_t acc_empty;
@@ -611,6 +613,7 @@ nvf4_fewrows_kernel(const __grid_constant__ CUtensorMap tm_wc, const __grid_cons
       mbar_init(smem_u32(&bars->full[s]), 1);
       mbar_init(smem_u32(&bars->split_full[s]), kWSplitWarps + kXSplitWarps);
       mbar_init(smem_u32(&bars->sf_full[s]), kCopyWarps);
+      mbar_init(smem_u32(&bars->sf_ready[s]), kWSplitWarps + kXSplitWarps);
       mbar_init(smem_u32(&bars->empty[s]), 1);
     }
     mbar_init(smem_u32(&bars->acc_full), 1);
@@ -682,7 +685,8 @@ nvf4_fewrows_kernel(const __grid_constant__ CUtensorMap tm_wc, const __grid_cons
         bool first = true;
         for (; u < run_end; ++u, ++it) {
           const int s = it % NST;
-          if (!mbar_wait(smem_u32(&bars->sf_full[s]), (uint32_t)((it / NST) & 1), abort_flag, kWaitLimitNs)) {
+          if (!mbar_wait(smem_u32(&bars->split_full[s]), (uint32_t)((it / NST) & 1), abort_flag, kWaitLimitNs) ||
+              !mbar_wait(smem_u32(&bars->sf_full[s]), (uint32_t)((it / NST) & 1), abort_flag, kWaitLimitNs)) {
             fail(4u);
             ok = false;
             break;
@@ -705,18 +709,19 @@ nvf4_fewrows_kernel(const __grid_constant__ CUtensorMap tm_wc, const __grid_cons
     }
   } else if (warp >= kCopyWarp) {
     // ---------------- scale copies ----------------
-    // Once a stage's scale tiles are written, the A tile's scales, the weight
-    // main rows' scales and the weight residual rows' scales go to tensor
-    // memory (tcgen05.cp, replicated to the four lane quarters) and the
-    // commit tells the MMA thread; the two copy warps take K steps 0-1 and
-    // 2-3.  A stage's columns are rewritten only after its next split, which
+    // Once a stage's scale tiles are written (before its residual rows), the
+    // A tile's scales, the weight main rows' scales and the weight residual
+    // rows' scales go to tensor memory (tcgen05.cp, replicated to the four
+    // lane quarters) and the commit tells the MMA thread, which also waits
+    // for the residual rows; the two copy warps take K steps 0-1 and 2-3.  A
+    // stage's columns are rewritten only after its next TMA landing, which
     // follows the MMAs that read them.
     const int j0 = 2 * (warp - kCopyWarp);
     if (lane == 0) {
       int it = 0;
       for (long long u = u_begin; u < u_end; ++u, ++it) {
         const int s = it % NST;
-        if (!mbar_wait(smem_u32(&bars->split_full[s]), (uint32_t)((it / NST) & 1), abort_flag, kWaitLimitNs)) {
+        if (!mbar_wait(smem_u32(&bars->sf_ready[s]), (uint32_t)((it / NST) & 1), abort_flag, kWaitLimitNs)) {
           fail(128u);
           break;
         }
@@ -753,16 +758,30 @@ nvf4_fewrows_kernel(const __grid_constant__ CUtensorMap tm_wc, const __grid_cons
       if (is_w) {
         const int row = t >> 2, q4 = t & 3;
         const uint32_t swz = (uint32_t)(row & 7);
+        {
+          const uint32_t sw = lds32(sp + OWS + (uint32_t)row * 16 + (uint32_t)q4 * 4);
+          sts32(sp + OSFB + q4 * 512 + sf_offset(row), sw & 0x7F7F7F7Fu);
+          sts32(sp + OSFR + q4 * 512 + sf_offset(row), residual_scales(sw));
+        }
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(smem_u32(&bars->sf_ready[s]));
 #pragma unroll
         for (int k = 0; k < 2; ++k) {
           const uint32_t a = sp + OB + (uint32_t)row * ROWB + ((((uint32_t)(2 * q4 + k)) ^ swz) << 4);
           const uint4 c = lds128(a);
           sts128(a + WR * ROWB, residual_word(c.x), residual_word(c.y), residual_word(c.z), residual_word(c.w));
         }
-        const uint32_t sw = lds32(sp + OWS + (uint32_t)row * 16 + (uint32_t)q4 * 4);
-        sts32(sp + OSFB + q4 * 512 + sf_offset(row), sw & 0x7F7F7F7Fu);
-        sts32(sp + OSFR + q4 * 512 + sf_offset(row), residual_scales(sw));
       } else {
+        for (int q = t; q < nx * 4; q += kXSplitWarps * 32) {  // scale word q % 4 of row q / 4
+          const int row = q >> 2, j = q & 3;
+          const uint32_t sw = lds32(sp + OXS + (uint32_t)row * 16 + (uint32_t)j * 4);
+          sts32(sp + OSFA + j * 512 + sf_offset(row), sw & 0x7F7F7F7Fu);
+          sts32(sp + OSFA + j * 512 + sf_offset(row + XR), residual_scales(sw));
+        }
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(smem_u32(&bars->sf_ready[s]));
 #pragma unroll 1
         for (int q = t; q < nx * 8; q += kXSplitWarps * 32) {
           const int row = q >> 3, c8 = q & 7;
@@ -770,11 +789,6 @@ nvf4_fewrows_kernel(const __grid_constant__ CUtensorMap tm_wc, const __grid_cons
           const uint4 c = lds128(a);
           sts128(a + (uint32_t)XR * ROWB, residual_word(c.x), residual_word(c.y), residual_word(c.z),
                  residual_word(c.w));
-          if (c8 < 4) {  // scale word c8 = K step c8, for the main and residual rows
-            const uint32_t sw = lds32(sp + OXS + (uint32_t)row * 16 + (uint32_t)c8 * 4);
-            sts32(sp + OSFA + c8 * 512 + sf_offset(row), sw & 0x7F7F7F7Fu);
-            sts32(sp + OSFA + c8 * 512 + sf_offset(row + XR), residual_scales(sw));
-          }
         }
       }
       fence_proxy_async_smem();
