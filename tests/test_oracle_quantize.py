@@ -156,6 +156,46 @@ def test_brute_force_tiny_blocks(oracle):
                 assert T == 1  # strict "<" of Alg. 1: ties go to E1M2
 
 
+def _rne_codebook(y, book):
+    """R4: the codebook value nearest to the fp32 quotient y, ties to the
+    even payload, saturating at the largest value (exact comparisons)."""
+    yq = Fraction(float(y))
+    return min(range(8), key=lambda p: (abs(Fraction(book[p]) - yq), p % 2))
+
+
+def test_error_sums_match_exact_mse(oracle):
+    """Both candidates' error sums S (the comparison of Algorithm 1) against
+    the exact rational sum of squared errors of the codes that reading R4
+    defines: |S - S_exact| <= 16 u S_exact (u = 2^-24; each fma chain adds
+    at most 8 roundings, the final sum one).  Random bf16 normals with
+    outlier channels, both block types, every block; a dropped term, a wrong
+    sign or a swapped operand in the error shows up here."""
+    rng = np.random.default_rng(77)
+    rows, nb = 16, 8
+    x = rng.standard_normal((rows, nb * 16)).astype(np.float32)
+    x[:, rng.integers(0, nb * 16, 6)] *= 40.0
+    bits = torch.tensor(x).to(torch.bfloat16).view(torch.int16).numpy().view(np.uint16)
+    xf = bits_to_f32(bits)
+    codes, scales, s32, e2, e1 = oracle.quantize(bits, want_errors=True)
+    books = [[oracle.fp4_value(f, p) for p in range(8)] for f in (0, 1)]
+    u = Fraction(1, 2 ** 24)
+    checked = 0
+    for r in range(rows):
+        for b in range(nb):
+            a = np.abs(xf[r, b * 16:(b + 1) * 16]) / np.float32(s32)   # fl32(|x| / s32)
+            B = np.float32(a.max())
+            for fmt, S in ((0, float(e2[r, b])), (1, float(e1[r, b]))):
+                c = np.float32(6.0 if fmt == 0 else 7.0)
+                s8 = oracle.e4m3_value(oracle.e4m3_rne(float(np.float32(B / c))))
+                exact = Fraction(0)
+                for ai in a:
+                    q = _rne_codebook(np.float32(ai) / np.float32(s8), books[fmt]) if s8 > 0 else 0
+                    exact += (Fraction(books[fmt][q]) * Fraction(s8) - Fraction(float(ai))) ** 2
+                assert abs(Fraction(S) - exact) <= 16 * u * exact, (r, b, fmt, S, float(exact))
+                checked += 1
+    assert checked == rows * nb * 2
+
+
 def test_type_bit_consistency(oracle):
     """App. B.3: a MixFP4 block with T=0 is byte-identical to the E2M1-only
     (NVFP4) quantization of the same block, and with T=1 to the E1M2-only one."""
