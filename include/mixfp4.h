@@ -337,13 +337,19 @@ int mixfp4_gemm_native(const uint8_t* a_main, const uint8_t* a_res, const uint8_
 /*
  * mixfp4_gemm_native_fewrows -- the native block-scaled FP4 variant for few
  * activation rows (decode-shaped GEMMs, M <= 64), taking the MixFP4 operands
- * as stored (the arguments of mixfp4_gemm): each 128-row x 256-K unit of B
- * and the matching slice of A are split into E2M1 main + residual parts in
- * shared memory (as mixfp4_split_native defines them) and contracted by
- * tcgen05.mma kind::mxf4nvf4, one instruction per 64-K step covering all four
- * products (main and residual stacked on the M and N sides).  C is the same
- * product as mixfp4_gemm's up to fp32 summation order; the host zeroes C
- * first and the partial sums of the K slices are added into it.
+ * as stored (the arguments of mixfp4_gemm).  Each operand is the sum of two
+ * E2M1 parts with ue4m3 block-16 scales: the stored codes read as E2M1 codes
+ * (scale: the block scale without its type bit), and a residual whose
+ * payload is {0,1,2,3,4,4,4,2}[p] of the stored payload p (scale: the block
+ * scale for an E1M2 block, 0 for an E2M1 block); for an E1M2 block the two
+ * E2M1 values add up to the E1M2 value p, for an E2M1 block the residual
+ * vanishes.  Each 128-row x 256-K unit of B and the matching slice of A are
+ * loaded as stored, their residual rows and scale tiles are written in
+ * shared memory, and tcgen05.mma kind::mxf4nvf4 contracts them, one
+ * instruction per 64-K step covering all four products (main and residual
+ * stacked on the M and N sides).  C is the same product as mixfp4_gemm's up
+ * to fp32 summation order; the host zeroes C first and the partial sums of
+ * the K slices are added into it.
  * M            0 <= M <= 64 (else MIXFP4_ERR_SHAPE).
  * Other arguments, alignment and errors: as mixfp4_gemm.
  */
