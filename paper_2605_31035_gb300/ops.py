@@ -507,7 +507,8 @@ def mixfp4_gemm_native(a: NativeTensor, b: NativeTensor, out: torch.Tensor | Non
 def mixfp4_gemm_native_fewrows(a: QTensor, b: QTensor, out: torch.Tensor | None = None,
                                status_word: torch.Tensor | None = None, stream=None) -> torch.Tensor:
     """C = A_deq . B_deq^T for a with at most 64 rows, on the block-scaled FP4
-    tensor path with the operands split on the fly."""
+    tensor path: the stored codes are the main E2M1 operands, their residual
+    rows and scale tiles are formed on the fly."""
     _check_operand(a, "a")
     _check_operand(b, "b")
     _require(a.K == b.K and a.rows <= 64 and a.codes.device == b.codes.device,
