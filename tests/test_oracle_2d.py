@@ -112,6 +112,60 @@ def test_2d_brute_force_dyadic_tiles(oracle):
     assert checked > 0
 
 
+def test_2d_random_tiles_codes_and_choice(oracle):
+    """Full-precision tiles (Student-t values with outlier columns, computed
+    s32): every code is reading R4 applied to the fp32 quotient fl32(a / s8)
+    with a = fl32(|x| / s32), the scale byte is the E4M3 cast of
+    fl32(tile_max / c), and the chosen format has the smaller exact tile
+    error (rational sum over the 256 elements of the R4 codes) whenever the
+    two exact errors differ by more than 64 u of the larger: the tree of
+    fp32 row sums cannot reverse such a comparison."""
+    rng = np.random.default_rng(21)
+    rows, K = 64, 96
+    z = rng.standard_normal((4, rows, K)).astype(np.float32)
+    x = z[0] / np.sqrt((z[1] ** 2 + z[2] ** 2 + z[3] ** 2) / 3.0) * 0.5
+    x[:, rng.integers(0, K, 3)] *= 30.0
+    bits = torch.tensor(x).to(torch.bfloat16).view(torch.int16).numpy().view(np.uint16)
+    xf = (bits.astype(np.uint32) << 16).view(np.float32)
+    codes, scales, s32 = oracle.quantize_2d(bits)
+    books = [[oracle.fp4_value(f, p) for p in range(8)] for f in (0, 1)]
+    u = Fraction(1, 2 ** 24)
+
+    def r4(yq, book):
+        yy = Fraction(float(yq))
+        return min(range(8), key=lambda p: (abs(Fraction(book[p]) - yy), p % 2))
+
+    decided = 0
+    for t in range(rows // 16):
+        for b in range(K // 16):
+            a = np.abs(xf[16 * t:16 * t + 16, 16 * b:16 * b + 16]) / np.float32(s32)   # fl32(|x| / s32)
+            B = np.float32(a.max())
+            sb = scales[16 * t:16 * t + 16, b]
+            assert np.all(sb == sb[0])
+            T = sb[0] >> 7
+            errs, s8s = [], []
+            for fmt in (0, 1):
+                code = oracle.e4m3_rne(float(np.float32(B / np.float32(6.0 if fmt == 0 else 7.0))))
+                s8 = oracle.e4m3_value(code)
+                s8s.append((code, s8))
+                e = Fraction(0)
+                for v in a.ravel():
+                    q = r4(np.float32(v) / np.float32(s8), books[fmt]) if s8 > 0 else 0
+                    e += (Fraction(books[fmt][q]) * Fraction(s8) - Fraction(float(v))) ** 2
+                errs.append(e)
+            assert sb[0] & 0x7F == s8s[T][0]
+            s8 = s8s[T][1]
+            for i in range(16):
+                for k in range(16):
+                    nib = (codes[16 * t + i, 8 * b + k // 2] >> (4 * (k & 1))) & 0xF
+                    q = r4(np.float32(a[i, k]) / np.float32(s8), books[T]) if s8 > 0 else 0
+                    assert (nib & 7) == q, (t, b, i, k)
+            if abs(errs[0] - errs[1]) > 64 * u * max(errs):
+                assert T == (0 if errs[0] < errs[1] else 1), (t, b)
+                decided += 1
+    assert decided >= (rows // 16) * (K // 16) // 2
+
+
 def test_2d_negation_and_power_of_two(oracle):
     """Negating X flips only the nibble sign bits; X x 2^k leaves codes and
     scale bytes unchanged and scales s32 by 2^k."""
