@@ -272,7 +272,7 @@ int mixfp4_dequantize(const uint8_t* codes, const uint8_t* scales, const float* 
  * mixfp4_gemm -- MixFP4 x MixFP4 GEMM, C = A_deq . B_deq^T:
  *   C[m][n] = s32A * s32B * sum_blocks (sA * sB) * sum_i vA_i * vB_i
  * (App. B.1 Eq. (factor)), where each block's codes are decoded to the unified
- * E2M2 value (Sec. 3.3, App. B.5) times its E4M3 scale -- exact in bf16 -- and
+ * E2M2 value (Sec. 3.3, App. B.5) times its E4M3 scale -- exact in f16 -- and
  * contracted on the tensor cores with fp32 accumulation.
  *
  * a_codes/a_scales/a_ts   A = activations, M x K, quantized by mixfp4_quantize.
