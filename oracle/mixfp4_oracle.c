@@ -61,6 +61,9 @@
  *   R5 block error: d_i = fl32(q_i*s8 - |a_i|) (the product is exact);
  *      S_even = fma chain over i = 0,2,..,14 from +0, S_odd over 1,3,..,15,
  *      S = fl32(S_even + S_odd); the division by 16 of the mean is omitted.
+ *      The order is a definition (the paper names only the MSE); the sums
+ *      are pinned to the exact rational sum of squares within 16 ulp-units
+ *      by the tests, and the choice to the exact comparison beyond that.
  *   R6 E2M1 is chosen iff S_E2M1 < S_E1M2 (strict), otherwise E1M2 with T=1.
  *   R7 s8 == 0 gives all-zero magnitudes and d_i = -|a_i|; s32 == 0 gives a_i = 0.
  *   R9 element 2j in the low nibble of byte j; codes [rows][K/2], scales
